@@ -1,0 +1,208 @@
+/*
+ * agnes.h -- C ABI of libagnes.so: block-wise, hyperbatch-based multi-hop
+ * neighbour sampling and feature gathering on one GB300 GPU (sm_103a), after
+ * AGNES (arXiv 2601.01473).
+ *
+ * The operation (Algorithm 1, Sec. 3.5): given a graph's topology B_g and
+ * features B_f cut into fixed-size blocks (Sec. 3.2, storage layer) and the
+ * target nodes of a hyperbatch of H minibatches (Sec. 3.3), run K hops of
+ * sampling -- each hop buckets the frontier by (block, minibatch) (the
+ * bucket matrix Bck of Sec. 3.4 (3)), visits every non-empty block row once
+ * for all minibatches, draws up to fanout[h] neighbours per frontier node
+ * and unions the draws per minibatch -- then gather every sampled node's
+ * feature row block by block (Algorithm 1's gathering loop).  The sampled
+ * nodes N_s and gathered features F_g (Algorithm 1's outputs) stay in device
+ * memory, one view per minibatch.
+ *
+ * Semantics fixed by this library where the paper is silent:
+ *  - Sampling is uniform without replacement over a node's adjacency
+ *    positions; a node with deg <= fanout takes all neighbours in CSR order;
+ *    otherwise Floyd's algorithm with Philox4x32-10 draws keyed on
+ *    key = (lo32 seed, hi32 seed), ctr = (v, (hop << 24) | slot,
+ *    lo32 g, hi32 g), g = first_minibatch_id + j, hop = 1..K, and
+ *    t = floor(((x1 << 32) | x0) * (J + 1) / 2^64).  Draws therefore depend
+ *    on the global minibatch id, never on H, the block size or the order of
+ *    work, and results are bit-exact and deterministic.
+ *  - Per hop h of minibatch j: dst_h = the frontier, new_h = the ascending
+ *    unique sampled ids not in dst_h, src_h = dst_h ++ new_h, and
+ *    dst_{h+1} = src_h (hop 1's dst is the targets, in the caller's order).
+ *    col[e] indexes the e-th sampled neighbour in src_h; edges are grouped by
+ *    dst position (indptr) and in draw order within a dst.
+ *  - Feature rows are copied byte for byte (fp32 / fp16 bit patterns,
+ *    NaN payloads included).
+ *
+ * Conventions: every call returns an agnes_status and never throws; on
+ * failure agnes_last_error(ctx) gives a message.  All work of a call is
+ * enqueued on the caller's CUDA stream (NULL = the legacy default stream);
+ * calls on one ctx must not overlap.  Pointers are host or device memory as
+ * stated per argument; the library detects which with
+ * cudaPointerGetAttributes where both are allowed.
+ */
+#ifndef AGNES_H
+#define AGNES_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AGNES_MAX_HOPS 8
+#define AGNES_MAX_FANOUT 1024
+
+typedef enum {
+  AGNES_OK = 0,
+  AGNES_EINVAL = 1,   /* invalid argument or input data */
+  AGNES_ERANGE = 2,   /* sizes overflow the library's index types */
+  AGNES_ENOMEM = 3,   /* device or pinned host allocation failed */
+  AGNES_ECUDA = 4,    /* a CUDA runtime call failed */
+  AGNES_ESTATE = 5,   /* call out of order (e.g. fetch before prepare) */
+  AGNES_ETIMEOUT = 6, /* a bounded host-side wait ran out */
+  AGNES_EKERNEL = 7   /* a kernel reported an internal inconsistency */
+} agnes_status;
+
+typedef enum { AGNES_F32 = 0, AGNES_F16 = 1 } agnes_dtype;
+
+typedef struct agnes_ctx agnes_ctx; /* opaque, owned by the library */
+
+/* Graph description for agnes_load_graph (CSR + row-major features).
+ *  num_nodes   N, 1 <= N < 2^31.
+ *  num_edges   E = offsets[N] (offsets[0] must be 0).
+ *  offsets     N+1 entries of offsets_bits (32 or 64) bits; host or device.
+ *  indices     E int32 neighbour ids in [0, N); host or device.
+ *  features    N x feat_dim elements of feat_dtype, row-major; host or
+ *              device, or pinned host memory when features_on_host = 1.
+ *  adj_block_bytes   size of a topology block (Sec. 3.2); >= 64.
+ *  feat_block_bytes  size of a feature block; >= one feature row.
+ * Host arrays are copied to device memory the library owns.  Device arrays
+ * are borrowed: the caller keeps them alive and unchanged until
+ * agnes_free.  With features_on_host = 1 the feature matrix stays in pinned
+ * host memory (borrowed) and each hyperbatch streams the feature blocks it
+ * needs into device staging slots on a side stream (the asynchronous
+ * block I/O of Sec. 3.4 (4), with the host link standing in for the SSD). */
+typedef struct {
+  int64_t num_nodes;
+  int64_t num_edges;
+  const void* offsets;
+  int32_t offsets_bits;
+  const int32_t* indices;
+  const void* features;
+  int32_t feat_dtype; /* agnes_dtype */
+  int64_t feat_dim;
+  int32_t features_on_host;
+  int64_t adj_block_bytes;
+  int64_t feat_block_bytes;
+} agnes_graph_desc;
+
+/* Loads a graph on `device` and builds its block tables: the object index
+ * table T^g_obj of Sec. 3.2 (greedy in-order packing of objects of
+ * offsets_bits/8 + 4*deg bytes into adj_block_bytes blocks; an object larger
+ * than a block starts a fresh block and spans ceil(size/block) blocks) and
+ * the feature blocks (feat_block_bytes / row_bytes rows each).  Enqueued on
+ * cuda_stream and synchronised before return.  *out receives a new ctx (NULL
+ * on failure).  Errors: EINVAL (bad desc), ERANGE, ENOMEM, ECUDA. */
+agnes_status agnes_load_graph(const agnes_graph_desc* desc, int device, void* cuda_stream,
+                              agnes_ctx** out);
+
+/* Samples K hops and gathers features for a hyperbatch of H minibatches of
+ * B targets each (Algorithm 1).
+ *  targets   H*B int32 node ids, row j = minibatch j's targets (distinct
+ *            within a row); host or device memory.  Host memory is copied
+ *            inside the call (pinned memory makes that copy asynchronous).
+ *  fanouts   K host int32 values, fanouts[0] for the targets' hop;
+ *            1 <= fanouts[h] <= AGNES_MAX_FANOUT, 1 <= K <= AGNES_MAX_HOPS.
+ *  seed, first_minibatch_id  key the random draws (see above).
+ * Stream-ordered: returns once the work is enqueued.  Element-wise checks of
+ * targets (range, distinctness) run on the device and are reported by the
+ * next agnes_fetch_minibatch / agnes_hyperbatch_stats call as EINVAL.
+ * Errors here: EINVAL (bad scalar args), ERANGE (H * capacity >= 2^31 output
+ * rows), ENOMEM, ECUDA. */
+agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, int32_t H,
+                                      int32_t B, const int32_t* fanouts, int32_t K,
+                                      uint64_t seed, uint64_t first_minibatch_id,
+                                      void* cuda_stream);
+
+/* View of minibatch j of the last prepared hyperbatch.  Per hop h (0-based
+ * index, hop number h+1): the bipartite block has num_dst[h] dst nodes
+ * (= nodes[0 .. num_dst[h])) and num_src[h] src nodes
+ * (= nodes[0 .. num_src[h])); indptr[h] (num_dst[h]+1 int64, device) groups
+ * the num_edges[h] edges by dst; col[h] (num_edges[h] int32, device) gives
+ * each edge's src index.  nodes (num_nodes int32, device) = src_K in global
+ * ids; feats (num_nodes x feat_dim of feat_dtype, device, row-major) their
+ * gathered rows.  All pointers are owned by ctx and stay valid until the
+ * next agnes_prepare_hyperbatch or agnes_free. */
+typedef struct {
+  int32_t K;
+  int64_t num_dst[AGNES_MAX_HOPS];
+  int64_t num_src[AGNES_MAX_HOPS];
+  int64_t num_edges[AGNES_MAX_HOPS];
+  const int64_t* indptr[AGNES_MAX_HOPS];
+  const int32_t* col[AGNES_MAX_HOPS];
+  const int32_t* nodes;
+  int64_t num_nodes;
+  const void* feats;
+  int32_t feat_dtype;
+  int64_t feat_dim;
+} agnes_minibatch_view;
+
+/* Fills *out for minibatch j (0 <= j < H).  The first fetch after a prepare
+ * waits for that hyperbatch's work (host-side, on an event) and reads its
+ * sizes back once.  Errors: ESTATE (no hyperbatch), EINVAL (bad j, or bad
+ * targets found on the device), ECUDA. */
+agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_view* out);
+
+/* Blocks touched by the last hyperbatch (the block-wise I/Os of Sec. 3.3 and
+ * Fig. 7): out[h] for h < K = distinct topology blocks holding a node of
+ * some minibatch's hop-(h+1) frontier; out[K] = distinct feature blocks
+ * holding a gathered node.  out has K+1 host entries.  Waits like fetch. */
+agnes_status agnes_hyperbatch_stats(agnes_ctx* ctx, int64_t* out);
+
+/* Whole-hyperbatch totals of the last hyperbatch, for byte accounting.
+ * Waits like fetch. */
+typedef struct {
+  int32_t K;
+  int64_t frontier[AGNES_MAX_HOPS]; /* sum over minibatches of num_dst[h] */
+  int64_t edges[AGNES_MAX_HOPS];    /* sum over minibatches of num_edges[h] */
+  int64_t rows;                     /* sum over minibatches of num_nodes */
+  int64_t distinct_rows;            /* distinct node ids among all gathered rows */
+  int64_t row_bytes;
+} agnes_counters;
+agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
+
+/* Static facts about the loaded graph.  adj_blocks counts continuation
+ * blocks of split objects; tiles is the number of (topology block x
+ * feature block x 4096-id chunk) cells the buckets are kept in. */
+typedef struct {
+  int64_t num_nodes, num_edges;
+  int64_t adj_blocks, adj_block_starts, feat_blocks, feat_rows_per_block, tiles;
+  int64_t row_bytes;
+} agnes_graph_info;
+agnes_status agnes_get_graph_info(agnes_ctx* ctx, agnes_graph_info* out);
+
+/* Copies the object index table to host memory: for each of the first
+ * min(cap, adj_block_starts) block starts, the first node whose object
+ * starts there (start_node) and that block's index (start_block).
+ * Continuation blocks of a split object are implied by the gaps between
+ * consecutive start_block values. */
+agnes_status agnes_copy_adj_blocks(agnes_ctx* ctx, int32_t* start_node, int32_t* start_block,
+                                   int64_t cap);
+
+/* Optional per-phase timing of later prepares with CUDA events on the
+ * caller's stream (off by default).  agnes_phase_times writes up to n
+ * milliseconds of the last prepare, in order: [0] bucketing of the targets,
+ * then per hop h (3 each): [1+3h] count+scan, [2+3h] sampling,
+ * [3+3h] dedup+relabel, then [1+3K] gather; returns the count written via
+ * *n_out.  Waits like fetch. */
+agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable);
+agnes_status agnes_phase_times(agnes_ctx* ctx, float* ms, int32_t n, int32_t* n_out);
+
+/* Releases everything the ctx owns (after synchronising its streams). */
+agnes_status agnes_free(agnes_ctx* ctx);
+
+const char* agnes_status_string(agnes_status s);
+const char* agnes_last_error(agnes_ctx* ctx); /* "" when none; ctx may be NULL */
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,809 @@
+// api.cu -- the C ABI of libagnes.so (declared in include/agnes.h).
+//
+// Orchestrates one hyperbatch (Algorithm 1, Sec. 3.5) on the caller's stream:
+//   bucket the targets by (tile, minibatch)                   [sample.cu]
+//   for each hop: count min(deg, k) per frontier entry, scan to indptr,
+//                 sample in bucket order                      [sample.cu, scan.cu]
+//                 bucket the samples, dedup + relabel, carry the bucket
+//                                                             [dedup.cu]
+//   gather the final bucket's rows block by block             [gather.cu]
+//   count the blocks touched (the paper's block-wise I/Os)   [gather.cu]
+// Everything is sized for the worst case up front (per-minibatch capacities
+// cap_h = min(N, B * prod(1 + k))), so no kernel's launch waits on a count
+// from the device and the host synchronises only when a view is fetched.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <new>
+
+#include "../../include/agnes.h"
+#include "common.cuh"
+#include "internal.h"
+
+using namespace agnes;
+
+namespace {
+
+constexpr int kMaxPhases = 2 + 3 * AGNES_MAX_HOPS;
+
+struct Workspace {
+  int32_t H = 0, B = 0, K = 0;
+  int32_t fan[AGNES_MAX_HOPS] = {0};
+  int64_t cap[AGNES_MAX_HOPS + 1] = {0};
+  int64_t capK = 0, ecap_max = 0, cap_prev_max = 0;
+  bool valid = false;
+
+  int32_t* nodes = nullptr;
+  int32_t* fb_id[2] = {nullptr, nullptr};
+  int32_t* fb_pos[2] = {nullptr, nullptr};
+  int32_t* fcell_off[2] = {nullptr, nullptr};
+  int32_t* fcnt = nullptr;
+  int32_t* scnt = nullptr;
+  int32_t* soff = nullptr;
+  int32_t* nfcnt = nullptr;
+  int32_t* newcnt = nullptr;
+  int32_t* newbase = nullptr;
+  int32_t* newtot = nullptr;
+  int32_t* nsz = nullptr;   // (K+1) x H
+  int32_t* ecnt = nullptr;  // K x H
+  int64_t* indptr[AGNES_MAX_HOPS] = {nullptr};
+  int32_t* col[AGNES_MAX_HOPS] = {nullptr};
+  int32_t* nbr = nullptr;
+  int32_t* stile = nullptr;
+  int32_t* sb_u = nullptr;
+  int32_t* sb_e = nullptr;
+  int32_t* cnt = nullptr;
+  void* feats_out = nullptr;
+  uint8_t* adj_flags = nullptr;
+  uint8_t* feat_flags = nullptr;
+  int64_t* stats = nullptr;  // K+1
+  int64_t* scan_scratch = nullptr;
+  int32_t* status = nullptr;
+  unsigned long long* distinct = nullptr;
+
+  // pinned host readback: [status][nsz (K+1)H][ecnt KH] then int64 stats (K+1)
+  void* h_back = nullptr;
+  size_t h_back_bytes = 0;
+};
+
+}  // namespace
+
+struct agnes_ctx {
+  int device = 0;
+  int num_sms = 0;
+  cudaStream_t load_stream = nullptr;
+
+  int64_t N = 0, E = 0;
+  int offsets_bits = 64;
+  void* offsets = nullptr;
+  int32_t* indices = nullptr;
+  void* features = nullptr;
+  bool own_offsets = false, own_indices = false, own_features = false;
+  int32_t feat_dtype = 0;
+  int64_t feat_dim = 0, row_bytes = 0;
+  int32_t features_on_host = 0;
+  int64_t adj_block_bytes = 0, feat_block_bytes = 0;
+  BlockTables bt;
+
+  Workspace ws;
+  bool prepared = false;
+  bool synced = false;
+  int cur = 0;  // which frontier buffer holds the final bucket
+  cudaEvent_t done = nullptr;
+
+  bool profiling = false;
+  int n_phases = 0;
+  cudaEvent_t ev[kMaxPhases + 1] = {nullptr};
+  bool ev_created = false;
+
+  char err[512] = {0};
+};
+
+static thread_local char g_err[512];
+
+static void set_err(agnes_ctx* ctx, const char* fmt, ...) {
+  char* dst = ctx ? ctx->err : g_err;
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(dst, 512, fmt, ap);
+  va_end(ap);
+  if (ctx) snprintf(g_err, sizeof(g_err), "%s", ctx->err);
+}
+
+#define CK(ctx, call)                                                            \
+  do {                                                                           \
+    cudaError_t e_ = (call);                                                     \
+    if (e_ != cudaSuccess) {                                                     \
+      set_err(ctx, "%s failed: %s", #call, cudaGetErrorString(e_));              \
+      return e_ == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;       \
+    }                                                                            \
+  } while (0)
+
+static bool is_device_ptr(const void* p) {
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged;
+}
+
+static bool is_pinned_host_ptr(const void* p) {
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return attr.type == cudaMemoryTypeHost;
+}
+
+__global__ static void fill_i32_kernel(int32_t* p, int64_t n, int32_t v) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    p[i] = v;
+}
+
+static void free_workspace(Workspace* w) {
+  cudaFree(w->nodes);
+  for (int b = 0; b < 2; ++b) {
+    cudaFree(w->fb_id[b]);
+    cudaFree(w->fb_pos[b]);
+    cudaFree(w->fcell_off[b]);
+  }
+  cudaFree(w->fcnt);
+  cudaFree(w->scnt);
+  cudaFree(w->soff);
+  cudaFree(w->nfcnt);
+  cudaFree(w->newcnt);
+  cudaFree(w->newbase);
+  cudaFree(w->newtot);
+  cudaFree(w->nsz);
+  cudaFree(w->ecnt);
+  for (int h = 0; h < AGNES_MAX_HOPS; ++h) {
+    cudaFree(w->indptr[h]);
+    cudaFree(w->col[h]);
+  }
+  cudaFree(w->nbr);
+  cudaFree(w->stile);
+  cudaFree(w->sb_u);
+  cudaFree(w->sb_e);
+  cudaFree(w->cnt);
+  cudaFree(w->feats_out);
+  cudaFree(w->adj_flags);
+  cudaFree(w->feat_flags);
+  cudaFree(w->stats);
+  cudaFree(w->scan_scratch);
+  cudaFree(w->status);
+  cudaFree(w->distinct);
+  if (w->h_back) cudaFreeHost(w->h_back);
+  *w = Workspace();
+}
+
+template <typename T>
+static cudaError_t dalloc(T** p, int64_t n) {
+  return cudaMalloc((void**)p, sizeof(T) * (size_t)(n > 0 ? n : 1));
+}
+
+static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const int32_t* fan,
+                                     int32_t K, const int64_t* cap) {
+  Workspace& w = ctx->ws;
+  bool same = w.valid && w.H == H && w.B == B && w.K == K;
+  for (int h = 0; same && h < K; ++h) same = w.fan[h] == fan[h];
+  if (same) return AGNES_OK;
+  cudaDeviceSynchronize();
+  free_workspace(&w);
+  w.H = H;
+  w.B = B;
+  w.K = K;
+  for (int h = 0; h < K; ++h) w.fan[h] = fan[h];
+  for (int h = 0; h <= K; ++h) w.cap[h] = cap[h];
+  w.capK = cap[K];
+  w.ecap_max = 0;
+  w.cap_prev_max = 0;
+  for (int h = 0; h < K; ++h) {
+    const int64_t e = cap[h] * fan[h];
+    if (e > w.ecap_max) w.ecap_max = e;
+    if (cap[h] > w.cap_prev_max) w.cap_prev_max = cap[h];
+  }
+  const int64_t T = ctx->bt.T;
+  const int64_t cells = T * H;
+  const int64_t rows = (int64_t)H * w.capK;
+  const int64_t edges = (int64_t)H * w.ecap_max;
+  const int64_t nb = ctx->bt.n_blocks;
+  const int64_t nfb = ctx->bt.n_feat_blocks;
+  int64_t scratch = scan_scratch_elems(1, cells);
+  const int64_t s2 = scan_scratch_elems(1, ctx->N);
+  const int64_t s3 = scan_scratch_elems(H, w.cap_prev_max);
+  const int64_t s4 = scan_scratch_elems(H, T);
+  if (s2 > scratch) scratch = s2;
+  if (s3 > scratch) scratch = s3;
+  if (s4 > scratch) scratch = s4;
+
+#define WA(p, n)                                                                             \
+  do {                                                                                       \
+    if (dalloc(&(p), (n)) != cudaSuccess) {                                                  \
+      cudaGetLastError();                                                                    \
+      free_workspace(&w);                                                                    \
+      set_err(ctx, "out of device memory allocating %s (%lld elements)", #p, (long long)(n)); \
+      return AGNES_ENOMEM;                                                                   \
+    }                                                                                        \
+  } while (0)
+
+  WA(w.nodes, rows);
+  for (int b = 0; b < 2; ++b) {
+    WA(w.fb_id[b], rows);
+    WA(w.fb_pos[b], rows);
+    WA(w.fcell_off[b], cells + 1);
+  }
+  WA(w.fcnt, cells);
+  WA(w.scnt, cells);
+  WA(w.soff, cells + 1);
+  WA(w.nfcnt, cells);
+  WA(w.newcnt, cells);
+  WA(w.newbase, cells);
+  WA(w.newtot, H);
+  WA(w.nsz, (int64_t)(K + 1) * H);
+  WA(w.ecnt, (int64_t)K * H);
+  for (int h = 0; h < K; ++h) {
+    WA(w.indptr[h], (int64_t)H * (cap[h] + 1));
+    WA(w.col[h], (int64_t)H * cap[h] * fan[h]);
+  }
+  WA(w.nbr, edges);
+  WA(w.stile, edges);
+  WA(w.sb_u, edges > rows ? edges : rows);
+  WA(w.sb_e, edges > rows ? edges : rows);
+  WA(w.cnt, (int64_t)H * w.cap_prev_max);
+  {
+    uint8_t* f = nullptr;
+    WA(f, rows * ctx->row_bytes);
+    w.feats_out = f;
+  }
+  WA(w.adj_flags, (int64_t)K * nb);
+  WA(w.feat_flags, nfb);
+  WA(w.stats, K + 1);
+  WA(w.scan_scratch, scratch);
+  WA(w.status, 1);
+  WA(w.distinct, 1);
+#undef WA
+  w.h_back_bytes = sizeof(int32_t) * (1 + (size_t)(K + 1) * H + (size_t)K * H + 1) +
+                   sizeof(int64_t) * (K + 2);
+  if (cudaMallocHost(&w.h_back, w.h_back_bytes) != cudaSuccess) {
+    cudaGetLastError();
+    w.h_back = nullptr;
+    free_workspace(&w);
+    set_err(ctx, "out of pinned host memory");
+    return AGNES_ENOMEM;
+  }
+  if (cudaMemset(w.fcnt, 0, sizeof(int32_t) * cells) != cudaSuccess ||
+      cudaMemset(w.scnt, 0, sizeof(int32_t) * cells) != cudaSuccess) {
+    free_workspace(&w);
+    set_err(ctx, "cudaMemset failed");
+    return AGNES_ECUDA;
+  }
+  w.valid = true;
+  return AGNES_OK;
+}
+
+// Host view of the readback buffer.
+struct Back {
+  int32_t* status;
+  int32_t* nsz;
+  int32_t* ecnt;
+  int64_t* stats;
+};
+
+static Back back_of(Workspace& w) {
+  Back b;
+  int32_t* p = (int32_t*)w.h_back;
+  b.status = p;
+  b.nsz = p + 1;
+  b.ecnt = b.nsz + (size_t)(w.K + 1) * w.H;
+  size_t off32 = 1 + (size_t)(w.K + 1) * w.H + (size_t)w.K * w.H + 1;
+  b.stats = (int64_t*)((char*)w.h_back + ((off32 * sizeof(int32_t) + 7) & ~(size_t)7));
+  return b;
+}
+
+static agnes_status wait_prepared(agnes_ctx* ctx) {
+  if (!ctx) return AGNES_EINVAL;
+  if (!ctx->prepared) {
+    set_err(ctx, "no hyperbatch has been prepared");
+    return AGNES_ESTATE;
+  }
+  if (!ctx->synced) {
+    cudaSetDevice(ctx->device);
+    cudaError_t e = cudaEventSynchronize(ctx->done);
+    if (e != cudaSuccess) {
+      set_err(ctx, "waiting for the hyperbatch failed: %s", cudaGetErrorString(e));
+      return AGNES_ECUDA;
+    }
+    ctx->synced = true;
+  }
+  const Back b = back_of(ctx->ws);
+  const int32_t s = *b.status;
+  if (s != 0) {
+    if (s & kErrTargetRange) {
+      set_err(ctx, "a target id is outside [0, %lld)", (long long)ctx->N);
+      return AGNES_EINVAL;
+    }
+    if (s & kErrTargetDup) {
+      set_err(ctx, "a target id is repeated within a minibatch");
+      return AGNES_EINVAL;
+    }
+    set_err(ctx, "device status word 0x%x", s);
+    return AGNES_EKERNEL;
+  }
+  return AGNES_OK;
+}
+
+// ============================================================================
+// Public API
+// ============================================================================
+
+extern "C" {
+
+const char* agnes_status_string(agnes_status s) {
+  switch (s) {
+    case AGNES_OK: return "ok";
+    case AGNES_EINVAL: return "invalid argument";
+    case AGNES_ERANGE: return "size out of range";
+    case AGNES_ENOMEM: return "out of memory";
+    case AGNES_ECUDA: return "CUDA error";
+    case AGNES_ESTATE: return "call out of order";
+    case AGNES_ETIMEOUT: return "timed out";
+    case AGNES_EKERNEL: return "kernel reported an inconsistency";
+  }
+  return "unknown status";
+}
+
+const char* agnes_last_error(agnes_ctx* ctx) { return ctx ? ctx->err : g_err; }
+
+agnes_status agnes_free(agnes_ctx* ctx) {
+  if (!ctx) return AGNES_OK;
+  cudaSetDevice(ctx->device);
+  cudaDeviceSynchronize();
+  free_workspace(&ctx->ws);
+  free_block_tables(&ctx->bt);
+  if (ctx->own_offsets) cudaFree(ctx->offsets);
+  if (ctx->own_indices) cudaFree(ctx->indices);
+  if (ctx->own_features) cudaFree(ctx->features);
+  if (ctx->done) cudaEventDestroy(ctx->done);
+  if (ctx->ev_created)
+    for (int i = 0; i <= kMaxPhases; ++i) cudaEventDestroy(ctx->ev[i]);
+  delete ctx;
+  return AGNES_OK;
+}
+
+static agnes_status adopt_or_copy(agnes_ctx* ctx, const void* src, size_t bytes, void** dst,
+                                  bool* own, cudaStream_t st) {
+  if (is_device_ptr(src)) {
+    *dst = const_cast<void*>(src);
+    *own = false;
+    return AGNES_OK;
+  }
+  CK(ctx, cudaMalloc(dst, bytes ? bytes : 1));
+  *own = true;
+  CK(ctx, cudaMemcpyAsync(*dst, src, bytes, cudaMemcpyHostToDevice, st));
+  return AGNES_OK;
+}
+
+agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_stream,
+                              agnes_ctx** out) {
+  if (!out) {
+    set_err(nullptr, "out is NULL");
+    return AGNES_EINVAL;
+  }
+  *out = nullptr;
+  if (!d) {
+    set_err(nullptr, "desc is NULL");
+    return AGNES_EINVAL;
+  }
+  if (d->num_nodes < 1 || d->num_nodes >= ((int64_t)1 << 31)) {
+    set_err(nullptr, "num_nodes must be in [1, 2^31)");
+    return d->num_nodes < 1 ? AGNES_EINVAL : AGNES_ERANGE;
+  }
+  if (d->offsets_bits != 32 && d->offsets_bits != 64) {
+    set_err(nullptr, "offsets_bits must be 32 or 64");
+    return AGNES_EINVAL;
+  }
+  if (d->num_edges < 0 || (d->offsets_bits == 32 && d->num_edges >= ((int64_t)1 << 31))) {
+    set_err(nullptr, "num_edges out of range for the offsets type");
+    return AGNES_ERANGE;
+  }
+  if (!d->offsets || (d->num_edges > 0 && !d->indices) || !d->features) {
+    set_err(nullptr, "offsets, indices and features must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  if (d->feat_dtype != AGNES_F32 && d->feat_dtype != AGNES_F16) {
+    set_err(nullptr, "feat_dtype must be AGNES_F32 or AGNES_F16");
+    return AGNES_EINVAL;
+  }
+  const int64_t esize = d->feat_dtype == AGNES_F32 ? 4 : 2;
+  if (d->feat_dim < 1 || d->feat_dim > (1 << 20)) {
+    set_err(nullptr, "feat_dim must be in [1, 2^20]");
+    return AGNES_EINVAL;
+  }
+  const int64_t row_bytes = d->feat_dim * esize;
+  if (d->adj_block_bytes < 64 || d->adj_block_bytes > ((int64_t)1 << 34)) {
+    set_err(nullptr, "adj_block_bytes must be in [64, 2^34]");
+    return AGNES_EINVAL;
+  }
+  if (d->feat_block_bytes < row_bytes || d->feat_block_bytes > ((int64_t)1 << 34)) {
+    set_err(nullptr, "feat_block_bytes must hold at least one feature row");
+    return AGNES_EINVAL;
+  }
+  if (d->features_on_host && !is_pinned_host_ptr(d->features)) {
+    set_err(nullptr, "features_on_host requires pinned host memory");
+    return AGNES_EINVAL;
+  }
+  if (cudaSetDevice(device) != cudaSuccess) {
+    cudaGetLastError();
+    set_err(nullptr, "invalid device %d", device);
+    return AGNES_EINVAL;
+  }
+  agnes_ctx* ctx = new (std::nothrow) agnes_ctx();
+  if (!ctx) {
+    set_err(nullptr, "out of host memory");
+    return AGNES_ENOMEM;
+  }
+  ctx->device = device;
+  cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device);
+  if (ctx->num_sms < 1) ctx->num_sms = 1;
+  ctx->N = d->num_nodes;
+  ctx->E = d->num_edges;
+  ctx->offsets_bits = d->offsets_bits;
+  ctx->feat_dtype = d->feat_dtype;
+  ctx->feat_dim = d->feat_dim;
+  ctx->row_bytes = row_bytes;
+  ctx->features_on_host = d->features_on_host;
+  ctx->adj_block_bytes = d->adj_block_bytes;
+  ctx->feat_block_bytes = d->feat_block_bytes;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+
+  agnes_status rc;
+  const size_t off_bytes = (size_t)(d->num_nodes + 1) * (d->offsets_bits / 8);
+  rc = adopt_or_copy(ctx, d->offsets, off_bytes, &ctx->offsets, &ctx->own_offsets, st);
+  if (rc == AGNES_OK && d->num_edges > 0)
+    rc = adopt_or_copy(ctx, d->indices, (size_t)d->num_edges * 4, (void**)&ctx->indices,
+                       &ctx->own_indices, st);
+  if (rc == AGNES_OK) {
+    if (d->features_on_host) {
+      ctx->features = const_cast<void*>(d->features);
+      ctx->own_features = false;
+    } else {
+      rc = adopt_or_copy(ctx, d->features, (size_t)(d->num_nodes * row_bytes), &ctx->features,
+                         &ctx->own_features, st);
+    }
+  }
+  if (rc == AGNES_OK) {
+    int64_t ends[2] = {0, 0};
+    cudaError_t e;
+    if (d->offsets_bits == 32) {
+      int32_t v[2];
+      e = cudaMemcpyAsync(&v[0], ctx->offsets, 4, cudaMemcpyDeviceToHost, st);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&v[1], (int32_t*)ctx->offsets + d->num_nodes, 4,
+                            cudaMemcpyDeviceToHost, st);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+      ends[0] = v[0];
+      ends[1] = v[1];
+    } else {
+      e = cudaMemcpyAsync(&ends[0], ctx->offsets, 8, cudaMemcpyDeviceToHost, st);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&ends[1], (int64_t*)ctx->offsets + d->num_nodes, 8,
+                            cudaMemcpyDeviceToHost, st);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    }
+    if (e != cudaSuccess) {
+      set_err(ctx, "reading offsets failed: %s", cudaGetErrorString(e));
+      rc = AGNES_ECUDA;
+    } else if (ends[0] != 0 || ends[1] != d->num_edges) {
+      set_err(ctx, "offsets[0] must be 0 and offsets[N] must equal num_edges");
+      rc = AGNES_EINVAL;
+    }
+  }
+  if (rc == AGNES_OK) {
+    const int64_t rpb = d->feat_block_bytes / row_bytes;
+    cudaError_t e = build_block_tables(ctx->offsets, d->offsets_bits, d->num_nodes, d->num_edges,
+                                       d->adj_block_bytes, rpb, &ctx->bt, st, ctx->err,
+                                       sizeof(ctx->err));
+    if (e != cudaSuccess) rc = e == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;
+  }
+  if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
+    set_err(ctx, "cudaEventCreate failed");
+    rc = AGNES_ECUDA;
+  }
+  if (rc != AGNES_OK) {
+    snprintf(g_err, sizeof(g_err), "%s", ctx->err);
+    agnes_free(ctx);
+    return rc;
+  }
+  *out = ctx;
+  return AGNES_OK;
+}
+
+agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, int32_t H,
+                                      int32_t B, const int32_t* fanouts, int32_t K,
+                                      uint64_t seed, uint64_t first_minibatch_id,
+                                      void* cuda_stream) {
+  if (!ctx) {
+    set_err(nullptr, "ctx is NULL");
+    return AGNES_EINVAL;
+  }
+  if (!targets || !fanouts) {
+    set_err(ctx, "targets and fanouts must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  if (H < 1 || H > 65535 || B < 1 || K < 1 || K > AGNES_MAX_HOPS) {
+    set_err(ctx, "need 1 <= H <= 65535, B >= 1, 1 <= K <= %d", AGNES_MAX_HOPS);
+    return AGNES_EINVAL;
+  }
+  if (B > ctx->N) {
+    set_err(ctx, "B = %d distinct targets exceed N = %lld", B, (long long)ctx->N);
+    return AGNES_EINVAL;
+  }
+  int64_t cap[AGNES_MAX_HOPS + 1];
+  cap[0] = B;
+  for (int h = 0; h < K; ++h) {
+    if (fanouts[h] < 1 || fanouts[h] > AGNES_MAX_FANOUT) {
+      set_err(ctx, "fanouts[%d] = %d outside [1, %d]", h, fanouts[h], AGNES_MAX_FANOUT);
+      return AGNES_EINVAL;
+    }
+    const int64_t grown = cap[h] * (1 + (int64_t)fanouts[h]);
+    cap[h + 1] = grown < ctx->N ? grown : ctx->N;
+  }
+  const int64_t lim = ((int64_t)1 << 31) - 1;
+  for (int h = 0; h < K; ++h) {
+    if ((int64_t)H * cap[h] * fanouts[h] > lim) {
+      set_err(ctx, "H x edge capacity of hop %d exceeds 2^31", h + 1);
+      return AGNES_ERANGE;
+    }
+  }
+  if ((int64_t)H * cap[K] > lim) {
+    set_err(ctx, "H x node capacity (%lld) exceeds 2^31", (long long)(H * cap[K]));
+    return AGNES_ERANGE;
+  }
+  if (ctx->features_on_host) {
+    set_err(ctx, "streaming of host-resident features is not available in this build");
+    return AGNES_EINVAL;
+  }
+  if (cudaSetDevice(ctx->device) != cudaSuccess) {
+    cudaGetLastError();
+    set_err(ctx, "cudaSetDevice failed");
+    return AGNES_ECUDA;
+  }
+  agnes_status rc = ensure_workspace(ctx, H, B, fanouts, K, cap);
+  if (rc != AGNES_OK) return rc;
+
+  Workspace& w = ctx->ws;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const int32_t T = (int32_t)ctx->bt.T;
+  const int64_t cells = (int64_t)T * H;
+  const int nsm = ctx->num_sms;
+  ctx->prepared = false;
+  ctx->synced = false;
+
+  if (ctx->profiling && !ctx->ev_created) {
+    for (int i = 0; i <= kMaxPhases; ++i) CK(ctx, cudaEventCreate(&ctx->ev[i]));
+    ctx->ev_created = true;
+  }
+  int ph = 0;
+  auto mark = [&]() {
+    if (ctx->profiling) cudaEventRecord(ctx->ev[ph++], st);
+  };
+
+  mark();
+  CK(ctx, cudaMemsetAsync(w.status, 0, sizeof(int32_t), st));
+  CK(ctx, cudaMemsetAsync(w.fcnt, 0, sizeof(int32_t) * cells, st));
+  CK(ctx, cudaMemsetAsync(w.scnt, 0, sizeof(int32_t) * cells, st));
+  CK(ctx, cudaMemsetAsync(w.adj_flags, 0, (size_t)K * ctx->bt.n_blocks, st));
+  CK(ctx, cudaMemsetAsync(w.feat_flags, 0, (size_t)ctx->bt.n_feat_blocks, st));
+  CK(ctx, cudaMemsetAsync(w.stats, 0, sizeof(int64_t) * (K + 1), st));
+  CK(ctx, cudaMemcpy2DAsync(w.nodes, sizeof(int32_t) * w.capK, targets, sizeof(int32_t) * B,
+                            sizeof(int32_t) * B, H, cudaMemcpyDefault, st));
+  fill_i32_kernel<<<(H + 255) / 256, 256, 0, st>>>(w.nsz, H, B);
+  CK(ctx, cudaGetLastError());
+  CK(ctx, launch_bucket_targets(w.nodes, w.capK, H, B, (int32_t)ctx->N, ctx->bt.tile_first,
+                                ctx->bt.chunk_tile, T, w.fcnt, w.fcell_off[0], w.sb_u, w.sb_e,
+                                w.fb_id[0], w.fb_pos[0], w.scan_scratch, w.status, nsm, st));
+  int cur = 0;
+  for (int h = 0; h < K; ++h) {
+    mark();
+    HopArgs a;
+    a.offsets = ctx->offsets;
+    a.offsets_bits = ctx->offsets_bits;
+    a.indices = ctx->indices;
+    a.N = (int32_t)ctx->N;
+    a.tile_first = ctx->bt.tile_first;
+    a.chunk_tile = ctx->bt.chunk_tile;
+    a.T = T;
+    a.H = H;
+    a.capK = w.capK;
+    a.cap_prev = cap[h];
+    a.ecap = cap[h] * fanouts[h];
+    a.k = fanouts[h];
+    a.hop = h + 1;
+    a.seed = seed;
+    a.first_gid = first_minibatch_id;
+    a.status = w.status;
+    int32_t* nsz_prev = w.nsz + (int64_t)h * H;
+    int32_t* ecnt = w.ecnt + (int64_t)h * H;
+    CK(ctx, launch_sample_count(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.cnt, nsm, st));
+    CK(ctx, (seg_scan<int32_t, int64_t>(w.cnt, cap[h], w.indptr[h], cap[h] + 1, nsz_prev, 0, H,
+                                         cap[h], true, ecnt, w.scan_scratch, w.status, st)));
+    mark();
+    CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h],
+                               w.nbr, nsm, st));
+    mark();
+    DedupBufs d;
+    d.nbr = w.nbr;
+    d.ecnt = ecnt;
+    d.stile = w.stile;
+    d.scnt = w.scnt;
+    d.soff = w.soff;
+    d.sb_u = w.sb_u;
+    d.sb_e = w.sb_e;
+    d.fb_id = w.fb_id[cur];
+    d.fb_pos = w.fb_pos[cur];
+    d.fcell_off = w.fcell_off[cur];
+    d.newcnt = w.newcnt;
+    d.newbase = w.newbase;
+    d.newtot = w.newtot;
+    d.nfcnt = w.nfcnt;
+    d.nfcell_off = w.fcell_off[1 - cur];
+    d.nfb_id = w.fb_id[1 - cur];
+    d.nfb_pos = w.fb_pos[1 - cur];
+    d.nsz_prev = nsz_prev;
+    d.nsz_next = w.nsz + (int64_t)(h + 1) * H;
+    d.nodes = w.nodes;
+    d.col = w.col[h];
+    d.tile_adj_block = ctx->bt.tile_adj_block;
+    d.adj_flags = w.adj_flags + (int64_t)h * ctx->bt.n_blocks;
+    d.scan_scratch = w.scan_scratch;
+    CK(ctx, launch_dedup(a, d, nsm, st));
+    cur = 1 - cur;
+  }
+  mark();
+  CK(ctx, launch_gather(ctx->features, ctx->row_bytes, w.fb_id[cur], w.fb_pos[cur],
+                        w.fcell_off[cur] + cells, w.feats_out, w.status, nsm, st));
+  mark();
+  for (int h = 0; h < K; ++h)
+    CK(ctx, launch_mark_count(nullptr, T, H, nullptr, w.adj_flags + (int64_t)h * ctx->bt.n_blocks,
+                              ctx->bt.n_blocks, w.stats + h, w.status, st));
+  CK(ctx, launch_mark_count(w.fcell_off[cur], T, H, ctx->bt.tile_feat_block, w.feat_flags,
+                            ctx->bt.n_feat_blocks, w.stats + K, w.status, st));
+  const Back b = back_of(w);
+  CK(ctx, cudaMemcpyAsync(b.status, w.status, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(b.nsz, w.nsz, sizeof(int32_t) * (K + 1) * H, cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(b.ecnt, w.ecnt, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(b.stats, w.stats, sizeof(int64_t) * (K + 1), cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaEventRecord(ctx->done, st));
+  ctx->n_phases = ctx->profiling ? ph - 1 : 0;
+  ctx->cur = cur;
+  ctx->prepared = true;
+  return AGNES_OK;
+}
+
+agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_view* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  agnes_status rc = wait_prepared(ctx);
+  if (rc != AGNES_OK) return rc;
+  Workspace& w = ctx->ws;
+  if (j < 0 || j >= w.H) {
+    set_err(ctx, "minibatch %d outside [0, %d)", j, w.H);
+    return AGNES_EINVAL;
+  }
+  const Back b = back_of(w);
+  memset(out, 0, sizeof(*out));
+  out->K = w.K;
+  for (int h = 0; h < w.K; ++h) {
+    out->num_dst[h] = b.nsz[(size_t)h * w.H + j];
+    out->num_src[h] = b.nsz[(size_t)(h + 1) * w.H + j];
+    out->num_edges[h] = b.ecnt[(size_t)h * w.H + j];
+    out->indptr[h] = w.indptr[h] + (int64_t)j * (w.cap[h] + 1);
+    out->col[h] = w.col[h] + (int64_t)j * w.cap[h] * w.fan[h];
+  }
+  out->nodes = w.nodes + (int64_t)j * w.capK;
+  out->num_nodes = b.nsz[(size_t)w.K * w.H + j];
+  out->feats = (const char*)w.feats_out + (int64_t)j * w.capK * ctx->row_bytes;
+  out->feat_dtype = ctx->feat_dtype;
+  out->feat_dim = ctx->feat_dim;
+  return AGNES_OK;
+}
+
+agnes_status agnes_hyperbatch_stats(agnes_ctx* ctx, int64_t* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  agnes_status rc = wait_prepared(ctx);
+  if (rc != AGNES_OK) return rc;
+  const Back b = back_of(ctx->ws);
+  for (int h = 0; h <= ctx->ws.K; ++h) out[h] = b.stats[h];
+  return AGNES_OK;
+}
+
+agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  agnes_status rc = wait_prepared(ctx);
+  if (rc != AGNES_OK) return rc;
+  Workspace& w = ctx->ws;
+  const Back b = back_of(w);
+  memset(out, 0, sizeof(*out));
+  out->K = w.K;
+  for (int h = 0; h < w.K; ++h)
+    for (int j = 0; j < w.H; ++j) {
+      out->frontier[h] += b.nsz[(size_t)h * w.H + j];
+      out->edges[h] += b.ecnt[(size_t)h * w.H + j];
+    }
+  for (int j = 0; j < w.H; ++j) out->rows += b.nsz[(size_t)w.K * w.H + j];
+  out->row_bytes = ctx->row_bytes;
+  cudaSetDevice(ctx->device);
+  unsigned long long distinct = 0;
+  CK(ctx, cudaMemset(w.distinct, 0, sizeof(unsigned long long)));
+  CK(ctx, launch_distinct_rows(w.fb_id[ctx->cur], w.fcell_off[ctx->cur], ctx->bt.tile_first,
+                               (int32_t)ctx->bt.T, w.H, w.distinct, nullptr));
+  CK(ctx, cudaMemcpy(&distinct, w.distinct, sizeof(distinct), cudaMemcpyDeviceToHost));
+  out->distinct_rows = (int64_t)distinct;
+  return AGNES_OK;
+}
+
+agnes_status agnes_get_graph_info(agnes_ctx* ctx, agnes_graph_info* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  out->num_nodes = ctx->N;
+  out->num_edges = ctx->E;
+  out->adj_blocks = ctx->bt.n_blocks;
+  out->adj_block_starts = ctx->bt.n_starts;
+  out->feat_blocks = ctx->bt.n_feat_blocks;
+  out->feat_rows_per_block = ctx->bt.rows_per_feat_block;
+  out->tiles = ctx->bt.T;
+  out->row_bytes = ctx->row_bytes;
+  return AGNES_OK;
+}
+
+agnes_status agnes_copy_adj_blocks(agnes_ctx* ctx, int32_t* start_node, int32_t* start_block,
+                                   int64_t cap) {
+  if (!ctx || !start_node || !start_block || cap < 0) {
+    set_err(ctx, "invalid arguments");
+    return AGNES_EINVAL;
+  }
+  const int64_t n = cap < ctx->bt.n_starts ? cap : ctx->bt.n_starts;
+  cudaSetDevice(ctx->device);
+  CK(ctx, cudaMemcpy(start_node, ctx->bt.start_node, sizeof(int32_t) * n, cudaMemcpyDeviceToHost));
+  CK(ctx, cudaMemcpy(start_block, ctx->bt.start_block, sizeof(int32_t) * n,
+                     cudaMemcpyDeviceToHost));
+  return AGNES_OK;
+}
+
+agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable) {
+  if (!ctx) return AGNES_EINVAL;
+  ctx->profiling = enable != 0;
+  return AGNES_OK;
+}
+
+agnes_status agnes_phase_times(agnes_ctx* ctx, float* ms, int32_t n, int32_t* n_out) {
+  if (!ctx || (!ms && n > 0) || !n_out) {
+    set_err(ctx, "invalid arguments");
+    return AGNES_EINVAL;
+  }
+  *n_out = 0;
+  agnes_status rc = wait_prepared(ctx);
+  if (rc != AGNES_OK) return rc;
+  int cnt = ctx->n_phases < n ? ctx->n_phases : n;
+  for (int i = 0; i < cnt; ++i) {
+    CK(ctx, cudaEventElapsedTime(&ms[i], ctx->ev[i], ctx->ev[i + 1]));
+  }
+  *n_out = cnt;
+  return AGNES_OK;
+}
+
+}  // extern "C"

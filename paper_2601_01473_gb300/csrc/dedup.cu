@@ -1,0 +1,309 @@
+// dedup.cu -- per-minibatch union / dedup and relabelling of a hop's samples
+// (Algorithm 1: N^j_out <- N^j_out u Sample(j, ...), N_in <- N_out).
+//
+// The sampled ids of every minibatch are bucketed by (tile, minibatch) cell
+// (histogram -> scan -> scatter, the bucket matrix of Sec. 3.4 (3)).  A cell
+// covers at most 4096 consecutive ids, so one warp resolves it with two
+// shared-memory bitmaps over the tile: D = the cell's frontier (dst_h) ids and
+// S = its sampled ids.  new = S & ~D in ascending id order is the cell's part
+// of new_h (tiles ascend in id, so a per-minibatch scan of the cells' new
+// counts over tiles gives each new node its index in src_h = dst_h ++ new_h);
+// popcount ranks in D and new give every sampled edge its col; and D | new in
+// ascending order, with each node's output row, is the cell of the next hop's
+// frontier bucket -- the bucket is carried from hop to hop and never rebuilt.
+#include "common.cuh"
+#include "internal.h"
+
+namespace agnes {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+
+__global__ void __launch_bounds__(kThreads)
+dedup_hist_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict__ ecnt, int64_t ecap,
+                  int32_t H, TileMap tm, int32_t* __restrict__ stile, int32_t* __restrict__ scnt,
+                  const int32_t* status) {
+  if (failed(status)) return;
+  const int32_t j = blockIdx.y;
+  const int64_t E = ecnt[j];
+  const int32_t* src = nbr + j * ecap;
+  int32_t* til = stile + j * ecap;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; e0 < E;
+       e0 += stride) {
+    const int64_t e = e0 + lane_id();
+    const bool active = e < E;
+    int64_t cell = 0;
+    if (active) {
+      const int32_t t = tile_of(tm, src[e]);
+      til[e] = t;
+      cell = (int64_t)t * H + j;
+    }
+    warp_agg_inc(scnt, cell, active);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict__ ecnt,
+                     int64_t ecap, int32_t H, const int32_t* __restrict__ stile,
+                     int32_t* __restrict__ scnt, const int32_t* __restrict__ soff,
+                     int32_t* __restrict__ sb_u, int32_t* __restrict__ sb_e,
+                     const int32_t* status) {
+  if (failed(status)) return;
+  const int32_t j = blockIdx.y;
+  const int64_t E = ecnt[j];
+  const int32_t* src = nbr + j * ecap;
+  const int32_t* til = stile + j * ecap;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; e0 < E;
+       e0 += stride) {
+    const int64_t e = e0 + lane_id();
+    const bool active = e < E;
+    const unsigned mask = __ballot_sync(0xffffffffu, active);
+    if (active) {
+      const int64_t cell = (int64_t)til[e] * H + j;
+      const int32_t slot = soff[cell] + warp_agg_take(scnt, cell, mask);
+      sb_u[slot] = src[e];
+      sb_e[slot] = (int32_t)e;
+    }
+  }
+}
+
+struct CellArgs {
+  TileMap tm;
+  int32_t H;
+  int64_t ncells;
+  int64_t capK, ecap;
+  const int32_t* fb_id;
+  const int32_t* fb_pos;
+  const int32_t* fcell_off;
+  const int32_t* sb_u;
+  const int32_t* sb_e;
+  const int32_t* soff;
+  const int32_t* tile_adj_block;
+  uint8_t* adj_flags;
+  int32_t* newcnt;
+  const int32_t* newbase;
+  int32_t* nfcnt;
+  const int32_t* nfcell_off;
+  int32_t* nfb_id;
+  int32_t* nfb_pos;
+  const int32_t* nsz_prev;
+  int32_t* nodes;
+  int32_t* col;
+  const int32_t* status;
+};
+
+// Marks the cell's frontier ids in D and sampled ids in S (tile-local bits).
+__device__ __forceinline__ void mark_cell(const CellArgs& a, uint32_t* D, uint32_t* S, int32_t base,
+                                          int32_t words, int32_t fo, int32_t fn, int32_t so,
+                                          int32_t sn) {
+  const int lane = lane_id();
+  for (int w = lane; w < words; w += 32) {
+    D[w] = 0;
+    S[w] = 0;
+  }
+  __syncwarp();
+  for (int32_t i = lane; i < fn; i += 32) {
+    const int32_t lu = a.fb_id[fo + i] - base;
+    atomicOr(&D[lu >> 5], 1u << (lu & 31));
+  }
+  for (int32_t i = lane; i < sn; i += 32) {
+    const int32_t lu = a.sb_u[so + i] - base;
+    atomicOr(&S[lu >> 5], 1u << (lu & 31));
+  }
+  __syncwarp();
+}
+
+__global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
+  if (failed(a.status)) return;
+  __shared__ uint32_t D_s[kWarps][kTileWords];
+  __shared__ uint32_t S_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  uint32_t* D = D_s[warp];
+  uint32_t* S = S_s[warp];
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t cell = blockIdx.x * (int64_t)kWarps + warp; cell < a.ncells; cell += nwarps) {
+    const int32_t t = (int32_t)(cell / a.H);
+    const int32_t j = (int32_t)(cell - (int64_t)t * a.H);
+    const int32_t fo = a.fcell_off[cell], fn = a.fcell_off[cell + 1] - fo;
+    const int32_t so = a.soff[cell], sn = a.soff[cell + 1] - so;
+    int32_t cnt = 0;
+    if (sn > 0) {
+      const int32_t base = a.tm.tile_first[t];
+      const int32_t words = (a.tm.tile_first[t + 1] - base + 31) >> 5;
+      mark_cell(a, D, S, base, words, fo, fn, so, sn);
+      for (int w = lane; w < words; w += 32) cnt += __popc(S[w] & ~D[w]);
+      cnt = warp_sum(cnt);
+      __syncwarp();
+    }
+    if (lane == 0) {
+      a.newcnt[(int64_t)j * a.tm.T + t] = cnt;
+      a.nfcnt[cell] = fn + cnt;
+      if (fn > 0) a.adj_flags[a.tile_adj_block[t]] = 1;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
+  if (failed(a.status)) return;
+  __shared__ uint32_t D_s[kWarps][kTileWords];
+  __shared__ uint32_t N_s[kWarps][kTileWords];
+  __shared__ int32_t pD_s[kWarps][kTileWords];
+  __shared__ int32_t pN_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  uint32_t* D = D_s[warp];
+  uint32_t* Nw = N_s[warp];
+  int32_t* pD = pD_s[warp];
+  int32_t* pN = pN_s[warp];
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t cell = blockIdx.x * (int64_t)kWarps + warp; cell < a.ncells; cell += nwarps) {
+    const int32_t fo = a.fcell_off[cell], fn = a.fcell_off[cell + 1] - fo;
+    const int32_t so = a.soff[cell], sn = a.soff[cell + 1] - so;
+    if (fn + sn == 0) continue;
+    const int32_t nfo = a.nfcell_off[cell];
+    if (sn == 0) {  // nothing sampled here: the frontier cell carries over unchanged
+      for (int32_t i = lane; i < fn; i += 32) {
+        a.nfb_id[nfo + i] = a.fb_id[fo + i];
+        a.nfb_pos[nfo + i] = a.fb_pos[fo + i];
+      }
+      continue;
+    }
+    const int32_t t = (int32_t)(cell / a.H);
+    const int32_t j = (int32_t)(cell - (int64_t)t * a.H);
+    const int32_t base = a.tm.tile_first[t];
+    const int32_t words = (a.tm.tile_first[t + 1] - base + 31) >> 5;
+    mark_cell(a, D, Nw, base, words, fo, fn, so, sn);
+
+    // new = S & ~D; per-word exclusive ranks of D and new
+    uint32_t dw[4], nw[4];
+    int32_t sd = 0, sn_ = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      dw[q] = w < words ? D[w] : 0u;
+      nw[q] = w < words ? (Nw[w] & ~dw[q]) : 0u;
+      sd += __popc(dw[q]);
+      sn_ += __popc(nw[q]);
+    }
+    int32_t rd = warp_incl_scan(sd) - sd;
+    int32_t rn = warp_incl_scan(sn_) - sn_;
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      Nw[w] = nw[q];
+      pD[w] = rd;
+      pN[w] = rn;
+      rd += __popc(dw[q]);
+      rn += __popc(nw[q]);
+    }
+    __syncwarp();
+
+    const int64_t jcap = (int64_t)j * a.capK;
+    const int32_t nb = a.nsz_prev[j] + a.newbase[(int64_t)j * a.tm.T + t];
+    int32_t* col = a.col + (int64_t)j * a.ecap;
+    for (int32_t i = lane; i < sn; i += 32) {
+      const int32_t lu = a.sb_u[so + i] - base;
+      const int32_t w = lu >> 5;
+      const uint32_t bit = 1u << (lu & 31), below = bit - 1u;
+      int32_t c;
+      if (D[w] & bit)
+        c = (int32_t)(a.fb_pos[fo + pD[w] + __popc(D[w] & below)] - jcap);
+      else
+        c = nb + pN[w] + __popc(Nw[w] & below);
+      col[a.sb_e[so + i]] = c;
+    }
+
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      if (w >= words) break;
+      const uint32_t d = dw[q], n = nw[q];
+      uint32_t rest = d | n;
+      const int32_t r0 = pD[w] + pN[w];
+      while (rest) {
+        const int b = __ffs(rest) - 1;
+        rest &= rest - 1u;
+        const uint32_t below = (1u << b) - 1u;
+        const int32_t id = base + w * 32 + b;
+        const int32_t r = r0 + __popc((d | n) & below);
+        int32_t g;
+        if ((d >> b) & 1u) {
+          g = a.fb_pos[fo + pD[w] + __popc(d & below)];
+        } else {
+          g = (int32_t)(jcap + nb + pN[w] + __popc(n & below));
+          a.nodes[g] = id;
+        }
+        a.nfb_id[nfo + r] = id;
+        a.nfb_pos[nfo + r] = g;
+      }
+    }
+    __syncwarp();
+  }
+}
+
+__global__ void add_sizes_kernel(const int32_t* __restrict__ prev, const int32_t* __restrict__ add,
+                                 int32_t* __restrict__ next, int32_t H, const int32_t* status) {
+  if (failed(status)) return;
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < H; j += gridDim.x * blockDim.x)
+    next[j] = prev[j] + add[j];
+}
+
+}  // namespace
+
+cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cudaStream_t st) {
+  const TileMap tm{a.tile_first, a.chunk_tile, a.T};
+  const int64_t ncells = (int64_t)a.T * a.H;
+  int gx = (num_sms * 8 + a.H - 1) / a.H;
+  if (gx < 1) gx = 1;
+  const dim3 egrid(gx, a.H);
+  dedup_hist_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, a.H, tm, d.stile, d.scnt,
+                                                a.status);
+  cudaError_t e = seg_scan<int32_t, int32_t>(d.scnt, 0, d.soff, 0, nullptr, ncells, 1, ncells,
+                                             true, nullptr, d.scan_scratch, a.status, st);
+  if (e != cudaSuccess) return e;
+  dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, a.H, d.stile, d.scnt,
+                                                   d.soff, d.sb_u, d.sb_e, a.status);
+
+  CellArgs c;
+  c.tm = tm;
+  c.H = a.H;
+  c.ncells = ncells;
+  c.capK = a.capK;
+  c.ecap = a.ecap;
+  c.fb_id = d.fb_id;
+  c.fb_pos = d.fb_pos;
+  c.fcell_off = d.fcell_off;
+  c.sb_u = d.sb_u;
+  c.sb_e = d.sb_e;
+  c.soff = d.soff;
+  c.tile_adj_block = d.tile_adj_block;
+  c.adj_flags = d.adj_flags;
+  c.newcnt = d.newcnt;
+  c.newbase = d.newbase;
+  c.nfcnt = d.nfcnt;
+  c.nfcell_off = d.nfcell_off;
+  c.nfb_id = d.nfb_id;
+  c.nfb_pos = d.nfb_pos;
+  c.nsz_prev = d.nsz_prev;
+  c.nodes = d.nodes;
+  c.col = d.col;
+  c.status = a.status;
+  const int cgrid = num_sms * 8;
+  dedup_count_kernel<<<cgrid, kThreads, 0, st>>>(c);
+  e = seg_scan<int32_t, int32_t>(d.newcnt, a.T, d.newbase, a.T, nullptr, a.T, a.H, a.T, false,
+                                 d.newtot, d.scan_scratch, a.status, st);
+  if (e != cudaSuccess) return e;
+  add_sizes_kernel<<<(a.H + 255) / 256, 256, 0, st>>>(d.nsz_prev, d.newtot, d.nsz_next, a.H,
+                                                      a.status);
+  e = seg_scan<int32_t, int32_t>(d.nfcnt, 0, d.nfcell_off, 0, nullptr, ncells, 1, ncells, true,
+                                 nullptr, d.scan_scratch, a.status, st);
+  if (e != cudaSuccess) return e;
+  dedup_emit_kernel<<<cgrid, kThreads, 0, st>>>(c);
+  return cudaGetLastError();
+}
+
+}  // namespace agnes

@@ -1,0 +1,178 @@
+// gather.cu -- block-wise feature gathering (Algorithm 1's gathering loop,
+// Sec. 3.4 (2)) and the bookkeeping kernels for blocks-touched statistics.
+//
+// The final frontier bucket lists every gathered node once per minibatch, in
+// (tile, minibatch, id) order, with its output row.  Tiles never straddle a
+// feature block, so walking the bucket in order visits each feature block
+// once for all minibatches: a row requested by several minibatches is read
+// from HBM once and served from L2 afterwards.  Rows are copied as 16-byte
+// vectors (bit-exact, no float conversion); a group of row_bytes/16 lanes
+// moves one row, each lane keeping U rows in flight; output stores are
+// streaming (evict-first) so they do not push the feature rows out of L2.
+#include "common.cuh"
+#include "internal.h"
+
+namespace agnes {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+
+// LPR lanes per row, row = LPR 16-byte vectors, U rows in flight per lane.
+template <int LPR, int U>
+__global__ void __launch_bounds__(kThreads)
+gather_vec_kernel(const uint4* __restrict__ feats, const int32_t* __restrict__ fb_id,
+                  const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
+                  uint4* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  constexpr int kRowsPerWarp = 32 / LPR;
+  constexpr int kStep = kRowsPerWarp * U;
+  const int64_t total = *total_ptr;
+  const int lane = lane_id();
+  const int sub = lane / LPR, l = lane % LPR;
+  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t r0 = warp0 * kStep; r0 < total; r0 += nwarps * kStep) {
+    uint4 v[U];
+    int32_t g[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t i = r0 + u * kRowsPerWarp + sub;
+      g[u] = -1;
+      if (i < total) {
+        const int32_t id = __ldg(fb_id + i);
+        g[u] = __ldg(fb_pos + i);
+        v[u] = __ldg(feats + (int64_t)id * LPR + l);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (g[u] >= 0) __stcs(out + (int64_t)g[u] * LPR + l, v[u]);
+  }
+}
+
+// Any row size that is a multiple of 16 bytes: one warp per row.
+__global__ void __launch_bounds__(kThreads)
+gather_rows_kernel(const uint4* __restrict__ feats, int64_t vecs, const int32_t* __restrict__ fb_id,
+                   const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
+                   uint4* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  const int64_t total = *total_ptr;
+  const int lane = lane_id();
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
+    const int64_t src = (int64_t)__ldg(fb_id + i) * vecs;
+    const int64_t dst = (int64_t)__ldg(fb_pos + i) * vecs;
+    for (int64_t c = lane; c < vecs; c += 32) __stcs(out + dst + c, __ldg(feats + src + c));
+  }
+}
+
+// Rows whose size is not a multiple of 16 bytes: byte copy, one warp per row.
+__global__ void __launch_bounds__(kThreads)
+gather_bytes_kernel(const uint8_t* __restrict__ feats, int64_t row_bytes,
+                    const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
+                    const int32_t* total_ptr, uint8_t* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  const int64_t total = *total_ptr;
+  const int lane = lane_id();
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
+    const int64_t src = (int64_t)__ldg(fb_id + i) * row_bytes;
+    const int64_t dst = (int64_t)__ldg(fb_pos + i) * row_bytes;
+    for (int64_t c = lane; c < row_bytes; c += 32) out[dst + c] = __ldg(feats + src + c);
+  }
+}
+
+__global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
+                            const int32_t* __restrict__ map, uint8_t* __restrict__ flags,
+                            const int32_t* status) {
+  if (failed(status)) return;
+  const int64_t ncells = (int64_t)T * H;
+  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < ncells;
+       c += (int64_t)gridDim.x * blockDim.x)
+    if (cell_off[c + 1] > cell_off[c]) flags[map[c / H]] = 1;
+}
+
+__global__ void count_flags_kernel(const uint8_t* __restrict__ flags, int64_t n,
+                                   int64_t* __restrict__ count) {
+  int64_t local = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    local += flags[i] != 0;
+  local = warp_sum(local);
+  if (lane_id() == 0 && local) atomicAdd((unsigned long long*)count, (unsigned long long)local);
+}
+
+// One warp per tile: union of the tile's cells over all minibatches.
+__global__ void __launch_bounds__(kThreads)
+distinct_rows_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict__ cell_off,
+                     const int32_t* __restrict__ tile_first, int32_t T, int32_t H,
+                     unsigned long long* count) {
+  __shared__ uint32_t bits_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  uint32_t* bits = bits_s[warp];
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t t = blockIdx.x * (int64_t)kWarps + warp; t < T; t += nwarps) {
+    const int32_t base = tile_first[t];
+    const int32_t words = (tile_first[t + 1] - base + 31) >> 5;
+    for (int w = lane; w < words; w += 32) bits[w] = 0;
+    __syncwarp();
+    const int32_t o = cell_off[t * H], e = cell_off[(t + 1) * H];
+    for (int32_t i = o + lane; i < e; i += 32) {
+      const int32_t lu = fb_id[i] - base;
+      atomicOr(&bits[lu >> 5], 1u << (lu & 31));
+    }
+    __syncwarp();
+    uint32_t c = 0;
+    for (int w = lane; w < words; w += 32) c += __popc(bits[w]);
+    c = warp_sum(c);
+    if (lane == 0 && c) atomicAdd(count, (unsigned long long)c);
+    __syncwarp();
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
+                          const int32_t* fb_pos, const int32_t* total, void* out,
+                          const int32_t* status, int num_sms, cudaStream_t st) {
+  const int grid = num_sms * 8;
+  const bool aligned = (row_bytes % 16 == 0) && ((uintptr_t)feats % 16 == 0) &&
+                       ((uintptr_t)out % 16 == 0);
+  if (aligned) {
+    const int64_t vecs = row_bytes / 16;
+    const uint4* f = (const uint4*)feats;
+    uint4* o = (uint4*)out;
+    if (vecs == 8)
+      gather_vec_kernel<8, 4><<<grid, kThreads, 0, st>>>(f, fb_id, fb_pos, total, o, status);
+    else if (vecs == 16)
+      gather_vec_kernel<16, 4><<<grid, kThreads, 0, st>>>(f, fb_id, fb_pos, total, o, status);
+    else if (vecs == 32)
+      gather_vec_kernel<32, 4><<<grid, kThreads, 0, st>>>(f, fb_id, fb_pos, total, o, status);
+    else
+      gather_rows_kernel<<<grid, kThreads, 0, st>>>(f, vecs, fb_id, fb_pos, total, o, status);
+  } else {
+    gather_bytes_kernel<<<grid, kThreads, 0, st>>>((const uint8_t*)feats, row_bytes, fb_id,
+                                                   fb_pos, total, (uint8_t*)out, status);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, const int32_t* map,
+                              uint8_t* flags, int64_t n_flags, int64_t* count,
+                              const int32_t* status, cudaStream_t st) {
+  if (cell_off && map)
+    mark_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, map, flags, status);
+  count_flags_kernel<<<256, 256, 0, st>>>(flags, n_flags, count);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_distinct_rows(const int32_t* fb_id, const int32_t* cell_off,
+                                 const int32_t* tile_first, int32_t T, int32_t H,
+                                 unsigned long long* count, cudaStream_t st) {
+  distinct_rows_kernel<<<1184, kThreads, 0, st>>>(fb_id, cell_off, tile_first, T, H, count);
+  return cudaGetLastError();
+}
+
+}  // namespace agnes

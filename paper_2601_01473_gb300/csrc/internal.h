@@ -1,0 +1,128 @@
+// internal.h -- host-side launchers shared between the libagnes translation
+// units.  Not part of the public ABI (include/agnes.h is).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace agnes {
+
+// ---- scan.cu ---------------------------------------------------------------
+// Exclusive scan of nseg segments.  Segment s reads in[s*in_stride + i] for
+// i < len(s) and writes out[s*out_stride + i]; len(s) = d_len[s] when d_len is
+// non-null, else const_len.  With write_end, out[s*out_stride + len(s)] gets
+// the segment total; seg_total (if non-null) gets it too.  max_len bounds
+// every len(s).  scratch needs scan_scratch_elems(nseg, max_len) int64s.
+int64_t scan_scratch_elems(int64_t nseg, int64_t max_len);
+
+template <typename InT, typename OutT>
+cudaError_t seg_scan(const InT* in, int64_t in_stride, OutT* out, int64_t out_stride,
+                     const int32_t* d_len, int64_t const_len, int32_t nseg, int64_t max_len,
+                     bool write_end, int32_t* seg_total, int64_t* scratch,
+                     const int32_t* status, cudaStream_t st);
+
+// ---- blocks.cu -------------------------------------------------------------
+struct BlockTables {
+  int32_t* start_node = nullptr;   // first node of each block start
+  int32_t* start_block = nullptr;  // block index of each start
+  int64_t n_starts = 0;
+  int64_t n_blocks = 0;            // incl. continuation blocks of split objects
+  int32_t* tile_first = nullptr;   // T+1
+  int32_t* chunk_tile = nullptr;   // C+1
+  int32_t* tile_adj_block = nullptr;
+  int32_t* tile_feat_block = nullptr;
+  int64_t T = 0;
+  int64_t n_feat_blocks = 0;
+  int64_t rows_per_feat_block = 0;
+};
+
+// Builds the block tables on the device; allocates the arrays in *bt.
+cudaError_t build_block_tables(const void* d_offsets, int offsets_bits, int64_t N, int64_t E,
+                               int64_t adj_block_bytes, int64_t rows_per_feat_block,
+                               BlockTables* bt, cudaStream_t st, char* err, size_t errlen);
+void free_block_tables(BlockTables* bt);
+
+// ---- sample.cu -------------------------------------------------------------
+struct HopArgs {
+  // graph
+  const void* offsets;
+  int offsets_bits;
+  const int32_t* indices;
+  int32_t N;
+  // tiles
+  const int32_t* tile_first;
+  const int32_t* chunk_tile;
+  int32_t T;
+  // hyperbatch shape
+  int32_t H;
+  int64_t capK;      // node capacity per minibatch
+  int64_t cap_prev;  // frontier capacity per minibatch at this hop
+  int64_t ecap;      // edge capacity per minibatch at this hop
+  int32_t k;         // fanout
+  int32_t hop;       // 1-based
+  uint64_t seed;
+  uint64_t first_gid;
+  int32_t* status;
+};
+
+cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32_t B, int32_t N,
+                                  const int32_t* tile_first, const int32_t* chunk_tile, int32_t T,
+                                  int32_t* fcnt, int32_t* fcell_off, int32_t* tmp_id,
+                                  int32_t* tmp_pos, int32_t* fb_id, int32_t* fb_pos,
+                                  int64_t* scan_scratch, int32_t* status, int num_sms,
+                                  cudaStream_t st);
+
+cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
+                                const int32_t* fcell_off, int32_t* cnt, int num_sms,
+                                cudaStream_t st);
+
+cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
+                               const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
+                               int num_sms, cudaStream_t st);
+
+// ---- dedup.cu --------------------------------------------------------------
+struct DedupBufs {
+  const int32_t* nbr;       // H x ecap sampled ids
+  const int32_t* ecnt;      // H edge counts
+  int32_t* stile;           // H x ecap scratch (tile of each sampled id)
+  int32_t* scnt;            // T*H counters, zero on entry and exit
+  int32_t* soff;            // T*H+1
+  int32_t* sb_u;            // bucketed sampled ids
+  int32_t* sb_e;            // their edge index in the minibatch
+  const int32_t* fb_id;     // current frontier bucket
+  const int32_t* fb_pos;
+  const int32_t* fcell_off;
+  int32_t* newcnt;          // H x T (minibatch-major)
+  int32_t* newbase;         // H x T
+  int32_t* newtot;          // H
+  int32_t* nfcnt;           // T*H
+  int32_t* nfcell_off;      // T*H+1
+  int32_t* nfb_id;          // next frontier bucket
+  int32_t* nfb_pos;
+  const int32_t* nsz_prev;  // H frontier sizes
+  int32_t* nsz_next;        // H
+  int32_t* nodes;           // H x capK
+  int32_t* col;             // H x ecap
+  const int32_t* tile_adj_block;
+  uint8_t* adj_flags;       // per topology block: touched at this hop
+  int64_t* scan_scratch;
+};
+
+cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cudaStream_t st);
+
+// ---- gather.cu -------------------------------------------------------------
+cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
+                          const int32_t* fb_pos, const int32_t* total, void* out,
+                          const int32_t* status, int num_sms, cudaStream_t st);
+
+// Marks flags[map[t]] for every tile t whose cells (t, 0..H-1) in cell_off
+// hold an entry, then counts set flags into *count (int64).
+cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, const int32_t* map,
+                              uint8_t* flags, int64_t n_flags, int64_t* count,
+                              const int32_t* status, cudaStream_t st);
+
+cudaError_t launch_distinct_rows(const int32_t* fb_id, const int32_t* cell_off,
+                                 const int32_t* tile_first, int32_t T, int32_t H,
+                                 unsigned long long* count, cudaStream_t st);
+
+}  // namespace agnes

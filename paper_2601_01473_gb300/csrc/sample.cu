@@ -1,0 +1,350 @@
+// sample.cu -- bucketing of the targets and per-hop neighbour sampling.
+//
+// Bucket matrix (Sec. 3.4 (3), Algorithm 1's Bck_{i,j}): frontier entries are
+// kept per (tile, minibatch) cell in tile-major, minibatch-minor order, sorted
+// by node id inside a cell, each with its global output row
+// g = j * capK + position.  A topology block's requests are therefore one
+// contiguous run of the bucket, and sampling walks the bucket in order, so the
+// block is read once for all minibatches of the hyperbatch (Sec. 3.3) and its
+// adjacency data is reused out of L2.
+//
+// Sampling (Sec. 3.1, Algorithm 1's Sample): up to k neighbours per frontier
+// node, uniformly without replacement; all of them in CSR order when
+// deg <= k, else Floyd's algorithm (Bentley & Floyd, CACM 1987) with
+// Philox4x32-10 draws keyed on (seed; v, hop, slot, g).  A group of G >= k
+// lanes handles one frontier node: lane s draws slot s's candidate in
+// parallel and the k-step collision resolution runs over in-group shuffles.
+#include "common.cuh"
+#include "internal.h"
+
+namespace agnes {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+
+// ---- bucketing of the targets ------------------------------------------------
+
+__global__ void __launch_bounds__(kThreads)
+targets_count_kernel(const int32_t* __restrict__ nodes, int64_t capK, int32_t H, int32_t B,
+                     int32_t N, TileMap tm, int32_t* __restrict__ fcnt, int32_t* status) {
+  const int64_t total = (int64_t)H * B;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; i0 < total;
+       i0 += stride) {
+    const int64_t i = i0 + lane_id();
+    bool active = i < total;
+    int64_t cell = 0;
+    if (active) {
+      const int32_t j = (int32_t)(i / B);
+      const int32_t v = nodes[j * capK + (i - (int64_t)j * B)];
+      if (v < 0 || v >= N) {
+        atomicOr(status, kErrTargetRange);
+        active = false;
+      } else {
+        cell = (int64_t)tile_of(tm, v) * H + j;
+      }
+    }
+    warp_agg_inc(fcnt, cell, active);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+targets_scatter_kernel(const int32_t* __restrict__ nodes, int64_t capK, int32_t H, int32_t B,
+                       int32_t N, TileMap tm, int32_t* __restrict__ fcnt,
+                       const int32_t* __restrict__ fcell_off, int32_t* __restrict__ tmp_id,
+                       int32_t* __restrict__ tmp_pos, const int32_t* status) {
+  if (failed(status)) return;
+  const int64_t total = (int64_t)H * B;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; i0 < total;
+       i0 += stride) {
+    const int64_t i = i0 + lane_id();
+    bool active = i < total;
+    int32_t v = 0, j = 0;
+    int64_t cell = 0;
+    if (active) {
+      j = (int32_t)(i / B);
+      v = nodes[j * capK + (i - (int64_t)j * B)];
+      active = v >= 0 && v < N;
+      if (active) cell = (int64_t)tile_of(tm, v) * H + j;
+    }
+    const unsigned mask = __ballot_sync(0xffffffffu, active);
+    if (active) {
+      const int32_t slot = fcell_off[cell] + warp_agg_take(fcnt, cell, mask);
+      tmp_id[slot] = v;
+      tmp_pos[slot] = (int32_t)(j * capK + (i - (int64_t)j * B));
+    }
+  }
+}
+
+// One warp per cell: orders the cell's targets by id (rank in the cell's
+// membership bitmap) and flags a target repeated within a minibatch.
+__global__ void __launch_bounds__(kThreads)
+targets_sort_kernel(const int32_t* __restrict__ fcell_off, int64_t ncells, int32_t H, TileMap tm,
+                    const int32_t* __restrict__ tmp_id, const int32_t* __restrict__ tmp_pos,
+                    int32_t* __restrict__ fb_id, int32_t* __restrict__ fb_pos, int32_t* status) {
+  if (failed(status)) return;
+  __shared__ uint32_t bits_s[kWarps][kTileWords];
+  __shared__ int32_t pref_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  uint32_t* bits = bits_s[warp];
+  int32_t* pref = pref_s[warp];
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t cell = blockIdx.x * (int64_t)kWarps + warp; cell < ncells; cell += nwarps) {
+    const int32_t o = fcell_off[cell];
+    const int32_t n = fcell_off[cell + 1] - o;
+    if (n == 0) continue;
+    const int32_t t = (int32_t)(cell / H);
+    const int32_t base = tm.tile_first[t];
+    const int32_t words = (tm.tile_first[t + 1] - base + 31) >> 5;
+    for (int w = lane; w < words; w += 32) bits[w] = 0;
+    __syncwarp();
+    for (int32_t i = lane; i < n; i += 32) {
+      const int32_t lu = tmp_id[o + i] - base;
+      const uint32_t bit = 1u << (lu & 31);
+      if (atomicOr(&bits[lu >> 5], bit) & bit) atomicOr(status, kErrTargetDup);
+    }
+    __syncwarp();
+    int32_t c[4], sum = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      c[q] = w < words ? __popc(bits[w]) : 0;
+      sum += c[q];
+    }
+    int32_t run = warp_incl_scan(sum) - sum;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      pref[lane * 4 + q] = run;
+      run += c[q];
+    }
+    __syncwarp();
+    for (int32_t i = lane; i < n; i += 32) {
+      const int32_t v = tmp_id[o + i];
+      const int32_t lu = v - base;
+      const int32_t w = lu >> 5;
+      const int32_t r = pref[w] + __popc(bits[w] & ((1u << (lu & 31)) - 1u));
+      fb_id[o + r] = v;
+      fb_pos[o + r] = tmp_pos[o + i];
+    }
+    __syncwarp();
+  }
+}
+
+// ---- sampling --------------------------------------------------------------------
+
+template <typename OffT>
+__global__ void __launch_bounds__(kThreads)
+sample_count_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
+                    const int32_t* total_ptr, const OffT* __restrict__ off, int64_t capK,
+                    int64_t cap_prev, int32_t k, int32_t* __restrict__ cnt,
+                    const int32_t* status) {
+  if (failed(status)) return;
+  const int64_t total = *total_ptr;
+  const uint32_t capk32 = (uint32_t)capK;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t v = fb_id[i];
+    const uint32_t g = (uint32_t)fb_pos[i];
+    const uint32_t j = g / capk32;
+    const uint32_t pos = g - j * capk32;
+    const int64_t d = (int64_t)__ldg(off + v + 1) - (int64_t)__ldg(off + v);
+    cnt[j * cap_prev + pos] = (int32_t)(d < k ? d : k);
+  }
+}
+
+struct FillArgs {
+  const int32_t* fb_id;
+  const int32_t* fb_pos;
+  const int32_t* total_ptr;
+  const int64_t* indptr;
+  const int32_t* indices;
+  int32_t* nbr;
+  int64_t capK, cap_prev, ecap;
+  int32_t k, hop;
+  uint32_t key_lo, key_hi;
+  uint64_t first_gid;
+  const int32_t* status;
+};
+
+__device__ __forceinline__ int64_t draw(const FillArgs& a, int32_t v, int32_t s, uint64_t gid,
+                                        int64_t J) {
+  const uint4 x = philox4x32_10(
+      make_uint4((uint32_t)v, ((uint32_t)a.hop << 24) | (uint32_t)s, (uint32_t)gid,
+                 (uint32_t)(gid >> 32)),
+      make_uint2(a.key_lo, a.key_hi));
+  const uint64_t r = ((uint64_t)x.y << 32) | (uint64_t)x.x;
+  return (int64_t)__umul64hi(r, (uint64_t)(J + 1));
+}
+
+// G lanes per frontier node, k <= G.
+template <typename OffT, int G>
+__global__ void __launch_bounds__(kThreads)
+sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
+  if (failed(a.status)) return;
+  const int64_t total = *a.total_ptr;
+  constexpr int kGroups = 32 / G;
+  const int lane = lane_id();
+  const int sub = lane / G, s = lane % G;
+  const unsigned gmask = G == 32 ? 0xffffffffu : (((1u << G) - 1u) << (sub * G));
+  const uint32_t capk32 = (uint32_t)a.capK;
+  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t e0 = warp0 * kGroups; e0 < total; e0 += nwarps * kGroups) {
+    const int64_t i = e0 + sub;
+    if (i >= total) continue;  // whole group skips together
+    const int32_t v = a.fb_id[i];
+    const uint32_t g = (uint32_t)a.fb_pos[i];
+    const uint32_t j = g / capk32;
+    const uint32_t pos = g - j * capk32;
+    const int64_t base = (int64_t)__ldg(off + v);
+    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
+    int32_t* out = a.nbr + j * a.ecap + a.indptr[j * (a.cap_prev + 1) + pos];
+    if (d <= a.k) {
+      for (int64_t q = s; q < d; q += G) out[q] = __ldg(a.indices + base + q);
+      continue;
+    }
+    const int64_t J = d - a.k + s;
+    const int64_t t = s < a.k ? draw(a, v, s, a.first_gid + j, J) : -1;
+    bool collided = false;
+    for (int q = 0; q < a.k; ++q) {
+      const int64_t mine = collided ? J : t;
+      const int64_t cq = __shfl_sync(gmask, mine, q, G);
+      if (s > q && t == cq) collided = true;
+    }
+    if (s < a.k) out[s] = __ldg(a.indices + base + (collided ? J : t));
+  }
+}
+
+// One warp per frontier node for fanouts above 32: slots are drawn 32 at a
+// time; each candidate is checked against the choices of earlier chunks (kept
+// in shared memory) and then resolved within its chunk by shuffles.
+template <typename OffT>
+__global__ void __launch_bounds__(kThreads)
+sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
+  if (failed(a.status)) return;
+  __shared__ int32_t chosen_s[kWarps][kMaxFanout];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  int32_t* chosen = chosen_s[warp];
+  const int64_t total = *a.total_ptr;
+  const uint32_t capk32 = (uint32_t)a.capK;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total;
+       i += nwarps) {
+    const int32_t v = a.fb_id[i];
+    const uint32_t g = (uint32_t)a.fb_pos[i];
+    const uint32_t j = g / capk32;
+    const uint32_t pos = g - j * capk32;
+    const int64_t base = (int64_t)__ldg(off + v);
+    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
+    int32_t* out = a.nbr + j * a.ecap + a.indptr[j * (a.cap_prev + 1) + pos];
+    if (d <= a.k) {
+      for (int64_t q = lane; q < d; q += 32) out[q] = __ldg(a.indices + base + q);
+      continue;
+    }
+    for (int c0 = 0; c0 < a.k; c0 += 32) {
+      const int s = c0 + lane;
+      const bool valid = s < a.k;
+      const int64_t J = d - a.k + s;
+      const int64_t t = valid ? draw(a, v, s, a.first_gid + j, J) : -1;
+      bool collided = false;
+      for (int q = 0; q < c0; ++q) collided |= (chosen[q] == t);
+      const int m = min(32, a.k - c0);
+      for (int q = 0; q < m; ++q) {
+        const int64_t mine = collided ? J : t;
+        const int64_t cq = __shfl_sync(0xffffffffu, mine, q);
+        if (lane > q && t == cq) collided = true;
+      }
+      const int64_t c = collided ? J : t;
+      if (valid) {
+        chosen[s] = (int32_t)c;
+        out[s] = __ldg(a.indices + base + c);
+      }
+      __syncwarp();
+    }
+  }
+}
+
+int grid_for(int num_sms, int per_sm) { return num_sms * per_sm; }
+
+}  // namespace
+
+cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32_t B, int32_t N,
+                                  const int32_t* tile_first, const int32_t* chunk_tile, int32_t T,
+                                  int32_t* fcnt, int32_t* fcell_off, int32_t* tmp_id,
+                                  int32_t* tmp_pos, int32_t* fb_id, int32_t* fb_pos,
+                                  int64_t* scan_scratch, int32_t* status, int num_sms,
+                                  cudaStream_t st) {
+  const TileMap tm{tile_first, chunk_tile, T};
+  const int64_t ncells = (int64_t)T * H;
+  const int grid = grid_for(num_sms, 8);
+  targets_count_kernel<<<grid, kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, status);
+  cudaError_t e = seg_scan<int32_t, int32_t>(fcnt, 0, fcell_off, 0, nullptr, ncells, 1, ncells,
+                                             true, nullptr, scan_scratch, status, st);
+  if (e != cudaSuccess) return e;
+  targets_scatter_kernel<<<grid, kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, fcell_off,
+                                                    tmp_id, tmp_pos, status);
+  targets_sort_kernel<<<grid, kThreads, 0, st>>>(fcell_off, ncells, H, tm, tmp_id, tmp_pos,
+                                                 fb_id, fb_pos, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
+                                const int32_t* fcell_off, int32_t* cnt, int num_sms,
+                                cudaStream_t st) {
+  const int32_t* total = fcell_off + (int64_t)a.T * a.H;
+  const int grid = grid_for(num_sms, 8);
+  if (a.offsets_bits == 32)
+    sample_count_kernel<int32_t><<<grid, kThreads, 0, st>>>(
+        fb_id, fb_pos, total, (const int32_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt, a.status);
+  else
+    sample_count_kernel<int64_t><<<grid, kThreads, 0, st>>>(
+        fb_id, fb_pos, total, (const int64_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt, a.status);
+  return cudaGetLastError();
+}
+
+template <typename OffT>
+static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int grid,
+                              cudaStream_t st) {
+  if (k <= 4)
+    sample_fill_kernel<OffT, 4><<<grid, kThreads, 0, st>>>(f, off);
+  else if (k <= 8)
+    sample_fill_kernel<OffT, 8><<<grid, kThreads, 0, st>>>(f, off);
+  else if (k <= 16)
+    sample_fill_kernel<OffT, 16><<<grid, kThreads, 0, st>>>(f, off);
+  else if (k <= 32)
+    sample_fill_kernel<OffT, 32><<<grid, kThreads, 0, st>>>(f, off);
+  else
+    sample_fill_wide_kernel<OffT><<<grid, kThreads, 0, st>>>(f, off);
+}
+
+cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
+                               const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
+                               int num_sms, cudaStream_t st) {
+  FillArgs f;
+  f.fb_id = fb_id;
+  f.fb_pos = fb_pos;
+  f.total_ptr = fcell_off + (int64_t)a.T * a.H;
+  f.indptr = indptr;
+  f.indices = a.indices;
+  f.nbr = nbr;
+  f.capK = a.capK;
+  f.cap_prev = a.cap_prev;
+  f.ecap = a.ecap;
+  f.k = a.k;
+  f.hop = a.hop;
+  f.key_lo = (uint32_t)a.seed;
+  f.key_hi = (uint32_t)(a.seed >> 32);
+  f.first_gid = a.first_gid;
+  f.status = a.status;
+  const int grid = grid_for(num_sms, 8);
+  if (a.offsets_bits == 32)
+    launch_fill_typed<int32_t>(f, (const int32_t*)a.offsets, a.k, grid, st);
+  else
+    launch_fill_typed<int64_t>(f, (const int64_t*)a.offsets, a.k, grid, st);
+  return cudaGetLastError();
+}
+
+}  // namespace agnes

@@ -1,0 +1,164 @@
+// scan.cu -- segmented exclusive scans (reduce / scan-of-partials / downsweep).
+//
+// Used for every prefix sum on the path: the per-minibatch indptr of a hop,
+// the cell offsets of the bucket matrix, the per-minibatch offsets of the new
+// nodes of each (tile, minibatch) cell, and the tile compaction at load time.
+// Three launches per scan and no inter-block waiting, so no kernel ever spins
+// on another block's progress.
+#include "common.cuh"
+#include "internal.h"
+
+namespace agnes {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kItems = 8;
+constexpr int kChunk = kThreads * kItems;  // elements per block and chunk
+
+__device__ __forceinline__ int64_t seg_len(const int32_t* d_len, int64_t const_len, int s) {
+  return d_len ? (int64_t)d_len[s] : const_len;
+}
+
+// Exclusive block-wide scan of one int64 per thread; *total gets the sum.
+__device__ __forceinline__ int64_t block_excl_scan(int64_t v, int64_t* total) {
+  __shared__ int64_t warp_tot[kThreads / 32];
+  __shared__ int64_t block_tot;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t incl = warp_incl_scan(v);
+  if (lane == 31) warp_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const int64_t w = lane < kThreads / 32 ? warp_tot[lane] : 0;
+    const int64_t wi = warp_incl_scan(w);
+    if (lane < kThreads / 32) warp_tot[lane] = wi - w;
+    if (lane == kThreads / 32 - 1) block_tot = wi;
+  }
+  __syncthreads();
+  const int64_t out = warp_tot[warp] + incl - v;
+  *total = block_tot;
+  __syncthreads();  // warp_tot / block_tot are reused by the next call
+  return out;
+}
+
+template <typename InT>
+__global__ void __launch_bounds__(kThreads)
+scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t* d_len,
+                   int64_t const_len, int64_t chunks, int64_t* __restrict__ partial,
+                   const int32_t* status) {
+  if (status && failed(status)) return;
+  const int s = blockIdx.y;
+  const int64_t c = blockIdx.x;
+  const int64_t len = seg_len(d_len, const_len, s);
+  const int64_t begin = c * kChunk;
+  int64_t sum = 0;
+  if (begin < len) {
+    const InT* p = in + (int64_t)s * in_stride;
+    const int64_t end = min(len, begin + kChunk);
+    for (int64_t i = begin + threadIdx.x; i < end; i += kThreads) sum += (int64_t)p[i];
+  }
+  __shared__ int64_t wsum[kThreads / 32];
+  sum = warp_sum(sum);
+  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = sum;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    int64_t v = threadIdx.x < kThreads / 32 ? wsum[threadIdx.x] : 0;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) partial[(int64_t)s * chunks + c] = v;
+  }
+}
+
+template <typename OutT>
+__global__ void __launch_bounds__(kThreads)
+scan_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, const int32_t* d_len,
+                     int64_t const_len, OutT* __restrict__ out, int64_t out_stride, bool write_end,
+                     int32_t* seg_total, const int32_t* status) {
+  if (status && failed(status)) return;
+  const int s = blockIdx.x;
+  int64_t* p = partial + (int64_t)s * chunks;
+  int64_t carry = 0;
+  for (int64_t base = 0; base < chunks; base += kThreads) {
+    const int64_t i = base + threadIdx.x;
+    const int64_t v = i < chunks ? p[i] : 0;
+    int64_t tot;
+    const int64_t ex = block_excl_scan(v, &tot);
+    if (i < chunks) p[i] = carry + ex;
+    carry += tot;
+  }
+  if (threadIdx.x == 0) {
+    const int64_t len = seg_len(d_len, const_len, s);
+    if (write_end) out[(int64_t)s * out_stride + len] = (OutT)carry;
+    if (seg_total) seg_total[s] = (int32_t)carry;
+  }
+}
+
+template <typename InT, typename OutT>
+__global__ void __launch_bounds__(kThreads)
+scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict__ out,
+                 int64_t out_stride, const int32_t* d_len, int64_t const_len, int64_t chunks,
+                 const int64_t* __restrict__ partial, const int32_t* status) {
+  if (status && failed(status)) return;
+  const int s = blockIdx.y;
+  const int64_t c = blockIdx.x;
+  const int64_t len = seg_len(d_len, const_len, s);
+  const int64_t begin = c * kChunk;
+  if (begin >= len) return;
+  const int64_t n = min((int64_t)kChunk, len - begin);
+  const InT* p = in + (int64_t)s * in_stride + begin;
+  OutT* q = out + (int64_t)s * out_stride + begin;
+
+  __shared__ int64_t stage[kChunk];
+  for (int i = threadIdx.x; i < kChunk; i += kThreads) stage[i] = i < n ? (int64_t)p[i] : 0;
+  __syncthreads();
+  int64_t local[kItems];
+  int64_t run = 0;
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) {
+    local[k] = run;
+    run += stage[threadIdx.x * kItems + k];
+  }
+  int64_t tot;
+  const int64_t ex = block_excl_scan(run, &tot) + partial[(int64_t)s * chunks + c];
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) stage[threadIdx.x * kItems + k] = ex + local[k];
+  __syncthreads();
+  for (int i = threadIdx.x; i < n; i += kThreads) q[i] = (OutT)stage[i];
+}
+
+}  // namespace
+
+int64_t scan_scratch_elems(int64_t nseg, int64_t max_len) {
+  int64_t chunks = (max_len + kChunk - 1) / kChunk;
+  if (chunks < 1) chunks = 1;
+  return nseg * chunks;
+}
+
+template <typename InT, typename OutT>
+cudaError_t seg_scan(const InT* in, int64_t in_stride, OutT* out, int64_t out_stride,
+                     const int32_t* d_len, int64_t const_len, int32_t nseg, int64_t max_len,
+                     bool write_end, int32_t* seg_total, int64_t* scratch,
+                     const int32_t* status, cudaStream_t st) {
+  if (nseg <= 0) return cudaSuccess;
+  int64_t chunks = (max_len + kChunk - 1) / kChunk;
+  if (chunks < 1) chunks = 1;
+  const dim3 grid((unsigned)chunks, (unsigned)nseg);
+  scan_reduce_kernel<InT><<<grid, kThreads, 0, st>>>(in, in_stride, d_len, const_len, chunks,
+                                                      scratch, status);
+  scan_partials_kernel<OutT><<<nseg, kThreads, 0, st>>>(scratch, chunks, d_len, const_len, out,
+                                                        out_stride, write_end, seg_total, status);
+  scan_down_kernel<InT, OutT><<<grid, kThreads, 0, st>>>(in, in_stride, out, out_stride, d_len,
+                                                         const_len, chunks, scratch, status);
+  return cudaGetLastError();
+}
+
+template cudaError_t seg_scan<int32_t, int32_t>(const int32_t*, int64_t, int32_t*, int64_t,
+                                                const int32_t*, int64_t, int32_t, int64_t, bool,
+                                                int32_t*, int64_t*, const int32_t*, cudaStream_t);
+template cudaError_t seg_scan<int32_t, int64_t>(const int32_t*, int64_t, int64_t*, int64_t,
+                                                const int32_t*, int64_t, int32_t, int64_t, bool,
+                                                int32_t*, int64_t*, const int32_t*, cudaStream_t);
+template cudaError_t seg_scan<uint8_t, int32_t>(const uint8_t*, int64_t, int32_t*, int64_t,
+                                                const int32_t*, int64_t, int32_t, int64_t, bool,
+                                                int32_t*, int64_t*, const int32_t*, cudaStream_t);
+
+}  // namespace agnes

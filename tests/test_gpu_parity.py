@@ -1,0 +1,223 @@
+"""Parity of the CUDA path (through the C ABI) with the oracle: bit-exact
+sampled subgraphs, relabelled edges, node lists, gathered feature bytes and
+blocks-touched statistics, on small seeded inputs that span many tiles and
+blocks, plus edge cases and error reporting."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from agnes_inputs import WORKLOADS, build_workload, synth, targets_for_step
+from paper_2601_01473_gb300 import AgnesError, Graph
+
+pytestmark = pytest.mark.gpu
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _bytes(t: torch.Tensor) -> np.ndarray:
+    t = t.detach().cpu().contiguous()
+    return t.view(torch.uint8).numpy() if t.numel() else np.zeros(0, np.uint8)
+
+
+def compare(g: Graph, og: oracle.Graph, targets: np.ndarray, fanouts, seed, gid0, adj_bb, feat_bb,
+            check_stats=True, only=None):
+    """Compares every (or the listed) minibatch of g's last hyperbatch with
+    the oracle."""
+    H = targets.shape[0]
+    js = range(H) if only is None else only
+    if check_stats:
+        ref, ref_stats = oracle.hyperbatch(og, targets, fanouts, seed, gid0, True, adj_bb, feat_bb)
+        assert g.stats() == ref_stats
+    else:
+        ref = {j: oracle.sample_minibatch(og, targets[j], fanouts, seed, gid0 + j) for j in js}
+    for j in js:
+        v, r = g.fetch(j), ref[j]
+        assert np.array_equal(v.nodes.cpu().numpy(), r["nodes"]), f"nodes of minibatch {j}"
+        for h in range(len(fanouts)):
+            hv, hr = v.hops[h], r["hops"][h]
+            assert (hv.num_dst, hv.num_src, hv.num_edges) == (
+                hr["num_dst"], hr["num_src"], hr["num_edges"]), f"sizes of hop {h}, mb {j}"
+            assert np.array_equal(hv.indptr.cpu().numpy(), hr["indptr"]), f"indptr {h} mb {j}"
+            assert np.array_equal(hv.col.cpu().numpy(), hr["col"]), f"col {h} mb {j}"
+        assert np.array_equal(_bytes(v.feats), r["feats"].view(np.uint8).reshape(-1)
+                              if r["feats"].size else np.zeros(0, np.uint8)), f"feats mb {j}"
+
+
+def make(n, deg, a=0.57, b=0.19, c=0.19, seed=0, bits=64, dtype=torch.float16, dim=64):
+    off, ind = synth.rmat_csr(n, deg, a, b, c, seed,
+                              offsets_dtype=torch.int32 if bits == 32 else torch.int64)
+    feats = synth.normal_features(n, dim, dtype, seed + 100)
+    return off, ind, feats
+
+
+def load(off, ind, feats, adj_bb, feat_bb):
+    dev = torch.device("cuda:0")
+    return Graph(off.to(dev), ind.to(dev), feats.to(dev), adj_block_bytes=adj_bb,
+                 feat_block_bytes=feat_bb)
+
+
+def test_golden_fixture(cuda_device):
+    with open(os.path.join(GOLDEN, "oracle_tiny.json")) as f:
+        d = json.load(f)
+    off = torch.tensor(d["offsets"], dtype=torch.int32)
+    ind = torch.tensor(d["indices"], dtype=torch.int32)
+    feats = torch.tensor(d["features"], dtype=torch.float32)
+    targets = torch.tensor(d["targets"], dtype=torch.int32)
+    g = load(off, ind, feats, d["adj_block_bytes"], d["feat_block_bytes"])
+    g.prepare(targets.to(cuda_device), d["fanouts"], d["seed"], d["first_gid"])
+    assert g.stats() == d["stats"]
+    for j, ref in enumerate(d["minibatches"]):
+        v = g.fetch(j)
+        assert v.nodes.cpu().tolist() == ref["nodes"]
+        for hv, hr in zip(v.hops, ref["hops"]):
+            assert hv.num_dst == hr["num_dst"]
+            assert hv.indptr.cpu().tolist() == hr["indptr"]
+            assert hv.col.cpu().tolist() == hr["col"]
+    g.close()
+
+
+@pytest.mark.parametrize("bits,dtype,fanouts", [
+    (32, torch.float32, (10, 5)),
+    (64, torch.float16, (15, 10, 5)),
+    (64, torch.float16, (25, 10)),
+    (32, torch.float16, (3,)),
+    (64, torch.float32, (1, 1, 1, 1)),
+    (64, torch.float16, (40, 3)),      # fanout above one warp
+    (32, torch.float32, (33, 2)),
+    (64, torch.float16, (4, 8, 16, 32)),
+])
+def test_parity_small_rmat(cuda_device, bits, dtype, fanouts):
+    off, ind, feats = make(30000, 12, seed=len(fanouts) * 7 + bits, bits=bits, dtype=dtype)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), 5, 100, 11, bits)
+    adj_bb, feat_bb = 8192, 4096
+    g = load(off, ind, feats, adj_bb, feat_bb)
+    g.prepare(targets.to(cuda_device), list(fanouts), 0xDEADBEEF12345678, 1000)
+    compare(g, og, targets.numpy(), list(fanouts), 0xDEADBEEF12345678, 1000, adj_bb, feat_bb)
+    g.close()
+
+
+def test_block_table_matches_oracle(cuda_device):
+    for bits, bb in ((32, 64), (64, 256), (64, 4096), (32, 65536)):
+        off, ind, feats = make(20000, 20, a=0.6, b=0.2, c=0.15, seed=bb, bits=bits)
+        og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+        node_block, nb = oracle.build_adj_blocks(og, bb)
+        starts = np.flatnonzero(np.r_[True, node_block[1:] != node_block[:-1]])
+        g = load(off, ind, feats, bb, 4096)
+        sn, sb = g.adj_blocks()
+        assert np.array_equal(sn.numpy(), starts)
+        assert np.array_equal(sb.numpy(), node_block[starts])
+        assert g.info()["adj_blocks"] == nb
+        g.close()
+
+
+def test_degenerate_graphs(cuda_device):
+    # a star plus isolated nodes: most targets have degree 0
+    n = 5000
+    deg = np.zeros(n, np.int64)
+    deg[0] = n - 1
+    deg[1:50] = 1
+    off = torch.tensor(np.r_[0, np.cumsum(deg)], dtype=torch.int64)
+    rows = [np.arange(1, n)] + [np.array([0])] * 49
+    ind = torch.tensor(np.concatenate(rows), dtype=torch.int32)
+    feats = synth.normal_features(n, 8, torch.float32, 1)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    g = load(off, ind, feats, 1024, 64)
+    for targets in (np.arange(4000, 4064, dtype=np.int32).reshape(1, 64),   # all degree 0
+                    np.array([[0, 1, 2, 3], [4999, 10, 0, 7]], np.int32),
+                    np.arange(n, dtype=np.int32).reshape(1, n)):          # B = N
+        for fan in ([5], [2, 2], [1024]):
+            g.prepare(torch.tensor(targets).to(cuda_device), fan, 3, 9)
+            compare(g, og, targets, fan, 3, 9, 1024, 64)
+    g.close()
+
+
+def test_hyperbatch_size_and_block_size_do_not_change_results(cuda_device):
+    """Global minibatch 502 gives the same output inside hyperbatches of 16, 3
+    and 1 minibatches and under different block sizes."""
+    off, ind, feats = make(40000, 14, seed=21)
+    targets = synth.hyperbatch_targets(torch.arange(40000, dtype=torch.int32), 16, 128, 4, 0)
+    fan, seed = [8, 4, 2], 99
+    ref = None
+    # (first row, H, block bytes): row 2 of targets is global minibatch 502
+    for first, H, bb in ((0, 16, 1 << 20), (1, 3, 65536), (2, 1, 4096), (0, 16, 2048)):
+        g = load(off, ind, feats, bb, bb)
+        g.prepare(targets[first:first + H].contiguous().to(cuda_device), fan, seed, 500 + first)
+        v = g.fetch(2 - first)
+        got = (v.nodes.cpu().numpy(), [h.col.cpu().numpy() for h in v.hops], _bytes(v.feats))
+        if ref is None:
+            ref = got
+        else:
+            assert np.array_equal(got[0], ref[0])
+            assert all(np.array_equal(a, b) for a, b in zip(got[1], ref[1]))
+            assert np.array_equal(got[2], ref[2])
+        g.close()
+
+
+def test_host_targets_equal_device_targets(cuda_device):
+    off, ind, feats = make(20000, 10, seed=3)
+    targets = synth.hyperbatch_targets(torch.arange(20000, dtype=torch.int32), 4, 256, 1, 0)
+    g = load(off, ind, feats, 16384, 16384)
+    g.prepare(targets.to(cuda_device), [10, 5], 5, 0)
+    a = [g.fetch(j).nodes.cpu().clone() for j in range(4)]
+    g.prepare(targets.pin_memory(), [10, 5], 5, 0)
+    b = [g.fetch(j).nodes.cpu().clone() for j in range(4)]
+    g.prepare(targets.clone(), [10, 5], 5, 0)  # pageable host memory
+    c = [g.fetch(j).nodes.cpu().clone() for j in range(4)]
+    assert all(torch.equal(x, y) and torch.equal(x, z) for x, y, z in zip(a, b, c))
+    g.close()
+
+
+@pytest.mark.parametrize("dtype,dim", [(torch.float16, 3), (torch.float32, 100),
+                                       (torch.float32, 32), (torch.float16, 256),
+                                       (torch.float32, 1000)])
+def test_row_sizes(cuda_device, dtype, dim):
+    off, ind, feats = make(8000, 8, seed=dim, dtype=dtype, dim=dim)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    targets = synth.hyperbatch_targets(torch.arange(8000, dtype=torch.int32), 3, 50, 2, dim)
+    rb = feats.shape[1] * feats.element_size()
+    g = load(off, ind, feats, 4096, max(4096, rb))
+    g.prepare(targets.to(cuda_device), [6, 3], 17, 3)
+    compare(g, og, targets.numpy(), [6, 3], 17, 3, 4096, max(4096, rb))
+    g.close()
+
+
+def test_invalid_targets_are_reported_and_ctx_stays_usable(cuda_device):
+    off, ind, feats = make(3000, 6, seed=8)
+    g = load(off, ind, feats, 4096, 4096)
+    bad_range = torch.tensor([[1, 2, 3000]], dtype=torch.int32)
+    bad_dup = torch.tensor([[5, 9, 5, 7]], dtype=torch.int32)
+    for bad in (bad_range, bad_dup, torch.tensor([[-1, 4]], dtype=torch.int32)):
+        g.prepare(bad.to(cuda_device), [3], 1, 0)
+        with pytest.raises(AgnesError) as e:
+            g.fetch(0)
+        assert e.value.status == 1
+    with pytest.raises(AgnesError):
+        g.prepare(torch.tensor([[1]], dtype=torch.int32, device=cuda_device), [0], 1, 0)
+    with pytest.raises(AgnesError):
+        g.prepare(torch.tensor([[1]], dtype=torch.int32, device=cuda_device), [2000], 1, 0)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    ok = np.array([[1, 2, 3, 4]], np.int32)
+    g.prepare(torch.tensor(ok).to(cuda_device), [3, 2], 1, 0)
+    compare(g, og, ok, [3, 2], 1, 0, 4096, 4096)
+    g.close()
+
+
+@pytest.mark.parametrize("name", ["rmat100k", "mini100m", "mini_skew"])
+def test_workload_parity_all_minibatches(cuda_device, name):
+    w = WORKLOADS[name]
+    data = build_workload(w, "cpu")
+    og = oracle.Graph(data["offsets"].numpy(), data["indices"].numpy(), data["features"].numpy())
+    g = load(data["offsets"], data["indices"], data["features"], w.adj_block_bytes,
+             w.feat_block_bytes)
+    targets = targets_for_step(w, data["pool"], 0)
+    g.prepare(targets.to(cuda_device), list(w.fanouts), w.seed, 0)
+    compare(g, og, targets.numpy(), list(w.fanouts), w.seed, 0, w.adj_block_bytes,
+            w.feat_block_bytes)
+    c = g.counters()
+    assert c["rows"] == sum(g.sizes(j)["num_nodes"] for j in range(w.H))
+    assert 0 < c["distinct_rows"] <= c["rows"]
+    g.close()
