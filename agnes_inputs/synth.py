@@ -154,19 +154,17 @@ def _normal_table(device) -> torch.Tensor:
 def normal_features(num_nodes: int, dim: int, dtype, seed: int, device="cpu",
                     chunk_rows: int = 1 << 20) -> torch.Tensor:
     """[N, dim] features ~ N(0,1) (inverse-CDF of 16-bit uniforms), as dtype."""
-    if dim % 2:
-        raise ValueError("feature dim must be even")
     table = _normal_table(device)
     out = torch.empty((num_nodes, dim), dtype=dtype, device=device)
-    half = dim // 2
+    half = (dim + 1) // 2
     for r0 in range(0, num_nodes, chunk_rows):
         r1 = min(num_nodes, r0 + chunk_rows)
         rows = torch.arange(r0, r1, dtype=torch.int64, device=device)
         ctr = (rows[:, None] * half + torch.arange(half, dtype=torch.int64, device=device))
         ctr = ctr.flatten()
         h = hash32(ctr, seed, 0x46454154)
-        u = torch.stack([h & 0xFFFF, h >> 16], dim=1).flatten()
-        out[r0:r1] = table[u].view(r1 - r0, dim).to(dtype)
+        u = torch.stack([h & 0xFFFF, h >> 16], dim=1).view(r1 - r0, 2 * half)[:, :dim]
+        out[r0:r1] = table[u].to(dtype)
     return out
 
 

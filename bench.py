@@ -1,0 +1,411 @@
+"""Benchmark: hyperbatch sampling + gathering on one (or N replica) GB300s.
+
+One step = one hyperbatch through the whole path (bucketing, K hops of
+sampling + dedup/relabel, block-wise feature gather) via the C ABI, on the
+100M-node RMAT workload (fp16 x128 features, 1 MB blocks, 128 minibatches x
+1024 targets from a 1% train split, fanouts [15, 10, 5]).  Inputs are
+generated on the device before timing; the graph (~33 GB) is far larger than
+L2, so no L2 flush is needed between steps.
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle
+instead (bounded sample, host cores).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from agnes_inputs import WORKLOADS, build_graph, target_pool, targets_for_step  # noqa: E402
+
+METRIC = "sampled+gathered minibatches/sec per hyperbatch; achieved HBM GB/s vs ~8 TB/s"
+UNIT = "minibatches/s"
+DEFAULT_WORKLOAD = "rmat100m"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ----------------------------------------------------------------------------
+# helpers
+# ----------------------------------------------------------------------------
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return None
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+def kernel_launches_per_step(K: int) -> int:
+    """Kernels libagnes launches per hyperbatch: target bucketing 6 (count,
+    3-kernel scan, scatter, sort) + 1 size fill; per hop 19 (count, 3 scan,
+    fill, hist, 3 scan, scatter, dedup count, 3 scan, size add, 3 scan,
+    emit); 1 gather; K+2 for the blocks-touched counts."""
+    return 7 + 19 * K + 1 + K + 2
+
+
+def algorithmic_bytes(c: dict, off_bytes: int) -> dict:
+    """Bytes the method must move per hyperbatch (per-unit model):
+    per hop h: frontier offsets pair, sampled-id read, col write, indptr,
+    node-list write; gather: one read per distinct row, one write per row,
+    8 index bytes per row."""
+    rb = c["row_bytes"]
+    K = len(c["frontier"])
+    hop = 0
+    for h in range(K):
+        f, e = c["frontier"][h], c["edges"][h]
+        src = c["frontier"][h + 1] if h + 1 < K else c["rows"]
+        hop += f * 2 * off_bytes + e * 4 + e * 4 + f * 8 + (src - f) * 4
+    gather = c["rows"] * (rb + 8) + c["distinct_rows"] * rb
+    return {"sampling": hop, "gather": gather, "total": hop + gather}
+
+
+def gather_traffic_from_profile():
+    """Per-launch DRAM traffic of the gather kernel from the committed ncu
+    summary, if it was taken on the current gather source."""
+    path = os.path.join(ROOT, "profiles", "gather_rmat100m.md")
+    src = os.path.join(ROOT, "paper_2601_01473_gb300", "csrc", "gather.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        vals = {}
+        for line in open(path):
+            if ":" in line and line.strip().startswith("- "):
+                k, v = line.strip()[2:].split(":", 1)
+                vals[k.strip()] = v.strip()
+        if vals.get("gather.cu sha256[:16]") != sha:
+            return None
+        return float(vals["dram bytes per launch (full workload)"])
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------
+# oracle (CPU baseline / reference arm)
+# ----------------------------------------------------------------------------
+
+def time_oracle(host_graph, w, targets_cpu, seconds_budget: float, max_mbs: int):
+    """Runs the oracle (as it stands) on a sample of the workload's
+    minibatches on the host cores; returns (minibatches/s, cores, sample)."""
+    import concurrent.futures as cf
+
+    import oracle
+    og = oracle.Graph(*host_graph)
+    cores = max(1, min(os.cpu_count() or 1, max_mbs))
+    # calibrate on one minibatch, then size the sample to the budget
+    t0 = time.perf_counter()
+    oracle.sample_minibatch(og, targets_cpu[0], list(w.fanouts), w.seed, 0)
+    one = time.perf_counter() - t0
+    n = int(max(cores, min(max_mbs, (seconds_budget / max(one, 1e-3)) * cores)))
+    n = max(1, min(n, targets_cpu.shape[0] * 64))
+    rows = [targets_cpu[i % targets_cpu.shape[0]] for i in range(n)]
+
+    def run(i):
+        oracle.sample_minibatch(og, rows[i], list(w.fanouts), w.seed, i)
+        return i
+
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(max_workers=cores) as ex:
+        list(ex.map(run, range(n)))
+    dt = time.perf_counter() - t0
+    return n / dt, cores, f"{n} minibatches of the workload (B={w.B}, fanouts {list(w.fanouts)}) on {cores} threads, {dt:.1f} s"
+
+
+def host_copy(offsets, indices, features):
+    return (offsets.cpu().numpy(), indices.cpu().numpy(), features.cpu().numpy())
+
+
+# ----------------------------------------------------------------------------
+# main
+# ----------------------------------------------------------------------------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="agnes", choices=["agnes", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(WORKLOADS))
+    ap.add_argument("--H", type=int, default=None, help="override minibatches per hyperbatch")
+    ap.add_argument("--block", type=int, default=None, help="override block bytes")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+
+    world, rank, local = dist_env()
+    if args.warmup < 3:
+        args.warmup = 3
+    w = WORKLOADS[args.workload]
+    if args.H:
+        w = w.with_(H=args.H)
+    if args.block:
+        w = w.with_(adj_block_bytes=args.block, feat_block_bytes=args.block)
+
+    if args.impl == "reference":
+        return run_reference(args, w, world, rank)
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+
+    from paper_2601_01473_gb300 import Graph
+
+    t_gen = time.perf_counter()
+    offsets, indices, features = build_graph(w, dev)
+    pool = target_pool(w, dev)
+    n_steps = args.warmup + args.steps
+    # each rank draws its own hyperbatches (weak scaling: fixed work per GPU)
+    step_targets = [targets_for_step(w, pool, rank * 1000 + s) for s in range(n_steps)]
+    torch.cuda.synchronize()
+    gen_s = time.perf_counter() - t_gen
+    torch.cuda.empty_cache()
+
+    stream = torch.cuda.current_stream(dev)
+    g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes, device=local,
+              stream=stream)
+    info = g.info()
+    fan = list(w.fanouts)
+    K = len(fan)
+    gid = lambda s: (rank * 1000 + s) * w.H  # noqa: E731
+
+    # warm-up (also allocates the workspace)
+    for s in range(args.warmup):
+        g.prepare(step_targets[s], fan, w.seed, gid(s), stream)
+    torch.cuda.synchronize()
+
+    # timed: device-resident inputs, CUDA events on the launching stream; the
+    # library records per-phase events on the same stream (ring of 64)
+    g.set_profiling(True)
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    gpu_index = local
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")
+    if len(vis) > local and vis[local].strip().isdigit():
+        gpu_index = int(vis[local])
+    with ClockSampler(gpu_index) as clk:
+        ev0.record(stream)
+        for s in range(args.warmup, n_steps):
+            g.prepare(step_targets[s], fan, w.seed, gid(s), stream)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    phases = [g.phase_times(ago) for ago in range(min(args.steps, 64))]
+    g.set_profiling(False)
+    if pg:
+        t = torch.tensor([elapsed_ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    clocks = clk.summary()
+    gather_ms = [p[1 + 3 * K] for p in phases if len(p) > 1 + 3 * K]
+
+    # byte accounting: rerun the timed steps untimed to read their counters
+    counters = []
+    for s in range(args.warmup, n_steps):
+        g.prepare(step_targets[s], fan, w.seed, gid(s), stream)
+        counters.append(g.counters())
+    off_bytes = offsets.element_size()
+    algo = [algorithmic_bytes(c, off_bytes) for c in counters]
+    gather_bytes = statistics.mean(a["gather"] for a in algo)
+    total_bytes = statistics.mean(a["total"] for a in algo)
+    stats = g.stats()
+
+    # end to end through the C ABI: host (pinned) targets in, views out
+    e2e = None
+    if not args.no_e2e:
+        host_targets = [t.cpu().pin_memory() for t in step_targets]
+        for s in range(2):
+            g.prepare(host_targets[s], fan, w.seed, gid(s), stream)
+            for j in range(w.H):
+                g.sizes(j)
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for s in range(args.warmup, n_steps):
+            g.prepare(host_targets[s], fan, w.seed, gid(s), stream)
+            for j in range(w.H):
+                g.fetch(j)
+        torch.cuda.synchronize()
+        e2e_s = time.perf_counter() - t0
+        if pg:
+            t = torch.tensor([e2e_s], device=dev)
+            pg.all_reduce(t, op=pg.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        d2h = 4 * (1 + (K + 1) * w.H + K * w.H) + 8 * (K + 1)
+        e2e = {"value": world * w.H * args.steps / e2e_s, "unit": UNIT,
+               "h2d_bytes_per_step": w.H * w.B * 4, "d2h_bytes_per_step": d2h}
+
+    value = world * w.H * args.steps / (elapsed_ms / 1e3)
+    peak, peak_kind = measured_peak()
+    g_ms = statistics.mean(gather_ms) if gather_ms else None
+    achieved = gather_bytes / (g_ms / 1e3) / 1e9 if g_ms else None
+    roofline = {"bound": "hbm", "kernel": "gather_vec_kernel<16,4>",
+                "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak if achieved else None,
+                "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
+                if peak_kind == "measured" else "fallback 6.8 TB/s",
+                "traffic": gather_traffic_from_profile(),
+                "algorithmic_bytes_per_launch": gather_bytes,
+                "avg_launch_ms": g_ms,
+                "path_algorithmic_bytes_per_step": total_bytes,
+                "path_GBps": total_bytes / (elapsed_ms / args.steps / 1e3) / 1e9}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        host_graph = host_copy(offsets, indices, features)
+        tcpu = step_targets[args.warmup].cpu().numpy()
+        v, cores, sample = time_oracle(host_graph, w, tcpu, args.cpu_seconds, 256)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        mean_phases = [statistics.mean(p[i] for p in phases) for i in range(len(phases[0]))] \
+            if phases else []
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+            "data": "synthetic",
+            "config": {"workload": f"{w.name}: {w.describe()}",
+                       "graph": {"nodes": info["num_nodes"], "edges": info["num_edges"],
+                                 "adj_blocks": info["adj_blocks"], "tiles": info["tiles"],
+                                 "feat_blocks": info["feat_blocks"]},
+                       "H": w.H, "B": w.B, "fanouts": fan, "parallelism": f"replicas{world}",
+                       "l2": "inputs larger than L2 (graph ~%.0f GB vs 129 MB L2), no flush"
+                             % ((offsets.numel() * offsets.element_size()
+                                 + indices.numel() * 4
+                                 + features.numel() * features.element_size()) / 1e9),
+                       "blocks_touched_last_step": stats,
+                       "counters_last_step": counters[-1] if counters else None,
+                       "gen_seconds": round(gen_s, 1)},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": kernel_launches_per_step(K) * args.steps,
+            "clocks": clocks,
+            "phases_ms": {"names": ["bucket_targets"] + [f"hop{h + 1}_{p}" for h in range(K)
+                                                         for p in ("count_scan", "sample", "dedup")]
+                          + ["gather"], "mean": mean_phases},
+        }
+        print(json.dumps(out), flush=True)
+    g.close()
+    if pg:
+        pg.destroy_process_group()
+
+
+def run_reference(args, w, world, rank):
+    """The oracle as the reference arm: bounded sample on the host cores."""
+    if rank != 0:
+        return
+    t0 = time.perf_counter()
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    offsets, indices, features = build_graph(w, dev)
+    pool = target_pool(w, dev)
+    targets = targets_for_step(w, pool, 0)
+    host_graph = host_copy(offsets, indices, features)
+    del offsets, indices, features
+    tcpu = targets.cpu().numpy()
+    budget = max(5.0, min(60.0, 120.0 / max(1, args.steps)))
+    vals, cores, sample = [], 1, ""
+    for _ in range(args.warmup if args.warmup < 1 else 1):
+        time_oracle(host_graph, w, tcpu, 2.0, 8)
+    for _ in range(args.steps):
+        v, cores, sample = time_oracle(host_graph, w, tcpu, budget / 4, 64)
+        vals.append(v)
+    value = statistics.median(vals)
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "int32", "data": "synthetic", "impl": "reference",
+           "config": {"workload": f"{w.name}: {w.describe()}", "H": w.H, "B": w.B,
+                      "fanouts": list(w.fanouts)},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                            "sample": sample},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0},
+           "wall_s": round(time.perf_counter() - t0, 1)}
+    print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -188,13 +188,16 @@ agnes_status agnes_copy_adj_blocks(agnes_ctx* ctx, int32_t* start_node, int32_t*
                                    int64_t cap);
 
 /* Optional per-phase timing of later prepares with CUDA events on the
- * caller's stream (off by default).  agnes_phase_times writes up to n
- * milliseconds of the last prepare, in order: [0] bucketing of the targets,
- * then per hop h (3 each): [1+3h] count+scan, [2+3h] sampling,
- * [3+3h] dedup+relabel, then [1+3K] gather; returns the count written via
- * *n_out.  Waits like fetch. */
+ * caller's stream (off by default; the events of the last 64 prepares are
+ * kept).  agnes_phase_times writes up to n milliseconds of the prepare
+ * issued `ago` calls before the latest one (0 = the latest, < 64), in
+ * order: [0] bucketing of the targets, then per hop h (3 each): [1+3h]
+ * count+scan, [2+3h] sampling, [3+3h] dedup+relabel, then [1+3K] gather;
+ * *n_out receives the count (0 if that prepare was not profiled).  Waits
+ * for the latest prepare like fetch.  Errors: EINVAL (ago out of range). */
 agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable);
-agnes_status agnes_phase_times(agnes_ctx* ctx, float* ms, int32_t n, int32_t* n_out);
+agnes_status agnes_phase_times(agnes_ctx* ctx, int32_t ago, float* ms, int32_t n,
+                               int32_t* n_out);
 
 /* Releases everything the ctx owns (after synchronising its streams). */
 agnes_status agnes_free(agnes_ctx* ctx);

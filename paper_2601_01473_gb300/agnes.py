@@ -98,7 +98,8 @@ SIGNATURES = {
     "agnes_get_graph_info": ([_P, ctypes.POINTER(_GraphInfo)], ctypes.c_int),
     "agnes_copy_adj_blocks": ([_P, _P, _P, ctypes.c_int64], ctypes.c_int),
     "agnes_set_profiling": ([_P, ctypes.c_int32], ctypes.c_int),
-    "agnes_phase_times": ([_P, _P, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)], ctypes.c_int),
+    "agnes_phase_times": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)],
+                          ctypes.c_int),
     "agnes_free": ([_P], ctypes.c_int),
     "agnes_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "agnes_last_error": ([_P], ctypes.c_char_p),
@@ -293,8 +294,10 @@ class Graph:
     def set_profiling(self, enable: bool):
         _check(lib().agnes_set_profiling(self._ctx, int(enable)), self._ctx)
 
-    def phase_times(self) -> list:
+    def phase_times(self, ago: int = 0) -> list:
+        """Per-phase milliseconds of the prepare issued ``ago`` calls before
+        the latest (profiling must have been on for it)."""
         buf = (ctypes.c_float * (2 + 3 * MAX_HOPS))()
         n = ctypes.c_int32(0)
-        _check(lib().agnes_phase_times(self._ctx, buf, len(buf), ctypes.byref(n)), self._ctx)
+        _check(lib().agnes_phase_times(self._ctx, ago, buf, len(buf), ctypes.byref(n)), self._ctx)
         return list(buf[:n.value])

@@ -26,6 +26,7 @@ using namespace agnes;
 namespace {
 
 constexpr int kMaxPhases = 2 + 3 * AGNES_MAX_HOPS;
+constexpr int kEventRing = 64;  // prepares whose phase times stay readable
 
 struct Workspace {
   int32_t H = 0, B = 0, K = 0;
@@ -93,8 +94,9 @@ struct agnes_ctx {
   cudaEvent_t done = nullptr;
 
   bool profiling = false;
-  int n_phases = 0;
-  cudaEvent_t ev[kMaxPhases + 1] = {nullptr};
+  int64_t n_prepared = 0;                  // prepares issued so far
+  int n_phases[kEventRing] = {0};          // per ring slot; 0 = not profiled
+  cudaEvent_t ev[kEventRing][kMaxPhases + 1] = {{nullptr}};
   bool ev_created = false;
 
   char err[512] = {0};
@@ -369,7 +371,8 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (ctx->own_features) cudaFree(ctx->features);
   if (ctx->done) cudaEventDestroy(ctx->done);
   if (ctx->ev_created)
-    for (int i = 0; i <= kMaxPhases; ++i) cudaEventDestroy(ctx->ev[i]);
+    for (int r = 0; r < kEventRing; ++r)
+      for (int i = 0; i <= kMaxPhases; ++i) cudaEventDestroy(ctx->ev[r][i]);
   delete ctx;
   return AGNES_OK;
 }
@@ -584,12 +587,15 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   ctx->synced = false;
 
   if (ctx->profiling && !ctx->ev_created) {
-    for (int i = 0; i <= kMaxPhases; ++i) CK(ctx, cudaEventCreate(&ctx->ev[i]));
+    for (int r = 0; r < kEventRing; ++r)
+      for (int i = 0; i <= kMaxPhases; ++i) CK(ctx, cudaEventCreate(&ctx->ev[r][i]));
     ctx->ev_created = true;
   }
+  const int ring = (int)(ctx->n_prepared % kEventRing);
+  ctx->n_phases[ring] = 0;
   int ph = 0;
   auto mark = [&]() {
-    if (ctx->profiling) cudaEventRecord(ctx->ev[ph++], st);
+    if (ctx->profiling) cudaEventRecord(ctx->ev[ring][ph++], st);
   };
 
   mark();
@@ -678,7 +684,8 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   CK(ctx, cudaMemcpyAsync(b.ecnt, w.ecnt, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.stats, w.stats, sizeof(int64_t) * (K + 1), cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaEventRecord(ctx->done, st));
-  ctx->n_phases = ctx->profiling ? ph - 1 : 0;
+  ctx->n_phases[ring] = ctx->profiling ? ph - 1 : 0;
+  ctx->n_prepared += 1;
   ctx->cur = cur;
   ctx->prepared = true;
   return AGNES_OK;
@@ -790,18 +797,23 @@ agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable) {
   return AGNES_OK;
 }
 
-agnes_status agnes_phase_times(agnes_ctx* ctx, float* ms, int32_t n, int32_t* n_out) {
-  if (!ctx || (!ms && n > 0) || !n_out) {
+agnes_status agnes_phase_times(agnes_ctx* ctx, int32_t ago, float* ms, int32_t n,
+                               int32_t* n_out) {
+  if (!ctx || (!ms && n > 0) || !n_out || ago < 0 || ago >= kEventRing) {
     set_err(ctx, "invalid arguments");
     return AGNES_EINVAL;
   }
   *n_out = 0;
   agnes_status rc = wait_prepared(ctx);
   if (rc != AGNES_OK) return rc;
-  int cnt = ctx->n_phases < n ? ctx->n_phases : n;
-  for (int i = 0; i < cnt; ++i) {
-    CK(ctx, cudaEventElapsedTime(&ms[i], ctx->ev[i], ctx->ev[i + 1]));
+  if (ago >= ctx->n_prepared) {
+    set_err(ctx, "only %lld hyperbatches prepared", (long long)ctx->n_prepared);
+    return AGNES_EINVAL;
   }
+  const int ring = (int)((ctx->n_prepared - 1 - ago) % kEventRing);
+  const int cnt = ctx->n_phases[ring] < n ? ctx->n_phases[ring] : n;
+  for (int i = 0; i < cnt; ++i)
+    CK(ctx, cudaEventElapsedTime(&ms[i], ctx->ev[ring][i], ctx->ev[ring][i + 1]));
   *n_out = cnt;
   return AGNES_OK;
 }

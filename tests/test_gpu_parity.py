@@ -19,7 +19,7 @@ GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
 def _bytes(t: torch.Tensor) -> np.ndarray:
     t = t.detach().cpu().contiguous()
-    return t.view(torch.uint8).numpy() if t.numel() else np.zeros(0, np.uint8)
+    return t.view(torch.uint8).numpy().reshape(-1) if t.numel() else np.zeros(0, np.uint8)
 
 
 def compare(g: Graph, og: oracle.Graph, targets: np.ndarray, fanouts, seed, gid0, adj_bb, feat_bb,
