@@ -117,6 +117,87 @@ __device__ __forceinline__ void mark_cell(const CellArgs& a, uint32_t* D, uint32
   __syncwarp();
 }
 
+// A cell (t, j): its frontier entries [fo, fo+fn) and sampled entries
+// [so, so+sn).
+struct Cell {
+  int32_t fo, fn, so, sn, t, j;
+};
+
+// Loads the cell of this lane (one cell per lane, 32 consecutive cells per
+// warp); returns false past the last cell.
+__device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell* c) {
+  if (cell >= a.ncells) {
+    *c = Cell{0, 0, 0, 0, 0, 0};
+    return false;
+  }
+  c->fo = a.fcell_off[cell];
+  c->fn = a.fcell_off[cell + 1] - c->fo;
+  c->so = a.soff[cell];
+  c->sn = a.soff[cell + 1] - c->so;
+  c->t = (int32_t)(cell / a.H);
+  c->j = (int32_t)(cell - (int64_t)c->t * a.H);
+  return true;
+}
+
+__device__ __forceinline__ Cell bcast(const Cell& c, int k) {
+  Cell o;
+  o.fo = __shfl_sync(0xffffffffu, c.fo, k);
+  o.fn = __shfl_sync(0xffffffffu, c.fn, k);
+  o.so = __shfl_sync(0xffffffffu, c.so, k);
+  o.sn = __shfl_sync(0xffffffffu, c.sn, k);
+  o.t = __shfl_sync(0xffffffffu, c.t, k);
+  o.j = __shfl_sync(0xffffffffu, c.j, k);
+  return o;
+}
+
+// Small cells (fn + sn <= 32): one entry per lane; equal ids are found with
+// match_any, ranks by comparing against every other lane's id.
+struct SmallCell {
+  int32_t id;
+  int32_t extra;     // frontier: output row g; sampled: edge index e
+  bool act, isF, inD, leader;
+  unsigned fmask, peers, lmask;
+};
+
+__device__ __forceinline__ SmallCell small_cell(const CellArgs& a, const Cell& c) {
+  SmallCell s;
+  const int lane = lane_id();
+  const int n = c.fn + c.sn;
+  s.act = lane < n;
+  s.isF = lane < c.fn;
+  s.id = 0x7fffffff;
+  s.extra = 0;
+  if (s.act) {
+    if (s.isF) {
+      s.id = a.fb_id[c.fo + lane];
+      s.extra = a.fb_pos[c.fo + lane];
+    } else {
+      s.id = a.sb_u[c.so + lane - c.fn];
+      s.extra = a.sb_e[c.so + lane - c.fn];
+    }
+  }
+  const unsigned amask = n >= 32 ? 0xffffffffu : ((1u << n) - 1u);
+  s.fmask = c.fn >= 32 ? 0xffffffffu : ((1u << c.fn) - 1u);
+  s.peers = __match_any_sync(0xffffffffu, s.id) & amask;
+  s.inD = (s.peers & s.fmask) != 0;
+  s.leader = s.act && !s.isF && !s.inD && lane == __ffs(s.peers) - 1;
+  s.lmask = __ballot_sync(0xffffffffu, s.leader);
+  return s;
+}
+
+// Cells with more than 32 entries: bitmaps over the tile.
+__device__ __forceinline__ int32_t big_count(const CellArgs& a, const Cell& c, uint32_t* D,
+                                             uint32_t* S) {
+  const int32_t base = a.tm.tile_first[c.t];
+  const int32_t words = (a.tm.tile_first[c.t + 1] - base + 31) >> 5;
+  mark_cell(a, D, S, base, words, c.fo, c.fn, c.so, c.sn);
+  int32_t cnt = 0;
+  for (int w = lane_id(); w < words; w += 32) cnt += __popc(S[w] & ~D[w]);
+  cnt = warp_sum(cnt);
+  __syncwarp();
+  return cnt;
+}
+
 __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
   if (failed(a.status)) return;
   __shared__ uint32_t D_s[kWarps][kTileWords];
@@ -124,27 +205,132 @@ __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
   const int warp = threadIdx.x >> 5, lane = lane_id();
   uint32_t* D = D_s[warp];
   uint32_t* S = S_s[warp];
+  const int64_t nchunks = (a.ncells + 31) / 32;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  for (int64_t cell = blockIdx.x * (int64_t)kWarps + warp; cell < a.ncells; cell += nwarps) {
-    const int32_t t = (int32_t)(cell / a.H);
-    const int32_t j = (int32_t)(cell - (int64_t)t * a.H);
-    const int32_t fo = a.fcell_off[cell], fn = a.fcell_off[cell + 1] - fo;
-    const int32_t so = a.soff[cell], sn = a.soff[cell + 1] - so;
-    int32_t cnt = 0;
-    if (sn > 0) {
-      const int32_t base = a.tm.tile_first[t];
-      const int32_t words = (a.tm.tile_first[t + 1] - base + 31) >> 5;
-      mark_cell(a, D, S, base, words, fo, fn, so, sn);
-      for (int w = lane; w < words; w += 32) cnt += __popc(S[w] & ~D[w]);
-      cnt = warp_sum(cnt);
-      __syncwarp();
+  for (int64_t ch = blockIdx.x * (int64_t)kWarps + warp; ch < nchunks; ch += nwarps) {
+    const int64_t my_cell = ch * 32 + lane;
+    Cell mine;
+    const bool valid = load_cell(a, my_cell, &mine);
+    int32_t my_cnt = 0;
+    unsigned todo = __ballot_sync(0xffffffffu, valid && mine.sn > 0);
+    while (todo) {
+      const int k = __ffs(todo) - 1;
+      todo &= todo - 1u;
+      const Cell c = bcast(mine, k);
+      int32_t cnt;
+      if (c.fn + c.sn <= 32)
+        cnt = __popc(small_cell(a, c).lmask);
+      else
+        cnt = big_count(a, c, D, S);
+      if (lane == k) my_cnt = cnt;
     }
-    if (lane == 0) {
-      a.newcnt[(int64_t)j * a.tm.T + t] = cnt;
-      a.nfcnt[cell] = fn + cnt;
-      if (fn > 0) a.adj_flags[a.tile_adj_block[t]] = 1;
+    if (valid) {
+      a.newcnt[(int64_t)mine.j * a.tm.T + mine.t] = my_cnt;
+      a.nfcnt[my_cell] = mine.fn + my_cnt;
+      if (mine.fn > 0) a.adj_flags[a.tile_adj_block[mine.t]] = 1;
     }
   }
+}
+
+__device__ __forceinline__ void small_emit(const CellArgs& a, const Cell& c, int32_t nb,
+                                           int32_t nfo) {
+  const SmallCell s = small_cell(a, c);
+  const int n = c.fn + c.sn;
+  int32_t lessF = 0, lessN = 0;
+  for (int k = 0; k < n; ++k) {
+    const int32_t idk = __shfl_sync(0xffffffffu, s.id, k);
+    if (idk < s.id) {
+      lessF += (s.fmask >> k) & 1u;
+      lessN += (s.lmask >> k) & 1u;
+    }
+  }
+  const int lane = lane_id();
+  const int src = s.inD ? __ffs(s.peers & s.fmask) - 1 : lane;
+  const int32_t fpos = __shfl_sync(0xffffffffu, s.extra, src);
+  const int64_t jcap = (int64_t)c.j * a.capK;
+  if (s.act && !s.isF)
+    a.col[(int64_t)c.j * a.ecap + s.extra] = s.inD ? (int32_t)(fpos - jcap) : nb + lessN;
+  if (s.act && (s.isF || s.leader)) {
+    const int32_t r = nfo + lessF + lessN;
+    int32_t g = s.extra;
+    if (s.leader) {
+      g = (int32_t)(jcap + nb + lessN);
+      a.nodes[g] = s.id;
+    }
+    a.nfb_id[r] = s.id;
+    a.nfb_pos[r] = g;
+  }
+}
+
+__device__ __forceinline__ void big_emit(const CellArgs& a, const Cell& c, int32_t nb, int32_t nfo,
+                                         uint32_t* D, uint32_t* Nw, int32_t* pD, int32_t* pN) {
+  const int lane = lane_id();
+  const int32_t base = a.tm.tile_first[c.t];
+  const int32_t words = (a.tm.tile_first[c.t + 1] - base + 31) >> 5;
+  mark_cell(a, D, Nw, base, words, c.fo, c.fn, c.so, c.sn);
+  // new = S & ~D; per-word exclusive ranks of D and new
+  uint32_t dw[4], nw[4];
+  int32_t sd = 0, sn_ = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int w = lane * 4 + q;
+    dw[q] = w < words ? D[w] : 0u;
+    nw[q] = w < words ? (Nw[w] & ~dw[q]) : 0u;
+    sd += __popc(dw[q]);
+    sn_ += __popc(nw[q]);
+  }
+  int32_t rd = warp_incl_scan(sd) - sd;
+  int32_t rn = warp_incl_scan(sn_) - sn_;
+  __syncwarp();
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int w = lane * 4 + q;
+    Nw[w] = nw[q];
+    pD[w] = rd;
+    pN[w] = rn;
+    rd += __popc(dw[q]);
+    rn += __popc(nw[q]);
+  }
+  __syncwarp();
+
+  const int64_t jcap = (int64_t)c.j * a.capK;
+  int32_t* col = a.col + (int64_t)c.j * a.ecap;
+  for (int32_t i = lane; i < c.sn; i += 32) {
+    const int32_t lu = a.sb_u[c.so + i] - base;
+    const int32_t w = lu >> 5;
+    const uint32_t bit = 1u << (lu & 31), below = bit - 1u;
+    int32_t cv;
+    if (D[w] & bit)
+      cv = (int32_t)(a.fb_pos[c.fo + pD[w] + __popc(D[w] & below)] - jcap);
+    else
+      cv = nb + pN[w] + __popc(Nw[w] & below);
+    col[a.sb_e[c.so + i]] = cv;
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int w = lane * 4 + q;
+    if (w >= words) break;
+    const uint32_t d = dw[q], n = nw[q];
+    uint32_t rest = d | n;
+    const int32_t r0 = pD[w] + pN[w];
+    while (rest) {
+      const int b = __ffs(rest) - 1;
+      rest &= rest - 1u;
+      const uint32_t below = (1u << b) - 1u;
+      const int32_t id = base + w * 32 + b;
+      const int32_t r = r0 + __popc((d | n) & below);
+      int32_t g;
+      if ((d >> b) & 1u) {
+        g = a.fb_pos[c.fo + pD[w] + __popc(d & below)];
+      } else {
+        g = (int32_t)(jcap + nb + pN[w] + __popc(n & below));
+        a.nodes[g] = id;
+      }
+      a.nfb_id[nfo + r] = id;
+      a.nfb_pos[nfo + r] = g;
+    }
+  }
+  __syncwarp();
 }
 
 __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
@@ -154,94 +340,35 @@ __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
   __shared__ int32_t pD_s[kWarps][kTileWords];
   __shared__ int32_t pN_s[kWarps][kTileWords];
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  uint32_t* D = D_s[warp];
-  uint32_t* Nw = N_s[warp];
-  int32_t* pD = pD_s[warp];
-  int32_t* pN = pN_s[warp];
+  const int64_t nchunks = (a.ncells + 31) / 32;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  for (int64_t cell = blockIdx.x * (int64_t)kWarps + warp; cell < a.ncells; cell += nwarps) {
-    const int32_t fo = a.fcell_off[cell], fn = a.fcell_off[cell + 1] - fo;
-    const int32_t so = a.soff[cell], sn = a.soff[cell + 1] - so;
-    if (fn + sn == 0) continue;
-    const int32_t nfo = a.nfcell_off[cell];
-    if (sn == 0) {  // nothing sampled here: the frontier cell carries over unchanged
-      for (int32_t i = lane; i < fn; i += 32) {
-        a.nfb_id[nfo + i] = a.fb_id[fo + i];
-        a.nfb_pos[nfo + i] = a.fb_pos[fo + i];
-      }
-      continue;
+  for (int64_t ch = blockIdx.x * (int64_t)kWarps + warp; ch < nchunks; ch += nwarps) {
+    const int64_t my_cell = ch * 32 + lane;
+    Cell mine;
+    const bool valid = load_cell(a, my_cell, &mine);
+    int32_t my_nfo = 0, my_nb = 0;
+    if (valid && mine.fn + mine.sn > 0) {
+      my_nfo = a.nfcell_off[my_cell];
+      if (mine.sn > 0) my_nb = a.nsz_prev[mine.j] + a.newbase[(int64_t)mine.j * a.tm.T + mine.t];
     }
-    const int32_t t = (int32_t)(cell / a.H);
-    const int32_t j = (int32_t)(cell - (int64_t)t * a.H);
-    const int32_t base = a.tm.tile_first[t];
-    const int32_t words = (a.tm.tile_first[t + 1] - base + 31) >> 5;
-    mark_cell(a, D, Nw, base, words, fo, fn, so, sn);
-
-    // new = S & ~D; per-word exclusive ranks of D and new
-    uint32_t dw[4], nw[4];
-    int32_t sd = 0, sn_ = 0;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int w = lane * 4 + q;
-      dw[q] = w < words ? D[w] : 0u;
-      nw[q] = w < words ? (Nw[w] & ~dw[q]) : 0u;
-      sd += __popc(dw[q]);
-      sn_ += __popc(nw[q]);
-    }
-    int32_t rd = warp_incl_scan(sd) - sd;
-    int32_t rn = warp_incl_scan(sn_) - sn_;
-    __syncwarp();
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int w = lane * 4 + q;
-      Nw[w] = nw[q];
-      pD[w] = rd;
-      pN[w] = rn;
-      rd += __popc(dw[q]);
-      rn += __popc(nw[q]);
-    }
-    __syncwarp();
-
-    const int64_t jcap = (int64_t)j * a.capK;
-    const int32_t nb = a.nsz_prev[j] + a.newbase[(int64_t)j * a.tm.T + t];
-    int32_t* col = a.col + (int64_t)j * a.ecap;
-    for (int32_t i = lane; i < sn; i += 32) {
-      const int32_t lu = a.sb_u[so + i] - base;
-      const int32_t w = lu >> 5;
-      const uint32_t bit = 1u << (lu & 31), below = bit - 1u;
-      int32_t c;
-      if (D[w] & bit)
-        c = (int32_t)(a.fb_pos[fo + pD[w] + __popc(D[w] & below)] - jcap);
-      else
-        c = nb + pN[w] + __popc(Nw[w] & below);
-      col[a.sb_e[so + i]] = c;
-    }
-
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int w = lane * 4 + q;
-      if (w >= words) break;
-      const uint32_t d = dw[q], n = nw[q];
-      uint32_t rest = d | n;
-      const int32_t r0 = pD[w] + pN[w];
-      while (rest) {
-        const int b = __ffs(rest) - 1;
-        rest &= rest - 1u;
-        const uint32_t below = (1u << b) - 1u;
-        const int32_t id = base + w * 32 + b;
-        const int32_t r = r0 + __popc((d | n) & below);
-        int32_t g;
-        if ((d >> b) & 1u) {
-          g = a.fb_pos[fo + pD[w] + __popc(d & below)];
-        } else {
-          g = (int32_t)(jcap + nb + pN[w] + __popc(n & below));
-          a.nodes[g] = id;
+    unsigned todo = __ballot_sync(0xffffffffu, valid && mine.fn + mine.sn > 0);
+    while (todo) {
+      const int k = __ffs(todo) - 1;
+      todo &= todo - 1u;
+      const Cell c = bcast(mine, k);
+      const int32_t nfo = __shfl_sync(0xffffffffu, my_nfo, k);
+      const int32_t nb = __shfl_sync(0xffffffffu, my_nb, k);
+      if (c.sn == 0) {  // nothing sampled here: the frontier cell carries over unchanged
+        for (int32_t i = lane; i < c.fn; i += 32) {
+          a.nfb_id[nfo + i] = a.fb_id[c.fo + i];
+          a.nfb_pos[nfo + i] = a.fb_pos[c.fo + i];
         }
-        a.nfb_id[nfo + r] = id;
-        a.nfb_pos[nfo + r] = g;
+      } else if (c.fn + c.sn <= 32) {
+        small_emit(a, c, nb, nfo);
+      } else {
+        big_emit(a, c, nb, nfo, D_s[warp], N_s[warp], pD_s[warp], pN_s[warp]);
       }
     }
-    __syncwarp();
   }
 }
 

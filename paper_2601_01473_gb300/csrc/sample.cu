@@ -79,8 +79,10 @@ targets_scatter_kernel(const int32_t* __restrict__ nodes, int64_t capK, int32_t 
   }
 }
 
-// One warp per cell: orders the cell's targets by id (rank in the cell's
-// membership bitmap) and flags a target repeated within a minibatch.
+// Orders each cell's targets by id and flags a target repeated within a
+// minibatch.  A warp scans 32 consecutive cells and skips empty ones; a cell
+// of at most 32 targets is ranked in registers (each lane counts the smaller
+// ids), a bigger one by popcount ranks in a bitmap over its tile.
 __global__ void __launch_bounds__(kThreads)
 targets_sort_kernel(const int32_t* __restrict__ fcell_off, int64_t ncells, int32_t H, TileMap tm,
                     const int32_t* __restrict__ tmp_id, const int32_t* __restrict__ tmp_pos,
@@ -91,45 +93,71 @@ targets_sort_kernel(const int32_t* __restrict__ fcell_off, int64_t ncells, int32
   const int warp = threadIdx.x >> 5, lane = lane_id();
   uint32_t* bits = bits_s[warp];
   int32_t* pref = pref_s[warp];
+  const int64_t nchunks = (ncells + 31) / 32;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  for (int64_t cell = blockIdx.x * (int64_t)kWarps + warp; cell < ncells; cell += nwarps) {
-    const int32_t o = fcell_off[cell];
-    const int32_t n = fcell_off[cell + 1] - o;
-    if (n == 0) continue;
-    const int32_t t = (int32_t)(cell / H);
-    const int32_t base = tm.tile_first[t];
-    const int32_t words = (tm.tile_first[t + 1] - base + 31) >> 5;
-    for (int w = lane; w < words; w += 32) bits[w] = 0;
-    __syncwarp();
-    for (int32_t i = lane; i < n; i += 32) {
-      const int32_t lu = tmp_id[o + i] - base;
-      const uint32_t bit = 1u << (lu & 31);
-      if (atomicOr(&bits[lu >> 5], bit) & bit) atomicOr(status, kErrTargetDup);
+  for (int64_t ch = blockIdx.x * (int64_t)kWarps + warp; ch < nchunks; ch += nwarps) {
+    const int64_t my_cell = ch * 32 + lane;
+    int32_t my_o = 0, my_n = 0;
+    if (my_cell < ncells) {
+      my_o = fcell_off[my_cell];
+      my_n = fcell_off[my_cell + 1] - my_o;
     }
-    __syncwarp();
-    int32_t c[4], sum = 0;
+    unsigned todo = __ballot_sync(0xffffffffu, my_n > 0);
+    while (todo) {
+      const int k = __ffs(todo) - 1;
+      todo &= todo - 1u;
+      const int32_t o = __shfl_sync(0xffffffffu, my_o, k);
+      const int32_t n = __shfl_sync(0xffffffffu, my_n, k);
+      if (n <= 32) {
+        const bool act = lane < n;
+        const int32_t v = act ? tmp_id[o + lane] : 0x7fffffff;
+        const int32_t p = act ? tmp_pos[o + lane] : 0;
+        const unsigned amask = n >= 32 ? 0xffffffffu : ((1u << n) - 1u);
+        const unsigned peers = __match_any_sync(0xffffffffu, v);  // every lane takes part
+        if (act && __popc(peers & amask) > 1) atomicOr(status, kErrTargetDup);
+        int32_t r = 0;
+        for (int q = 0; q < n; ++q) r += __shfl_sync(0xffffffffu, v, q) < v;
+        if (act) {
+          fb_id[o + r] = v;
+          fb_pos[o + r] = p;
+        }
+        continue;
+      }
+      const int32_t t = (int32_t)((ch * 32 + k) / H);
+      const int32_t base = tm.tile_first[t];
+      const int32_t words = (tm.tile_first[t + 1] - base + 31) >> 5;
+      for (int w = lane; w < words; w += 32) bits[w] = 0;
+      __syncwarp();
+      for (int32_t i = lane; i < n; i += 32) {
+        const int32_t lu = tmp_id[o + i] - base;
+        const uint32_t bit = 1u << (lu & 31);
+        if (atomicOr(&bits[lu >> 5], bit) & bit) atomicOr(status, kErrTargetDup);
+      }
+      __syncwarp();
+      int32_t c[4], sum = 0;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int w = lane * 4 + q;
-      c[q] = w < words ? __popc(bits[w]) : 0;
-      sum += c[q];
-    }
-    int32_t run = warp_incl_scan(sum) - sum;
+      for (int q = 0; q < 4; ++q) {
+        const int w = lane * 4 + q;
+        c[q] = w < words ? __popc(bits[w]) : 0;
+        sum += c[q];
+      }
+      int32_t run = warp_incl_scan(sum) - sum;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      pref[lane * 4 + q] = run;
-      run += c[q];
+      for (int q = 0; q < 4; ++q) {
+        pref[lane * 4 + q] = run;
+        run += c[q];
+      }
+      __syncwarp();
+      for (int32_t i = lane; i < n; i += 32) {
+        const int32_t v = tmp_id[o + i];
+        const int32_t lu = v - base;
+        const int32_t w = lu >> 5;
+        const int32_t r = pref[w] + __popc(bits[w] & ((1u << (lu & 31)) - 1u));
+        fb_id[o + r] = v;
+        fb_pos[o + r] = tmp_pos[o + i];
+      }
+      __syncwarp();
     }
-    __syncwarp();
-    for (int32_t i = lane; i < n; i += 32) {
-      const int32_t v = tmp_id[o + i];
-      const int32_t lu = v - base;
-      const int32_t w = lu >> 5;
-      const int32_t r = pref[w] + __popc(bits[w] & ((1u << (lu & 31)) - 1u));
-      fb_id[o + r] = v;
-      fb_pos[o + r] = tmp_pos[o + i];
-    }
-    __syncwarp();
   }
 }
 
