@@ -51,7 +51,8 @@ struct Workspace {
   int64_t* indptr[AGNES_MAX_HOPS] = {nullptr};
   int32_t* col[AGNES_MAX_HOPS] = {nullptr};
   int32_t* nbr = nullptr;
-  int32_t* stile = nullptr;
+  int32_t* scell = nullptr;
+  int32_t* srank = nullptr;
   int32_t* sb_u = nullptr;
   int32_t* sb_e = nullptr;
   int32_t* cnt = nullptr;
@@ -167,7 +168,8 @@ static void free_workspace(Workspace* w) {
     cudaFree(w->col[h]);
   }
   cudaFree(w->nbr);
-  cudaFree(w->stile);
+  cudaFree(w->scell);
+  cudaFree(w->srank);
   cudaFree(w->sb_u);
   cudaFree(w->sb_e);
   cudaFree(w->cnt);
@@ -252,7 +254,8 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
     WA(w.col[h], (int64_t)H * cap[h] * fan[h]);
   }
   WA(w.nbr, edges);
-  WA(w.stile, edges);
+  WA(w.scell, edges);
+  WA(w.srank, edges);
   WA(w.sb_u, edges > rows ? edges : rows);
   WA(w.sb_e, edges > rows ? edges : rows);
   WA(w.cnt, (int64_t)H * w.cap_prev_max);
@@ -601,7 +604,6 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   mark();
   CK(ctx, cudaMemsetAsync(w.status, 0, sizeof(int32_t), st));
   CK(ctx, cudaMemsetAsync(w.fcnt, 0, sizeof(int32_t) * cells, st));
-  CK(ctx, cudaMemsetAsync(w.scnt, 0, sizeof(int32_t) * cells, st));
   CK(ctx, cudaMemsetAsync(w.adj_flags, 0, (size_t)K * ctx->bt.n_blocks, st));
   CK(ctx, cudaMemsetAsync(w.feat_flags, 0, (size_t)ctx->bt.n_feat_blocks, st));
   CK(ctx, cudaMemsetAsync(w.stats, 0, sizeof(int64_t) * (K + 1), st));
@@ -638,13 +640,15 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     CK(ctx, (seg_scan<int32_t, int64_t>(w.cnt, cap[h], w.indptr[h], cap[h] + 1, nsz_prev, 0, H,
                                          cap[h], true, ecnt, w.scan_scratch, w.status, st)));
     mark();
+    CK(ctx, cudaMemsetAsync(w.scnt, 0, sizeof(int32_t) * cells, st));
     CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h],
-                               w.nbr, nsm, st));
+                               w.nbr, w.scnt, w.scell, w.srank, nsm, st));
     mark();
     DedupBufs d;
     d.nbr = w.nbr;
     d.ecnt = ecnt;
-    d.stile = w.stile;
+    d.scell = w.scell;
+    d.srank = w.srank;
     d.scnt = w.scnt;
     d.soff = w.soff;
     d.sb_u = w.sb_u;

@@ -84,6 +84,19 @@ __device__ __forceinline__ int32_t warp_agg_take(int32_t* counters, int64_t idx,
   return old - 1 - __popc(peers & ((1u << lane) - 1u));
 }
 
+// Adds one per active lane to counters[idx] (one atomic per distinct idx) and
+// returns this lane's rank among all additions to idx: the counter's value
+// before it plus its rank among the warp's peers.
+__device__ __forceinline__ int32_t warp_agg_add(int32_t* counters, int64_t idx, unsigned mask) {
+  const unsigned peers = __match_any_sync(mask, (unsigned long long)idx);
+  const int leader = __ffs(peers) - 1;
+  const int lane = lane_id();
+  int32_t old = 0;
+  if (lane == leader) old = atomicAdd(counters + idx, __popc(peers));
+  old = __shfl_sync(peers, old, leader);
+  return old + __popc(peers & ((1u << lane) - 1u));
+}
+
 template <typename T>
 __device__ __forceinline__ T warp_incl_scan(T x) {
 #pragma unroll

@@ -21,53 +21,23 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 
-__global__ void __launch_bounds__(kThreads)
-dedup_hist_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict__ ecnt, int64_t ecap,
-                  int32_t H, TileMap tm, int32_t* __restrict__ stile, int32_t* __restrict__ scnt,
-                  const int32_t* status) {
-  if (failed(status)) return;
-  const int32_t j = blockIdx.y;
-  const int64_t E = ecnt[j];
-  const int32_t* src = nbr + j * ecap;
-  int32_t* til = stile + j * ecap;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; e0 < E;
-       e0 += stride) {
-    const int64_t e = e0 + lane_id();
-    const bool active = e < E;
-    int64_t cell = 0;
-    if (active) {
-      const int32_t t = tile_of(tm, src[e]);
-      til[e] = t;
-      cell = (int64_t)t * H + j;
-    }
-    warp_agg_inc(scnt, cell, active);
-  }
-}
-
+// Places every sampled edge of minibatch j at soff[cell] + rank (cell and
+// rank were recorded while sampling), building the sampled bucket.
 __global__ void __launch_bounds__(kThreads)
 dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict__ ecnt,
-                     int64_t ecap, int32_t H, const int32_t* __restrict__ stile,
-                     int32_t* __restrict__ scnt, const int32_t* __restrict__ soff,
+                     int64_t ecap, const int32_t* __restrict__ scell,
+                     const int32_t* __restrict__ srank, const int32_t* __restrict__ soff,
                      int32_t* __restrict__ sb_u, int32_t* __restrict__ sb_e,
                      const int32_t* status) {
   if (failed(status)) return;
   const int32_t j = blockIdx.y;
   const int64_t E = ecnt[j];
-  const int32_t* src = nbr + j * ecap;
-  const int32_t* til = stile + j * ecap;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; e0 < E;
-       e0 += stride) {
-    const int64_t e = e0 + lane_id();
-    const bool active = e < E;
-    const unsigned mask = __ballot_sync(0xffffffffu, active);
-    if (active) {
-      const int64_t cell = (int64_t)til[e] * H + j;
-      const int32_t slot = soff[cell] + warp_agg_take(scnt, cell, mask);
-      sb_u[slot] = src[e];
-      sb_e[slot] = (int32_t)e;
-    }
+  const int64_t o = (int64_t)j * ecap;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < E;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t slot = soff[scell[o + e]] + srank[o + e];
+    sb_u[slot] = nbr[o + e];
+    sb_e[slot] = (int32_t)e;
   }
 }
 
@@ -150,39 +120,82 @@ __device__ __forceinline__ Cell bcast(const Cell& c, int k) {
   return o;
 }
 
-// Small cells (fn + sn <= 32): one entry per lane; equal ids are found with
-// match_any, ranks by comparing against every other lane's id.
-struct SmallCell {
-  int32_t id;
-  int32_t extra;     // frontier: output row g; sampled: edge index e
-  bool act, isF, inD, leader;
-  unsigned fmask, peers, lmask;
+// Small cells (at most 32 entries) are packed several to a warp pass: the
+// cells of the pass take consecutive lanes (cell r owns lanes
+// [start_r, start_r + n_r)), one entry per lane, frontier entries first.
+// Equal ids of one cell are found with match_any on (r, id); ranks are
+// counted against the other lanes of the same cell.
+struct Pass {
+  unsigned cells;  // lanes (of the 32-cell chunk) whose cell is in this pass
+  int used;        // entry lanes used
 };
 
-__device__ __forceinline__ SmallCell small_cell(const CellArgs& a, const Cell& c) {
-  SmallCell s;
+struct Slot {
+  bool act, isF, inD, leader;
+  int r, cl;        // rank of the slot's cell in the pass, lane owning it
+  int32_t id;
+  int32_t extra;    // frontier: output row; sampled: edge index
+  unsigned long long key;
+  unsigned peers, fm, lm;
+  Cell c;
+};
+
+// Chooses the next pass among the remaining small cells (in lane order, as
+// many as fit in 32 lanes); returns this lane's first entry lane in *start.
+__device__ __forceinline__ Pass next_pass(unsigned* remaining, int n, int* start) {
   const int lane = lane_id();
-  const int n = c.fn + c.sn;
-  s.act = lane < n;
-  s.isF = lane < c.fn;
-  s.id = 0x7fffffff;
+  const bool rem = (*remaining >> lane) & 1u;
+  const int mine = rem ? n : 0;
+  const int incl = warp_incl_scan(mine);
+  const bool fits = rem && incl <= 32;
+  Pass p;
+  p.cells = __ballot_sync(0xffffffffu, fits);
+  p.used = __shfl_sync(0xffffffffu, incl, 31 - __clz(p.cells));
+  *remaining &= ~p.cells;
+  *start = incl - mine;
+  return p;
+}
+
+__device__ __forceinline__ Slot load_slot(const CellArgs& a, const Pass& p, const Cell& mine,
+                                          int start, int* cell_lane) {
+  const int lane = lane_id();
+  const bool in_pass = (p.cells >> lane) & 1u;
+  if (in_pass) cell_lane[__popc(p.cells & ((1u << lane) - 1u))] = lane;
+  __syncwarp();
+  const unsigned starts = __reduce_or_sync(0xffffffffu, in_pass ? (1u << start) : 0u);
+  Slot s;
+  s.act = lane < p.used;
+  s.r = s.act ? __popc(starts & ((2u << lane) - 1u)) - 1 : 0;
+  s.cl = s.act ? cell_lane[s.r] : 0;
+  __syncwarp();
+  s.c = bcast(mine, s.cl);
+  const int st = __shfl_sync(0xffffffffu, start, s.cl);
+  const int q = lane - st;
+  s.isF = s.act && q < s.c.fn;
+  s.id = 0;
   s.extra = 0;
   if (s.act) {
     if (s.isF) {
-      s.id = a.fb_id[c.fo + lane];
-      s.extra = a.fb_pos[c.fo + lane];
+      s.id = a.fb_id[s.c.fo + q];
+      s.extra = a.fb_pos[s.c.fo + q];
     } else {
-      s.id = a.sb_u[c.so + lane - c.fn];
-      s.extra = a.sb_e[c.so + lane - c.fn];
+      s.id = a.sb_u[s.c.so + q - s.c.fn];
+      s.extra = a.sb_e[s.c.so + q - s.c.fn];
     }
   }
-  const unsigned amask = n >= 32 ? 0xffffffffu : ((1u << n) - 1u);
-  s.fmask = c.fn >= 32 ? 0xffffffffu : ((1u << c.fn) - 1u);
-  s.peers = __match_any_sync(0xffffffffu, s.id) & amask;
-  s.inD = (s.peers & s.fmask) != 0;
+  s.key = s.act ? (((unsigned long long)s.r << 32) | (uint32_t)s.id)
+                : (0xffffffff00000000ull | (unsigned)lane);
+  s.peers = __match_any_sync(0xffffffffu, s.key);
+  s.fm = __ballot_sync(0xffffffffu, s.isF);
+  s.inD = (s.peers & s.fm) != 0;
   s.leader = s.act && !s.isF && !s.inD && lane == __ffs(s.peers) - 1;
-  s.lmask = __ballot_sync(0xffffffffu, s.leader);
+  s.lm = __ballot_sync(0xffffffffu, s.leader);
   return s;
+}
+
+// Lanes [start, start + n) as a mask (n <= 32).
+__device__ __forceinline__ unsigned lane_range(int start, int n) {
+  return n >= 32 ? 0xffffffffu : (((1u << n) - 1u) << start);
 }
 
 // Cells with more than 32 entries: bitmaps over the tile.
@@ -207,22 +220,28 @@ __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
   uint32_t* S = S_s[warp];
   const int64_t nchunks = (a.ncells + 31) / 32;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  __shared__ int cell_lane_s[kWarps][32];
   for (int64_t ch = blockIdx.x * (int64_t)kWarps + warp; ch < nchunks; ch += nwarps) {
     const int64_t my_cell = ch * 32 + lane;
     Cell mine;
     const bool valid = load_cell(a, my_cell, &mine);
+    const int n = mine.fn + mine.sn;
     int32_t my_cnt = 0;
-    unsigned todo = __ballot_sync(0xffffffffu, valid && mine.sn > 0);
+    // cells with more than 32 entries, one at a time, on bitmaps
+    unsigned todo = __ballot_sync(0xffffffffu, valid && mine.sn > 0 && n > 32);
     while (todo) {
       const int k = __ffs(todo) - 1;
       todo &= todo - 1u;
-      const Cell c = bcast(mine, k);
-      int32_t cnt;
-      if (c.fn + c.sn <= 32)
-        cnt = __popc(small_cell(a, c).lmask);
-      else
-        cnt = big_count(a, c, D, S);
+      const int32_t cnt = big_count(a, bcast(mine, k), D, S);
       if (lane == k) my_cnt = cnt;
+    }
+    // small cells, packed
+    unsigned remaining = __ballot_sync(0xffffffffu, valid && mine.sn > 0 && n <= 32);
+    while (remaining) {
+      int start;
+      const Pass p = next_pass(&remaining, n, &start);
+      const Slot sl = load_slot(a, p, mine, start, cell_lane_s[warp]);
+      if ((p.cells >> lane) & 1u) my_cnt = __popc(sl.lm & lane_range(start, n));
     }
     if (valid) {
       a.newcnt[(int64_t)mine.j * a.tm.T + mine.t] = my_cnt;
@@ -232,24 +251,27 @@ __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
   }
 }
 
-__device__ __forceinline__ void small_emit(const CellArgs& a, const Cell& c, int32_t nb,
-                                           int32_t nfo) {
-  const SmallCell s = small_cell(a, c);
-  const int n = c.fn + c.sn;
+// Emits a pass of small cells: col of every sampled entry, the new nodes
+// (ascending, after the cell's new base nb), and the next frontier cell
+// (frontier and new ids merged in ascending order at nfo).
+__device__ __forceinline__ void small_emit(const CellArgs& a, const Pass& p, const Slot& s,
+                                           int32_t my_nb, int32_t my_nfo) {
+  const int32_t nb = __shfl_sync(0xffffffffu, my_nb, s.cl);
+  const int32_t nfo = __shfl_sync(0xffffffffu, my_nfo, s.cl);
   int32_t lessF = 0, lessN = 0;
-  for (int k = 0; k < n; ++k) {
-    const int32_t idk = __shfl_sync(0xffffffffu, s.id, k);
-    if (idk < s.id) {
-      lessF += (s.fmask >> k) & 1u;
-      lessN += (s.lmask >> k) & 1u;
+  for (int k = 0; k < p.used; ++k) {
+    const unsigned long long kk = __shfl_sync(0xffffffffu, s.key, k);
+    if ((kk >> 32) == (s.key >> 32) && (uint32_t)kk < (uint32_t)s.id) {
+      lessF += (s.fm >> k) & 1u;
+      lessN += (s.lm >> k) & 1u;
     }
   }
   const int lane = lane_id();
-  const int src = s.inD ? __ffs(s.peers & s.fmask) - 1 : lane;
+  const int src = s.inD ? __ffs(s.peers & s.fm) - 1 : lane;
   const int32_t fpos = __shfl_sync(0xffffffffu, s.extra, src);
-  const int64_t jcap = (int64_t)c.j * a.capK;
+  const int64_t jcap = (int64_t)s.c.j * a.capK;
   if (s.act && !s.isF)
-    a.col[(int64_t)c.j * a.ecap + s.extra] = s.inD ? (int32_t)(fpos - jcap) : nb + lessN;
+    a.col[(int64_t)s.c.j * a.ecap + s.extra] = s.inD ? (int32_t)(fpos - jcap) : nb + lessN;
   if (s.act && (s.isF || s.leader)) {
     const int32_t r = nfo + lessF + lessN;
     int32_t g = s.extra;
@@ -339,6 +361,7 @@ __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
   __shared__ uint32_t N_s[kWarps][kTileWords];
   __shared__ int32_t pD_s[kWarps][kTileWords];
   __shared__ int32_t pN_s[kWarps][kTileWords];
+  __shared__ int cell_lane_s[kWarps][32];
   const int warp = threadIdx.x >> 5, lane = lane_id();
   const int64_t nchunks = (a.ncells + 31) / 32;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
@@ -346,12 +369,14 @@ __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
     const int64_t my_cell = ch * 32 + lane;
     Cell mine;
     const bool valid = load_cell(a, my_cell, &mine);
+    const int n = mine.fn + mine.sn;
     int32_t my_nfo = 0, my_nb = 0;
-    if (valid && mine.fn + mine.sn > 0) {
+    if (valid && n > 0) {
       my_nfo = a.nfcell_off[my_cell];
       if (mine.sn > 0) my_nb = a.nsz_prev[mine.j] + a.newbase[(int64_t)mine.j * a.tm.T + mine.t];
     }
-    unsigned todo = __ballot_sync(0xffffffffu, valid && mine.fn + mine.sn > 0);
+    // cells with more than 32 entries, one at a time
+    unsigned todo = __ballot_sync(0xffffffffu, valid && n > 32);
     while (todo) {
       const int k = __ffs(todo) - 1;
       todo &= todo - 1u;
@@ -363,11 +388,17 @@ __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
           a.nfb_id[nfo + i] = a.fb_id[c.fo + i];
           a.nfb_pos[nfo + i] = a.fb_pos[c.fo + i];
         }
-      } else if (c.fn + c.sn <= 32) {
-        small_emit(a, c, nb, nfo);
       } else {
         big_emit(a, c, nb, nfo, D_s[warp], N_s[warp], pD_s[warp], pN_s[warp]);
       }
+    }
+    // small cells (including frontier-only ones), packed
+    unsigned remaining = __ballot_sync(0xffffffffu, valid && n > 0 && n <= 32);
+    while (remaining) {
+      int start;
+      const Pass p = next_pass(&remaining, n, &start);
+      const Slot sl = load_slot(a, p, mine, start, cell_lane_s[warp]);
+      small_emit(a, p, sl, my_nb, my_nfo);
     }
   }
 }
@@ -387,12 +418,10 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   int gx = (num_sms * 8 + a.H - 1) / a.H;
   if (gx < 1) gx = 1;
   const dim3 egrid(gx, a.H);
-  dedup_hist_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, a.H, tm, d.stile, d.scnt,
-                                                a.status);
   cudaError_t e = seg_scan<int32_t, int32_t>(d.scnt, 0, d.soff, 0, nullptr, ncells, 1, ncells,
                                              true, nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
-  dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, a.H, d.stile, d.scnt,
+  dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, d.scell, d.srank,
                                                    d.soff, d.sb_u, d.sb_e, a.status);
 
   CellArgs c;

@@ -76,16 +76,21 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
                                 const int32_t* fcell_off, int32_t* cnt, int num_sms,
                                 cudaStream_t st);
 
+// Samples every frontier entry and records, per sampled edge, its
+// neighbour id (nbr), its (tile, minibatch) cell (scell) and its rank within
+// that cell (srank), counting the cells in scnt (zero on entry).
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
                                const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
-                               int num_sms, cudaStream_t st);
+                               int32_t* scnt, int32_t* scell, int32_t* srank, int num_sms,
+                               cudaStream_t st);
 
 // ---- dedup.cu --------------------------------------------------------------
 struct DedupBufs {
   const int32_t* nbr;       // H x ecap sampled ids
   const int32_t* ecnt;      // H edge counts
-  int32_t* stile;           // H x ecap scratch (tile of each sampled id)
-  int32_t* scnt;            // T*H counters, zero on entry and exit
+  const int32_t* scell;     // H x ecap: cell of each sampled id
+  const int32_t* srank;     // H x ecap: its rank within the cell
+  const int32_t* scnt;      // T*H per-cell counts of sampled ids
   int32_t* soff;            // T*H+1
   int32_t* sb_u;            // bucketed sampled ids
   int32_t* sb_e;            // their edge index in the minibatch

@@ -184,6 +184,11 @@ sample_count_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict
 }
 
 struct FillArgs {
+  TileMap tm;
+  int32_t H;
+  int32_t* scnt;   // T*H per-cell counters of sampled ids (zero on entry)
+  int32_t* scell;  // per edge: its (tile, minibatch) cell
+  int32_t* srank;  // per edge: its rank within the cell
   const int32_t* fb_id;
   const int32_t* fb_pos;
   const int32_t* total_ptr;
@@ -207,6 +212,23 @@ __device__ __forceinline__ int64_t draw(const FillArgs& a, int32_t v, int32_t s,
   return (int64_t)__umul64hi(r, (uint64_t)(J + 1));
 }
 
+// Records sampled edge e = (j, eidx) with neighbour u: its id, its
+// (tile, minibatch) cell and its rank within the cell (warp-aggregated
+// atomic), so the bucketing scatter after the scan needs no atomics.
+__device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t u, uint32_t j,
+                                           int64_t eidx) {
+  int64_t cell = 0;
+  if (has) cell = (int64_t)tile_of(a.tm, u) * a.H + j;
+  const unsigned m = __ballot_sync(0xffffffffu, has);
+  if (has) {
+    const int32_t rank = warp_agg_add(a.scnt, cell, m);
+    const int64_t at = (int64_t)j * a.ecap + eidx;
+    a.nbr[at] = u;
+    a.scell[at] = (int32_t)cell;
+    a.srank[at] = rank;
+  }
+}
+
 // G lanes per frontier node, k <= G.
 template <typename OffT, int G>
 __global__ void __launch_bounds__(kThreads)
@@ -222,27 +244,39 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t e0 = warp0 * kGroups; e0 < total; e0 += nwarps * kGroups) {
     const int64_t i = e0 + sub;
-    if (i >= total) continue;  // whole group skips together
-    const int32_t v = a.fb_id[i];
-    const uint32_t g = (uint32_t)a.fb_pos[i];
-    const uint32_t j = g / capk32;
-    const uint32_t pos = g - j * capk32;
-    const int64_t base = (int64_t)__ldg(off + v);
-    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
-    int32_t* out = a.nbr + j * a.ecap + a.indptr[j * (a.cap_prev + 1) + pos];
-    if (d <= a.k) {
-      for (int64_t q = s; q < d; q += G) out[q] = __ldg(a.indices + base + q);
-      continue;
+    bool has = false;
+    int32_t u = 0;
+    uint32_t j = 0;
+    int64_t eidx = 0;
+    if (i < total) {  // whole group takes the same branches
+      const int32_t v = a.fb_id[i];
+      const uint32_t g = (uint32_t)a.fb_pos[i];
+      j = g / capk32;
+      const uint32_t pos = g - j * capk32;
+      const int64_t base = (int64_t)__ldg(off + v);
+      const int64_t d = (int64_t)__ldg(off + v + 1) - base;
+      eidx = a.indptr[j * (a.cap_prev + 1) + pos] + s;
+      if (d <= a.k) {
+        if (s < d) {
+          u = __ldg(a.indices + base + s);
+          has = true;
+        }
+      } else {
+        const int64_t J = d - a.k + s;
+        const int64_t t = s < a.k ? draw(a, v, s, a.first_gid + j, J) : -1;
+        bool collided = false;
+        for (int q = 0; q < a.k; ++q) {
+          const int64_t mine = collided ? J : t;
+          const int64_t cq = __shfl_sync(gmask, mine, q, G);
+          if (s > q && t == cq) collided = true;
+        }
+        if (s < a.k) {
+          u = __ldg(a.indices + base + (collided ? J : t));
+          has = true;
+        }
+      }
     }
-    const int64_t J = d - a.k + s;
-    const int64_t t = s < a.k ? draw(a, v, s, a.first_gid + j, J) : -1;
-    bool collided = false;
-    for (int q = 0; q < a.k; ++q) {
-      const int64_t mine = collided ? J : t;
-      const int64_t cq = __shfl_sync(gmask, mine, q, G);
-      if (s > q && t == cq) collided = true;
-    }
-    if (s < a.k) out[s] = __ldg(a.indices + base + (collided ? J : t));
+    emit_edges(a, has, u, j, eidx);
   }
 }
 
@@ -267,9 +301,13 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
     const uint32_t pos = g - j * capk32;
     const int64_t base = (int64_t)__ldg(off + v);
     const int64_t d = (int64_t)__ldg(off + v + 1) - base;
-    int32_t* out = a.nbr + j * a.ecap + a.indptr[j * (a.cap_prev + 1) + pos];
+    const int64_t ebase = a.indptr[j * (a.cap_prev + 1) + pos];
     if (d <= a.k) {
-      for (int64_t q = lane; q < d; q += 32) out[q] = __ldg(a.indices + base + q);
+      for (int64_t q0 = 0; q0 < d; q0 += 32) {
+        const int64_t q = q0 + lane;
+        const bool has = q < d;
+        emit_edges(a, has, has ? __ldg(a.indices + base + q) : 0, j, ebase + q);
+      }
       continue;
     }
     for (int c0 = 0; c0 < a.k; c0 += 32) {
@@ -286,10 +324,8 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
         if (lane > q && t == cq) collided = true;
       }
       const int64_t c = collided ? J : t;
-      if (valid) {
-        chosen[s] = (int32_t)c;
-        out[s] = __ldg(a.indices + base + c);
-      }
+      if (valid) chosen[s] = (int32_t)c;
+      emit_edges(a, valid, valid ? __ldg(a.indices + base + c) : 0, j, ebase + s);
       __syncwarp();
     }
   }
@@ -350,8 +386,14 @@ static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int gri
 
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
                                const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
-                               int num_sms, cudaStream_t st) {
+                               int32_t* scnt, int32_t* scell, int32_t* srank, int num_sms,
+                               cudaStream_t st) {
   FillArgs f;
+  f.tm = TileMap{a.tile_first, a.chunk_tile, a.T};
+  f.H = a.H;
+  f.scnt = scnt;
+  f.scell = scell;
+  f.srank = srank;
   f.fb_id = fb_id;
   f.fb_pos = fb_pos;
   f.total_ptr = fcell_off + (int64_t)a.T * a.H;

@@ -92,6 +92,8 @@ scan_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, const int32_
   }
 }
 
+// Each warp scans 256 consecutive elements as 8 coalesced 32-wide slices
+// (carry passed slice to slice), then the warps' totals are scanned.
 template <typename InT, typename OutT>
 __global__ void __launch_bounds__(kThreads)
 scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict__ out,
@@ -103,26 +105,39 @@ scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict
   const int64_t len = seg_len(d_len, const_len, s);
   const int64_t begin = c * kChunk;
   if (begin >= len) return;
-  const int64_t n = min((int64_t)kChunk, len - begin);
-  const InT* p = in + (int64_t)s * in_stride + begin;
-  OutT* q = out + (int64_t)s * out_stride + begin;
-
-  __shared__ int64_t stage[kChunk];
-  for (int i = threadIdx.x; i < kChunk; i += kThreads) stage[i] = i < n ? (int64_t)p[i] : 0;
-  __syncthreads();
-  int64_t local[kItems];
-  int64_t run = 0;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t wbase = begin + (int64_t)warp * (32 * kItems);
+  const InT* p = in + (int64_t)s * in_stride;
+  OutT* q = out + (int64_t)s * out_stride;
+  int64_t v[kItems];
 #pragma unroll
   for (int k = 0; k < kItems; ++k) {
-    local[k] = run;
-    run += stage[threadIdx.x * kItems + k];
+    const int64_t i = wbase + k * 32 + lane;
+    v[k] = i < len ? (int64_t)p[i] : 0;
   }
-  int64_t tot;
-  const int64_t ex = block_excl_scan(run, &tot) + partial[(int64_t)s * chunks + c];
+  int64_t carry = 0;
 #pragma unroll
-  for (int k = 0; k < kItems; ++k) stage[threadIdx.x * kItems + k] = ex + local[k];
+  for (int k = 0; k < kItems; ++k) {
+    const int64_t inc = warp_incl_scan(v[k]);
+    const int64_t x = v[k];
+    v[k] = carry + inc - x;
+    carry += __shfl_sync(0xffffffffu, inc, 31);
+  }
+  __shared__ int64_t wtot[kThreads / 32];
+  if (lane == 0) wtot[warp] = carry;
   __syncthreads();
-  for (int i = threadIdx.x; i < n; i += kThreads) q[i] = (OutT)stage[i];
+  if (warp == 0) {
+    const int64_t w = lane < kThreads / 32 ? wtot[lane] : 0;
+    const int64_t wi = warp_incl_scan(w);
+    if (lane < kThreads / 32) wtot[lane] = wi - w;
+  }
+  __syncthreads();
+  const int64_t off = partial[(int64_t)s * chunks + c] + wtot[warp];
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) {
+    const int64_t i = wbase + k * 32 + lane;
+    if (i < len) q[i] = (OutT)(off + v[k]);
+  }
 }
 
 }  // namespace
