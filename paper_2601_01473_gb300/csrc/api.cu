@@ -53,8 +53,11 @@ struct Workspace {
   int32_t* nbr = nullptr;
   int32_t* scell = nullptr;
   int32_t* srank = nullptr;
-  int32_t* sb_u = nullptr;
-  int32_t* sb_e = nullptr;
+  int2* sb = nullptr;
+  int32_t* big_list = nullptr;
+  int32_t* big_n = nullptr;
+  int32_t* tmp_id = nullptr;
+  int32_t* tmp_pos = nullptr;
   int32_t* cnt = nullptr;
   void* feats_out = nullptr;
   uint8_t* adj_flags = nullptr;
@@ -170,8 +173,11 @@ static void free_workspace(Workspace* w) {
   cudaFree(w->nbr);
   cudaFree(w->scell);
   cudaFree(w->srank);
-  cudaFree(w->sb_u);
-  cudaFree(w->sb_e);
+  cudaFree(w->sb);
+  cudaFree(w->big_list);
+  cudaFree(w->big_n);
+  cudaFree(w->tmp_id);
+  cudaFree(w->tmp_pos);
   cudaFree(w->cnt);
   cudaFree(w->feats_out);
   cudaFree(w->adj_flags);
@@ -256,8 +262,11 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.nbr, edges);
   WA(w.scell, edges);
   WA(w.srank, edges);
-  WA(w.sb_u, edges > rows ? edges : rows);
-  WA(w.sb_e, edges > rows ? edges : rows);
+  WA(w.sb, edges);
+  WA(w.big_list, (rows + edges) / 33 + 1);
+  WA(w.big_n, 1);
+  WA(w.tmp_id, (int64_t)H * B);
+  WA(w.tmp_pos, (int64_t)H * B);
   WA(w.cnt, (int64_t)H * w.cap_prev_max);
   {
     uint8_t* f = nullptr;
@@ -612,7 +621,7 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   fill_i32_kernel<<<(H + 255) / 256, 256, 0, st>>>(w.nsz, H, B);
   CK(ctx, cudaGetLastError());
   CK(ctx, launch_bucket_targets(w.nodes, w.capK, H, B, (int32_t)ctx->N, ctx->bt.tile_first,
-                                ctx->bt.chunk_tile, T, w.fcnt, w.fcell_off[0], w.sb_u, w.sb_e,
+                                ctx->bt.chunk_tile, T, w.fcnt, w.fcell_off[0], w.tmp_id, w.tmp_pos,
                                 w.fb_id[0], w.fb_pos[0], w.scan_scratch, w.status, nsm, st));
   int cur = 0;
   for (int h = 0; h < K; ++h) {
@@ -651,8 +660,9 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     d.srank = w.srank;
     d.scnt = w.scnt;
     d.soff = w.soff;
-    d.sb_u = w.sb_u;
-    d.sb_e = w.sb_e;
+    d.sb = w.sb;
+    d.big_list = w.big_list;
+    d.big_n = w.big_n;
     d.fb_id = w.fb_id[cur];
     d.fb_pos = w.fb_pos[cur];
     d.fcell_off = w.fcell_off[cur];

@@ -27,8 +27,7 @@ __global__ void __launch_bounds__(kThreads)
 dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict__ ecnt,
                      int64_t ecap, const int32_t* __restrict__ scell,
                      const int32_t* __restrict__ srank, const int32_t* __restrict__ soff,
-                     int32_t* __restrict__ sb_u, int32_t* __restrict__ sb_e,
-                     const int32_t* status) {
+                     int2* __restrict__ sb, const int32_t* status) {
   if (failed(status)) return;
   const int32_t j = blockIdx.y;
   const int64_t E = ecnt[j];
@@ -36,8 +35,7 @@ dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict_
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < E;
        e += (int64_t)gridDim.x * blockDim.x) {
     const int32_t slot = soff[scell[o + e]] + srank[o + e];
-    sb_u[slot] = nbr[o + e];
-    sb_e[slot] = (int32_t)e;
+    sb[slot] = make_int2(nbr[o + e], (int32_t)e);
   }
 }
 
@@ -49,9 +47,10 @@ struct CellArgs {
   const int32_t* fb_id;
   const int32_t* fb_pos;
   const int32_t* fcell_off;
-  const int32_t* sb_u;
-  const int32_t* sb_e;
+  const int2* sb;        // sampled bucket: (id, edge index) per slot
   const int32_t* soff;
+  int32_t* big_list;     // cells with more than 32 entries
+  int32_t* big_n;
   const int32_t* tile_adj_block;
   uint8_t* adj_flags;
   int32_t* newcnt;
@@ -76,13 +75,22 @@ __device__ __forceinline__ void mark_cell(const CellArgs& a, uint32_t* D, uint32
     S[w] = 0;
   }
   __syncwarp();
-  for (int32_t i = lane; i < fn; i += 32) {
-    const int32_t lu = a.fb_id[fo + i] - base;
-    atomicOr(&D[lu >> 5], 1u << (lu & 31));
+  // four entries in flight per lane
+  for (int32_t i0 = lane; i0 < fn; i0 += 128) {
+    int32_t v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = i0 + 32 * q < fn ? a.fb_id[fo + i0 + 32 * q] - base : -1;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (v[q] >= 0) atomicOr(&D[v[q] >> 5], 1u << (v[q] & 31));
   }
-  for (int32_t i = lane; i < sn; i += 32) {
-    const int32_t lu = a.sb_u[so + i] - base;
-    atomicOr(&S[lu >> 5], 1u << (lu & 31));
+  for (int32_t i0 = lane; i0 < sn; i0 += 128) {
+    int32_t v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = i0 + 32 * q < sn ? a.sb[so + i0 + 32 * q].x - base : -1;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (v[q] >= 0) atomicOr(&S[v[q] >> 5], 1u << (v[q] & 31));
   }
   __syncwarp();
 }
@@ -179,8 +187,9 @@ __device__ __forceinline__ Slot load_slot(const CellArgs& a, const Pass& p, cons
       s.id = a.fb_id[s.c.fo + q];
       s.extra = a.fb_pos[s.c.fo + q];
     } else {
-      s.id = a.sb_u[s.c.so + q - s.c.fn];
-      s.extra = a.sb_e[s.c.so + q - s.c.fn];
+      const int2 e = a.sb[s.c.so + q - s.c.fn];
+      s.id = e.x;
+      s.extra = e.y;
     }
   }
   s.key = s.act ? (((unsigned long long)s.r << 32) | (uint32_t)s.id)
@@ -213,11 +222,7 @@ __device__ __forceinline__ int32_t big_count(const CellArgs& a, const Cell& c, u
 
 __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
   if (failed(a.status)) return;
-  __shared__ uint32_t D_s[kWarps][kTileWords];
-  __shared__ uint32_t S_s[kWarps][kTileWords];
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  uint32_t* D = D_s[warp];
-  uint32_t* S = S_s[warp];
   const int64_t nchunks = (a.ncells + 31) / 32;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
   __shared__ int cell_lane_s[kWarps][32];
@@ -227,13 +232,15 @@ __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
     const bool valid = load_cell(a, my_cell, &mine);
     const int n = mine.fn + mine.sn;
     int32_t my_cnt = 0;
-    // cells with more than 32 entries, one at a time, on bitmaps
-    unsigned todo = __ballot_sync(0xffffffffu, valid && mine.sn > 0 && n > 32);
-    while (todo) {
-      const int k = __ffs(todo) - 1;
-      todo &= todo - 1u;
-      const int32_t cnt = big_count(a, bcast(mine, k), D, S);
-      if (lane == k) my_cnt = cnt;
+    // cells with more than 32 entries go to the big-cell list (one warp each
+    // in the next kernel, so a hub tile's cells spread over the GPU)
+    const bool big = valid && n > 32;
+    const unsigned bm = __ballot_sync(0xffffffffu, big);
+    if (bm) {
+      int32_t base = 0;
+      if (lane == __ffs(bm) - 1) base = atomicAdd(a.big_n, __popc(bm));
+      base = __shfl_sync(0xffffffffu, base, __ffs(bm) - 1);
+      if (big) a.big_list[base + __popc(bm & ((1u << lane) - 1u))] = (int32_t)my_cell;
     }
     // small cells, packed
     unsigned remaining = __ballot_sync(0xffffffffu, valid && mine.sn > 0 && n <= 32);
@@ -243,10 +250,30 @@ __global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
       const Slot sl = load_slot(a, p, mine, start, cell_lane_s[warp]);
       if ((p.cells >> lane) & 1u) my_cnt = __popc(sl.lm & lane_range(start, n));
     }
-    if (valid) {
+    if (valid && !big) {
       a.newcnt[(int64_t)mine.j * a.tm.T + mine.t] = my_cnt;
       a.nfcnt[my_cell] = mine.fn + my_cnt;
-      if (mine.fn > 0) a.adj_flags[a.tile_adj_block[mine.t]] = 1;
+    }
+    if (valid && mine.fn > 0) a.adj_flags[a.tile_adj_block[mine.t]] = 1;
+  }
+}
+
+// One warp per big cell (listed by dedup_count_kernel).
+__global__ void __launch_bounds__(kThreads) dedup_count_big_kernel(CellArgs a) {
+  if (failed(a.status)) return;
+  __shared__ uint32_t D_s[kWarps][kTileWords];
+  __shared__ uint32_t S_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  const int32_t nbig = *a.big_n;
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t b = blockIdx.x * (int64_t)kWarps + warp; b < nbig; b += nwarps) {
+    const int64_t cell = a.big_list[b];
+    Cell c;
+    load_cell(a, cell, &c);
+    const int32_t cnt = c.sn > 0 ? big_count(a, c, D_s[warp], S_s[warp]) : 0;
+    if (lane == 0) {
+      a.newcnt[(int64_t)c.j * a.tm.T + c.t] = cnt;
+      a.nfcnt[cell] = c.fn + cnt;
     }
   }
 }
@@ -318,7 +345,8 @@ __device__ __forceinline__ void big_emit(const CellArgs& a, const Cell& c, int32
   const int64_t jcap = (int64_t)c.j * a.capK;
   int32_t* col = a.col + (int64_t)c.j * a.ecap;
   for (int32_t i = lane; i < c.sn; i += 32) {
-    const int32_t lu = a.sb_u[c.so + i] - base;
+    const int2 se = a.sb[c.so + i];
+    const int32_t lu = se.x - base;
     const int32_t w = lu >> 5;
     const uint32_t bit = 1u << (lu & 31), below = bit - 1u;
     int32_t cv;
@@ -326,7 +354,7 @@ __device__ __forceinline__ void big_emit(const CellArgs& a, const Cell& c, int32
       cv = (int32_t)(a.fb_pos[c.fo + pD[w] + __popc(D[w] & below)] - jcap);
     else
       cv = nb + pN[w] + __popc(Nw[w] & below);
-    col[a.sb_e[c.so + i]] = cv;
+    col[se.y] = cv;
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -357,10 +385,6 @@ __device__ __forceinline__ void big_emit(const CellArgs& a, const Cell& c, int32
 
 __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
   if (failed(a.status)) return;
-  __shared__ uint32_t D_s[kWarps][kTileWords];
-  __shared__ uint32_t N_s[kWarps][kTileWords];
-  __shared__ int32_t pD_s[kWarps][kTileWords];
-  __shared__ int32_t pN_s[kWarps][kTileWords];
   __shared__ int cell_lane_s[kWarps][32];
   const int warp = threadIdx.x >> 5, lane = lane_id();
   const int64_t nchunks = (a.ncells + 31) / 32;
@@ -371,26 +395,9 @@ __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
     const bool valid = load_cell(a, my_cell, &mine);
     const int n = mine.fn + mine.sn;
     int32_t my_nfo = 0, my_nb = 0;
-    if (valid && n > 0) {
+    if (valid && n > 0 && n <= 32) {
       my_nfo = a.nfcell_off[my_cell];
       if (mine.sn > 0) my_nb = a.nsz_prev[mine.j] + a.newbase[(int64_t)mine.j * a.tm.T + mine.t];
-    }
-    // cells with more than 32 entries, one at a time
-    unsigned todo = __ballot_sync(0xffffffffu, valid && n > 32);
-    while (todo) {
-      const int k = __ffs(todo) - 1;
-      todo &= todo - 1u;
-      const Cell c = bcast(mine, k);
-      const int32_t nfo = __shfl_sync(0xffffffffu, my_nfo, k);
-      const int32_t nb = __shfl_sync(0xffffffffu, my_nb, k);
-      if (c.sn == 0) {  // nothing sampled here: the frontier cell carries over unchanged
-        for (int32_t i = lane; i < c.fn; i += 32) {
-          a.nfb_id[nfo + i] = a.fb_id[c.fo + i];
-          a.nfb_pos[nfo + i] = a.fb_pos[c.fo + i];
-        }
-      } else {
-        big_emit(a, c, nb, nfo, D_s[warp], N_s[warp], pD_s[warp], pN_s[warp]);
-      }
     }
     // small cells (including frontier-only ones), packed
     unsigned remaining = __ballot_sync(0xffffffffu, valid && n > 0 && n <= 32);
@@ -400,6 +407,33 @@ __global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
       const Slot sl = load_slot(a, p, mine, start, cell_lane_s[warp]);
       small_emit(a, p, sl, my_nb, my_nfo);
     }
+  }
+}
+
+// One warp per big cell (the list built by dedup_count_kernel).
+__global__ void __launch_bounds__(kThreads) dedup_emit_big_kernel(CellArgs a) {
+  if (failed(a.status)) return;
+  __shared__ uint32_t D_s[kWarps][kTileWords];
+  __shared__ uint32_t N_s[kWarps][kTileWords];
+  __shared__ int32_t pD_s[kWarps][kTileWords];
+  __shared__ int32_t pN_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  const int32_t nbig = *a.big_n;
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t b = blockIdx.x * (int64_t)kWarps + warp; b < nbig; b += nwarps) {
+    const int64_t cell = a.big_list[b];
+    Cell c;
+    load_cell(a, cell, &c);
+    const int32_t nfo = a.nfcell_off[cell];
+    if (c.sn == 0) {  // nothing sampled here: the frontier cell carries over unchanged
+      for (int32_t i = lane; i < c.fn; i += 32) {
+        a.nfb_id[nfo + i] = a.fb_id[c.fo + i];
+        a.nfb_pos[nfo + i] = a.fb_pos[c.fo + i];
+      }
+      continue;
+    }
+    const int32_t nb = a.nsz_prev[c.j] + a.newbase[(int64_t)c.j * a.tm.T + c.t];
+    big_emit(a, c, nb, nfo, D_s[warp], N_s[warp], pD_s[warp], pN_s[warp]);
   }
 }
 
@@ -422,7 +456,9 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
                                              true, nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
   dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, d.scell, d.srank,
-                                                   d.soff, d.sb_u, d.sb_e, a.status);
+                                                   d.soff, d.sb, a.status);
+  e = cudaMemsetAsync(d.big_n, 0, sizeof(int32_t), st);
+  if (e != cudaSuccess) return e;
 
   CellArgs c;
   c.tm = tm;
@@ -433,8 +469,9 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   c.fb_id = d.fb_id;
   c.fb_pos = d.fb_pos;
   c.fcell_off = d.fcell_off;
-  c.sb_u = d.sb_u;
-  c.sb_e = d.sb_e;
+  c.sb = d.sb;
+  c.big_list = d.big_list;
+  c.big_n = d.big_n;
   c.soff = d.soff;
   c.tile_adj_block = d.tile_adj_block;
   c.adj_flags = d.adj_flags;
@@ -450,6 +487,7 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   c.status = a.status;
   const int cgrid = num_sms * 8;
   dedup_count_kernel<<<cgrid, kThreads, 0, st>>>(c);
+  dedup_count_big_kernel<<<cgrid, kThreads, 0, st>>>(c);
   e = seg_scan<int32_t, int32_t>(d.newcnt, a.T, d.newbase, a.T, nullptr, a.T, a.H, a.T, false,
                                  d.newtot, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
@@ -459,6 +497,7 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
                                  nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
   dedup_emit_kernel<<<cgrid, kThreads, 0, st>>>(c);
+  dedup_emit_big_kernel<<<cgrid, kThreads, 0, st>>>(c);
   return cudaGetLastError();
 }
 

@@ -92,8 +92,9 @@ struct DedupBufs {
   const int32_t* srank;     // H x ecap: its rank within the cell
   const int32_t* scnt;      // T*H per-cell counts of sampled ids
   int32_t* soff;            // T*H+1
-  int32_t* sb_u;            // bucketed sampled ids
-  int32_t* sb_e;            // their edge index in the minibatch
+  int2* sb;                 // bucketed (sampled id, edge index in the minibatch)
+  int32_t* big_list;        // cells with more than 32 entries (capacity: entries / 33 + 1)
+  int32_t* big_n;           // their count
   const int32_t* fb_id;     // current frontier bucket
   const int32_t* fb_pos;
   const int32_t* fcell_off;
