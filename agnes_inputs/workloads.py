@@ -65,6 +65,10 @@ WORKLOADS = {
     # small stand-ins with the same structure, for parity tests the oracle finishes in seconds
     "mini100m": Workload("mini100m", 2_000_000, 16, 0.57, 0.19, 0.19, "int64", "float16", 128,
                          MB, MB, 16, 1024, (15, 10, 5), 0.05, 1),
+    # profiling stand-in for rmat100m: same cell density per (tile, minibatch) at hop 3
+    # (~6 entries) with ~4 GB on the device
+    "prof5m": Workload("prof5m", 5_000_000, 16, 0.57, 0.19, 0.19, "int64", "float16", 128,
+                       MB, MB, 128, 64, (15, 10, 5), 0.05, 3),
     "mini_skew": Workload("mini_skew", 1_000_000, 28, 0.6, 0.2, 0.15, "int64", "float16", 256,
                           MB, MB, 8, 1024, (25, 10), None, 2),
 }

@@ -45,7 +45,6 @@ struct Workspace {
   int32_t* nfcnt = nullptr;
   int32_t* newcnt = nullptr;
   int32_t* newbase = nullptr;
-  int32_t* newtot = nullptr;
   int32_t* nsz = nullptr;   // (K+1) x H
   int32_t* ecnt = nullptr;  // K x H
   int64_t* indptr[AGNES_MAX_HOPS] = {nullptr};
@@ -54,6 +53,7 @@ struct Workspace {
   int32_t* scell = nullptr;
   int32_t* srank = nullptr;
   int2* sb = nullptr;
+  int2* tmp = nullptr;
   int32_t* big_list = nullptr;
   int32_t* big_n = nullptr;
   int32_t* tmp_id = nullptr;
@@ -163,7 +163,6 @@ static void free_workspace(Workspace* w) {
   cudaFree(w->nfcnt);
   cudaFree(w->newcnt);
   cudaFree(w->newbase);
-  cudaFree(w->newtot);
   cudaFree(w->nsz);
   cudaFree(w->ecnt);
   for (int h = 0; h < AGNES_MAX_HOPS; ++h) {
@@ -174,6 +173,7 @@ static void free_workspace(Workspace* w) {
   cudaFree(w->scell);
   cudaFree(w->srank);
   cudaFree(w->sb);
+  cudaFree(w->tmp);
   cudaFree(w->big_list);
   cudaFree(w->big_n);
   cudaFree(w->tmp_id);
@@ -225,7 +225,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   int64_t scratch = scan_scratch_elems(1, cells);
   const int64_t s2 = scan_scratch_elems(1, ctx->N);
   const int64_t s3 = scan_scratch_elems(H, w.cap_prev_max);
-  const int64_t s4 = scan_scratch_elems(H, T);
+  const int64_t s4 = col_scan_scratch_elems(T, H);
   if (s2 > scratch) scratch = s2;
   if (s3 > scratch) scratch = s3;
   if (s4 > scratch) scratch = s4;
@@ -252,7 +252,6 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.nfcnt, cells);
   WA(w.newcnt, cells);
   WA(w.newbase, cells);
-  WA(w.newtot, H);
   WA(w.nsz, (int64_t)(K + 1) * H);
   WA(w.ecnt, (int64_t)K * H);
   for (int h = 0; h < K; ++h) {
@@ -263,6 +262,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.scell, edges);
   WA(w.srank, edges);
   WA(w.sb, edges);
+  WA(w.tmp, rows + edges);
   WA(w.big_list, (rows + edges) / 33 + 1);
   WA(w.big_n, 1);
   WA(w.tmp_id, (int64_t)H * B);
@@ -661,6 +661,7 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     d.scnt = w.scnt;
     d.soff = w.soff;
     d.sb = w.sb;
+    d.tmp = w.tmp;
     d.big_list = w.big_list;
     d.big_n = w.big_n;
     d.fb_id = w.fb_id[cur];
@@ -668,7 +669,6 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     d.fcell_off = w.fcell_off[cur];
     d.newcnt = w.newcnt;
     d.newbase = w.newbase;
-    d.newtot = w.newtot;
     d.nfcnt = w.nfcnt;
     d.nfcell_off = w.fcell_off[1 - cur];
     d.nfb_id = w.fb_id[1 - cur];

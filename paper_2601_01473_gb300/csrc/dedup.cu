@@ -2,15 +2,16 @@
 // (Algorithm 1: N^j_out <- N^j_out u Sample(j, ...), N_in <- N_out).
 //
 // The sampled ids of every minibatch are bucketed by (tile, minibatch) cell
-// (histogram -> scan -> scatter, the bucket matrix of Sec. 3.4 (3)).  A cell
-// covers at most 4096 consecutive ids, so one warp resolves it with two
-// shared-memory bitmaps over the tile: D = the cell's frontier (dst_h) ids and
-// S = its sampled ids.  new = S & ~D in ascending id order is the cell's part
-// of new_h (tiles ascend in id, so a per-minibatch scan of the cells' new
-// counts over tiles gives each new node its index in src_h = dst_h ++ new_h);
-// popcount ranks in D and new give every sampled edge its col; and D | new in
-// ascending order, with each node's output row, is the cell of the next hop's
-// frontier bucket -- the bucket is carried from hop to hop and never rebuilt.
+// (histogram -> scan -> scatter, the bucket matrix of Sec. 3.4 (3)); each
+// cell is then resolved once against the same cell of the frontier bucket:
+// D = the cell's frontier (dst_h) ids, S = its sampled ids, new = S \ D.
+// Tiles ascend in id, so new_h in ascending order is the cells' new ids in
+// tile order, and a per-minibatch scan of the cells' new counts over tiles
+// places every new node in src_h = dst_h ++ new_h.  Resolving a cell gives,
+// with ranks local to the cell, each sampled edge's col and the cell of the
+// next hop's frontier bucket (D | new in ascending id); after the scans, a
+// fix-up pass and a compaction pass turn the local ranks into final indices.
+// The bucket is carried from hop to hop and never rebuilt.
 #include "common.cuh"
 #include "internal.h"
 
@@ -44,56 +45,21 @@ struct CellArgs {
   int32_t H;
   int64_t ncells;
   int64_t capK, ecap;
-  const int32_t* fb_id;
+  const int32_t* fb_id;      // frontier bucket (ids sorted inside a cell)
   const int32_t* fb_pos;
   const int32_t* fcell_off;
-  const int2* sb;        // sampled bucket: (id, edge index) per slot
+  const int2* sb;            // sampled bucket: (id, edge index)
   const int32_t* soff;
-  int32_t* big_list;     // cells with more than 32 entries
-  int32_t* big_n;
   const int32_t* tile_adj_block;
   uint8_t* adj_flags;
-  int32_t* newcnt;
-  const int32_t* newbase;
-  int32_t* nfcnt;
-  const int32_t* nfcell_off;
-  int32_t* nfb_id;
-  int32_t* nfb_pos;
-  const int32_t* nsz_prev;
-  int32_t* nodes;
-  int32_t* col;
+  int32_t* newcnt;           // per cell: new ids
+  int32_t* nfcnt;            // per cell: next-frontier entries
+  int2* tmp;                 // per cell at fcell_off + soff: next-frontier entries, local ranks
+  int32_t* col;              // H x ecap: final col, or -(1 + local new rank)
+  int32_t* big_list;         // cells with more than 32 entries
+  int32_t* big_n;
   const int32_t* status;
 };
-
-// Marks the cell's frontier ids in D and sampled ids in S (tile-local bits).
-__device__ __forceinline__ void mark_cell(const CellArgs& a, uint32_t* D, uint32_t* S, int32_t base,
-                                          int32_t words, int32_t fo, int32_t fn, int32_t so,
-                                          int32_t sn) {
-  const int lane = lane_id();
-  for (int w = lane; w < words; w += 32) {
-    D[w] = 0;
-    S[w] = 0;
-  }
-  __syncwarp();
-  // four entries in flight per lane
-  for (int32_t i0 = lane; i0 < fn; i0 += 128) {
-    int32_t v[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) v[q] = i0 + 32 * q < fn ? a.fb_id[fo + i0 + 32 * q] - base : -1;
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (v[q] >= 0) atomicOr(&D[v[q] >> 5], 1u << (v[q] & 31));
-  }
-  for (int32_t i0 = lane; i0 < sn; i0 += 128) {
-    int32_t v[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) v[q] = i0 + 32 * q < sn ? a.sb[so + i0 + 32 * q].x - base : -1;
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (v[q] >= 0) atomicOr(&S[v[q] >> 5], 1u << (v[q] & 31));
-  }
-  __syncwarp();
-}
 
 // A cell (t, j): its frontier entries [fo, fo+fn) and sampled entries
 // [so, so+sn).
@@ -101,8 +67,6 @@ struct Cell {
   int32_t fo, fn, so, sn, t, j;
 };
 
-// Loads the cell of this lane (one cell per lane, 32 consecutive cells per
-// warp); returns false past the last cell.
 __device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell* c) {
   if (cell >= a.ncells) {
     *c = Cell{0, 0, 0, 0, 0, 0};
@@ -117,331 +81,392 @@ __device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell*
   return true;
 }
 
-__device__ __forceinline__ Cell bcast(const Cell& c, int k) {
-  Cell o;
-  o.fo = __shfl_sync(0xffffffffu, c.fo, k);
-  o.fn = __shfl_sync(0xffffffffu, c.fn, k);
-  o.so = __shfl_sync(0xffffffffu, c.so, k);
-  o.sn = __shfl_sync(0xffffffffu, c.sn, k);
-  o.t = __shfl_sync(0xffffffffu, c.t, k);
-  o.j = __shfl_sync(0xffffffffu, c.j, k);
-  return o;
-}
+// ---- small cells: entry-parallel -----------------------------------------------
+//
+// A CTA takes 256 consecutive cells and stages the entries of the cells with
+// samples and at most 32 entries in shared memory, each cell's frontier
+// entries (sorted) followed by its sampled entries.  Every thread then
+// resolves one entry against the entries of its own cell:
+//   phase 1, sampled entry u: inD = u is a frontier id of the cell (binary
+//            search) and which; leader = not inD and no earlier sampled entry
+//            of the cell is u;
+//   phase 2: lessN = leaders of the cell smaller than u, lessF = frontier ids
+//            smaller than u (a frontier entry's own index); the entry's rank
+//            in the next-frontier cell is lessF + lessN and a new node's rank
+//            among the cell's new ids is lessN.
+// Cells with more than 32 entries go to the big-cell list.
+constexpr int kGroupCells = 256;
+constexpr int kSlotCap = 2048;
+constexpr int kSmallMax = 32;
+constexpr int kRoundFill = kSlotCap - kSmallMax;  // a cell starting below this fits
 
-// Small cells (at most 32 entries) are packed several to a warp pass: the
-// cells of the pass take consecutive lanes (cell r owns lanes
-// [start_r, start_r + n_r)), one entry per lane, frontier entries first.
-// Equal ids of one cell are found with match_any on (r, id); ranks are
-// counted against the other lanes of the same cell.
-struct Pass {
-  unsigned cells;  // lanes (of the 32-cell chunk) whose cell is in this pass
-  int used;        // entry lanes used
+enum : uint8_t { kSlotF = 1, kSlotLeader = 2, kSlotInD = 4 };
+
+struct GroupSmem {
+  int32_t fn[kGroupCells];
+  int32_t ps[kGroupCells + 1];  // staged-slot prefix of the group's cells
+  int32_t tb[kGroupCells];      // tmp base of the cell
+  int32_t j[kGroupCells];
+  int32_t wsum[kGroupCells / 32];
+  int32_t id[kSlotCap];
+  int32_t x[kSlotCap];       // frontier: output row; sampled: edge index
+  int16_t fidx[kSlotCap];    // sampled inD: slot of the matching frontier entry
+  uint8_t cell[kSlotCap];
+  uint8_t flag[kSlotCap];
 };
 
-struct Slot {
-  bool act, isF, inD, leader;
-  int r, cl;        // rank of the slot's cell in the pass, lane owning it
-  int32_t id;
-  int32_t extra;    // frontier: output row; sampled: edge index
-  unsigned long long key;
-  unsigned peers, fm, lm;
-  Cell c;
-};
-
-// Chooses the next pass among the remaining small cells (in lane order, as
-// many as fit in 32 lanes); returns this lane's first entry lane in *start.
-__device__ __forceinline__ Pass next_pass(unsigned* remaining, int n, int* start) {
-  const int lane = lane_id();
-  const bool rem = (*remaining >> lane) & 1u;
-  const int mine = rem ? n : 0;
-  const int incl = warp_incl_scan(mine);
-  const bool fits = rem && incl <= 32;
-  Pass p;
-  p.cells = __ballot_sync(0xffffffffu, fits);
-  p.used = __shfl_sync(0xffffffffu, incl, 31 - __clz(p.cells));
-  *remaining &= ~p.cells;
-  *start = incl - mine;
-  return p;
+__device__ __forceinline__ void put_tmp(const CellArgs& a, int32_t at, int32_t id, int32_t x) {
+  a.tmp[at] = make_int2(id, x);
 }
 
-__device__ __forceinline__ Slot load_slot(const CellArgs& a, const Pass& p, const Cell& mine,
-                                          int start, int* cell_lane) {
-  const int lane = lane_id();
-  const bool in_pass = (p.cells >> lane) & 1u;
-  if (in_pass) cell_lane[__popc(p.cells & ((1u << lane) - 1u))] = lane;
-  __syncwarp();
-  const unsigned starts = __reduce_or_sync(0xffffffffu, in_pass ? (1u << start) : 0u);
-  Slot s;
-  s.act = lane < p.used;
-  s.r = s.act ? __popc(starts & ((2u << lane) - 1u)) - 1 : 0;
-  s.cl = s.act ? cell_lane[s.r] : 0;
-  __syncwarp();
-  s.c = bcast(mine, s.cl);
-  const int st = __shfl_sync(0xffffffffu, start, s.cl);
-  const int q = lane - st;
-  s.isF = s.act && q < s.c.fn;
-  s.id = 0;
-  s.extra = 0;
-  if (s.act) {
-    if (s.isF) {
-      s.id = a.fb_id[s.c.fo + q];
-      s.extra = a.fb_pos[s.c.fo + q];
-    } else {
-      const int2 e = a.sb[s.c.so + q - s.c.fn];
-      s.id = e.x;
-      s.extra = e.y;
-    }
-  }
-  s.key = s.act ? (((unsigned long long)s.r << 32) | (uint32_t)s.id)
-                : (0xffffffff00000000ull | (unsigned)lane);
-  s.peers = __match_any_sync(0xffffffffu, s.key);
-  s.fm = __ballot_sync(0xffffffffu, s.isF);
-  s.inD = (s.peers & s.fm) != 0;
-  s.leader = s.act && !s.isF && !s.inD && lane == __ffs(s.peers) - 1;
-  s.lm = __ballot_sync(0xffffffffu, s.leader);
-  return s;
-}
-
-// Lanes [start, start + n) as a mask (n <= 32).
-__device__ __forceinline__ unsigned lane_range(int start, int n) {
-  return n >= 32 ? 0xffffffffu : (((1u << n) - 1u) << start);
-}
-
-// Cells with more than 32 entries: bitmaps over the tile.
-__device__ __forceinline__ int32_t big_count(const CellArgs& a, const Cell& c, uint32_t* D,
-                                             uint32_t* S) {
-  const int32_t base = a.tm.tile_first[c.t];
-  const int32_t words = (a.tm.tile_first[c.t + 1] - base + 31) >> 5;
-  mark_cell(a, D, S, base, words, c.fo, c.fn, c.so, c.sn);
-  int32_t cnt = 0;
-  for (int w = lane_id(); w < words; w += 32) cnt += __popc(S[w] & ~D[w]);
-  cnt = warp_sum(cnt);
-  __syncwarp();
-  return cnt;
-}
-
-__global__ void __launch_bounds__(kThreads) dedup_count_kernel(CellArgs a) {
+__global__ void __launch_bounds__(kThreads) dedup_cells_kernel(CellArgs a) {
   if (failed(a.status)) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int64_t nchunks = (a.ncells + 31) / 32;
-  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  __shared__ int cell_lane_s[kWarps][32];
-  for (int64_t ch = blockIdx.x * (int64_t)kWarps + warp; ch < nchunks; ch += nwarps) {
-    const int64_t my_cell = ch * 32 + lane;
-    Cell mine;
-    const bool valid = load_cell(a, my_cell, &mine);
-    const int n = mine.fn + mine.sn;
-    int32_t my_cnt = 0;
-    // cells with more than 32 entries go to the big-cell list (one warp each
-    // in the next kernel, so a hub tile's cells spread over the GPU)
-    const bool big = valid && n > 32;
-    const unsigned bm = __ballot_sync(0xffffffffu, big);
-    if (bm) {
-      int32_t base = 0;
-      if (lane == __ffs(bm) - 1) base = atomicAdd(a.big_n, __popc(bm));
-      base = __shfl_sync(0xffffffffu, base, __ffs(bm) - 1);
-      if (big) a.big_list[base + __popc(bm & ((1u << lane) - 1u))] = (int32_t)my_cell;
-    }
-    // small cells, packed
-    unsigned remaining = __ballot_sync(0xffffffffu, valid && mine.sn > 0 && n <= 32);
-    while (remaining) {
-      int start;
-      const Pass p = next_pass(&remaining, n, &start);
-      const Slot sl = load_slot(a, p, mine, start, cell_lane_s[warp]);
-      if ((p.cells >> lane) & 1u) my_cnt = __popc(sl.lm & lane_range(start, n));
-    }
-    if (valid && !big) {
-      a.newcnt[(int64_t)mine.j * a.tm.T + mine.t] = my_cnt;
-      a.nfcnt[my_cell] = mine.fn + my_cnt;
-    }
-    if (valid && mine.fn > 0) a.adj_flags[a.tile_adj_block[mine.t]] = 1;
-  }
-}
-
-// One warp per big cell (listed by dedup_count_kernel).
-__global__ void __launch_bounds__(kThreads) dedup_count_big_kernel(CellArgs a) {
-  if (failed(a.status)) return;
-  __shared__ uint32_t D_s[kWarps][kTileWords];
-  __shared__ uint32_t S_s[kWarps][kTileWords];
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int32_t nbig = *a.big_n;
-  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  for (int64_t b = blockIdx.x * (int64_t)kWarps + warp; b < nbig; b += nwarps) {
-    const int64_t cell = a.big_list[b];
+  __shared__ GroupSmem sm;
+  const int tid = threadIdx.x, lane = lane_id(), warp = tid >> 5;
+  const int64_t ngroups = (a.ncells + kGroupCells - 1) / kGroupCells;
+  for (int64_t grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
+    const int64_t c0 = grp * kGroupCells;
+    const int64_t my_cell = c0 + tid;
+    // per-cell facts, one thread per cell
     Cell c;
-    load_cell(a, cell, &c);
-    const int32_t cnt = c.sn > 0 ? big_count(a, c, D_s[warp], S_s[warp]) : 0;
-    if (lane == 0) {
-      a.newcnt[(int64_t)c.j * a.tm.T + c.t] = cnt;
-      a.nfcnt[cell] = c.fn + cnt;
-    }
-  }
-}
-
-// Emits a pass of small cells: col of every sampled entry, the new nodes
-// (ascending, after the cell's new base nb), and the next frontier cell
-// (frontier and new ids merged in ascending order at nfo).
-__device__ __forceinline__ void small_emit(const CellArgs& a, const Pass& p, const Slot& s,
-                                           int32_t my_nb, int32_t my_nfo) {
-  const int32_t nb = __shfl_sync(0xffffffffu, my_nb, s.cl);
-  const int32_t nfo = __shfl_sync(0xffffffffu, my_nfo, s.cl);
-  int32_t lessF = 0, lessN = 0;
-  for (int k = 0; k < p.used; ++k) {
-    const unsigned long long kk = __shfl_sync(0xffffffffu, s.key, k);
-    if ((kk >> 32) == (s.key >> 32) && (uint32_t)kk < (uint32_t)s.id) {
-      lessF += (s.fm >> k) & 1u;
-      lessN += (s.lm >> k) & 1u;
-    }
-  }
-  const int lane = lane_id();
-  const int src = s.inD ? __ffs(s.peers & s.fm) - 1 : lane;
-  const int32_t fpos = __shfl_sync(0xffffffffu, s.extra, src);
-  const int64_t jcap = (int64_t)s.c.j * a.capK;
-  if (s.act && !s.isF)
-    a.col[(int64_t)s.c.j * a.ecap + s.extra] = s.inD ? (int32_t)(fpos - jcap) : nb + lessN;
-  if (s.act && (s.isF || s.leader)) {
-    const int32_t r = nfo + lessF + lessN;
-    int32_t g = s.extra;
-    if (s.leader) {
-      g = (int32_t)(jcap + nb + lessN);
-      a.nodes[g] = s.id;
-    }
-    a.nfb_id[r] = s.id;
-    a.nfb_pos[r] = g;
-  }
-}
-
-__device__ __forceinline__ void big_emit(const CellArgs& a, const Cell& c, int32_t nb, int32_t nfo,
-                                         uint32_t* D, uint32_t* Nw, int32_t* pD, int32_t* pN) {
-  const int lane = lane_id();
-  const int32_t base = a.tm.tile_first[c.t];
-  const int32_t words = (a.tm.tile_first[c.t + 1] - base + 31) >> 5;
-  mark_cell(a, D, Nw, base, words, c.fo, c.fn, c.so, c.sn);
-  // new = S & ~D; per-word exclusive ranks of D and new
-  uint32_t dw[4], nw[4];
-  int32_t sd = 0, sn_ = 0;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int w = lane * 4 + q;
-    dw[q] = w < words ? D[w] : 0u;
-    nw[q] = w < words ? (Nw[w] & ~dw[q]) : 0u;
-    sd += __popc(dw[q]);
-    sn_ += __popc(nw[q]);
-  }
-  int32_t rd = warp_incl_scan(sd) - sd;
-  int32_t rn = warp_incl_scan(sn_) - sn_;
-  __syncwarp();
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int w = lane * 4 + q;
-    Nw[w] = nw[q];
-    pD[w] = rd;
-    pN[w] = rn;
-    rd += __popc(dw[q]);
-    rn += __popc(nw[q]);
-  }
-  __syncwarp();
-
-  const int64_t jcap = (int64_t)c.j * a.capK;
-  int32_t* col = a.col + (int64_t)c.j * a.ecap;
-  for (int32_t i = lane; i < c.sn; i += 32) {
-    const int2 se = a.sb[c.so + i];
-    const int32_t lu = se.x - base;
-    const int32_t w = lu >> 5;
-    const uint32_t bit = 1u << (lu & 31), below = bit - 1u;
-    int32_t cv;
-    if (D[w] & bit)
-      cv = (int32_t)(a.fb_pos[c.fo + pD[w] + __popc(D[w] & below)] - jcap);
-    else
-      cv = nb + pN[w] + __popc(Nw[w] & below);
-    col[se.y] = cv;
-  }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int w = lane * 4 + q;
-    if (w >= words) break;
-    const uint32_t d = dw[q], n = nw[q];
-    uint32_t rest = d | n;
-    const int32_t r0 = pD[w] + pN[w];
-    while (rest) {
-      const int b = __ffs(rest) - 1;
-      rest &= rest - 1u;
-      const uint32_t below = (1u << b) - 1u;
-      const int32_t id = base + w * 32 + b;
-      const int32_t r = r0 + __popc((d | n) & below);
-      int32_t g;
-      if ((d >> b) & 1u) {
-        g = a.fb_pos[c.fo + pD[w] + __popc(d & below)];
-      } else {
-        g = (int32_t)(jcap + nb + pN[w] + __popc(n & below));
-        a.nodes[g] = id;
+    const bool valid = load_cell(a, my_cell, &c);
+    const int n = c.fn + c.sn;
+    const bool staged = valid && c.sn > 0 && n <= kSmallMax;
+    if (valid) {
+      if (c.fn > 0) a.adj_flags[a.tile_adj_block[c.t]] = 1;
+      if (n > kSmallMax) {
+        a.big_list[atomicAdd(a.big_n, 1)] = (int32_t)my_cell;
+      } else if (c.sn == 0) {
+        a.newcnt[my_cell] = 0;
+        a.nfcnt[my_cell] = c.fn;
       }
-      a.nfb_id[nfo + r] = id;
-      a.nfb_pos[nfo + r] = g;
     }
+    const int32_t ns = staged ? n : 0;
+    sm.fn[tid] = c.fn;
+    sm.j[tid] = c.j;
+    sm.tb[tid] = c.fo + c.so;
+    const int32_t inc = warp_incl_scan(ns);
+    if (lane == 31) sm.wsum[warp] = inc;
+    __syncthreads();
+    {
+      int32_t off = 0, tot = 0;
+      for (int w = 0; w < kWarps; ++w) {
+        off += w < warp ? sm.wsum[w] : 0;
+        tot += sm.wsum[w];
+      }
+      sm.ps[tid] = off + inc - ns;
+      if (tid == 0) sm.ps[kGroupCells] = tot;
+    }
+    __syncthreads();
+    const int32_t total = sm.ps[kGroupCells];
+    // rounds: each starts at a cell start and takes the cells that start less
+    // than kRoundFill slots later (a cell has at most 32 entries, so a round
+    // never needs more than kSlotCap slots)
+    for (int32_t rbase = 0, rend = 0; rbase < total; rbase = rend) {
+      int32_t lo = 0, hi = kGroupCells;  // first cell with ps >= rbase + kRoundFill
+      while (lo < hi) {
+        const int32_t mid = (lo + hi) >> 1;
+        if (sm.ps[mid] < rbase + kRoundFill) lo = mid + 1; else hi = mid;
+      }
+      rend = min(total, sm.ps[lo]);  // slots [rbase, rend)
+      const int32_t used = rend - rbase;
+      const bool mine_in_round = staged && sm.ps[tid] >= rbase && sm.ps[tid] < rend;
+      // the owner of each cell of the round maps its slots to the cell
+      if (mine_in_round)
+        for (int q = 0; q < n; ++q) sm.cell[sm.ps[tid] - rbase + q] = (uint8_t)tid;
+      __syncthreads();
+      for (int32_t sl = tid; sl < used; sl += kThreads) {
+        const int l = sm.cell[sl];
+        const int32_t q = rbase + sl - sm.ps[l];
+        const int32_t fnl = sm.fn[l];
+        // this cell's frontier / sampled entries start at tb - so / tb - fo
+        if (q < fnl) {
+          const int32_t fo = __ldg(a.fcell_off + c0 + l);
+          sm.id[sl] = a.fb_id[fo + q];
+          sm.x[sl] = a.fb_pos[fo + q];
+          sm.flag[sl] = kSlotF;
+        } else {
+          const int32_t so = __ldg(a.soff + c0 + l);
+          const int2 e = a.sb[so + q - fnl];
+          sm.id[sl] = e.x;
+          sm.x[sl] = e.y;
+          sm.flag[sl] = 0;
+        }
+      }
+      __syncthreads();
+      // phase 1: membership and first occurrence of sampled ids
+      for (int32_t sl = tid; sl < used; sl += kThreads) {
+        if (sm.flag[sl] & kSlotF) continue;
+        const int l = sm.cell[sl];
+        const int32_t fs = sm.ps[l] - rbase, fe = fs + sm.fn[l];
+        const int32_t id = sm.id[sl];
+        int32_t lo2 = fs, hi2 = fe;  // first frontier id >= id (sorted)
+        while (lo2 < hi2) {
+          const int32_t mid = (lo2 + hi2) >> 1;
+          if (sm.id[mid] < id) lo2 = mid + 1; else hi2 = mid;
+        }
+        uint8_t fl = 0;
+        if (lo2 < fe && sm.id[lo2] == id) {
+          fl = kSlotInD;
+          sm.fidx[sl] = (int16_t)lo2;
+        } else {
+          bool dup = false;
+          for (int32_t q = fe; q < sl; ++q) dup |= sm.id[q] == id;
+          if (!dup) fl = kSlotLeader;
+        }
+        sm.flag[sl] = fl;
+      }
+      __syncthreads();
+      // the owner counts its cell's new ids
+      if (mine_in_round) {
+        const int32_t fs = sm.ps[tid] - rbase;
+        int32_t cnt = 0;
+        for (int32_t q = fs + c.fn; q < fs + n; ++q) cnt += (sm.flag[q] & kSlotLeader) != 0;
+        a.newcnt[my_cell] = cnt;
+        a.nfcnt[my_cell] = c.fn + cnt;
+      }
+      // phase 2: local ranks, col, next-frontier entries
+      for (int32_t sl = tid; sl < used; sl += kThreads) {
+        const int l = sm.cell[sl];
+        const int32_t fs = sm.ps[l] - rbase, fe = fs + sm.fn[l], se = sm.ps[l + 1] - rbase;
+        const int32_t id = sm.id[sl];
+        const uint8_t fl = sm.flag[sl];
+        int32_t lessN = 0;
+        for (int32_t q = fe; q < se; ++q) lessN += (sm.flag[q] & kSlotLeader) && sm.id[q] < id;
+        const int32_t tb = sm.tb[l];
+        if (fl & kSlotF) {
+          put_tmp(a, tb + (sl - fs) + lessN, id, sm.x[sl]);
+          continue;
+        }
+        const int64_t jrow = (int64_t)sm.j[l] * a.ecap;
+        if (fl & kSlotInD) {
+          a.col[jrow + sm.x[sl]] = (int32_t)(sm.x[sm.fidx[sl]] - (int64_t)sm.j[l] * a.capK);
+          continue;
+        }
+        a.col[jrow + sm.x[sl]] = -1 - lessN;
+        if (fl & kSlotLeader) {
+          int32_t lo2 = fs, hi2 = fe;  // frontier ids smaller than id
+          while (lo2 < hi2) {
+            const int32_t mid = (lo2 + hi2) >> 1;
+            if (sm.id[mid] < id) lo2 = mid + 1; else hi2 = mid;
+          }
+          put_tmp(a, tb + (lo2 - fs) + lessN, id, -1 - lessN);
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// ---- big cells: one warp each, bitmaps over the tile ---------------------------
+
+__device__ __forceinline__ void mark_bits(const CellArgs& a, const Cell& c, uint32_t* D,
+                                          uint32_t* S, int32_t base, int32_t words) {
+  const int lane = lane_id();
+  for (int w = lane; w < words; w += 32) {
+    D[w] = 0;
+    S[w] = 0;
+  }
+  __syncwarp();
+  for (int32_t i0 = lane; i0 < c.fn; i0 += 128) {  // four entries in flight per lane
+    int32_t v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = i0 + 32 * q < c.fn ? a.fb_id[c.fo + i0 + 32 * q] - base : -1;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (v[q] >= 0) atomicOr(&D[v[q] >> 5], 1u << (v[q] & 31));
+  }
+  for (int32_t i0 = lane; i0 < c.sn; i0 += 128) {
+    int32_t v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = i0 + 32 * q < c.sn ? a.sb[c.so + i0 + 32 * q].x - base : -1;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (v[q] >= 0) atomicOr(&S[v[q] >> 5], 1u << (v[q] & 31));
   }
   __syncwarp();
 }
 
-__global__ void __launch_bounds__(kThreads) dedup_emit_kernel(CellArgs a) {
-  if (failed(a.status)) return;
-  __shared__ int cell_lane_s[kWarps][32];
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int64_t nchunks = (a.ncells + 31) / 32;
-  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  for (int64_t ch = blockIdx.x * (int64_t)kWarps + warp; ch < nchunks; ch += nwarps) {
-    const int64_t my_cell = ch * 32 + lane;
-    Cell mine;
-    const bool valid = load_cell(a, my_cell, &mine);
-    const int n = mine.fn + mine.sn;
-    int32_t my_nfo = 0, my_nb = 0;
-    if (valid && n > 0 && n <= 32) {
-      my_nfo = a.nfcell_off[my_cell];
-      if (mine.sn > 0) my_nb = a.nsz_prev[mine.j] + a.newbase[(int64_t)mine.j * a.tm.T + mine.t];
-    }
-    // small cells (including frontier-only ones), packed
-    unsigned remaining = __ballot_sync(0xffffffffu, valid && n > 0 && n <= 32);
-    while (remaining) {
-      int start;
-      const Pass p = next_pass(&remaining, n, &start);
-      const Slot sl = load_slot(a, p, mine, start, cell_lane_s[warp]);
-      small_emit(a, p, sl, my_nb, my_nfo);
-    }
-  }
-}
-
-// One warp per big cell (the list built by dedup_count_kernel).
-__global__ void __launch_bounds__(kThreads) dedup_emit_big_kernel(CellArgs a) {
+__global__ void __launch_bounds__(kThreads) dedup_big_kernel(CellArgs a) {
   if (failed(a.status)) return;
   __shared__ uint32_t D_s[kWarps][kTileWords];
   __shared__ uint32_t N_s[kWarps][kTileWords];
   __shared__ int32_t pD_s[kWarps][kTileWords];
   __shared__ int32_t pN_s[kWarps][kTileWords];
   const int warp = threadIdx.x >> 5, lane = lane_id();
+  uint32_t* D = D_s[warp];
+  uint32_t* Nw = N_s[warp];
+  int32_t* pD = pD_s[warp];
+  int32_t* pN = pN_s[warp];
   const int32_t nbig = *a.big_n;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
   for (int64_t b = blockIdx.x * (int64_t)kWarps + warp; b < nbig; b += nwarps) {
     const int64_t cell = a.big_list[b];
     Cell c;
     load_cell(a, cell, &c);
-    const int32_t nfo = a.nfcell_off[cell];
-    if (c.sn == 0) {  // nothing sampled here: the frontier cell carries over unchanged
-      for (int32_t i = lane; i < c.fn; i += 32) {
-        a.nfb_id[nfo + i] = a.fb_id[c.fo + i];
-        a.nfb_pos[nfo + i] = a.fb_pos[c.fo + i];
+    if (c.sn == 0) {  // nothing sampled: the compaction copies the frontier cell
+      if (lane == 0) {
+        a.newcnt[cell] = 0;
+        a.nfcnt[cell] = c.fn;
       }
       continue;
     }
-    const int32_t nb = a.nsz_prev[c.j] + a.newbase[(int64_t)c.j * a.tm.T + c.t];
-    big_emit(a, c, nb, nfo, D_s[warp], N_s[warp], pD_s[warp], pN_s[warp]);
+    const int32_t base = a.tm.tile_first[c.t];
+    const int32_t words = (a.tm.tile_first[c.t + 1] - base + 31) >> 5;
+    mark_bits(a, c, D, Nw, base, words);
+    // new = S & ~D; per-word exclusive ranks of D and new
+    uint32_t dw[4], nw[4];
+    int32_t sd = 0, snw = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      dw[q] = w < words ? D[w] : 0u;
+      nw[q] = w < words ? (Nw[w] & ~dw[q]) : 0u;
+      sd += __popc(dw[q]);
+      snw += __popc(nw[q]);
+    }
+    const int32_t tot_new = warp_sum(snw);
+    int32_t rd = warp_incl_scan(sd) - sd;
+    int32_t rn = warp_incl_scan(snw) - snw;
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      Nw[w] = nw[q];
+      pD[w] = rd;
+      pN[w] = rn;
+      rd += __popc(dw[q]);
+      rn += __popc(nw[q]);
+    }
+    __syncwarp();
+    if (lane == 0) {
+      a.newcnt[cell] = tot_new;
+      a.nfcnt[cell] = c.fn + tot_new;
+    }
+    const int64_t jcap = (int64_t)c.j * a.capK;
+    int32_t* col = a.col + (int64_t)c.j * a.ecap;
+    for (int32_t i = lane; i < c.sn; i += 32) {
+      const int2 se = a.sb[c.so + i];
+      const int32_t lu = se.x - base;
+      const int32_t w = lu >> 5;
+      const uint32_t bit = 1u << (lu & 31), below = bit - 1u;
+      col[se.y] = (D[w] & bit) ? (int32_t)(a.fb_pos[c.fo + pD[w] + __popc(D[w] & below)] - jcap)
+                               : -1 - (pN[w] + __popc(Nw[w] & below));
+    }
+    const int32_t tb = c.fo + c.so;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int w = lane * 4 + q;
+      if (w >= words) break;
+      const uint32_t d = dw[q], nn = nw[q];
+      uint32_t rest = d | nn;
+      const int32_t r0 = pD[w] + pN[w];
+      while (rest) {
+        const int bb = __ffs(rest) - 1;
+        rest &= rest - 1u;
+        const uint32_t below = (1u << bb) - 1u;
+        const int32_t id = base + w * 32 + bb;
+        const int32_t r = r0 + __popc((d | nn) & below);
+        const int32_t x = ((d >> bb) & 1u) ? a.fb_pos[c.fo + pD[w] + __popc(d & below)]
+                                           : -1 - (pN[w] + __popc(nn & below));
+        put_tmp(a, tb + r, id, x);
+      }
+    }
+    __syncwarp();
   }
 }
 
-__global__ void add_sizes_kernel(const int32_t* __restrict__ prev, const int32_t* __restrict__ add,
-                                 int32_t* __restrict__ next, int32_t H, const int32_t* status) {
+// ---- fix-up and compaction (after the scans) --------------------------------------
+
+// col[e] = -(1 + r) becomes the new node's index in src_h:
+// |dst_h| + (new ids of the minibatch in earlier tiles) + r.
+__global__ void __launch_bounds__(kThreads)
+dedup_fix_col_kernel(int32_t* __restrict__ col, const int32_t* __restrict__ ecnt, int64_t ecap,
+                     const int32_t* __restrict__ scell, const int32_t* __restrict__ newbase,
+                     const int32_t* __restrict__ nsz_prev, const int32_t* status) {
   if (failed(status)) return;
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < H; j += gridDim.x * blockDim.x)
-    next[j] = prev[j] + add[j];
+  const int32_t j = blockIdx.y;
+  const int64_t E = ecnt[j];
+  const int64_t o = (int64_t)j * ecap;
+  const int32_t base = nsz_prev[j];
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < E;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t v = col[o + e];
+    if (v < 0) col[o + e] = base + newbase[scell[o + e]] + (-1 - v);
+  }
+}
+
+struct CompactArgs {
+  int64_t ncells;
+  int32_t H;
+  int64_t capK;
+  const int32_t* fb_id;
+  const int32_t* fb_pos;
+  const int32_t* fcell_off;
+  const int32_t* soff;
+  const int2* tmp;
+  const int32_t* nfcell_off;
+  const int32_t* newbase;
+  const int32_t* nsz_prev;
+  int32_t* nfb_id;
+  int32_t* nfb_pos;
+  int32_t* nodes;
+  const int32_t* status;
+};
+
+// Writes the next frontier bucket in cell order: a cell without samples is
+// copied from the current bucket, any other from its tmp entries, where a new
+// node (x = -(1 + r)) gets its output row j * capK + |dst_h| + newbase + r and
+// its id is appended to the minibatch's node list.
+__global__ void __launch_bounds__(kThreads) dedup_compact_kernel(CompactArgs a) {
+  if (failed(a.status)) return;
+  __shared__ int32_t s_nfo[kGroupCells + 1];
+  __shared__ int32_t s_src[kGroupCells];   // source base in fb (>= 0) or ~base in tmp
+  __shared__ int32_t s_row[kGroupCells];   // j * capK + |dst_h| + newbase
+  const int tid = threadIdx.x;
+  const int64_t ngroups = (a.ncells + kGroupCells - 1) / kGroupCells;
+  for (int64_t grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
+    const int64_t c0 = grp * kGroupCells;
+    const int64_t cell = c0 + tid;
+    const int64_t last = min(a.ncells, c0 + kGroupCells);
+    if (cell < a.ncells) {
+      const int32_t fo = a.fcell_off[cell];
+      const int32_t so = a.soff[cell];
+      const int32_t sn = a.soff[cell + 1] - so;
+      const int32_t j = (int32_t)(cell % a.H);
+      s_nfo[tid] = a.nfcell_off[cell];
+      s_src[tid] = sn == 0 ? fo : ~(fo + so);
+      s_row[tid] = (int32_t)((int64_t)j * a.capK + a.nsz_prev[j] + a.newbase[cell]);
+    }
+    if (tid == 0) s_nfo[last - c0] = a.nfcell_off[last];
+    __syncthreads();
+    const int32_t k0 = s_nfo[0], k1 = s_nfo[last - c0];
+    for (int32_t k = k0 + tid; k < k1; k += kThreads) {
+      int32_t lo = 0, hi = (int32_t)(last - c0);  // last cell with nfo <= k
+      while (hi - lo > 1) {
+        const int32_t mid = (lo + hi) >> 1;
+        if (s_nfo[mid] <= k) lo = mid; else hi = mid;
+      }
+      const int32_t r = k - s_nfo[lo];
+      const int32_t src = s_src[lo];
+      int32_t id, pos;
+      if (src >= 0) {
+        id = a.fb_id[src + r];
+        pos = a.fb_pos[src + r];
+      } else {
+        const int2 e = a.tmp[~src + r];
+        id = e.x;
+        pos = e.y;
+        if (pos < 0) {
+          pos = s_row[lo] + (-1 - pos);
+          a.nodes[pos] = id;
+        }
+      }
+      a.nfb_id[k] = id;
+      a.nfb_pos[k] = pos;
+    }
+    __syncthreads();
+  }
 }
 
 }  // namespace
@@ -470,34 +495,48 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   c.fb_pos = d.fb_pos;
   c.fcell_off = d.fcell_off;
   c.sb = d.sb;
-  c.big_list = d.big_list;
-  c.big_n = d.big_n;
   c.soff = d.soff;
   c.tile_adj_block = d.tile_adj_block;
   c.adj_flags = d.adj_flags;
   c.newcnt = d.newcnt;
-  c.newbase = d.newbase;
   c.nfcnt = d.nfcnt;
-  c.nfcell_off = d.nfcell_off;
-  c.nfb_id = d.nfb_id;
-  c.nfb_pos = d.nfb_pos;
-  c.nsz_prev = d.nsz_prev;
-  c.nodes = d.nodes;
+  c.tmp = d.tmp;
   c.col = d.col;
+  c.big_list = d.big_list;
+  c.big_n = d.big_n;
   c.status = a.status;
-  const int cgrid = num_sms * 8;
-  dedup_count_kernel<<<cgrid, kThreads, 0, st>>>(c);
-  dedup_count_big_kernel<<<cgrid, kThreads, 0, st>>>(c);
-  e = seg_scan<int32_t, int32_t>(d.newcnt, a.T, d.newbase, a.T, nullptr, a.T, a.H, a.T, false,
-                                 d.newtot, d.scan_scratch, a.status, st);
+  dedup_cells_kernel<<<resident_grid((const void*)dedup_cells_kernel, kThreads, num_sms), kThreads,
+                       0, st>>>(c);
+  dedup_big_kernel<<<resident_grid((const void*)dedup_big_kernel, kThreads, num_sms), kThreads, 0,
+                     st>>>(c);
+  // per-minibatch offsets of the new ids: scan down the tiles of the
+  // tile-major [T x H] count matrix; totals give the next frontier sizes
+  e = col_scan(d.newcnt, d.newbase, a.T, a.H, d.nsz_prev, d.nsz_next, d.scan_scratch, a.status,
+               st);
   if (e != cudaSuccess) return e;
-  add_sizes_kernel<<<(a.H + 255) / 256, 256, 0, st>>>(d.nsz_prev, d.newtot, d.nsz_next, a.H,
-                                                      a.status);
   e = seg_scan<int32_t, int32_t>(d.nfcnt, 0, d.nfcell_off, 0, nullptr, ncells, 1, ncells, true,
                                  nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
-  dedup_emit_kernel<<<cgrid, kThreads, 0, st>>>(c);
-  dedup_emit_big_kernel<<<cgrid, kThreads, 0, st>>>(c);
+  dedup_fix_col_kernel<<<egrid, kThreads, 0, st>>>(d.col, d.ecnt, a.ecap, d.scell, d.newbase,
+                                                   d.nsz_prev, a.status);
+  CompactArgs k;
+  k.ncells = ncells;
+  k.H = a.H;
+  k.capK = a.capK;
+  k.fb_id = d.fb_id;
+  k.fb_pos = d.fb_pos;
+  k.fcell_off = d.fcell_off;
+  k.soff = d.soff;
+  k.tmp = d.tmp;
+  k.nfcell_off = d.nfcell_off;
+  k.newbase = d.newbase;
+  k.nsz_prev = d.nsz_prev;
+  k.nfb_id = d.nfb_id;
+  k.nfb_pos = d.nfb_pos;
+  k.nodes = d.nodes;
+  k.status = a.status;
+  dedup_compact_kernel<<<resident_grid((const void*)dedup_compact_kernel, kThreads, num_sms),
+                         kThreads, 0, st>>>(k);
   return cudaGetLastError();
 }
 

@@ -137,25 +137,31 @@ distinct_rows_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restric
 cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
                           const int32_t* fb_pos, const int32_t* total, void* out,
                           const int32_t* status, int num_sms, cudaStream_t st) {
-  const int grid = num_sms * 8;
   const bool aligned = (row_bytes % 16 == 0) && ((uintptr_t)feats % 16 == 0) &&
                        ((uintptr_t)out % 16 == 0);
   if (aligned) {
     const int64_t vecs = row_bytes / 16;
     const uint4* f = (const uint4*)feats;
     uint4* o = (uint4*)out;
+#define AGNES_GRID(KERNEL) resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st
     if (vecs == 8)
-      gather_vec_kernel<8, 4><<<grid, kThreads, 0, st>>>(f, fb_id, fb_pos, total, o, status);
+      gather_vec_kernel<8, 4><<<AGNES_GRID((gather_vec_kernel<8, 4>))>>>(f, fb_id, fb_pos, total, o,
+                                                                         status);
     else if (vecs == 16)
-      gather_vec_kernel<16, 4><<<grid, kThreads, 0, st>>>(f, fb_id, fb_pos, total, o, status);
+      gather_vec_kernel<16, 4><<<AGNES_GRID((gather_vec_kernel<16, 4>))>>>(f, fb_id, fb_pos, total,
+                                                                           o, status);
     else if (vecs == 32)
-      gather_vec_kernel<32, 4><<<grid, kThreads, 0, st>>>(f, fb_id, fb_pos, total, o, status);
+      gather_vec_kernel<32, 4><<<AGNES_GRID((gather_vec_kernel<32, 4>))>>>(f, fb_id, fb_pos, total,
+                                                                           o, status);
     else
-      gather_rows_kernel<<<grid, kThreads, 0, st>>>(f, vecs, fb_id, fb_pos, total, o, status);
+      gather_rows_kernel<<<AGNES_GRID(gather_rows_kernel)>>>(f, vecs, fb_id, fb_pos, total, o,
+                                                             status);
   } else {
-    gather_bytes_kernel<<<grid, kThreads, 0, st>>>((const uint8_t*)feats, row_bytes, fb_id,
-                                                   fb_pos, total, (uint8_t*)out, status);
+    gather_bytes_kernel<<<AGNES_GRID(gather_bytes_kernel)>>>((const uint8_t*)feats, row_bytes,
+                                                             fb_id, fb_pos, total, (uint8_t*)out,
+                                                             status);
   }
+#undef AGNES_GRID
   return cudaGetLastError();
 }
 

@@ -8,6 +8,11 @@
 namespace agnes {
 
 // ---- scan.cu ---------------------------------------------------------------
+// CTAs of `threads` threads of `kernel` that are resident on all SMs at once
+// (occupancy API, cached per kernel): the grid of a persistent grid-stride
+// kernel, so no CTA waits for a second wave.
+int resident_grid(const void* kernel, int threads, int num_sms);
+
 // Exclusive scan of nseg segments.  Segment s reads in[s*in_stride + i] for
 // i < len(s) and writes out[s*out_stride + i]; len(s) = d_len[s] when d_len is
 // non-null, else const_len.  With write_end, out[s*out_stride + len(s)] gets
@@ -19,6 +24,15 @@ template <typename InT, typename OutT>
 cudaError_t seg_scan(const InT* in, int64_t in_stride, OutT* out, int64_t out_stride,
                      const int32_t* d_len, int64_t const_len, int32_t nseg, int64_t max_len,
                      bool write_end, int32_t* seg_total, int64_t* scratch,
+                     const int32_t* status, cudaStream_t st);
+
+// Exclusive scan down each column of a row-major [rows x cols] matrix:
+// out[r*cols + c] = sum of in[r'*cols + c] over r' < r (coalesced along
+// rows).  total_out[c] (if non-null) = column total + add_in[c] (add_in may be
+// null).  scratch needs col_scan_scratch_elems(rows, cols) int64s.
+int64_t col_scan_scratch_elems(int64_t rows, int32_t cols);
+cudaError_t col_scan(const int32_t* in, int32_t* out, int64_t rows, int32_t cols,
+                     const int32_t* add_in, int32_t* total_out, int64_t* scratch,
                      const int32_t* status, cudaStream_t st);
 
 // ---- blocks.cu -------------------------------------------------------------
@@ -93,14 +107,14 @@ struct DedupBufs {
   const int32_t* scnt;      // T*H per-cell counts of sampled ids
   int32_t* soff;            // T*H+1
   int2* sb;                 // bucketed (sampled id, edge index in the minibatch)
+  int2* tmp;                // per cell: next-frontier entries with local ranks
   int32_t* big_list;        // cells with more than 32 entries (capacity: entries / 33 + 1)
   int32_t* big_n;           // their count
   const int32_t* fb_id;     // current frontier bucket
   const int32_t* fb_pos;
   const int32_t* fcell_off;
-  int32_t* newcnt;          // H x T (minibatch-major)
-  int32_t* newbase;         // H x T
-  int32_t* newtot;          // H
+  int32_t* newcnt;          // T*H: new ids per cell
+  int32_t* newbase;         // T*H: per-minibatch exclusive scan of newcnt over tiles
   int32_t* nfcnt;           // T*H
   int32_t* nfcell_off;      // T*H+1
   int32_t* nfb_id;          // next frontier bucket

@@ -331,8 +331,6 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
   }
 }
 
-int grid_for(int num_sms, int per_sm) { return num_sms * per_sm; }
-
 }  // namespace
 
 cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32_t B, int32_t N,
@@ -343,14 +341,16 @@ cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32
                                   cudaStream_t st) {
   const TileMap tm{tile_first, chunk_tile, T};
   const int64_t ncells = (int64_t)T * H;
-  const int grid = grid_for(num_sms, 8);
+  const int grid = resident_grid((const void*)targets_count_kernel, kThreads, num_sms);
   targets_count_kernel<<<grid, kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, status);
   cudaError_t e = seg_scan<int32_t, int32_t>(fcnt, 0, fcell_off, 0, nullptr, ncells, 1, ncells,
                                              true, nullptr, scan_scratch, status, st);
   if (e != cudaSuccess) return e;
-  targets_scatter_kernel<<<grid, kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, fcell_off,
+  targets_scatter_kernel<<<resident_grid((const void*)targets_scatter_kernel, kThreads, num_sms),
+                           kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, fcell_off,
                                                     tmp_id, tmp_pos, status);
-  targets_sort_kernel<<<grid, kThreads, 0, st>>>(fcell_off, ncells, H, tm, tmp_id, tmp_pos,
+  targets_sort_kernel<<<resident_grid((const void*)targets_sort_kernel, kThreads, num_sms),
+                        kThreads, 0, st>>>(fcell_off, ncells, H, tm, tmp_id, tmp_pos,
                                                  fb_id, fb_pos, status);
   return cudaGetLastError();
 }
@@ -359,29 +359,35 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
                                 const int32_t* fcell_off, int32_t* cnt, int num_sms,
                                 cudaStream_t st) {
   const int32_t* total = fcell_off + (int64_t)a.T * a.H;
-  const int grid = grid_for(num_sms, 8);
   if (a.offsets_bits == 32)
-    sample_count_kernel<int32_t><<<grid, kThreads, 0, st>>>(
+    sample_count_kernel<int32_t><<<resident_grid((const void*)sample_count_kernel<int32_t>,
+                                                 kThreads, num_sms),
+                                   kThreads, 0, st>>>(
         fb_id, fb_pos, total, (const int32_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt, a.status);
   else
-    sample_count_kernel<int64_t><<<grid, kThreads, 0, st>>>(
+    sample_count_kernel<int64_t><<<resident_grid((const void*)sample_count_kernel<int64_t>,
+                                                 kThreads, num_sms),
+                                   kThreads, 0, st>>>(
         fb_id, fb_pos, total, (const int64_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt, a.status);
   return cudaGetLastError();
 }
 
 template <typename OffT>
-static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int grid,
+static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int num_sms,
                               cudaStream_t st) {
+#define AGNES_FILL(KERNEL)                                                                   \
+  KERNEL<<<resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st>>>(f, off)
   if (k <= 4)
-    sample_fill_kernel<OffT, 4><<<grid, kThreads, 0, st>>>(f, off);
+    AGNES_FILL((sample_fill_kernel<OffT, 4>));
   else if (k <= 8)
-    sample_fill_kernel<OffT, 8><<<grid, kThreads, 0, st>>>(f, off);
+    AGNES_FILL((sample_fill_kernel<OffT, 8>));
   else if (k <= 16)
-    sample_fill_kernel<OffT, 16><<<grid, kThreads, 0, st>>>(f, off);
+    AGNES_FILL((sample_fill_kernel<OffT, 16>));
   else if (k <= 32)
-    sample_fill_kernel<OffT, 32><<<grid, kThreads, 0, st>>>(f, off);
+    AGNES_FILL((sample_fill_kernel<OffT, 32>));
   else
-    sample_fill_wide_kernel<OffT><<<grid, kThreads, 0, st>>>(f, off);
+    AGNES_FILL((sample_fill_wide_kernel<OffT>));
+#undef AGNES_FILL
 }
 
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
@@ -409,11 +415,10 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.key_hi = (uint32_t)(a.seed >> 32);
   f.first_gid = a.first_gid;
   f.status = a.status;
-  const int grid = grid_for(num_sms, 8);
   if (a.offsets_bits == 32)
-    launch_fill_typed<int32_t>(f, (const int32_t*)a.offsets, a.k, grid, st);
+    launch_fill_typed<int32_t>(f, (const int32_t*)a.offsets, a.k, num_sms, st);
   else
-    launch_fill_typed<int64_t>(f, (const int64_t*)a.offsets, a.k, grid, st);
+    launch_fill_typed<int64_t>(f, (const int64_t*)a.offsets, a.k, num_sms, st);
   return cudaGetLastError();
 }
 

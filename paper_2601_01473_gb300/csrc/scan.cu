@@ -5,6 +5,9 @@
 // nodes of each (tile, minibatch) cell, and the tile compaction at load time.
 // Three launches per scan and no inter-block waiting, so no kernel ever spins
 // on another block's progress.
+#include <mutex>
+#include <unordered_map>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -140,7 +143,99 @@ scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict
   }
 }
 
+// ---- column scan of a row-major [rows x cols] matrix ----------------------------
+constexpr int kColRows = 64;  // rows per chunk
+
+__global__ void __launch_bounds__(128)
+col_reduce_kernel(const int32_t* __restrict__ in, int64_t rows, int32_t cols,
+                  int64_t* __restrict__ partial, const int32_t* status) {
+  if (status && failed(status)) return;
+  const int32_t c = blockIdx.y * 128 + threadIdx.x;
+  if (c >= cols) return;
+  const int64_t r0 = (int64_t)blockIdx.x * kColRows;
+  const int64_t r1 = min(rows, r0 + kColRows);
+  int64_t sum = 0;
+#pragma unroll 8
+  for (int64_t r = r0; r < r1; ++r) sum += in[r * cols + c];
+  partial[(int64_t)blockIdx.x * cols + c] = sum;
+}
+
+// One CTA per column: exclusive scan of its chunk partials (strided by cols).
+__global__ void __launch_bounds__(kThreads)
+col_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, int32_t cols,
+                    const int32_t* __restrict__ add_in, int32_t* __restrict__ total_out,
+                    const int32_t* status) {
+  if (status && failed(status)) return;
+  const int32_t c = blockIdx.x;
+  int64_t carry = 0;
+  for (int64_t base = 0; base < chunks; base += kThreads) {
+    const int64_t i = base + threadIdx.x;
+    const int64_t v = i < chunks ? partial[i * cols + c] : 0;
+    int64_t tot;
+    const int64_t ex = block_excl_scan(v, &tot);
+    if (i < chunks) partial[i * cols + c] = carry + ex;
+    carry += tot;
+  }
+  if (threadIdx.x == 0 && total_out)
+    total_out[c] = (int32_t)carry + (add_in ? add_in[c] : 0);
+}
+
+__global__ void __launch_bounds__(128)
+col_down_kernel(const int32_t* __restrict__ in, int32_t* __restrict__ out, int64_t rows,
+                int32_t cols, const int64_t* __restrict__ partial, const int32_t* status) {
+  if (status && failed(status)) return;
+  const int32_t c = blockIdx.y * 128 + threadIdx.x;
+  if (c >= cols) return;
+  const int64_t r0 = (int64_t)blockIdx.x * kColRows;
+  const int64_t r1 = min(rows, r0 + kColRows);
+  int64_t run = partial[(int64_t)blockIdx.x * cols + c];
+#pragma unroll 8
+  for (int64_t r = r0; r < r1; ++r) {
+    const int32_t v = in[r * cols + c];
+    out[r * cols + c] = (int32_t)run;
+    run += v;
+  }
+}
+
 }  // namespace
+
+int64_t col_scan_scratch_elems(int64_t rows, int32_t cols) {
+  return ((rows + kColRows - 1) / kColRows) * (int64_t)cols;
+}
+
+cudaError_t col_scan(const int32_t* in, int32_t* out, int64_t rows, int32_t cols,
+                     const int32_t* add_in, int32_t* total_out, int64_t* scratch,
+                     const int32_t* status, cudaStream_t st) {
+  if (rows <= 0 || cols <= 0) return cudaSuccess;
+  const int64_t chunks = (rows + kColRows - 1) / kColRows;
+  const dim3 grid((unsigned)chunks, (unsigned)((cols + 127) / 128));
+  col_reduce_kernel<<<grid, 128, 0, st>>>(in, rows, cols, scratch, status);
+  col_partials_kernel<<<cols, kThreads, 0, st>>>(scratch, chunks, cols, add_in, total_out, status);
+  col_down_kernel<<<grid, 128, 0, st>>>(in, out, rows, cols, scratch, status);
+  return cudaGetLastError();
+}
+
+int resident_grid(const void* kernel, int threads, int num_sms) {
+  static std::mutex mu;
+  static std::unordered_map<const void*, int> per_sm_cache;
+  int per_sm = 0;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = per_sm_cache.find(kernel);
+    if (it != per_sm_cache.end()) per_sm = it->second;
+  }
+  if (per_sm == 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0) !=
+            cudaSuccess ||
+        per_sm < 1) {
+      cudaGetLastError();
+      per_sm = 1;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    per_sm_cache[kernel] = per_sm;
+  }
+  return per_sm * num_sms;
+}
 
 int64_t scan_scratch_elems(int64_t nseg, int64_t max_len) {
   int64_t chunks = (max_len + kChunk - 1) / kChunk;
