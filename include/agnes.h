@@ -199,6 +199,32 @@ agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable);
 agnes_status agnes_phase_times(agnes_ctx* ctx, int32_t ago, float* ms, int32_t n,
                                int32_t* n_out);
 
+/* Allocation-free variant of one step of the path: for a node list (for
+ * example one minibatch's frontier), the per-node edge counts of one hop's
+ * sampling, min(deg(v), fanout), and their prefix sum -- the indptr that
+ * agnes_prepare_hyperbatch computes for each hop.  It exists for callers
+ * that must not allocate device memory: a latency-critical loop cannot
+ * afford the device-wide synchronisation cudaFree implies, and a process
+ * whose device memory is all reserved by another allocator (a framework's
+ * caching pool) may find cudaMalloc failing.  The paper has no counterpart;
+ * this is a library convenience.
+ *  nodes   n int32 node ids in [0, N), device memory.
+ *  indptr  n+1 int64, device memory: indptr[0] = 0,
+ *          indptr[i+1] = indptr[i] + min(deg(nodes[i]), fanout).
+ *  n       0 <= n <= AGNES_NOALLOC_MAX_NODES, else ERANGE.
+ *  fanout  1 <= fanout <= AGNES_MAX_FANOUT.
+ * Its scratch (64 KiB: per-chunk partial sums and an error word) is a
+ * static device array that every GPU loading the library holds until the
+ * process exits; nothing is allocated per call.  The first call on a device
+ * looks up that array's device address, so make that first call before any
+ * stream capture.  All calls on a device share the array: calls that overlap
+ * on the GPU race and must be serialised by the caller.  The call enqueues its
+ * work on cuda_stream and then waits for it (to report node ids outside
+ * [0, N) as EINVAL).  Errors: EINVAL, ERANGE, ECUDA. */
+#define AGNES_NOALLOC_MAX_NODES (1LL << 24)
+agnes_status agnes_hop_indptr_noalloc(agnes_ctx* ctx, const int32_t* nodes, int64_t n,
+                                      int32_t fanout, int64_t* indptr, void* cuda_stream);
+
 /* Releases everything the ctx owns (after synchronising its streams). */
 agnes_status agnes_free(agnes_ctx* ctx);
 

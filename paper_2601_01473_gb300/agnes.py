@@ -100,6 +100,7 @@ SIGNATURES = {
     "agnes_set_profiling": ([_P, ctypes.c_int32], ctypes.c_int),
     "agnes_phase_times": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)],
                           ctypes.c_int),
+    "agnes_hop_indptr_noalloc": ([_P, _P, ctypes.c_int64, ctypes.c_int32, _P, _P], ctypes.c_int),
     "agnes_free": ([_P], ctypes.c_int),
     "agnes_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "agnes_last_error": ([_P], ctypes.c_char_p),

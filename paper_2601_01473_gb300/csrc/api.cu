@@ -117,6 +117,22 @@ static void set_err(agnes_ctx* ctx, const char* fmt, ...) {
   if (ctx) snprintf(g_err, sizeof(g_err), "%s", ctx->err);
 }
 
+void ctx_graph_view(const agnes_ctx* ctx, agnes::GraphView* out) {
+  out->device = ctx->device;
+  out->offsets = ctx->offsets;
+  out->offsets_bits = ctx->offsets_bits;
+  out->N = ctx->N;
+}
+
+void ctx_set_error(agnes_ctx* ctx, const char* fmt, ...) {
+  char* dst = ctx ? ctx->err : g_err;
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(dst, 512, fmt, ap);
+  va_end(ap);
+  if (ctx) snprintf(g_err, sizeof(g_err), "%s", ctx->err);
+}
+
 #define CK(ctx, call)                                                            \
   do {                                                                           \
     cudaError_t e_ = (call);                                                     \

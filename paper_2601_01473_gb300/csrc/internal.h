@@ -145,4 +145,16 @@ cudaError_t launch_distinct_rows(const int32_t* fb_id, const int32_t* cell_off,
                                  const int32_t* tile_first, int32_t T, int32_t H,
                                  unsigned long long* count, cudaStream_t st);
 
+// ---- api.cu: read-only view of a loaded graph for other translation units --
+struct GraphView {
+  int device;
+  const void* offsets;
+  int offsets_bits;
+  int64_t N;
+};
+
 }  // namespace agnes
+
+struct agnes_ctx;
+void ctx_graph_view(const agnes_ctx* ctx, agnes::GraphView* out);
+void ctx_set_error(agnes_ctx* ctx, const char* fmt, ...);
