@@ -227,23 +227,33 @@ def sample_minibatch(graph: Graph, targets, fanouts, seed: int, gid: int, gather
 
 
 def hyperbatch(graph: Graph, targets, fanouts, seed: int, first_gid: int, gather: bool,
-               adj_block_bytes: int, feat_block_bytes: int):
+               adj_block_bytes: int, feat_block_bytes: int, threads: int = 1):
     """Runs every minibatch of a hyperbatch (targets: [H, B]) and the
     blocks-touched statistics.  Returns (list of per-minibatch dicts, stats
-    list of K+1 ints)."""
+    list of K+1 ints).  threads > 1 runs independent minibatches on host
+    threads (the C functions are reentrant and ctypes releases the GIL)."""
     t = np.ascontiguousarray(targets, dtype=np.int32)
     H = t.shape[0]
     f = np.ascontiguousarray(fanouts, dtype=np.int32)
     arr = (_OrcMinibatch * H)()
-    done = 0
+    status = [None] * H
+
+    def run(j):
+        status[j] = lib().orc_sample_minibatch(
+            ctypes.byref(graph._struct), _ptr(t[j]), t.shape[1], _ptr(f), f.shape[0],
+            seed, first_gid + j, int(gather), ctypes.byref(arr[j]))
+
     try:
+        if threads > 1:
+            import concurrent.futures as cf
+            with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+                list(ex.map(run, range(H)))
+        else:
+            for j in range(H):
+                run(j)
         for j in range(H):
-            rc = lib().orc_sample_minibatch(
-                ctypes.byref(graph._struct), _ptr(t[j]), t.shape[1], _ptr(f), f.shape[0],
-                seed, first_gid + j, int(gather), ctypes.byref(arr[j]))
-            if rc != 0:
-                raise OracleError(f"orc_sample_minibatch failed ({rc}) for minibatch {j}")
-            done += 1
+            if status[j] != 0:
+                raise OracleError(f"orc_sample_minibatch failed ({status[j]}) for minibatch {j}")
         rpb = feat_rows_per_block(graph, feat_block_bytes)
         stats = np.zeros(f.shape[0] + 1, dtype=np.int64)
         rc = lib().orc_hyperbatch_stats(ctypes.byref(graph._struct), arr, H, adj_block_bytes,
@@ -254,8 +264,9 @@ def hyperbatch(graph: Graph, targets, fanouts, seed: int, first_gid: int, gather
         mbs = [_to_dict(arr[j], graph.row_bytes, dt, tail) for j in range(H)]
         return mbs, [int(x) for x in stats]
     finally:
-        for j in range(done):
-            lib().orc_free_minibatch(ctypes.byref(arr[j]))
+        for j in range(H):
+            if status[j] == 0:
+                lib().orc_free_minibatch(ctypes.byref(arr[j]))
 
 
 def feat_rows_per_block(graph: Graph, feat_block_bytes: int) -> int:
