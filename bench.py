@@ -146,7 +146,7 @@ def gather_traffic_from_profile():
             if ":" in line and line.strip().startswith("- "):
                 k, v = line.strip()[2:].split(":", 1)
                 vals[k.strip()] = v.strip()
-        if vals.get("gather.cu sha256[:16]") != sha:
+        if vals.get("gather.cu sha256 prefix") != sha:
             return None
         return float(vals["dram bytes per launch (full workload)"])
     except Exception:
