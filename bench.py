@@ -184,6 +184,23 @@ def time_oracle(host_graph, w, targets_cpu, seconds_budget: float, max_mbs: int)
     return n / dt, cores, f"{n} minibatches of the workload (B={w.B}, fanouts {list(w.fanouts)}) on {cores} threads, {dt:.1f} s"
 
 
+def pinned_h2d_peak(dev, nbytes: int = 1 << 30, reps: int = 5) -> float:
+    """Measured pinned host -> device copy bandwidth (GB/s), best of reps."""
+    src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    best = 0.0
+    for _ in range(reps + 1):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        dst.copy_(src, non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize()
+        best = max(best, nbytes / (e0.elapsed_time(e1) / 1e3) / 1e9)
+    del src, dst
+    return best
+
+
 def host_copy(offsets, indices, features):
     return (offsets.cpu().numpy(), indices.cpu().numpy(), features.cpu().numpy())
 
@@ -204,6 +221,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--stream", action="store_true",
+                    help="features in pinned host memory, streamed block-wise per hyperbatch")
     args = ap.parse_args()
 
     world, rank, local = dist_env()
@@ -239,8 +258,13 @@ def main():
     torch.cuda.empty_cache()
 
     stream = torch.cuda.current_stream(dev)
+    host_link = None
+    if args.stream:
+        features = features.cpu().pin_memory()
+        torch.cuda.empty_cache()
+        host_link = {"h2d_peak_GBps": pinned_h2d_peak(dev)}
     g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes, device=local,
-              stream=stream)
+              stream=stream, features_on_host=args.stream)
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
@@ -333,6 +357,15 @@ def main():
                 "path_algorithmic_bytes_per_step": total_bytes,
                 "path_GBps": total_bytes / (elapsed_ms / args.steps / 1e3) / 1e9}
 
+    if host_link is not None:
+        sb = statistics.mean(c["streamed_bytes"] for c in counters)
+        host_link.update({"streamed_bytes_per_step": sb,
+                          "streamed_blocks_per_step": statistics.mean(c["streamed_blocks"]
+                                                                      for c in counters),
+                          "streamed_GBps": sb / (g_ms / 1e3) / 1e9 if g_ms else None})
+        host_link["frac"] = (host_link["streamed_GBps"] / host_link["h2d_peak_GBps"]
+                             if host_link["streamed_GBps"] else None)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         host_graph = host_copy(offsets, indices, features)
@@ -349,7 +382,8 @@ def main():
             "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int32",
             "data": "synthetic",
-            "config": {"workload": f"{w.name}: {w.describe()}",
+            "config": {"workload": f"{w.name}: {w.describe()}"
+                           + (" features streamed from pinned host memory" if args.stream else ""),
                        "graph": {"nodes": info["num_nodes"], "edges": info["num_edges"],
                                  "adj_blocks": info["adj_blocks"], "tiles": info["tiles"],
                                  "feat_blocks": info["feat_blocks"]},
@@ -361,7 +395,7 @@ def main():
                        "blocks_touched_last_step": stats,
                        "counters_last_step": counters[-1] if counters else None,
                        "gen_seconds": round(gen_s, 1)},
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "host_link": host_link,
             "gpu_launches": kernel_launches_per_step(K) * args.steps,
             "clocks": clocks,
             "phases_ms": {"names": ["bucket_targets"] + [f"hop{h + 1}_{p}" for h in range(K)
@@ -397,7 +431,8 @@ def run_reference(args, w, world, rank):
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "int32", "data": "synthetic", "impl": "reference",
-           "config": {"workload": f"{w.name}: {w.describe()}", "H": w.H, "B": w.B,
+           "config": {"workload": f"{w.name}: {w.describe()}"
+                           + (" features streamed from pinned host memory" if args.stream else ""), "H": w.H, "B": w.B,
                       "fanouts": list(w.fanouts)},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                             "sample": sample},

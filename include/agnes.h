@@ -166,6 +166,8 @@ typedef struct {
   int64_t rows;                     /* sum over minibatches of num_nodes */
   int64_t distinct_rows;            /* distinct node ids among all gathered rows */
   int64_t row_bytes;
+  int64_t streamed_bytes;           /* features_on_host: bytes copied host -> device */
+  int64_t streamed_blocks;          /* features_on_host: feature blocks copied */
 } agnes_counters;
 agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
 

@@ -73,6 +73,8 @@ class _Counters(ctypes.Structure):
         ("rows", ctypes.c_int64),
         ("distinct_rows", ctypes.c_int64),
         ("row_bytes", ctypes.c_int64),
+        ("streamed_bytes", ctypes.c_int64),
+        ("streamed_blocks", ctypes.c_int64),
     ]
 
 
@@ -277,7 +279,8 @@ class Graph:
         c = _Counters()
         _check(lib().agnes_hyperbatch_counters(self._ctx, ctypes.byref(c)), self._ctx)
         return {"frontier": list(c.frontier[:c.K]), "edges": list(c.edges[:c.K]),
-                "rows": c.rows, "distinct_rows": c.distinct_rows, "row_bytes": c.row_bytes}
+                "rows": c.rows, "distinct_rows": c.distinct_rows, "row_bytes": c.row_bytes,
+                "streamed_bytes": c.streamed_bytes, "streamed_blocks": c.streamed_blocks}
 
     def info(self) -> dict:
         g = _GraphInfo()

@@ -16,6 +16,7 @@
 #include <string.h>
 
 #include <new>
+#include <vector>
 
 #include "../../include/agnes.h"
 #include "common.cuh"
@@ -27,6 +28,10 @@ namespace {
 
 constexpr int kMaxPhases = 2 + 3 * AGNES_MAX_HOPS;
 constexpr int kEventRing = 64;  // prepares whose phase times stay readable
+// Streaming of host-resident features: a ring of staging slots in HBM, each
+// holding a batch of up to kStreamBatchBlocks touched feature blocks.
+constexpr int kStreamSlots = 4;
+constexpr int kStreamBatchBlocks = 64;
 
 struct Workspace {
   int32_t H = 0, B = 0, K = 0;
@@ -102,6 +107,19 @@ struct agnes_ctx {
   int n_phases[kEventRing] = {0};          // per ring slot; 0 = not profiled
   cudaEvent_t ev[kEventRing][kMaxPhases + 1] = {{nullptr}};
   bool ev_created = false;
+
+  // streaming of host-resident features (features_on_host)
+  cudaStream_t copy_stream = nullptr;
+  char* slots = nullptr;
+  int64_t slot_bytes = 0;
+  cudaEvent_t slot_copied[kStreamSlots] = {nullptr};
+  cudaEvent_t slot_free[kStreamSlots] = {nullptr};
+  bool slot_used[kStreamSlots] = {false};
+  uint8_t* h_flags = nullptr;    // pinned, one byte per feature block
+  int32_t* h_touched = nullptr;  // pinned, touched feature blocks of the last hyperbatch
+  int32_t* d_touched = nullptr;
+  std::vector<int32_t> fblock_first_tile;
+  int64_t streamed_bytes = 0, streamed_blocks = 0;
 
   char err[512] = {0};
 };
@@ -398,6 +416,15 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (ctx->own_indices) cudaFree(ctx->indices);
   if (ctx->own_features) cudaFree(ctx->features);
   if (ctx->done) cudaEventDestroy(ctx->done);
+  for (int i = 0; i < kStreamSlots; ++i) {
+    if (ctx->slot_copied[i]) cudaEventDestroy(ctx->slot_copied[i]);
+    if (ctx->slot_free[i]) cudaEventDestroy(ctx->slot_free[i]);
+  }
+  if (ctx->copy_stream) cudaStreamDestroy(ctx->copy_stream);
+  cudaFree(ctx->slots);
+  cudaFree(ctx->d_touched);
+  if (ctx->h_flags) cudaFreeHost(ctx->h_flags);
+  if (ctx->h_touched) cudaFreeHost(ctx->h_touched);
   if (ctx->ev_created)
     for (int r = 0; r < kEventRing; ++r)
       for (int i = 0; i <= kMaxPhases; ++i) cudaEventDestroy(ctx->ev[r][i]);
@@ -415,6 +442,26 @@ static agnes_status adopt_or_copy(agnes_ctx* ctx, const void* src, size_t bytes,
   CK(ctx, cudaMalloc(dst, bytes ? bytes : 1));
   *own = true;
   CK(ctx, cudaMemcpyAsync(*dst, src, bytes, cudaMemcpyHostToDevice, st));
+  return AGNES_OK;
+}
+
+// Staging ring, copy stream and host tables for host-resident features.
+static agnes_status setup_streaming(agnes_ctx* ctx, cudaStream_t st) {
+  const int64_t nfb = ctx->bt.n_feat_blocks;
+  ctx->slot_bytes = (int64_t)kStreamBatchBlocks * ctx->bt.rows_per_feat_block * ctx->row_bytes;
+  CK(ctx, cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking));
+  for (int i = 0; i < kStreamSlots; ++i) {
+    CK(ctx, cudaEventCreateWithFlags(&ctx->slot_copied[i], cudaEventDisableTiming));
+    CK(ctx, cudaEventCreateWithFlags(&ctx->slot_free[i], cudaEventDisableTiming));
+  }
+  CK(ctx, cudaMalloc((void**)&ctx->slots, (size_t)(ctx->slot_bytes * kStreamSlots)));
+  CK(ctx, cudaMalloc((void**)&ctx->d_touched, sizeof(int32_t) * (size_t)(nfb + 1)));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_flags, (size_t)(nfb + 1)));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_touched, sizeof(int32_t) * (size_t)(nfb + 1)));
+  ctx->fblock_first_tile.resize((size_t)(nfb + 1));
+  CK(ctx, cudaMemcpyAsync(ctx->fblock_first_tile.data(), ctx->bt.fblock_first_tile,
+                          sizeof(int32_t) * (size_t)(nfb + 1), cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
   return AGNES_OK;
 }
 
@@ -465,6 +512,10 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   }
   if (d->features_on_host && !is_pinned_host_ptr(d->features)) {
     set_err(nullptr, "features_on_host requires pinned host memory");
+    return AGNES_EINVAL;
+  }
+  if (d->features_on_host && (row_bytes % 16) != 0) {
+    set_err(nullptr, "features_on_host needs feature rows of a multiple of 16 bytes");
     return AGNES_EINVAL;
   }
   if (cudaSetDevice(device) != cudaSuccess) {
@@ -540,6 +591,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
                                        sizeof(ctx->err));
     if (e != cudaSuccess) rc = e == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;
   }
+  if (rc == AGNES_OK && d->features_on_host) rc = setup_streaming(ctx, st);
   if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
     set_err(ctx, "cudaEventCreate failed");
     rc = AGNES_ECUDA;
@@ -550,6 +602,58 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
     return rc;
   }
   *out = ctx;
+  return AGNES_OK;
+}
+
+// Gather with host-resident features (Sec. 3.4 (4) asynchronous I/O, the
+// host link standing in for the SSD): the touched feature blocks are read
+// back once, then copied batch by batch into the ring of HBM slots on the
+// side stream; each batch's gather waits for its slot's copy event and the
+// next copy into a slot waits for the gather that last read it.
+static agnes_status gather_streamed(agnes_ctx* ctx, int cur, cudaStream_t st) {
+  Workspace& w = ctx->ws;
+  const int64_t nfb = ctx->bt.n_feat_blocks;
+  const int64_t rpb = ctx->bt.rows_per_feat_block;
+  const int64_t rb = ctx->row_bytes;
+  const int32_t H = w.H;
+  CK(ctx, cudaMemcpyAsync(ctx->h_flags, w.feat_flags, (size_t)nfb, cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
+  int32_t n = 0;
+  for (int64_t b = 0; b < nfb; ++b)
+    if (ctx->h_flags[b]) ctx->h_touched[n++] = (int32_t)b;
+  if (n > 0)
+    CK(ctx, cudaMemcpyAsync(ctx->d_touched, ctx->h_touched, sizeof(int32_t) * n,
+                            cudaMemcpyHostToDevice, st));
+  int64_t bytes = 0;
+  for (int32_t i0 = 0, batch = 0; i0 < n; i0 += kStreamBatchBlocks, ++batch) {
+    const int32_t nb = n - i0 < kStreamBatchBlocks ? n - i0 : kStreamBatchBlocks;
+    const int s = batch % kStreamSlots;
+    char* slot = ctx->slots + (int64_t)s * ctx->slot_bytes;
+    if (ctx->slot_used[s]) CK(ctx, cudaStreamWaitEvent(ctx->copy_stream, ctx->slot_free[s], 0));
+    for (int32_t p = 0; p < nb;) {  // one copy per run of consecutive blocks
+      int32_t q = p;
+      while (q + 1 < nb && ctx->h_touched[i0 + q + 1] == ctx->h_touched[i0 + q] + 1) ++q;
+      const int64_t r0 = (int64_t)ctx->h_touched[i0 + p] * rpb;
+      int64_t r1 = ((int64_t)ctx->h_touched[i0 + q] + 1) * rpb;
+      if (r1 > ctx->N) r1 = ctx->N;
+      const int64_t nbytes = (r1 - r0) * rb;
+      CK(ctx, cudaMemcpyAsync(slot + (int64_t)p * rpb * rb, (const char*)ctx->features + r0 * rb,
+                              (size_t)nbytes, cudaMemcpyHostToDevice, ctx->copy_stream));
+      bytes += nbytes;
+      p = q + 1;
+    }
+    CK(ctx, cudaEventRecord(ctx->slot_copied[s], ctx->copy_stream));
+    CK(ctx, cudaStreamWaitEvent(st, ctx->slot_copied[s], 0));
+    const int64_t cell_lo = (int64_t)ctx->fblock_first_tile[ctx->h_touched[i0]] * H;
+    const int64_t cell_hi = (int64_t)ctx->fblock_first_tile[ctx->h_touched[i0 + nb - 1] + 1] * H;
+    CK(ctx, launch_gather_staged(slot, rb, rpb, ctx->d_touched + i0, nb, w.fb_id[cur],
+                                 w.fb_pos[cur], w.fcell_off[cur], cell_lo, cell_hi, w.feats_out,
+                                 w.status, ctx->num_sms, st));
+    CK(ctx, cudaEventRecord(ctx->slot_free[s], st));
+    ctx->slot_used[s] = true;
+  }
+  ctx->streamed_bytes = bytes;
+  ctx->streamed_blocks = n;
   return AGNES_OK;
 }
 
@@ -593,10 +697,6 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   if ((int64_t)H * cap[K] > lim) {
     set_err(ctx, "H x node capacity (%lld) exceeds 2^31", (long long)(H * cap[K]));
     return AGNES_ERANGE;
-  }
-  if (ctx->features_on_host) {
-    set_err(ctx, "streaming of host-resident features is not available in this build");
-    return AGNES_EINVAL;
   }
   if (cudaSetDevice(ctx->device) != cudaSuccess) {
     cudaGetLastError();
@@ -699,15 +799,21 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     CK(ctx, launch_dedup(a, d, nsm, st));
     cur = 1 - cur;
   }
+  // feature blocks touched by the hyperbatch (stats; also the streaming list)
+  CK(ctx, launch_mark_count(w.fcell_off[cur], T, H, ctx->bt.tile_feat_block, w.feat_flags,
+                            ctx->bt.n_feat_blocks, w.stats + K, w.status, st));
   mark();
-  CK(ctx, launch_gather(ctx->features, ctx->row_bytes, w.fb_id[cur], w.fb_pos[cur],
-                        w.fcell_off[cur] + cells, w.feats_out, w.status, nsm, st));
+  if (ctx->features_on_host) {
+    rc = gather_streamed(ctx, cur, st);
+    if (rc != AGNES_OK) return rc;
+  } else {
+    CK(ctx, launch_gather(ctx->features, ctx->row_bytes, w.fb_id[cur], w.fb_pos[cur],
+                          w.fcell_off[cur] + cells, w.feats_out, w.status, nsm, st));
+  }
   mark();
   for (int h = 0; h < K; ++h)
     CK(ctx, launch_mark_count(nullptr, T, H, nullptr, w.adj_flags + (int64_t)h * ctx->bt.n_blocks,
                               ctx->bt.n_blocks, w.stats + h, w.status, st));
-  CK(ctx, launch_mark_count(w.fcell_off[cur], T, H, ctx->bt.tile_feat_block, w.feat_flags,
-                            ctx->bt.n_feat_blocks, w.stats + K, w.status, st));
   const Back b = back_of(w);
   CK(ctx, cudaMemcpyAsync(b.status, w.status, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.nsz, w.nsz, sizeof(int32_t) * (K + 1) * H, cudaMemcpyDeviceToHost, st));
@@ -788,6 +894,8 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
                                (int32_t)ctx->bt.T, w.H, w.distinct, nullptr));
   CK(ctx, cudaMemcpy(&distinct, w.distinct, sizeof(distinct), cudaMemcpyDeviceToHost));
   out->distinct_rows = (int64_t)distinct;
+  out->streamed_bytes = ctx->features_on_host ? ctx->streamed_bytes : 0;
+  out->streamed_blocks = ctx->features_on_host ? ctx->streamed_blocks : 0;
   return AGNES_OK;
 }
 

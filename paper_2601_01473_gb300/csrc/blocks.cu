@@ -133,6 +133,19 @@ __global__ void tile_blocks_kernel(const int32_t* __restrict__ tile_first, int64
   }
 }
 
+// First tile of each feature block (multiples of rows_per_block start tiles).
+__global__ void fblock_first_tile_kernel(const int32_t* __restrict__ tile_first,
+                                         const int32_t* __restrict__ tile_feat_block, int64_t T,
+                                         int64_t rpb, int64_t nfb,
+                                         int32_t* __restrict__ fblock_first_tile) {
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t b = tile_feat_block[t];
+    if ((int64_t)tile_first[t] == (int64_t)b * rpb) fblock_first_tile[b] = (int32_t)t;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) fblock_first_tile[nfb] = (int32_t)T;
+}
+
 }  // namespace
 
 void free_block_tables(BlockTables* bt) {
@@ -142,6 +155,7 @@ void free_block_tables(BlockTables* bt) {
   cudaFree(bt->chunk_tile);
   cudaFree(bt->tile_adj_block);
   cudaFree(bt->tile_feat_block);
+  cudaFree(bt->fblock_first_tile);
   *bt = BlockTables();
 }
 
@@ -213,10 +227,14 @@ cudaError_t build_block_tables(const void* d_offsets, int offsets_bits, int64_t 
   BT_CHECK(cudaMalloc(&bt->chunk_tile, sizeof(int32_t) * (C + 1)));
   BT_CHECK(cudaMalloc(&bt->tile_adj_block, sizeof(int32_t) * bt->T));
   BT_CHECK(cudaMalloc(&bt->tile_feat_block, sizeof(int32_t) * bt->T));
+  BT_CHECK(cudaMalloc(&bt->fblock_first_tile, sizeof(int32_t) * (bt->n_feat_blocks + 1)));
   tile_compact_kernel<<<grid, 256, 0, st>>>(flags, rank, N, bt->tile_first, bt->chunk_tile);
   tile_blocks_kernel<<<grid, 256, 0, st>>>(bt->tile_first, bt->T, bt->start_node,
                                            bt->start_block, bt->n_starts, rows_per_feat_block,
                                            bt->tile_adj_block, bt->tile_feat_block);
+  fblock_first_tile_kernel<<<grid, 256, 0, st>>>(bt->tile_first, bt->tile_feat_block, bt->T,
+                                                 rows_per_feat_block, bt->n_feat_blocks,
+                                                 bt->fblock_first_tile);
   BT_CHECK(cudaGetLastError());
   BT_CHECK(cudaStreamSynchronize(st));
 

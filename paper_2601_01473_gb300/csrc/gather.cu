@@ -84,6 +84,38 @@ gather_bytes_kernel(const uint8_t* __restrict__ feats, int64_t row_bytes,
   }
 }
 
+// Streaming variant: rows come from an HBM staging slot holding the batch's
+// feature blocks (copied from pinned host memory on the side stream).  LPR
+// lanes per row, each lane moving the row's 16-byte vectors l, l+LPR, ...
+template <int LPR>
+__global__ void __launch_bounds__(kThreads)
+gather_staged_kernel(const uint4* __restrict__ slot, int64_t vecs, int64_t rpb,
+                     const int32_t* __restrict__ touched, int32_t nb,
+                     const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
+                     const int32_t* __restrict__ cell_off, int64_t cell_lo, int64_t cell_hi,
+                     uint4* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  constexpr int kRowsPerWarp = 32 / LPR;
+  const int64_t e0 = cell_off[cell_lo], e1 = cell_off[cell_hi];
+  const int lane = lane_id();
+  const int sub = lane / LPR, l = lane % LPR;
+  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = e0 + warp0 * kRowsPerWarp + sub; i < e1; i += nwarps * kRowsPerWarp) {
+    const int32_t v = __ldg(fb_id + i);
+    const int64_t g = __ldg(fb_pos + i);
+    const int32_t b = (int32_t)(v / rpb);
+    int32_t lo = 0, hi = nb;  // position of block b in the batch
+    while (hi - lo > 1) {
+      const int32_t mid = (lo + hi) >> 1;
+      if (__ldg(touched + mid) <= b) lo = mid; else hi = mid;
+    }
+    const int64_t row = (int64_t)lo * rpb + (v - (int64_t)b * rpb);
+    for (int64_t c = l; c < vecs; c += LPR)
+      __stcs(out + g * vecs + c, __ldg(slot + row * vecs + c));
+  }
+}
+
 __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
                             const int32_t* __restrict__ map, uint8_t* __restrict__ flags,
                             const int32_t* status) {
@@ -162,6 +194,29 @@ cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* f
                                                              status);
   }
 #undef AGNES_GRID
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_staged(const void* slot, int64_t row_bytes, int64_t rpb,
+                                 const int32_t* touched, int32_t nb, const int32_t* fb_id,
+                                 const int32_t* fb_pos, const int32_t* cell_off, int64_t cell_lo,
+                                 int64_t cell_hi, void* out, const int32_t* status, int num_sms,
+                                 cudaStream_t st) {
+  const int64_t vecs = row_bytes / 16;
+  const uint4* sl = (const uint4*)slot;
+  uint4* o = (uint4*)out;
+#define AGNES_STAGED(LPR)                                                                    \
+  gather_staged_kernel<LPR><<<resident_grid((const void*)gather_staged_kernel<LPR>, kThreads, \
+                                            num_sms),                                        \
+                              kThreads, 0, st>>>(sl, vecs, rpb, touched, nb, fb_id, fb_pos,   \
+                                                 cell_off, cell_lo, cell_hi, o, status)
+  if (vecs <= 8)
+    AGNES_STAGED(8);
+  else if (vecs <= 16)
+    AGNES_STAGED(16);
+  else
+    AGNES_STAGED(32);
+#undef AGNES_STAGED
   return cudaGetLastError();
 }
 

@@ -45,6 +45,7 @@ struct BlockTables {
   int32_t* chunk_tile = nullptr;   // C+1
   int32_t* tile_adj_block = nullptr;
   int32_t* tile_feat_block = nullptr;
+  int32_t* fblock_first_tile = nullptr;  // n_feat_blocks+1: first tile of each feature block
   int64_t T = 0;
   int64_t n_feat_blocks = 0;
   int64_t rows_per_feat_block = 0;
@@ -134,6 +135,16 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
 cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
                           const int32_t* fb_pos, const int32_t* total, void* out,
                           const int32_t* status, int num_sms, cudaStream_t st);
+
+// Gathers the rows of a batch of feature blocks staged in an HBM slot: the
+// batch's blocks are touched[0 .. nb) (ascending), packed in the slot one
+// block (rpb rows) after another; its bucket entries are those of cells
+// [cell_lo, cell_hi) of cell_off.  Rows must be a multiple of 16 bytes.
+cudaError_t launch_gather_staged(const void* slot, int64_t row_bytes, int64_t rpb,
+                                 const int32_t* touched, int32_t nb, const int32_t* fb_id,
+                                 const int32_t* fb_pos, const int32_t* cell_off, int64_t cell_lo,
+                                 int64_t cell_hi, void* out, const int32_t* status, int num_sms,
+                                 cudaStream_t st);
 
 // Marks flags[map[t]] for every tile t whose cells (t, 0..H-1) in cell_off
 // hold an entry, then counts set flags into *count (int64).

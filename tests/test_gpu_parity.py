@@ -221,3 +221,27 @@ def test_workload_parity_all_minibatches(cuda_device, name):
     assert c["rows"] == sum(g.sizes(j)["num_nodes"] for j in range(w.H))
     assert 0 < c["distinct_rows"] <= c["rows"]
     g.close()
+
+
+@pytest.mark.parametrize("dtype,dim,fbb,H", [
+    (torch.float32, 16, 1024, 6),     # ~1900 feature blocks: many batches, the slot ring wraps
+    (torch.float16, 128, 4096, 3),
+    (torch.float16, 128, 1 << 20, 1),  # one block per batch
+])
+def test_streamed_features_match_oracle(cuda_device, dtype, dim, fbb, H):
+    """Features in pinned host memory, streamed block by block through the HBM
+    slot ring: same bytes as the oracle, over two hyperbatches in a row."""
+    off, ind, feats = make(30000, 10, seed=dim + H, dtype=dtype, dim=dim)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    host_feats = feats.pin_memory()
+    g = Graph(off.to(cuda_device), ind.to(cuda_device), host_feats, adj_block_bytes=8192,
+              feat_block_bytes=fbb, features_on_host=True)
+    for step in range(2):
+        targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), H, 200, 7, step)
+        g.prepare(targets.to(cuda_device), [8, 4], 21, 100 * step)
+        compare(g, og, targets.numpy(), [8, 4], 21, 100 * step, 8192, fbb)
+        c = g.counters()
+        assert c["streamed_blocks"] == g.stats()[-1]
+        assert 0 < c["streamed_bytes"] <= c["streamed_blocks"] * (fbb // (dim * feats.element_size())) \
+            * dim * feats.element_size()
+    g.close()
