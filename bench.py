@@ -170,7 +170,7 @@ def time_oracle(host_graph, w, targets_cpu, seconds_budget: float, max_mbs: int)
     oracle.sample_minibatch(og, targets_cpu[0], list(w.fanouts), w.seed, 0)
     one = time.perf_counter() - t0
     n = int(max(cores, min(max_mbs, (seconds_budget / max(one, 1e-3)) * cores)))
-    n = max(1, min(n, targets_cpu.shape[0] * 64))
+    n = max(1, n)
     rows = [targets_cpu[i % targets_cpu.shape[0]] for i in range(n)]
 
     def run(i):
@@ -221,6 +221,11 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="hyperbatch size x block size sweep on the workload's graph (one JSON "
+                         "line per combination)")
+    ap.add_argument("--sweep-H", default="1,2,4,8,16,32,64,128,256")
+    ap.add_argument("--sweep-blocks", default="262144,524288,1048576,2097152,4194304")
     ap.add_argument("--stream", action="store_true",
                     help="features in pinned host memory, streamed block-wise per hyperbatch")
     args = ap.parse_args()
@@ -236,6 +241,8 @@ def main():
 
     if args.impl == "reference":
         return run_reference(args, w, world, rank)
+    if args.sweep:
+        return run_sweep(args, w)
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
@@ -370,7 +377,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         host_graph = host_copy(offsets, indices, features)
         tcpu = step_targets[args.warmup].cpu().numpy()
-        v, cores, sample = time_oracle(host_graph, w, tcpu, args.cpu_seconds, 256)
+        v, cores, sample = time_oracle(host_graph, w, tcpu, args.cpu_seconds, 8192)
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
 
     if rank == 0:
@@ -408,6 +415,45 @@ def main():
         pg.destroy_process_group()
 
 
+def run_sweep(args, w):
+    """Minibatches/s and blocks touched per hop (the block-wise I/Os of the
+    paper's Fig. 7) over hyperbatch sizes and block sizes on one graph."""
+    from paper_2601_01473_gb300 import Graph
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    offsets, indices, features = build_graph(w, dev)
+    pool = target_pool(w, dev)
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    stream = torch.cuda.current_stream(dev)
+    fan = list(w.fanouts)
+    for bb in [int(x) for x in args.sweep_blocks.split(",")]:
+        g = Graph(offsets, indices, features, bb, bb, device=0, stream=stream)
+        info = g.info()
+        for H in [int(x) for x in args.sweep_H.split(",")]:
+            wh = w.with_(H=H, adj_block_bytes=bb, feat_block_bytes=bb)
+            steps = [targets_for_step(wh, pool, s) for s in range(args.warmup + args.steps)]
+            for s in range(args.warmup):
+                g.prepare(steps[s], fan, w.seed, s * H, stream)
+            torch.cuda.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for s in range(args.warmup, args.warmup + args.steps):
+                g.prepare(steps[s], fan, w.seed, s * H, stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / args.steps
+            stats = g.stats()
+            print(json.dumps({"sweep": w.name, "block_bytes": bb, "H": H, "B": w.B,
+                              "minibatches_per_s": H / (ms / 1e3), "ms_per_step": ms,
+                              "adj_blocks_touched_per_hop": stats[:-1],
+                              "feat_blocks_touched": stats[-1],
+                              "adj_blocks": info["adj_blocks"], "feat_blocks": info["feat_blocks"],
+                              "block_io_bytes": (sum(stats[:-1]) + stats[-1]) * bb}), flush=True)
+        g.close()
+
+
 def run_reference(args, w, world, rank):
     """The oracle as the reference arm: bounded sample on the host cores."""
     if rank != 0:
@@ -420,12 +466,13 @@ def run_reference(args, w, world, rank):
     host_graph = host_copy(offsets, indices, features)
     del offsets, indices, features
     tcpu = targets.cpu().numpy()
-    budget = max(5.0, min(60.0, 120.0 / max(1, args.steps)))
+    # each step: a bounded sample of the workload's minibatches, ~8 s of host
+    # work at most, so --steps K --warmup W ends within a few minutes
+    budget = max(2.0, min(8.0, 150.0 / max(1, args.steps)))
     vals, cores, sample = [], 1, ""
-    for _ in range(args.warmup if args.warmup < 1 else 1):
-        time_oracle(host_graph, w, tcpu, 2.0, 8)
+    time_oracle(host_graph, w, tcpu, 1.0, 64)
     for _ in range(args.steps):
-        v, cores, sample = time_oracle(host_graph, w, tcpu, budget / 4, 64)
+        v, cores, sample = time_oracle(host_graph, w, tcpu, budget, 8192)
         vals.append(v)
     value = statistics.median(vals)
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
