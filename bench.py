@@ -46,6 +46,21 @@ def dist_env():
     return ws, rank, local
 
 
+def step_index(rank: int, s: int) -> int:
+    """Hyperbatch index of step s on a rank: ranks draw disjoint target sets
+    (weak scaling, one independent replica per GPU)."""
+    return rank * 1_000_003 + s
+
+
+def reduce_max(x: float, pg, device) -> float:
+    """Max of x over the ranks of the process group (x itself without one)."""
+    if pg is None:
+        return x
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
 def measured_peak():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -259,7 +274,7 @@ def main():
     pool = target_pool(w, dev)
     n_steps = args.warmup + args.steps
     # each rank draws its own hyperbatches (weak scaling: fixed work per GPU)
-    step_targets = [targets_for_step(w, pool, rank * 1000 + s) for s in range(n_steps)]
+    step_targets = [targets_for_step(w, pool, step_index(rank, s)) for s in range(n_steps)]
     torch.cuda.synchronize()
     gen_s = time.perf_counter() - t_gen
     torch.cuda.empty_cache()
@@ -275,7 +290,7 @@ def main():
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
-    gid = lambda s: (rank * 1000 + s) * w.H  # noqa: E731
+    gid = lambda s: step_index(rank, s) * w.H  # noqa: E731
 
     # warm-up (also allocates the workspace)
     for s in range(args.warmup):
@@ -305,10 +320,7 @@ def main():
     elapsed_ms = ev0.elapsed_time(ev1)
     phases = [g.phase_times(ago) for ago in range(min(args.steps, 64))]
     g.set_profiling(False)
-    if pg:
-        t = torch.tensor([elapsed_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = reduce_max(elapsed_ms, pg, dev)
     clocks = clk.summary()
     gather_ms = [p[1 + 3 * K] for p in phases if len(p) > 1 + 3 * K]
 
@@ -341,10 +353,7 @@ def main():
                 g.fetch(j)
         torch.cuda.synchronize()
         e2e_s = time.perf_counter() - t0
-        if pg:
-            t = torch.tensor([e2e_s], device=dev)
-            pg.all_reduce(t, op=pg.ReduceOp.MAX)
-            e2e_s = float(t.item())
+        e2e_s = reduce_max(e2e_s, pg, dev)
         d2h = 4 * (1 + (K + 1) * w.H + K * w.H) + 8 * (K + 1)
         e2e = {"value": world * w.H * args.steps / e2e_s, "unit": UNIT,
                "h2d_bytes_per_step": w.H * w.B * 4, "d2h_bytes_per_step": d2h}
