@@ -323,7 +323,8 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
     set_err(ctx, "out of pinned host memory");
     return AGNES_ENOMEM;
   }
-  if (cudaMemset(w.fcnt, 0, sizeof(int32_t) * cells) != cudaSuccess ||
+  if (cudaMemset(w.scan_scratch, 0, sizeof(int64_t) * scratch) != cudaSuccess ||
+      cudaMemset(w.fcnt, 0, sizeof(int32_t) * cells) != cudaSuccess ||
       cudaMemset(w.scnt, 0, sizeof(int32_t) * cells) != cudaSuccess) {
     free_workspace(&w);
     set_err(ctx, "cudaMemset failed");

@@ -215,6 +215,7 @@ cudaError_t build_block_tables(const void* d_offsets, int offsets_bits, int64_t 
   BT_CHECK(cudaMalloc(&flags, N));
   BT_CHECK(cudaMalloc(&rank, sizeof(int32_t) * (N + 1)));
   BT_CHECK(cudaMalloc(&scratch, sizeof(int64_t) * scan_scratch_elems(1, N)));
+  BT_CHECK(cudaMemsetAsync(scratch, 0, sizeof(int64_t) * scan_scratch_elems(1, N), st));
   tile_flags_kernel<<<grid, 256, 0, st>>>(flags, N, rows_per_feat_block);
   tile_flag_starts_kernel<<<grid, 256, 0, st>>>(flags, bt->start_node, bt->n_starts);
   BT_CHECK(cudaGetLastError());

@@ -17,7 +17,8 @@ int resident_grid(const void* kernel, int threads, int num_sms);
 // i < len(s) and writes out[s*out_stride + i]; len(s) = d_len[s] when d_len is
 // non-null, else const_len.  With write_end, out[s*out_stride + len(s)] gets
 // the segment total; seg_total (if non-null) gets it too.  max_len bounds
-// every len(s).  scratch needs scan_scratch_elems(nseg, max_len) int64s.
+// every len(s).  scratch needs scan_scratch_elems(nseg, max_len) int64s,
+// zeroed once before first use (the scan leaves its tickets at zero again).
 int64_t scan_scratch_elems(int64_t nseg, int64_t max_len);
 
 template <typename InT, typename OutT>

@@ -18,6 +18,10 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kItems = 8;
 constexpr int kChunk = kThreads * kItems;  // elements per block and chunk
+// Scratch layout shared by every scan: one ticket per segment (at most
+// kMaxSegments) first, kept at zero between scans, then the chunk sums.
+constexpr int64_t kMaxSegments = 65536;
+constexpr int64_t kTicketElems = kMaxSegments / 2;  // int64 slots holding the uint32 tickets
 
 __device__ __forceinline__ int64_t seg_len(const int32_t* d_len, int64_t const_len, int s) {
   return d_len ? (int64_t)d_len[s] : const_len;
@@ -44,11 +48,15 @@ __device__ __forceinline__ int64_t block_excl_scan(int64_t v, int64_t* total) {
   return out;
 }
 
-template <typename InT>
+// Chunk sums; the last chunk of a segment to finish (atomic ticket after a
+// fence, no waiting) then scans the segment's chunk sums in place, writes
+// the segment total, and resets the ticket for the next scan.
+template <typename InT, typename OutT>
 __global__ void __launch_bounds__(kThreads)
 scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t* d_len,
                    int64_t const_len, int64_t chunks, int64_t* __restrict__ partial,
-                   const int32_t* status) {
+                   unsigned int* __restrict__ tickets, OutT* __restrict__ out, int64_t out_stride,
+                   bool write_end, int32_t* seg_total, const int32_t* status) {
   if (status && failed(status)) return;
   const int s = blockIdx.y;
   const int64_t c = blockIdx.x;
@@ -61,37 +69,36 @@ scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t*
     for (int64_t i = begin + threadIdx.x; i < end; i += kThreads) sum += (int64_t)p[i];
   }
   __shared__ int64_t wsum[kThreads / 32];
+  __shared__ bool last;
   sum = warp_sum(sum);
   if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = sum;
   __syncthreads();
   if (threadIdx.x < 32) {
     int64_t v = threadIdx.x < kThreads / 32 ? wsum[threadIdx.x] : 0;
     v = warp_sum(v);
-    if (threadIdx.x == 0) partial[(int64_t)s * chunks + c] = v;
+    if (threadIdx.x == 0) {
+      partial[(int64_t)s * chunks + c] = v;
+      __threadfence();
+      last = atomicAdd(tickets + s, 1u) == (unsigned)(chunks - 1);
+    }
   }
-}
-
-template <typename OutT>
-__global__ void __launch_bounds__(kThreads)
-scan_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, const int32_t* d_len,
-                     int64_t const_len, OutT* __restrict__ out, int64_t out_stride, bool write_end,
-                     int32_t* seg_total, const int32_t* status) {
-  if (status && failed(status)) return;
-  const int s = blockIdx.x;
-  int64_t* p = partial + (int64_t)s * chunks;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  int64_t* ps = partial + (int64_t)s * chunks;
   int64_t carry = 0;
   for (int64_t base = 0; base < chunks; base += kThreads) {
     const int64_t i = base + threadIdx.x;
-    const int64_t v = i < chunks ? p[i] : 0;
+    const int64_t v = i < chunks ? *(volatile int64_t*)(ps + i) : 0;
     int64_t tot;
     const int64_t ex = block_excl_scan(v, &tot);
-    if (i < chunks) p[i] = carry + ex;
+    if (i < chunks) ps[i] = carry + ex;
     carry += tot;
   }
   if (threadIdx.x == 0) {
-    const int64_t len = seg_len(d_len, const_len, s);
     if (write_end) out[(int64_t)s * out_stride + len] = (OutT)carry;
     if (seg_total) seg_total[s] = (int32_t)carry;
+    tickets[s] = 0;
   }
 }
 
@@ -200,7 +207,7 @@ col_down_kernel(const int32_t* __restrict__ in, int32_t* __restrict__ out, int64
 }  // namespace
 
 int64_t col_scan_scratch_elems(int64_t rows, int32_t cols) {
-  return ((rows + kColRows - 1) / kColRows) * (int64_t)cols;
+  return kTicketElems + ((rows + kColRows - 1) / kColRows) * (int64_t)cols;
 }
 
 cudaError_t col_scan(const int32_t* in, int32_t* out, int64_t rows, int32_t cols,
@@ -209,9 +216,10 @@ cudaError_t col_scan(const int32_t* in, int32_t* out, int64_t rows, int32_t cols
   if (rows <= 0 || cols <= 0) return cudaSuccess;
   const int64_t chunks = (rows + kColRows - 1) / kColRows;
   const dim3 grid((unsigned)chunks, (unsigned)((cols + 127) / 128));
-  col_reduce_kernel<<<grid, 128, 0, st>>>(in, rows, cols, scratch, status);
-  col_partials_kernel<<<cols, kThreads, 0, st>>>(scratch, chunks, cols, add_in, total_out, status);
-  col_down_kernel<<<grid, 128, 0, st>>>(in, out, rows, cols, scratch, status);
+  int64_t* partial = scratch + kTicketElems;  // leave the seg_scan tickets untouched
+  col_reduce_kernel<<<grid, 128, 0, st>>>(in, rows, cols, partial, status);
+  col_partials_kernel<<<cols, kThreads, 0, st>>>(partial, chunks, cols, add_in, total_out, status);
+  col_down_kernel<<<grid, 128, 0, st>>>(in, out, rows, cols, partial, status);
   return cudaGetLastError();
 }
 
@@ -240,7 +248,7 @@ int resident_grid(const void* kernel, int threads, int num_sms) {
 int64_t scan_scratch_elems(int64_t nseg, int64_t max_len) {
   int64_t chunks = (max_len + kChunk - 1) / kChunk;
   if (chunks < 1) chunks = 1;
-  return nseg * chunks;
+  return kTicketElems + nseg * chunks;
 }
 
 template <typename InT, typename OutT>
@@ -252,12 +260,14 @@ cudaError_t seg_scan(const InT* in, int64_t in_stride, OutT* out, int64_t out_st
   int64_t chunks = (max_len + kChunk - 1) / kChunk;
   if (chunks < 1) chunks = 1;
   const dim3 grid((unsigned)chunks, (unsigned)nseg);
-  scan_reduce_kernel<InT><<<grid, kThreads, 0, st>>>(in, in_stride, d_len, const_len, chunks,
-                                                      scratch, status);
-  scan_partials_kernel<OutT><<<nseg, kThreads, 0, st>>>(scratch, chunks, d_len, const_len, out,
-                                                        out_stride, write_end, seg_total, status);
+  if (nseg > kMaxSegments) return cudaErrorInvalidValue;
+  unsigned int* tickets = (unsigned int*)scratch;
+  int64_t* partial = scratch + kTicketElems;
+  scan_reduce_kernel<InT, OutT><<<grid, kThreads, 0, st>>>(in, in_stride, d_len, const_len, chunks,
+                                                           partial, tickets, out, out_stride,
+                                                           write_end, seg_total, status);
   scan_down_kernel<InT, OutT><<<grid, kThreads, 0, st>>>(in, in_stride, out, out_stride, d_len,
-                                                         const_len, chunks, scratch, status);
+                                                         const_len, chunks, partial, status);
   return cudaGetLastError();
 }
 
