@@ -341,16 +341,14 @@ def main():
         host_targets = [t.cpu().pin_memory() for t in step_targets]
         for s in range(2):
             g.prepare(host_targets[s], fan, w.seed, gid(s), stream)
-            for j in range(w.H):
-                g.sizes(j)
+            g.fetch_all()
         if pg:
             pg.barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for s in range(args.warmup, n_steps):
             g.prepare(host_targets[s], fan, w.seed, gid(s), stream)
-            for j in range(w.H):
-                g.fetch(j)
+            g.fetch_all()
         torch.cuda.synchronize()
         e2e_s = time.perf_counter() - t0
         e2e_s = reduce_max(e2e_s, pg, dev)

@@ -151,6 +151,35 @@ typedef struct {
  * targets found on the device), ECUDA. */
 agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_view* out);
 
+/* All minibatches of the last hyperbatch at once, for callers that consume
+ * the whole hyperbatch (one wait and one size read-back for all H views).
+ * Minibatch j's arrays start at base + j * stride (elements), with the sizes
+ * of agnes_fetch_minibatch:
+ *   indptr[h] + j*indptr_stride[h]   num_dst = dst_size[h*H + j] (+1 entries)
+ *   col[h] + j*col_stride[h]         num_edges = edges[h*H + j]
+ *   nodes + j*nodes_stride           num_nodes = node_size[K*H + j]
+ *   feats + j*feats_stride_rows*row_bytes
+ * node_size[h*H + j] (0 <= h <= K) is |dst_{h+1}| = |src_h| of minibatch j
+ * (node_size[0..H) = B); edges is K x H.  node_size and edges are host
+ * memory owned by ctx.  Everything stays valid until the next prepare or
+ * free.  Errors as agnes_fetch_minibatch. */
+typedef struct {
+  int32_t K, H;
+  const int64_t* indptr[AGNES_MAX_HOPS];
+  int64_t indptr_stride[AGNES_MAX_HOPS];
+  const int32_t* col[AGNES_MAX_HOPS];
+  int64_t col_stride[AGNES_MAX_HOPS];
+  const int32_t* nodes;
+  int64_t nodes_stride;
+  const void* feats;
+  int64_t feats_stride_rows;
+  int32_t feat_dtype;
+  int64_t feat_dim;
+  const int32_t* node_size;
+  const int32_t* edges;
+} agnes_hyperbatch_view;
+agnes_status agnes_fetch_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out);
+
 /* Blocks touched by the last hyperbatch (the block-wise I/Os of Sec. 3.3 and
  * Fig. 7): out[h] for h < K = distinct topology blocks holding a node of
  * some minibatch's hop-(h+1) frontier; out[K] = distinct feature blocks

@@ -65,6 +65,18 @@ class _View(ctypes.Structure):
     ]
 
 
+class _HyperbatchView(ctypes.Structure):
+    _fields_ = [
+        ("K", ctypes.c_int32), ("H", ctypes.c_int32),
+        ("indptr", ctypes.c_void_p * MAX_HOPS), ("indptr_stride", ctypes.c_int64 * MAX_HOPS),
+        ("col", ctypes.c_void_p * MAX_HOPS), ("col_stride", ctypes.c_int64 * MAX_HOPS),
+        ("nodes", ctypes.c_void_p), ("nodes_stride", ctypes.c_int64),
+        ("feats", ctypes.c_void_p), ("feats_stride_rows", ctypes.c_int64),
+        ("feat_dtype", ctypes.c_int32), ("feat_dim", ctypes.c_int64),
+        ("node_size", ctypes.c_void_p), ("edges", ctypes.c_void_p),
+    ]
+
+
 class _Counters(ctypes.Structure):
     _fields_ = [
         ("K", ctypes.c_int32),
@@ -95,6 +107,7 @@ SIGNATURES = {
     "agnes_prepare_hyperbatch": ([_P, _P, ctypes.c_int32, ctypes.c_int32, _P, ctypes.c_int32,
                                   ctypes.c_uint64, ctypes.c_uint64, _P], ctypes.c_int),
     "agnes_fetch_minibatch": ([_P, ctypes.c_int32, ctypes.POINTER(_View)], ctypes.c_int),
+    "agnes_fetch_hyperbatch": ([_P, ctypes.POINTER(_HyperbatchView)], ctypes.c_int),
     "agnes_hyperbatch_stats": ([_P, _P], ctypes.c_int),
     "agnes_hyperbatch_counters": ([_P, ctypes.POINTER(_Counters)], ctypes.c_int),
     "agnes_get_graph_info": ([_P, ctypes.POINTER(_GraphInfo)], ctypes.c_int),
@@ -176,6 +189,36 @@ class MinibatchView:
     hops: list
     nodes: torch.Tensor   # int32 [num_nodes], device (src_K, global ids)
     feats: torch.Tensor   # [num_nodes, feat_dim], device
+
+
+class HyperbatchView:
+    """Every minibatch of a hyperbatch: one zero-copy tensor per output
+    buffer ([H, capacity, ...]) plus host size tables; ``view(j)`` slices
+    minibatch j out of them."""
+
+    def __init__(self, v: _HyperbatchView, device):
+        K, H = v.K, v.H
+        self.K, self.H = K, H
+        import numpy as np
+        sz = np.ctypeslib.as_array(ctypes.cast(v.node_size, ctypes.POINTER(ctypes.c_int32)),
+                                   shape=((K + 1) * H,)).reshape(K + 1, H).copy()
+        ed = np.ctypeslib.as_array(ctypes.cast(v.edges, ctypes.POINTER(ctypes.c_int32)),
+                                   shape=(K * H,)).reshape(K, H).copy()
+        self.node_size, self.edges = sz, ed
+        self.indptr = [_wrap(v.indptr[h], (H, v.indptr_stride[h]), torch.int64, device)
+                       for h in range(K)]
+        self.col = [_wrap(v.col[h], (H, v.col_stride[h]), torch.int32, device) for h in range(K)]
+        self.nodes = _wrap(v.nodes, (H, v.nodes_stride), torch.int32, device)
+        self.feats = _wrap(v.feats, (H, v.feats_stride_rows, v.feat_dim),
+                           _TORCH_OF[v.feat_dtype], device)
+
+    def view(self, j: int) -> "MinibatchView":
+        hops = []
+        for h in range(self.K):
+            nd, ns, ne = int(self.node_size[h, j]), int(self.node_size[h + 1, j]), int(self.edges[h, j])
+            hops.append(Hop(nd, ns, ne, self.indptr[h][j, :nd + 1], self.col[h][j, :ne]))
+        n = int(self.node_size[self.K, j])
+        return MinibatchView(hops, self.nodes[j, :n], self.feats[j, :n])
 
 
 class Graph:
@@ -262,6 +305,12 @@ class Graph:
         nodes = _wrap(v.nodes, (v.num_nodes,), torch.int32, self.device)
         feats = _wrap(v.feats, (v.num_nodes, v.feat_dim), _TORCH_OF[v.feat_dtype], self.device)
         return MinibatchView(hops, nodes, feats)
+
+    def fetch_all(self) -> HyperbatchView:
+        """All minibatches of the last hyperbatch (one wait, one size read-back)."""
+        v = _HyperbatchView()
+        _check(lib().agnes_fetch_hyperbatch(self._ctx, ctypes.byref(v)), self._ctx)
+        return HyperbatchView(v, self.device)
 
     def sizes(self, j: int) -> dict:
         """Host-side sizes of minibatch j (no device data touched)."""

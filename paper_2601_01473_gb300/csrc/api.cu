@@ -858,6 +858,35 @@ agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_vi
   return AGNES_OK;
 }
 
+agnes_status agnes_fetch_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  agnes_status rc = wait_prepared(ctx);
+  if (rc != AGNES_OK) return rc;
+  Workspace& w = ctx->ws;
+  const Back b = back_of(w);
+  memset(out, 0, sizeof(*out));
+  out->K = w.K;
+  out->H = w.H;
+  for (int h = 0; h < w.K; ++h) {
+    out->indptr[h] = w.indptr[h];
+    out->indptr_stride[h] = w.cap[h] + 1;
+    out->col[h] = w.col[h];
+    out->col_stride[h] = w.cap[h] * w.fan[h];
+  }
+  out->nodes = w.nodes;
+  out->nodes_stride = w.capK;
+  out->feats = w.feats_out;
+  out->feats_stride_rows = w.capK;
+  out->feat_dtype = ctx->feat_dtype;
+  out->feat_dim = ctx->feat_dim;
+  out->node_size = b.nsz;
+  out->edges = b.ecnt;
+  return AGNES_OK;
+}
+
 agnes_status agnes_hyperbatch_stats(agnes_ctx* ctx, int64_t* out) {
   if (!ctx || !out) {
     set_err(ctx, "ctx and out must be non-NULL");

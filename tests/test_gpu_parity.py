@@ -245,3 +245,19 @@ def test_streamed_features_match_oracle(cuda_device, dtype, dim, fbb, H):
         assert 0 < c["streamed_bytes"] <= c["streamed_blocks"] * (fbb // (dim * feats.element_size())) \
             * dim * feats.element_size()
     g.close()
+
+
+def test_fetch_all_equals_per_minibatch_fetch(cuda_device):
+    off, ind, feats = make(20000, 10, seed=31)
+    targets = synth.hyperbatch_targets(torch.arange(20000, dtype=torch.int32), 5, 128, 3, 0)
+    g = load(off, ind, feats, 16384, 16384)
+    g.prepare(targets.to(cuda_device), [9, 4, 2], 8, 40)
+    allv = g.fetch_all()
+    assert (allv.K, allv.H) == (3, 5)
+    for j in range(5):
+        a, b = g.fetch(j), allv.view(j)
+        assert torch.equal(a.nodes, b.nodes) and torch.equal(a.feats, b.feats)
+        for ha, hb in zip(a.hops, b.hops):
+            assert (ha.num_dst, ha.num_src, ha.num_edges) == (hb.num_dst, hb.num_src, hb.num_edges)
+            assert torch.equal(ha.indptr, hb.indptr) and torch.equal(ha.col, hb.col)
+    g.close()
