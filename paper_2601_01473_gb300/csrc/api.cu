@@ -297,7 +297,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.srank, edges);
   WA(w.sb, edges);
   WA(w.tmp, rows + edges);
-  WA(w.big_list, (rows + edges) / 33 + 1);
+  WA(w.big_list, (rows + edges) / (kDedupSmallMax + 1) + 1);
   WA(w.big_n, 1);
   WA(w.tmp_id, (int64_t)H * B);
   WA(w.tmp_pos, (int64_t)H * B);

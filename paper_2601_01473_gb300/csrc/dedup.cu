@@ -56,7 +56,7 @@ struct CellArgs {
   int32_t* nfcnt;            // per cell: next-frontier entries
   int2* tmp;                 // per cell at fcell_off + soff: next-frontier entries, local ranks
   int32_t* col;              // H x ecap: final col, or -(1 + local new rank)
-  int32_t* big_list;         // cells with more than 32 entries
+  int32_t* big_list;         // cells with more than kDedupSmallMax entries
   int32_t* big_n;
   const int32_t* status;
 };
@@ -83,7 +83,7 @@ __device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell*
 
 // ---- small cells: entry-parallel -----------------------------------------------
 //
-// A CTA takes 256 consecutive cells and stages the entries of the cells with
+// A CTA takes 128 consecutive cells and stages the entries of the cells with
 // samples and at most 32 entries in shared memory, each cell's frontier
 // entries (sorted) followed by its sampled entries.  Every thread then
 // resolves one entry against the entries of its own cell:
@@ -95,9 +95,10 @@ __device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell*
 //            in the next-frontier cell is lessF + lessN and a new node's rank
 //            among the cell's new ids is lessN.
 // Cells with more than 32 entries go to the big-cell list.
-constexpr int kGroupCells = 256;
-constexpr int kSlotCap = 2048;
-constexpr int kSmallMax = 32;
+constexpr int kCellThreads = 128;  // threads per CTA of the cells kernel
+constexpr int kGroupCells = kCellThreads;
+constexpr int kSlotCap = 1024;
+constexpr int kSmallMax = kDedupSmallMax;
 constexpr int kRoundFill = kSlotCap - kSmallMax;  // a cell starting below this fits
 
 enum : uint8_t { kSlotF = 1, kSlotLeader = 2, kSlotInD = 4 };
@@ -107,7 +108,7 @@ struct GroupSmem {
   int32_t ps[kGroupCells + 1];  // staged-slot prefix of the group's cells
   int32_t tb[kGroupCells];      // tmp base of the cell
   int32_t j[kGroupCells];
-  int32_t wsum[kGroupCells / 32];
+  int32_t wsum[kCellThreads / 32];
   int32_t id[kSlotCap];
   int32_t x[kSlotCap];       // frontier: output row; sampled: edge index
   int16_t fidx[kSlotCap];    // sampled inD: slot of the matching frontier entry
@@ -119,7 +120,7 @@ __device__ __forceinline__ void put_tmp(const CellArgs& a, int32_t at, int32_t i
   a.tmp[at] = make_int2(id, x);
 }
 
-__global__ void __launch_bounds__(kThreads) dedup_cells_kernel(CellArgs a) {
+__global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
   if (failed(a.status)) return;
   __shared__ GroupSmem sm;
   const int tid = threadIdx.x, lane = lane_id(), warp = tid >> 5;
@@ -150,7 +151,7 @@ __global__ void __launch_bounds__(kThreads) dedup_cells_kernel(CellArgs a) {
     __syncthreads();
     {
       int32_t off = 0, tot = 0;
-      for (int w = 0; w < kWarps; ++w) {
+      for (int w = 0; w < kCellThreads / 32; ++w) {
         off += w < warp ? sm.wsum[w] : 0;
         tot += sm.wsum[w];
       }
@@ -175,7 +176,7 @@ __global__ void __launch_bounds__(kThreads) dedup_cells_kernel(CellArgs a) {
       if (mine_in_round)
         for (int q = 0; q < n; ++q) sm.cell[sm.ps[tid] - rbase + q] = (uint8_t)tid;
       __syncthreads();
-      for (int32_t sl = tid; sl < used; sl += kThreads) {
+      for (int32_t sl = tid; sl < used; sl += kCellThreads) {
         const int l = sm.cell[sl];
         const int32_t q = rbase + sl - sm.ps[l];
         const int32_t fnl = sm.fn[l];
@@ -195,7 +196,7 @@ __global__ void __launch_bounds__(kThreads) dedup_cells_kernel(CellArgs a) {
       }
       __syncthreads();
       // phase 1: membership and first occurrence of sampled ids
-      for (int32_t sl = tid; sl < used; sl += kThreads) {
+      for (int32_t sl = tid; sl < used; sl += kCellThreads) {
         if (sm.flag[sl] & kSlotF) continue;
         const int l = sm.cell[sl];
         const int32_t fs = sm.ps[l] - rbase, fe = fs + sm.fn[l];
@@ -226,7 +227,7 @@ __global__ void __launch_bounds__(kThreads) dedup_cells_kernel(CellArgs a) {
         a.nfcnt[my_cell] = c.fn + cnt;
       }
       // phase 2: local ranks, col, next-frontier entries
-      for (int32_t sl = tid; sl < used; sl += kThreads) {
+      for (int32_t sl = tid; sl < used; sl += kCellThreads) {
         const int l = sm.cell[sl];
         const int32_t fs = sm.ps[l] - rbase, fe = fs + sm.fn[l], se = sm.ps[l + 1] - rbase;
         const int32_t id = sm.id[sl];
@@ -418,7 +419,7 @@ struct CompactArgs {
 // copied from the current bucket, any other from its tmp entries, where a new
 // node (x = -(1 + r)) gets its output row j * capK + |dst_h| + newbase + r and
 // its id is appended to the minibatch's node list.
-__global__ void __launch_bounds__(kThreads) dedup_compact_kernel(CompactArgs a) {
+__global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs a) {
   if (failed(a.status)) return;
   __shared__ int32_t s_nfo[kGroupCells + 1];
   __shared__ int32_t s_src[kGroupCells];   // source base in fb (>= 0) or ~base in tmp
@@ -441,7 +442,7 @@ __global__ void __launch_bounds__(kThreads) dedup_compact_kernel(CompactArgs a) 
     if (tid == 0) s_nfo[last - c0] = a.nfcell_off[last];
     __syncthreads();
     const int32_t k0 = s_nfo[0], k1 = s_nfo[last - c0];
-    for (int32_t k = k0 + tid; k < k1; k += kThreads) {
+    for (int32_t k = k0 + tid; k < k1; k += kCellThreads) {
       int32_t lo = 0, hi = (int32_t)(last - c0);  // last cell with nfo <= k
       while (hi - lo > 1) {
         const int32_t mid = (lo + hi) >> 1;
@@ -505,8 +506,8 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   c.big_list = d.big_list;
   c.big_n = d.big_n;
   c.status = a.status;
-  dedup_cells_kernel<<<resident_grid((const void*)dedup_cells_kernel, kThreads, num_sms), kThreads,
-                       0, st>>>(c);
+  dedup_cells_kernel<<<resident_grid((const void*)dedup_cells_kernel, kCellThreads, num_sms),
+                       kCellThreads, 0, st>>>(c);
   dedup_big_kernel<<<resident_grid((const void*)dedup_big_kernel, kThreads, num_sms), kThreads, 0,
                      st>>>(c);
   // per-minibatch offsets of the new ids: scan down the tiles of the
@@ -535,8 +536,8 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   k.nfb_pos = d.nfb_pos;
   k.nodes = d.nodes;
   k.status = a.status;
-  dedup_compact_kernel<<<resident_grid((const void*)dedup_compact_kernel, kThreads, num_sms),
-                         kThreads, 0, st>>>(k);
+  dedup_compact_kernel<<<resident_grid((const void*)dedup_compact_kernel, kCellThreads, num_sms),
+                         kCellThreads, 0, st>>>(k);
   return cudaGetLastError();
 }
 

@@ -101,6 +101,11 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
                                cudaStream_t st);
 
 // ---- dedup.cu --------------------------------------------------------------
+// Cells with more than this many entries (frontier + sampled) are resolved
+// on bitmaps, one warp each; the rest entry-parallel.  The big-cell list
+// therefore holds at most (entries) / (kDedupSmallMax + 1) cells.
+constexpr int kDedupSmallMax = 32;
+
 struct DedupBufs {
   const int32_t* nbr;       // H x ecap sampled ids
   const int32_t* ecnt;      // H edge counts
@@ -110,7 +115,7 @@ struct DedupBufs {
   int32_t* soff;            // T*H+1
   int2* sb;                 // bucketed (sampled id, edge index in the minibatch)
   int2* tmp;                // per cell: next-frontier entries with local ranks
-  int32_t* big_list;        // cells with more than 32 entries (capacity: entries / 33 + 1)
+  int32_t* big_list;        // cells with more than kDedupSmallMax entries
   int32_t* big_n;           // their count
   const int32_t* fb_id;     // current frontier bucket
   const int32_t* fb_pos;

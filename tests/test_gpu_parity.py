@@ -261,3 +261,13 @@ def test_fetch_all_equals_per_minibatch_fetch(cuda_device):
             assert (ha.num_dst, ha.num_src, ha.num_edges) == (hb.num_dst, hb.num_src, hb.num_edges)
             assert torch.equal(ha.indptr, hb.indptr) and torch.equal(ha.col, hb.col)
     g.close()
+
+
+def test_capacity_overflow_is_erange(cuda_device):
+    off, ind, feats = make(3000, 6, seed=9)
+    g = load(off, ind, feats, 4096, 4096)
+    big = torch.zeros((65535, 1), dtype=torch.int32, device=cuda_device)
+    with pytest.raises(AgnesError) as e:  # 65535 x 1 x (1+1024)^2 output rows > 2^31
+        g.prepare(big, [1024, 1024], 1, 0)
+    assert e.value.status == 2
+    g.close()
