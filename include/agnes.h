@@ -79,7 +79,15 @@ typedef struct agnes_ctx agnes_ctx; /* opaque, owned by the library */
  * agnes_free.  With features_on_host = 1 the feature matrix stays in pinned
  * host memory (borrowed) and each hyperbatch streams the feature blocks it
  * needs into device staging slots on a side stream (the asynchronous
- * block I/O of Sec. 3.4 (4), with the host link standing in for the SSD). */
+ * block I/O of Sec. 3.4 (4), with the host link standing in for the SSD).
+ * With topology_on_host = 1 the neighbour lists (indices, pinned host
+ * memory, borrowed) stay on the host; offsets are still copied or borrowed
+ * in device memory.  Each hop loads the topology blocks its frontier touches
+ * into an HBM graph buffer of graph_buffer_bytes (a whole number of blocks,
+ * at least the largest object), reusing resident blocks and evicting the
+ * least recently used unpinned ones; a block stays pinned until the hop has
+ * sampled all its requests (Sec. 3.4 (1)).  When a hop's blocks do not fit,
+ * the hop runs in waves of blocks in ascending order. */
 typedef struct {
   int64_t num_nodes;
   int64_t num_edges;
@@ -92,6 +100,8 @@ typedef struct {
   int32_t features_on_host;
   int64_t adj_block_bytes;
   int64_t feat_block_bytes;
+  int32_t topology_on_host; /* 1: indices stay in pinned host memory (see below) */
+  int64_t graph_buffer_bytes; /* HBM graph buffer for topology_on_host (0: whole topology) */
 } agnes_graph_desc;
 
 /* Loads a graph on `device` and builds its block tables: the object index
@@ -197,6 +207,10 @@ typedef struct {
   int64_t row_bytes;
   int64_t streamed_bytes;           /* features_on_host: bytes copied host -> device */
   int64_t streamed_blocks;          /* features_on_host: feature blocks copied */
+  int64_t topo_loaded_blocks;       /* topology_on_host: blocks copied into the graph buffer */
+  int64_t topo_loaded_bytes;
+  int64_t topo_hit_blocks;          /* needed blocks already resident */
+  int64_t topo_waves;               /* fill launches over all hops */
 } agnes_counters;
 agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
 

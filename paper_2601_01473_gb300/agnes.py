@@ -46,6 +46,8 @@ class _GraphDesc(ctypes.Structure):
         ("features_on_host", ctypes.c_int32),
         ("adj_block_bytes", ctypes.c_int64),
         ("feat_block_bytes", ctypes.c_int64),
+        ("topology_on_host", ctypes.c_int32),
+        ("graph_buffer_bytes", ctypes.c_int64),
     ]
 
 
@@ -87,6 +89,10 @@ class _Counters(ctypes.Structure):
         ("row_bytes", ctypes.c_int64),
         ("streamed_bytes", ctypes.c_int64),
         ("streamed_blocks", ctypes.c_int64),
+        ("topo_loaded_blocks", ctypes.c_int64),
+        ("topo_loaded_bytes", ctypes.c_int64),
+        ("topo_hit_blocks", ctypes.c_int64),
+        ("topo_waves", ctypes.c_int64),
     ]
 
 
@@ -226,7 +232,8 @@ class Graph:
 
     def __init__(self, offsets, indices, features, adj_block_bytes: int = 1 << 20,
                  feat_block_bytes: int | None = None, device: int = 0, stream=None,
-                 features_on_host: bool = False):
+                 features_on_host: bool = False, topology_on_host: bool = False,
+                 graph_buffer_bytes: int = 0):
         if offsets.dtype not in (torch.int32, torch.int64):
             raise TypeError("offsets must be int32 or int64")
         if indices.dtype != torch.int32:
@@ -252,6 +259,8 @@ class Graph:
         d.features_on_host = int(features_on_host)
         d.adj_block_bytes = adj_block_bytes
         d.feat_block_bytes = feat_block_bytes if feat_block_bytes is not None else adj_block_bytes
+        d.topology_on_host = int(topology_on_host)
+        d.graph_buffer_bytes = graph_buffer_bytes
         ctx = ctypes.c_void_p()
         with torch.cuda.device(self.device):
             rc = lib().agnes_load_graph(ctypes.byref(d), device, _stream_handle(stream),
@@ -329,7 +338,9 @@ class Graph:
         _check(lib().agnes_hyperbatch_counters(self._ctx, ctypes.byref(c)), self._ctx)
         return {"frontier": list(c.frontier[:c.K]), "edges": list(c.edges[:c.K]),
                 "rows": c.rows, "distinct_rows": c.distinct_rows, "row_bytes": c.row_bytes,
-                "streamed_bytes": c.streamed_bytes, "streamed_blocks": c.streamed_blocks}
+                "streamed_bytes": c.streamed_bytes, "streamed_blocks": c.streamed_blocks,
+                "topo_loaded_blocks": c.topo_loaded_blocks, "topo_loaded_bytes": c.topo_loaded_bytes,
+                "topo_hit_blocks": c.topo_hit_blocks, "topo_waves": c.topo_waves}
 
     def info(self) -> dict:
         g = _GraphInfo()

@@ -121,6 +121,31 @@ struct agnes_ctx {
   std::vector<int32_t> fblock_first_tile;
   int64_t streamed_bytes = 0, streamed_blocks = 0;
 
+  // topology in pinned host memory, HBM graph buffer with LRU + pinning
+  struct Topo {
+    bool on = false;
+    const int32_t* host_indices = nullptr;
+    int64_t slots = 0, epb = 0;
+    int32_t* gbuf = nullptr;
+    int32_t* d_slot = nullptr;          // n_blocks: slot of each physical block, -1 if absent
+    int32_t* h_slot_stage = nullptr;    // pinned staging for uploads of the slot table
+    std::vector<int32_t> slot_of;       // host: block -> slot
+    std::vector<int32_t> block_of;      // slot -> block or -1
+    std::vector<int32_t> prev, next;    // LRU list over slots (head = least recent)
+    int32_t head = -1, tail = -1;
+    std::vector<uint32_t> pinned;       // slot -> wave it is pinned for
+    uint32_t wave = 0;
+    std::vector<int64_t> e0, e1;        // block edge ranges
+    std::vector<int32_t> start_block;   // n_starts + 1 (sentinel n_blocks)
+    std::vector<int32_t> run_first_tile;
+    uint8_t* d_need = nullptr;
+    uint8_t* h_need = nullptr;
+    cudaStream_t copy = nullptr;
+    cudaEvent_t uploaded = nullptr, wave_done = nullptr;
+    bool uploaded_used = false;
+    int64_t loaded_blocks = 0, loaded_bytes = 0, hits = 0, waves = 0;
+  } topo;
+
   char err[512] = {0};
 };
 
@@ -426,6 +451,17 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   cudaFree(ctx->d_touched);
   if (ctx->h_flags) cudaFreeHost(ctx->h_flags);
   if (ctx->h_touched) cudaFreeHost(ctx->h_touched);
+  {
+    agnes_ctx::Topo& tp = ctx->topo;
+    if (tp.copy) cudaStreamDestroy(tp.copy);
+    if (tp.uploaded) cudaEventDestroy(tp.uploaded);
+    if (tp.wave_done) cudaEventDestroy(tp.wave_done);
+    cudaFree(tp.gbuf);
+    cudaFree(tp.d_slot);
+    cudaFree(tp.d_need);
+    if (tp.h_slot_stage) cudaFreeHost(tp.h_slot_stage);
+    if (tp.h_need) cudaFreeHost(tp.h_need);
+  }
   if (ctx->ev_created)
     for (int r = 0; r < kEventRing; ++r)
       for (int i = 0; i <= kMaxPhases; ++i) cudaEventDestroy(ctx->ev[r][i]);
@@ -466,6 +502,75 @@ static agnes_status setup_streaming(agnes_ctx* ctx, cudaStream_t st) {
   return AGNES_OK;
 }
 
+// Graph buffer, tables and copy stream for topology in pinned host memory.
+static agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStream_t st) {
+  agnes_ctx::Topo& tp = ctx->topo;
+  const int64_t nb = ctx->bt.n_blocks, ns = ctx->bt.n_starts;
+  tp.on = true;
+  tp.host_indices = d->indices;
+  tp.epb = d->adj_block_bytes / 4;
+  tp.e0.resize((size_t)nb);
+  tp.e1.resize((size_t)nb);
+  tp.start_block.resize((size_t)ns + 1);
+  tp.run_first_tile.resize((size_t)ns + 1);
+  CK(ctx, cudaMemcpyAsync(tp.e0.data(), ctx->bt.blk_e0, sizeof(int64_t) * nb,
+                          cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(tp.e1.data(), ctx->bt.blk_e1, sizeof(int64_t) * nb,
+                          cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(tp.start_block.data(), ctx->bt.start_block, sizeof(int32_t) * ns,
+                          cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(tp.run_first_tile.data(), ctx->bt.run_first_tile,
+                          sizeof(int32_t) * (ns + 1), cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
+  tp.start_block[(size_t)ns] = (int32_t)nb;
+  int64_t longest = 1;
+  for (int64_t r = 0; r < ns; ++r) {
+    const int64_t m = tp.start_block[(size_t)r + 1] - tp.start_block[(size_t)r];
+    if (m > longest) longest = m;
+  }
+  tp.slots = d->graph_buffer_bytes > 0 ? d->graph_buffer_bytes / d->adj_block_bytes : nb;
+  if (tp.slots > nb) tp.slots = nb;
+  if (tp.slots < longest) {
+    set_err(ctx, "graph_buffer_bytes holds %lld blocks; the largest object needs %lld",
+            (long long)tp.slots, (long long)longest);
+    return AGNES_EINVAL;
+  }
+  CK(ctx, cudaMalloc((void**)&tp.gbuf, sizeof(int32_t) * (size_t)(tp.slots * tp.epb)));
+  CK(ctx, cudaMalloc((void**)&tp.d_slot, sizeof(int32_t) * (size_t)nb));
+  CK(ctx, cudaMalloc((void**)&tp.d_need, (size_t)ns + 1));
+  CK(ctx, cudaMallocHost((void**)&tp.h_slot_stage, sizeof(int32_t) * (size_t)nb));
+  CK(ctx, cudaMallocHost((void**)&tp.h_need, (size_t)ns + 1));
+  CK(ctx, cudaMemsetAsync(tp.d_slot, 0xff, sizeof(int32_t) * (size_t)nb, st));
+  CK(ctx, cudaStreamCreateWithFlags(&tp.copy, cudaStreamNonBlocking));
+  CK(ctx, cudaEventCreateWithFlags(&tp.uploaded, cudaEventDisableTiming));
+  CK(ctx, cudaEventCreateWithFlags(&tp.wave_done, cudaEventDisableTiming));
+  tp.slot_of.assign((size_t)nb, -1);
+  tp.block_of.assign((size_t)tp.slots, -1);
+  tp.pinned.assign((size_t)tp.slots, 0);
+  tp.prev.resize((size_t)tp.slots);
+  tp.next.resize((size_t)tp.slots);
+  for (int64_t i = 0; i < tp.slots; ++i) {  // all slots free, in LRU order
+    tp.prev[(size_t)i] = (int32_t)i - 1;
+    tp.next[(size_t)i] = i + 1 < tp.slots ? (int32_t)i + 1 : -1;
+  }
+  tp.head = 0;
+  tp.tail = (int32_t)tp.slots - 1;
+  CK(ctx, cudaStreamSynchronize(st));
+  return AGNES_OK;
+}
+
+// LRU list: move slot i to the most-recent end.
+static void lru_touch(agnes_ctx::Topo& tp, int32_t i) {
+  if (tp.tail == i) return;
+  const int32_t p = tp.prev[(size_t)i], n = tp.next[(size_t)i];
+  if (p >= 0) tp.next[(size_t)p] = n; else tp.head = n;
+  if (n >= 0) tp.prev[(size_t)n] = p;
+  tp.prev[(size_t)i] = tp.tail;
+  tp.next[(size_t)i] = -1;
+  tp.next[(size_t)tp.tail] = i;
+  tp.tail = i;
+}
+
 agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_stream,
                               agnes_ctx** out) {
   if (!out) {
@@ -488,6 +593,10 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   if (d->num_edges < 0 || (d->offsets_bits == 32 && d->num_edges >= ((int64_t)1 << 31))) {
     set_err(nullptr, "num_edges out of range for the offsets type");
     return AGNES_ERANGE;
+  }
+  if (d->topology_on_host && (!d->indices || !is_pinned_host_ptr(d->indices))) {
+    set_err(nullptr, "topology_on_host requires indices in pinned host memory");
+    return AGNES_EINVAL;
   }
   if (!d->offsets || (d->num_edges > 0 && !d->indices) || !d->features) {
     set_err(nullptr, "offsets, indices and features must be non-NULL");
@@ -546,7 +655,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   agnes_status rc;
   const size_t off_bytes = (size_t)(d->num_nodes + 1) * (d->offsets_bits / 8);
   rc = adopt_or_copy(ctx, d->offsets, off_bytes, &ctx->offsets, &ctx->own_offsets, st);
-  if (rc == AGNES_OK && d->num_edges > 0)
+  if (rc == AGNES_OK && d->num_edges > 0 && !d->topology_on_host)
     rc = adopt_or_copy(ctx, d->indices, (size_t)d->num_edges * 4, (void**)&ctx->indices,
                        &ctx->own_indices, st);
   if (rc == AGNES_OK) {
@@ -593,6 +702,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
     if (e != cudaSuccess) rc = e == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;
   }
   if (rc == AGNES_OK && d->features_on_host) rc = setup_streaming(ctx, st);
+  if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0) rc = setup_topology(ctx, d, st);
   if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
     set_err(ctx, "cudaEventCreate failed");
     rc = AGNES_ECUDA;
@@ -603,6 +713,96 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
     return rc;
   }
   *out = ctx;
+  return AGNES_OK;
+}
+
+// Sampling with the topology in pinned host memory.  The block runs the
+// frontier touches are read back; runs are taken in ascending order into
+// waves that fit the graph buffer: each needed block is either resident
+// (a hit: pinned and moved to the recent end of the LRU list) or copied into
+// the least recently used unpinned slot on the side stream.  The slot table
+// is uploaded, the wave's cells are sampled, and the wave's blocks unpin when
+// the next wave starts (its copies wait for this wave's sampling to finish).
+static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int h,
+                                  cudaStream_t st) {
+  Workspace& w = ctx->ws;
+  agnes_ctx::Topo& tp = ctx->topo;
+  const int64_t ns = ctx->bt.n_starts, nb = ctx->bt.n_blocks;
+  const int32_t H = w.H, T = (int32_t)ctx->bt.T;
+  CK(ctx, launch_mark_runs(w.fcell_off[cur], T, H, ctx->bt.tile_adj_start, tp.d_need, ns, w.status,
+                           st));
+  CK(ctx, cudaMemcpyAsync(tp.h_need, tp.d_need, (size_t)ns, cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
+  int64_t r = 0;
+  while (r < ns && !tp.h_need[r]) ++r;
+  while (r < ns) {
+    tp.wave += 1;
+    const uint32_t wave = tp.wave;
+    int64_t pinned_now = 0;
+    const int64_t r_first = r;
+    int64_t r_last = r;
+    // the previous wave must be done before its slots can be overwritten
+    CK(ctx, cudaStreamWaitEvent(tp.copy, tp.wave_done, 0));
+    while (r < ns) {
+      if (!tp.h_need[r]) {
+        ++r;
+        continue;
+      }
+      const int32_t b0 = tp.start_block[(size_t)r], b1 = tp.start_block[(size_t)r + 1];
+      if (pinned_now + (b1 - b0) > tp.slots) break;  // wave full
+      for (int32_t b = b0; b < b1; ++b) {
+        int32_t sl = tp.slot_of[(size_t)b];
+        if (sl >= 0) {
+          tp.hits += 1;
+        } else {
+          sl = tp.head;  // least recently used slot that is not pinned for this wave
+          while (sl >= 0 && tp.pinned[(size_t)sl] == wave) sl = tp.next[(size_t)sl];
+          if (sl < 0) {
+            set_err(ctx, "graph buffer exhausted inside a wave");
+            return AGNES_EKERNEL;
+          }
+          const int32_t old = tp.block_of[(size_t)sl];
+          if (old >= 0) tp.slot_of[(size_t)old] = -1;
+          tp.block_of[(size_t)sl] = b;
+          tp.slot_of[(size_t)b] = sl;
+          const int64_t ne = tp.e1[(size_t)b] - tp.e0[(size_t)b];
+          if (ne > 0)
+            CK(ctx, cudaMemcpyAsync(tp.gbuf + (int64_t)sl * tp.epb, tp.host_indices + tp.e0[(size_t)b],
+                                    sizeof(int32_t) * (size_t)ne, cudaMemcpyHostToDevice, tp.copy));
+          tp.loaded_blocks += 1;
+          tp.loaded_bytes += sizeof(int32_t) * ne;
+        }
+        tp.pinned[(size_t)sl] = wave;
+        lru_touch(tp, sl);
+        ++pinned_now;
+      }
+      r_last = r;
+      ++r;
+    }
+    if (pinned_now == 0) break;
+    // upload the slot table (the staging buffer is free once the last upload ran)
+    if (tp.uploaded_used) CK(ctx, cudaEventSynchronize(tp.uploaded));
+    memcpy(tp.h_slot_stage, tp.slot_of.data(), sizeof(int32_t) * (size_t)nb);
+    CK(ctx, cudaMemcpyAsync(tp.d_slot, tp.h_slot_stage, sizeof(int32_t) * (size_t)nb,
+                            cudaMemcpyHostToDevice, tp.copy));
+    CK(ctx, cudaEventRecord(tp.uploaded, tp.copy));
+    tp.uploaded_used = true;
+    CK(ctx, cudaStreamWaitEvent(st, tp.uploaded, 0));
+    FillRange fr;
+    fr.cell_lo = (int64_t)tp.run_first_tile[(size_t)r_first] * H;
+    fr.cell_hi = (int64_t)tp.run_first_tile[(size_t)r_last + 1] * H;
+    fr.tile_adj_block = ctx->bt.tile_adj_block;
+    fr.blk_slot = tp.d_slot;
+    fr.blk_e0 = ctx->bt.blk_e0;
+    fr.gbuf = tp.gbuf;
+    fr.epb = tp.epb;
+    fr.bb = ctx->adj_block_bytes;
+    CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h], w.nbr,
+                               w.scnt, w.scell, w.srank, fr, ctx->num_sms, st));
+    CK(ctx, cudaEventRecord(tp.wave_done, st));
+    tp.waves += 1;
+    while (r < ns && !tp.h_need[r]) ++r;
+  }
   return AGNES_OK;
 }
 
@@ -767,8 +967,16 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
                                          cap[h], true, ecnt, w.scan_scratch, w.status, st)));
     mark();
     CK(ctx, cudaMemsetAsync(w.scnt, 0, sizeof(int32_t) * cells, st));
-    CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h],
-                               w.nbr, w.scnt, w.scell, w.srank, nsm, st));
+    if (ctx->topo.on) {
+      rc = fill_streamed(ctx, a, cur, h, st);
+      if (rc != AGNES_OK) return rc;
+    } else {
+      FillRange r;
+      r.cell_lo = 0;
+      r.cell_hi = cells;
+      CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h],
+                                 w.nbr, w.scnt, w.scell, w.srank, r, nsm, st));
+    }
     mark();
     DedupBufs d;
     d.nbr = w.nbr;
@@ -926,6 +1134,10 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
   out->distinct_rows = (int64_t)distinct;
   out->streamed_bytes = ctx->features_on_host ? ctx->streamed_bytes : 0;
   out->streamed_blocks = ctx->features_on_host ? ctx->streamed_blocks : 0;
+  out->topo_loaded_blocks = ctx->topo.loaded_blocks;
+  out->topo_loaded_bytes = ctx->topo.loaded_bytes;
+  out->topo_hit_blocks = ctx->topo.hits;
+  out->topo_waves = ctx->topo.waves;
   return AGNES_OK;
 }
 

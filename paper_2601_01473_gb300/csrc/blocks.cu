@@ -115,7 +115,9 @@ __global__ void tile_blocks_kernel(const int32_t* __restrict__ tile_first, int64
                                    const int32_t* __restrict__ start_node,
                                    const int32_t* __restrict__ start_block, int64_t n_starts,
                                    int64_t rpb, int32_t* __restrict__ tile_adj_block,
-                                   int32_t* __restrict__ tile_feat_block) {
+                                   int32_t* __restrict__ tile_feat_block,
+                                   int32_t* __restrict__ tile_adj_start,
+                                   int32_t* __restrict__ run_first_tile) {
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
        t += (int64_t)gridDim.x * blockDim.x) {
     const int32_t v = tile_first[t];
@@ -130,6 +132,43 @@ __global__ void tile_blocks_kernel(const int32_t* __restrict__ tile_first, int64
     }
     tile_adj_block[t] = start_block[lo];
     tile_feat_block[t] = (int32_t)(v / rpb);
+    tile_adj_start[t] = (int32_t)lo;
+    if (start_node[lo] == v) run_first_tile[lo] = (int32_t)t;  // block starts start tiles
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) run_first_tile[n_starts] = (int32_t)T;
+}
+
+// Edge range [e0, e1) of every physical block: a block of whole objects
+// holds the edges of its nodes; the i-th block of an object larger than a
+// block holds the edges whose bytes (after the hdr-byte header) fall in
+// [i*bb, (i+1)*bb) of the object.
+template <typename OffT>
+__global__ void block_edges_kernel(const OffT* __restrict__ off, int64_t N, int64_t hdr, int64_t bb,
+                                   const int32_t* __restrict__ start_node,
+                                   const int32_t* __restrict__ start_block, int64_t n_starts,
+                                   int64_t n_blocks, int64_t* __restrict__ e0,
+                                   int64_t* __restrict__ e1) {
+  for (int64_t s = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; s < n_starts;
+       s += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t v0 = start_node[s];
+    const int64_t v1 = s + 1 < n_starts ? start_node[s + 1] : N;
+    const int64_t b0 = start_block[s];
+    const int64_t b1 = s + 1 < n_starts ? start_block[s + 1] : n_blocks;
+    const int64_t a = (int64_t)off[v0], z = (int64_t)off[v1];
+    if (b1 - b0 == 1) {
+      e0[b0] = a;
+      e1[b0] = z;
+    } else {  // one big object
+      const int64_t deg = z - a;
+      for (int64_t i = 0; i < b1 - b0; ++i) {
+        int64_t lo = (i * bb - hdr + 3) / 4;
+        int64_t hi = ((i + 1) * bb - hdr + 3) / 4;
+        lo = lo < 0 ? 0 : (lo > deg ? deg : lo);
+        hi = hi < 0 ? 0 : (hi > deg ? deg : hi);
+        e0[b0 + i] = a + lo;
+        e1[b0 + i] = a + hi;
+      }
+    }
   }
 }
 
@@ -156,6 +195,10 @@ void free_block_tables(BlockTables* bt) {
   cudaFree(bt->tile_adj_block);
   cudaFree(bt->tile_feat_block);
   cudaFree(bt->fblock_first_tile);
+  cudaFree(bt->tile_adj_start);
+  cudaFree(bt->run_first_tile);
+  cudaFree(bt->blk_e0);
+  cudaFree(bt->blk_e1);
   *bt = BlockTables();
 }
 
@@ -229,10 +272,25 @@ cudaError_t build_block_tables(const void* d_offsets, int offsets_bits, int64_t 
   BT_CHECK(cudaMalloc(&bt->tile_adj_block, sizeof(int32_t) * bt->T));
   BT_CHECK(cudaMalloc(&bt->tile_feat_block, sizeof(int32_t) * bt->T));
   BT_CHECK(cudaMalloc(&bt->fblock_first_tile, sizeof(int32_t) * (bt->n_feat_blocks + 1)));
+  BT_CHECK(cudaMalloc(&bt->tile_adj_start, sizeof(int32_t) * bt->T));
+  BT_CHECK(cudaMalloc(&bt->run_first_tile, sizeof(int32_t) * (bt->n_starts + 1)));
+  BT_CHECK(cudaMalloc(&bt->blk_e0, sizeof(int64_t) * bt->n_blocks));
+  BT_CHECK(cudaMalloc(&bt->blk_e1, sizeof(int64_t) * bt->n_blocks));
   tile_compact_kernel<<<grid, 256, 0, st>>>(flags, rank, N, bt->tile_first, bt->chunk_tile);
   tile_blocks_kernel<<<grid, 256, 0, st>>>(bt->tile_first, bt->T, bt->start_node,
                                            bt->start_block, bt->n_starts, rows_per_feat_block,
-                                           bt->tile_adj_block, bt->tile_feat_block);
+                                           bt->tile_adj_block, bt->tile_feat_block,
+                                           bt->tile_adj_start, bt->run_first_tile);
+  if (offsets_bits == 32)
+    block_edges_kernel<int32_t><<<grid, 256, 0, st>>>((const int32_t*)d_offsets, N, hdr,
+                                                      adj_block_bytes, bt->start_node,
+                                                      bt->start_block, bt->n_starts, bt->n_blocks,
+                                                      bt->blk_e0, bt->blk_e1);
+  else
+    block_edges_kernel<int64_t><<<grid, 256, 0, st>>>((const int64_t*)d_offsets, N, hdr,
+                                                      adj_block_bytes, bt->start_node,
+                                                      bt->start_block, bt->n_starts, bt->n_blocks,
+                                                      bt->blk_e0, bt->blk_e1);
   fblock_first_tile_kernel<<<grid, 256, 0, st>>>(bt->tile_first, bt->tile_feat_block, bt->T,
                                                  rows_per_feat_block, bt->n_feat_blocks,
                                                  bt->fblock_first_tile);

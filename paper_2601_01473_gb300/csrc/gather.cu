@@ -126,6 +126,16 @@ __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int
     if (cell_off[c + 1] > cell_off[c]) flags[map[c / H]] = 1;
 }
 
+// need[tile_adj_start[t]] = 1 for every tile t with a frontier entry.
+__global__ void mark_runs_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
+                                 const int32_t* __restrict__ tile_adj_start,
+                                 uint8_t* __restrict__ need, const int32_t* status) {
+  if (failed(status)) return;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
+       t += (int64_t)gridDim.x * blockDim.x)
+    if (cell_off[(t + 1) * H] > cell_off[t * H]) need[tile_adj_start[t]] = 1;
+}
+
 __global__ void count_flags_kernel(const uint8_t* __restrict__ flags, int64_t n,
                                    int64_t* __restrict__ count) {
   int64_t local = 0;
@@ -226,6 +236,15 @@ cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, con
   if (cell_off && map)
     mark_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, map, flags, status);
   count_flags_kernel<<<256, 256, 0, st>>>(flags, n_flags, count);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mark_runs(const int32_t* cell_off, int32_t T, int32_t H,
+                             const int32_t* tile_adj_start, uint8_t* need, int64_t n_runs,
+                             const int32_t* status, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(need, 0, (size_t)n_runs, st);
+  if (e != cudaSuccess) return e;
+  mark_runs_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, tile_adj_start, need, status);
   return cudaGetLastError();
 }
 

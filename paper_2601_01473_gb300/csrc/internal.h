@@ -47,6 +47,10 @@ struct BlockTables {
   int32_t* tile_adj_block = nullptr;
   int32_t* tile_feat_block = nullptr;
   int32_t* fblock_first_tile = nullptr;  // n_feat_blocks+1: first tile of each feature block
+  int32_t* tile_adj_start = nullptr;     // T: block start (run) index of each tile
+  int32_t* run_first_tile = nullptr;     // n_starts+1: first tile of each block run
+  int64_t* blk_e0 = nullptr;             // n_blocks: first edge held by each physical block
+  int64_t* blk_e1 = nullptr;             // n_blocks: one past its last edge
   int64_t T = 0;
   int64_t n_feat_blocks = 0;
   int64_t rows_per_feat_block = 0;
@@ -92,13 +96,24 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
                                 const int32_t* fcell_off, int32_t* cnt, int num_sms,
                                 cudaStream_t st);
 
-// Samples every frontier entry and records, per sampled edge, its
-// neighbour id (nbr), its (tile, minibatch) cell (scell) and its rank within
-// that cell (srank), counting the cells in scnt (zero on entry).
+// Which frontier cells to sample and, for streamed topology, where their
+// edge lists are (gbuf == nullptr: the edges are read from HopArgs::indices).
+struct FillRange {
+  int64_t cell_lo = 0, cell_hi = 0;
+  const int32_t* tile_adj_block = nullptr;
+  const int32_t* blk_slot = nullptr;
+  const int64_t* blk_e0 = nullptr;
+  const int32_t* gbuf = nullptr;
+  int64_t epb = 0, bb = 0;
+};
+
+// Samples the frontier entries of cells [r.cell_lo, r.cell_hi) and records,
+// per sampled edge, its neighbour id (nbr), its (tile, minibatch) cell (scell)
+// and its rank within that cell (srank), counting the cells in scnt.
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
                                const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
-                               int32_t* scnt, int32_t* scell, int32_t* srank, int num_sms,
-                               cudaStream_t st);
+                               int32_t* scnt, int32_t* scell, int32_t* srank,
+                               const FillRange& r, int num_sms, cudaStream_t st);
 
 // ---- dedup.cu --------------------------------------------------------------
 // Cells with more than this many entries (frontier + sampled) are resolved
@@ -157,6 +172,12 @@ cudaError_t launch_gather_staged(const void* slot, int64_t row_bytes, int64_t rp
 cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, const int32_t* map,
                               uint8_t* flags, int64_t n_flags, int64_t* count,
                               const int32_t* status, cudaStream_t st);
+
+// need[r] = 1 for every block run r whose tiles hold a frontier entry
+// (need is cleared first).
+cudaError_t launch_mark_runs(const int32_t* cell_off, int32_t T, int32_t H,
+                             const int32_t* tile_adj_start, uint8_t* need, int64_t n_runs,
+                             const int32_t* status, cudaStream_t st);
 
 cudaError_t launch_distinct_rows(const int32_t* fb_id, const int32_t* cell_off,
                                  const int32_t* tile_first, int32_t T, int32_t H,

@@ -185,13 +185,22 @@ sample_count_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict
 
 struct FillArgs {
   TileMap tm;
+  // frontier entries [fcell_off[cell_lo], fcell_off[cell_hi]) are sampled
+  const int32_t* fcell_off;
+  int64_t cell_lo, cell_hi;
+  // streamed topology: edge lists of resident physical blocks in the graph
+  // buffer (slot * epb edges each); blk_slot[b] < 0 means not resident
+  const int32_t* tile_adj_block;
+  const int32_t* blk_slot;
+  const int64_t* blk_e0;
+  const int32_t* gbuf;
+  int64_t epb, hdr, bb;
   int32_t H;
   int32_t* scnt;   // T*H per-cell counters of sampled ids (zero on entry)
   int32_t* scell;  // per edge: its (tile, minibatch) cell
   int32_t* srank;  // per edge: its rank within the cell
   const int32_t* fb_id;
   const int32_t* fb_pos;
-  const int32_t* total_ptr;
   const int64_t* indptr;
   const int32_t* indices;
   int32_t* nbr;
@@ -199,8 +208,26 @@ struct FillArgs {
   int32_t k, hop;
   uint32_t key_lo, key_hi;
   uint64_t first_gid;
-  const int32_t* status;
+  int32_t* status;
 };
+
+// Neighbour at position pos of node v (edges off_v .. off_v + deg).  With
+// streamed topology the edge sits in the graph-buffer slot of its physical
+// block: v's first block, plus, for an object larger than a block, the block
+// its byte offset (after the header) falls in.
+template <bool kStreamed>
+__device__ __forceinline__ int32_t edge_at(const FillArgs& a, int32_t v, int64_t off_v,
+                                           int64_t deg, int64_t pos) {
+  if (!kStreamed) return __ldg(a.indices + off_v + pos);
+  int64_t b = __ldg(a.tile_adj_block + tile_of(a.tm, v));
+  if (a.hdr + 4 * deg > a.bb) b += (a.hdr + 4 * pos) / a.bb;
+  const int32_t slot = __ldg(a.blk_slot + b);
+  if (slot < 0) {  // cannot happen: the host made every needed block resident
+    atomicOr(a.status, kErrInternal);
+    return 0;
+  }
+  return __ldg(a.gbuf + (int64_t)slot * a.epb + (off_v + pos - __ldg(a.blk_e0 + b)));
+}
 
 __device__ __forceinline__ int64_t draw(const FillArgs& a, int32_t v, int32_t s, uint64_t gid,
                                         int64_t J) {
@@ -230,11 +257,11 @@ __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t 
 }
 
 // G lanes per frontier node, k <= G.
-template <typename OffT, int G>
+template <typename OffT, int G, bool kStreamed>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
   if (failed(a.status)) return;
-  const int64_t total = *a.total_ptr;
+  const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
   constexpr int kGroups = 32 / G;
   const int lane = lane_id();
   const int sub = lane / G, s = lane % G;
@@ -242,13 +269,13 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
   const uint32_t capk32 = (uint32_t)a.capK;
   const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t e0 = warp0 * kGroups; e0 < total; e0 += nwarps * kGroups) {
+  for (int64_t e0 = E0 + warp0 * kGroups; e0 < E1; e0 += nwarps * kGroups) {
     const int64_t i = e0 + sub;
     bool has = false;
     int32_t u = 0;
     uint32_t j = 0;
     int64_t eidx = 0;
-    if (i < total) {  // whole group takes the same branches
+    if (i < E1) {  // whole group takes the same branches
       const int32_t v = a.fb_id[i];
       const uint32_t g = (uint32_t)a.fb_pos[i];
       j = g / capk32;
@@ -258,7 +285,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
       eidx = a.indptr[j * (a.cap_prev + 1) + pos] + s;
       if (d <= a.k) {
         if (s < d) {
-          u = __ldg(a.indices + base + s);
+          u = edge_at<kStreamed>(a, v, base, d, s);
           has = true;
         }
       } else {
@@ -271,7 +298,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
           if (s > q && t == cq) collided = true;
         }
         if (s < a.k) {
-          u = __ldg(a.indices + base + (collided ? J : t));
+          u = edge_at<kStreamed>(a, v, base, d, collided ? J : t);
           has = true;
         }
       }
@@ -283,17 +310,17 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
 // One warp per frontier node for fanouts above 32: slots are drawn 32 at a
 // time; each candidate is checked against the choices of earlier chunks (kept
 // in shared memory) and then resolved within its chunk by shuffles.
-template <typename OffT>
+template <typename OffT, bool kStreamed>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
   if (failed(a.status)) return;
   __shared__ int32_t chosen_s[kWarps][kMaxFanout];
   const int warp = threadIdx.x >> 5, lane = lane_id();
   int32_t* chosen = chosen_s[warp];
-  const int64_t total = *a.total_ptr;
+  const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
   const uint32_t capk32 = (uint32_t)a.capK;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total;
+  for (int64_t i = E0 + ((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5); i < E1;
        i += nwarps) {
     const int32_t v = a.fb_id[i];
     const uint32_t g = (uint32_t)a.fb_pos[i];
@@ -306,7 +333,7 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
       for (int64_t q0 = 0; q0 < d; q0 += 32) {
         const int64_t q = q0 + lane;
         const bool has = q < d;
-        emit_edges(a, has, has ? __ldg(a.indices + base + q) : 0, j, ebase + q);
+        emit_edges(a, has, has ? edge_at<kStreamed>(a, v, base, d, q) : 0, j, ebase + q);
       }
       continue;
     }
@@ -325,7 +352,7 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
       }
       const int64_t c = collided ? J : t;
       if (valid) chosen[s] = (int32_t)c;
-      emit_edges(a, valid, valid ? __ldg(a.indices + base + c) : 0, j, ebase + s);
+      emit_edges(a, valid, valid ? edge_at<kStreamed>(a, v, base, d, c) : 0, j, ebase + s);
       __syncwarp();
     }
   }
@@ -372,37 +399,46 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
   return cudaGetLastError();
 }
 
-template <typename OffT>
+template <typename OffT, bool kStreamed>
 static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int num_sms,
                               cudaStream_t st) {
 #define AGNES_FILL(KERNEL)                                                                   \
   KERNEL<<<resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st>>>(f, off)
   if (k <= 4)
-    AGNES_FILL((sample_fill_kernel<OffT, 4>));
+    AGNES_FILL((sample_fill_kernel<OffT, 4, kStreamed>));
   else if (k <= 8)
-    AGNES_FILL((sample_fill_kernel<OffT, 8>));
+    AGNES_FILL((sample_fill_kernel<OffT, 8, kStreamed>));
   else if (k <= 16)
-    AGNES_FILL((sample_fill_kernel<OffT, 16>));
+    AGNES_FILL((sample_fill_kernel<OffT, 16, kStreamed>));
   else if (k <= 32)
-    AGNES_FILL((sample_fill_kernel<OffT, 32>));
+    AGNES_FILL((sample_fill_kernel<OffT, 32, kStreamed>));
   else
-    AGNES_FILL((sample_fill_wide_kernel<OffT>));
+    AGNES_FILL((sample_fill_wide_kernel<OffT, kStreamed>));
 #undef AGNES_FILL
 }
 
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
                                const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
-                               int32_t* scnt, int32_t* scell, int32_t* srank, int num_sms,
-                               cudaStream_t st) {
+                               int32_t* scnt, int32_t* scell, int32_t* srank,
+                               const FillRange& r, int num_sms, cudaStream_t st) {
   FillArgs f;
   f.tm = TileMap{a.tile_first, a.chunk_tile, a.T};
+  f.fcell_off = fcell_off;
+  f.cell_lo = r.cell_lo;
+  f.cell_hi = r.cell_hi;
+  f.tile_adj_block = r.tile_adj_block;
+  f.blk_slot = r.blk_slot;
+  f.blk_e0 = r.blk_e0;
+  f.gbuf = r.gbuf;
+  f.epb = r.epb;
+  f.hdr = a.offsets_bits / 8;
+  f.bb = r.bb;
   f.H = a.H;
   f.scnt = scnt;
   f.scell = scell;
   f.srank = srank;
   f.fb_id = fb_id;
   f.fb_pos = fb_pos;
-  f.total_ptr = fcell_off + (int64_t)a.T * a.H;
   f.indptr = indptr;
   f.indices = a.indices;
   f.nbr = nbr;
@@ -415,10 +451,18 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.key_hi = (uint32_t)(a.seed >> 32);
   f.first_gid = a.first_gid;
   f.status = a.status;
-  if (a.offsets_bits == 32)
-    launch_fill_typed<int32_t>(f, (const int32_t*)a.offsets, a.k, num_sms, st);
-  else
-    launch_fill_typed<int64_t>(f, (const int64_t*)a.offsets, a.k, num_sms, st);
+  const bool streamed = r.gbuf != nullptr;
+  if (a.offsets_bits == 32) {
+    if (streamed)
+      launch_fill_typed<int32_t, true>(f, (const int32_t*)a.offsets, a.k, num_sms, st);
+    else
+      launch_fill_typed<int32_t, false>(f, (const int32_t*)a.offsets, a.k, num_sms, st);
+  } else {
+    if (streamed)
+      launch_fill_typed<int64_t, true>(f, (const int64_t*)a.offsets, a.k, num_sms, st);
+    else
+      launch_fill_typed<int64_t, false>(f, (const int64_t*)a.offsets, a.k, num_sms, st);
+  }
   return cudaGetLastError();
 }
 

@@ -271,3 +271,40 @@ def test_capacity_overflow_is_erange(cuda_device):
         g.prepare(big, [1024, 1024], 1, 0)
     assert e.value.status == 2
     g.close()
+
+
+@pytest.mark.parametrize("a,b,c,bb,buf_blocks,fan", [
+    (0.57, 0.19, 0.19, 8192, 40, [8, 4]),      # buffer << topology: many waves, LRU evictions
+    (0.6, 0.2, 0.15, 4096, 64, [25, 10]),     # skewed: objects larger than a block
+    (0.57, 0.19, 0.19, 16384, 100000, [6, 4, 2]),  # buffer holds everything: hits from hop 2 on
+])
+def test_streamed_topology_matches_oracle(cuda_device, a, b, c, bb, buf_blocks, fan):
+    """Neighbour lists in pinned host memory, loaded block by block into an
+    HBM graph buffer with LRU + pinning: same samples as the oracle."""
+    off, ind = synth.rmat_csr(30000, 14, a, b, c, seed=int(bb + buf_blocks),
+                              offsets_dtype=torch.int64)
+    feats = synth.normal_features(30000, 32, torch.float16, 5)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    max_obj = 8 + 4 * int((off[1:] - off[:-1]).max())
+    host_ind = ind.pin_memory()
+    buf = max(buf_blocks, -(-max_obj // bb) + 1) * bb
+    g = Graph(off.to(cuda_device), host_ind, feats.to(cuda_device), adj_block_bytes=bb,
+              feat_block_bytes=4096, topology_on_host=True, graph_buffer_bytes=buf)
+    for step in range(2):
+        targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), 4, 150, 9, step)
+        g.prepare(targets.to(cuda_device), fan, 77, 10 * step)
+        compare(g, og, targets.numpy(), fan, 77, 10 * step, bb, 4096)
+    cnt = g.counters()
+    assert cnt["topo_loaded_blocks"] > 0 and cnt["topo_waves"] >= 2 * len(fan)
+    if buf_blocks >= 100000:
+        assert cnt["topo_hit_blocks"] > 0
+    g.close()
+
+
+def test_graph_buffer_smaller_than_an_object_is_rejected(cuda_device):
+    off, ind = synth.rmat_csr(5000, 30, 0.6, 0.2, 0.15, seed=1)
+    feats = synth.normal_features(5000, 8, torch.float32, 2)
+    with pytest.raises(AgnesError) as e:
+        Graph(off.to(cuda_device), ind.pin_memory(), feats.to(cuda_device), adj_block_bytes=1024,
+              feat_block_bytes=1024, topology_on_host=True, graph_buffer_bytes=1024)
+    assert e.value.status == 1
