@@ -241,6 +241,9 @@ def main():
                          "line per combination)")
     ap.add_argument("--sweep-H", default="1,2,4,8,16,32,64,128,256")
     ap.add_argument("--sweep-blocks", default="262144,524288,1048576,2097152,4194304")
+    ap.add_argument("--stream-topology", action="store_true",
+                    help="neighbour lists in pinned host memory, loaded into an HBM graph buffer")
+    ap.add_argument("--graph-buffer-gb", type=float, default=4.0)
     ap.add_argument("--stream", action="store_true",
                     help="features in pinned host memory, streamed block-wise per hyperbatch")
     args = ap.parse_args()
@@ -285,8 +288,16 @@ def main():
         features = features.cpu().pin_memory()
         torch.cuda.empty_cache()
         host_link = {"h2d_peak_GBps": pinned_h2d_peak(dev)}
+    topo = None
+    if args.stream_topology:
+        indices = indices.cpu().pin_memory()
+        torch.cuda.empty_cache()
+        topo = {"graph_buffer_bytes": int(args.graph_buffer_gb * 2**30)}
+        if host_link is None:
+            host_link = {"h2d_peak_GBps": pinned_h2d_peak(dev)}
     g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes, device=local,
-              stream=stream, features_on_host=args.stream)
+              stream=stream, features_on_host=args.stream, topology_on_host=args.stream_topology,
+              graph_buffer_bytes=topo["graph_buffer_bytes"] if topo else 0)
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
@@ -371,7 +382,21 @@ def main():
                 "path_algorithmic_bytes_per_step": total_bytes,
                 "path_GBps": total_bytes / (elapsed_ms / args.steps / 1e3) / 1e9}
 
-    if host_link is not None:
+    if topo is not None:
+        # counters are cumulative over the ctx: per-step figures from the timed
+        # region's re-run (first and last of the re-run steps)
+        c0, c1 = counters[0], counters[-1]
+        n = max(1, len(counters) - 1)
+        topo.update({
+            "loaded_bytes_per_step": (c1["topo_loaded_bytes"] - c0["topo_loaded_bytes"]) / n,
+            "loaded_blocks_per_step": (c1["topo_loaded_blocks"] - c0["topo_loaded_blocks"]) / n,
+            "hit_blocks_per_step": (c1["topo_hit_blocks"] - c0["topo_hit_blocks"]) / n,
+            "waves_per_step": (c1["topo_waves"] - c0["topo_waves"]) / n,
+            "topology_bytes": indices.numel() * 4})
+        hb, lb = topo["hit_blocks_per_step"], topo["loaded_blocks_per_step"]
+        topo["hit_rate"] = hb / (hb + lb) if hb + lb else None
+        topo["load_GBps_over_step"] = topo["loaded_bytes_per_step"] / (elapsed_ms / args.steps / 1e3) / 1e9
+    if host_link is not None and args.stream:
         sb = statistics.mean(c["streamed_bytes"] for c in counters)
         host_link.update({"streamed_bytes_per_step": sb,
                           "streamed_blocks_per_step": statistics.mean(c["streamed_blocks"]
@@ -397,7 +422,9 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "int32",
             "data": "synthetic",
             "config": {"workload": f"{w.name}: {w.describe()}"
-                           + (" features streamed from pinned host memory" if args.stream else ""),
+                           + (" features streamed from pinned host memory" if args.stream else "")
+                           + (f" topology in pinned host memory, {args.graph_buffer_gb:g} GB graph buffer"
+                              if args.stream_topology else ""),
                        "graph": {"nodes": info["num_nodes"], "edges": info["num_edges"],
                                  "adj_blocks": info["adj_blocks"], "tiles": info["tiles"],
                                  "feat_blocks": info["feat_blocks"]},
@@ -410,6 +437,7 @@ def main():
                        "counters_last_step": counters[-1] if counters else None,
                        "gen_seconds": round(gen_s, 1)},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "host_link": host_link,
+            "topology_streaming": topo,
             "gpu_launches": kernel_launches_per_step(K) * args.steps,
             "clocks": clocks,
             "phases_ms": {"names": ["bucket_targets"] + [f"hop{h + 1}_{p}" for h in range(K)
@@ -486,7 +514,9 @@ def run_reference(args, w, world, rank):
            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "int32", "data": "synthetic", "impl": "reference",
            "config": {"workload": f"{w.name}: {w.describe()}"
-                           + (" features streamed from pinned host memory" if args.stream else ""), "H": w.H, "B": w.B,
+                           + (" features streamed from pinned host memory" if args.stream else "")
+                           + (f" topology in pinned host memory, {args.graph_buffer_gb:g} GB graph buffer"
+                              if args.stream_topology else ""), "H": w.H, "B": w.B,
                       "fanouts": list(w.fanouts)},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                             "sample": sample},

@@ -125,7 +125,11 @@ struct agnes_ctx {
   struct Topo {
     bool on = false;
     const int32_t* host_indices = nullptr;
+    const int32_t* dev_view = nullptr;  // device address of host_indices
     int64_t slots = 0, epb = 0;
+    int2* d_jobs = nullptr;             // per wave: (block, slot) copies for the loader
+    int2* h_jobs = nullptr;             // pinned staging of the jobs
+    int32_t jobs_cap = 0;
     int32_t* gbuf = nullptr;
     int32_t* d_slot = nullptr;          // n_blocks: slot of each physical block, -1 if absent
     int32_t* h_slot_stage = nullptr;    // pinned staging for uploads of the slot table
@@ -133,15 +137,15 @@ struct agnes_ctx {
     std::vector<int32_t> block_of;      // slot -> block or -1
     std::vector<int32_t> prev, next;    // LRU list over slots (head = least recent)
     int32_t head = -1, tail = -1;
-    std::vector<uint32_t> pinned;       // slot -> wave it is pinned for
-    uint32_t wave = 0;
+    std::vector<uint32_t> pinned;       // slot -> wave it is pinned for (0: never)
+    uint32_t wave = 2;                  // waves count from 3, so 0 is always evictable
     std::vector<int64_t> e0, e1;        // block edge ranges
     std::vector<int32_t> start_block;   // n_starts + 1 (sentinel n_blocks)
     std::vector<int32_t> run_first_tile;
     uint8_t* d_need = nullptr;
     uint8_t* h_need = nullptr;
     cudaStream_t copy = nullptr;
-    cudaEvent_t uploaded = nullptr, wave_done = nullptr;
+    cudaEvent_t uploaded = nullptr, wave_done[2] = {nullptr, nullptr};
     bool uploaded_used = false;
     int64_t loaded_blocks = 0, loaded_bytes = 0, hits = 0, waves = 0;
   } topo;
@@ -455,7 +459,10 @@ agnes_status agnes_free(agnes_ctx* ctx) {
     agnes_ctx::Topo& tp = ctx->topo;
     if (tp.copy) cudaStreamDestroy(tp.copy);
     if (tp.uploaded) cudaEventDestroy(tp.uploaded);
-    if (tp.wave_done) cudaEventDestroy(tp.wave_done);
+    for (int i = 0; i < 2; ++i)
+      if (tp.wave_done[i]) cudaEventDestroy(tp.wave_done[i]);
+    cudaFree(tp.d_jobs);
+    if (tp.h_jobs) cudaFreeHost(tp.h_jobs);
     cudaFree(tp.gbuf);
     cudaFree(tp.d_slot);
     cudaFree(tp.d_need);
@@ -530,9 +537,9 @@ static agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cu
   }
   tp.slots = d->graph_buffer_bytes > 0 ? d->graph_buffer_bytes / d->adj_block_bytes : nb;
   if (tp.slots > nb) tp.slots = nb;
-  if (tp.slots < longest) {
-    set_err(ctx, "graph_buffer_bytes holds %lld blocks; the largest object needs %lld",
-            (long long)tp.slots, (long long)longest);
+  if (tp.slots < 2 * longest) {
+    set_err(ctx, "graph_buffer_bytes holds %lld blocks; two waves of the largest object need %lld",
+            (long long)tp.slots, (long long)(2 * longest));
     return AGNES_EINVAL;
   }
   CK(ctx, cudaMalloc((void**)&tp.gbuf, sizeof(int32_t) * (size_t)(tp.slots * tp.epb)));
@@ -543,7 +550,16 @@ static agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cu
   CK(ctx, cudaMemsetAsync(tp.d_slot, 0xff, sizeof(int32_t) * (size_t)nb, st));
   CK(ctx, cudaStreamCreateWithFlags(&tp.copy, cudaStreamNonBlocking));
   CK(ctx, cudaEventCreateWithFlags(&tp.uploaded, cudaEventDisableTiming));
-  CK(ctx, cudaEventCreateWithFlags(&tp.wave_done, cudaEventDisableTiming));
+  for (int i = 0; i < 2; ++i)
+    CK(ctx, cudaEventCreateWithFlags(&tp.wave_done[i], cudaEventDisableTiming));
+  {
+    void* dv = nullptr;
+    CK(ctx, cudaHostGetDevicePointer(&dv, const_cast<int32_t*>(d->indices), 0));
+    tp.dev_view = (const int32_t*)dv;
+  }
+  tp.jobs_cap = (int32_t)(tp.slots < nb ? tp.slots : nb);
+  CK(ctx, cudaMalloc((void**)&tp.d_jobs, sizeof(int2) * (size_t)tp.jobs_cap));
+  CK(ctx, cudaMallocHost((void**)&tp.h_jobs, sizeof(int2) * (size_t)tp.jobs_cap));
   tp.slot_of.assign((size_t)nb, -1);
   tp.block_of.assign((size_t)tp.slots, -1);
   tp.pinned.assign((size_t)tp.slots, 0);
@@ -729,6 +745,9 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
   agnes_ctx::Topo& tp = ctx->topo;
   const int64_t ns = ctx->bt.n_starts, nb = ctx->bt.n_blocks;
   const int32_t H = w.H, T = (int32_t)ctx->bt.T;
+  // a wave may use half the buffer: the previous wave's blocks stay pinned
+  // while it samples, so the next wave's blocks load at the same time
+  const int64_t wave_cap = tp.slots / 2;
   CK(ctx, launch_mark_runs(w.fcell_off[cur], T, H, ctx->bt.tile_adj_start, tp.d_need, ns, w.status,
                            st));
   CK(ctx, cudaMemcpyAsync(tp.h_need, tp.d_need, (size_t)ns, cudaMemcpyDeviceToHost, st));
@@ -736,27 +755,30 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
   int64_t r = 0;
   while (r < ns && !tp.h_need[r]) ++r;
   while (r < ns) {
+    // the staging buffers (jobs, slot table) are rewritten below: wait until
+    // the previous wave's upload and loads have consumed them
+    if (tp.uploaded_used) CK(ctx, cudaEventSynchronize(tp.uploaded));
     tp.wave += 1;
     const uint32_t wave = tp.wave;
     int64_t pinned_now = 0;
+    int32_t njobs = 0;
     const int64_t r_first = r;
     int64_t r_last = r;
-    // the previous wave must be done before its slots can be overwritten
-    CK(ctx, cudaStreamWaitEvent(tp.copy, tp.wave_done, 0));
     while (r < ns) {
       if (!tp.h_need[r]) {
         ++r;
         continue;
       }
       const int32_t b0 = tp.start_block[(size_t)r], b1 = tp.start_block[(size_t)r + 1];
-      if (pinned_now + (b1 - b0) > tp.slots) break;  // wave full
+      if (pinned_now > 0 && pinned_now + (b1 - b0) > wave_cap) break;  // wave full
       for (int32_t b = b0; b < b1; ++b) {
         int32_t sl = tp.slot_of[(size_t)b];
         if (sl >= 0) {
           tp.hits += 1;
         } else {
-          sl = tp.head;  // least recently used slot that is not pinned for this wave
-          while (sl >= 0 && tp.pinned[(size_t)sl] == wave) sl = tp.next[(size_t)sl];
+          // least recently used slot not pinned by this wave or the previous one
+          sl = tp.head;
+          while (sl >= 0 && tp.pinned[(size_t)sl] + 1 >= wave) sl = tp.next[(size_t)sl];
           if (sl < 0) {
             set_err(ctx, "graph buffer exhausted inside a wave");
             return AGNES_EKERNEL;
@@ -765,12 +787,9 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
           if (old >= 0) tp.slot_of[(size_t)old] = -1;
           tp.block_of[(size_t)sl] = b;
           tp.slot_of[(size_t)b] = sl;
-          const int64_t ne = tp.e1[(size_t)b] - tp.e0[(size_t)b];
-          if (ne > 0)
-            CK(ctx, cudaMemcpyAsync(tp.gbuf + (int64_t)sl * tp.epb, tp.host_indices + tp.e0[(size_t)b],
-                                    sizeof(int32_t) * (size_t)ne, cudaMemcpyHostToDevice, tp.copy));
+          tp.h_jobs[njobs++] = make_int2(b, sl);
           tp.loaded_blocks += 1;
-          tp.loaded_bytes += sizeof(int32_t) * ne;
+          tp.loaded_bytes += sizeof(int32_t) * (tp.e1[(size_t)b] - tp.e0[(size_t)b]);
         }
         tp.pinned[(size_t)sl] = wave;
         lru_touch(tp, sl);
@@ -779,12 +798,17 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
       r_last = r;
       ++r;
     }
-    if (pinned_now == 0) break;
-    // upload the slot table (the staging buffer is free once the last upload ran)
-    if (tp.uploaded_used) CK(ctx, cudaEventSynchronize(tp.uploaded));
+    // the slots taken now were last read by wave - 2 at the latest
+    CK(ctx, cudaStreamWaitEvent(tp.copy, tp.wave_done[wave & 1], 0));
     memcpy(tp.h_slot_stage, tp.slot_of.data(), sizeof(int32_t) * (size_t)nb);
     CK(ctx, cudaMemcpyAsync(tp.d_slot, tp.h_slot_stage, sizeof(int32_t) * (size_t)nb,
                             cudaMemcpyHostToDevice, tp.copy));
+    if (njobs > 0) {
+      CK(ctx, cudaMemcpyAsync(tp.d_jobs, tp.h_jobs, sizeof(int2) * (size_t)njobs,
+                              cudaMemcpyHostToDevice, tp.copy));
+      CK(ctx, launch_load_blocks(tp.dev_view, ctx->bt.blk_e0, ctx->bt.blk_e1, tp.d_jobs, njobs,
+                                 tp.gbuf, tp.epb, ctx->num_sms, tp.copy));
+    }
     CK(ctx, cudaEventRecord(tp.uploaded, tp.copy));
     tp.uploaded_used = true;
     CK(ctx, cudaStreamWaitEvent(st, tp.uploaded, 0));
@@ -799,7 +823,7 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
     fr.bb = ctx->adj_block_bytes;
     CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h], w.nbr,
                                w.scnt, w.scell, w.srank, fr, ctx->num_sms, st));
-    CK(ctx, cudaEventRecord(tp.wave_done, st));
+    CK(ctx, cudaEventRecord(tp.wave_done[wave & 1], st));
     tp.waves += 1;
     while (r < ns && !tp.h_need[r]) ++r;
   }

@@ -126,6 +126,37 @@ __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int
     if (cell_off[c + 1] > cell_off[c]) flags[map[c / H]] = 1;
 }
 
+// Copies the edge lists of physical blocks from pinned host memory (read in
+// place over the host link) into their graph-buffer slots: job i copies
+// block jobs[i].x into slot jobs[i].y.  One CTA per job; 16-byte vectors
+// where the source is aligned, single words for the ragged ends.
+__global__ void __launch_bounds__(kThreads)
+load_blocks_kernel(const int32_t* __restrict__ host_indices, const int64_t* __restrict__ e0,
+                   const int64_t* __restrict__ e1, const int2* __restrict__ jobs, int32_t njobs,
+                   int32_t* __restrict__ gbuf, int64_t epb) {
+  for (int32_t i = blockIdx.x; i < njobs; i += gridDim.x) {
+    const int2 jb = jobs[i];
+    const int64_t a = e0[jb.x], n = e1[jb.x] - a;
+    const int32_t* src = host_indices + a;
+    int32_t* dst = gbuf + (int64_t)jb.y * epb;
+    // head words until the source is 16-byte aligned (the slot start is)
+    int64_t head = (int64_t)((16 - ((uintptr_t)src & 15)) & 15) / 4;
+    if (head > n) head = n;
+    for (int64_t q = threadIdx.x; q < head; q += blockDim.x) dst[q] = src[q];
+    const int64_t nv = (n - head) / 4;
+    const int4* s4 = (const int4*)(src + head);
+    for (int64_t q = threadIdx.x; q < nv; q += blockDim.x) {
+      const int4 v = s4[q];
+      int32_t* d = dst + head + 4 * q;  // the slot may not be 16-byte aligned here
+      d[0] = v.x;
+      d[1] = v.y;
+      d[2] = v.z;
+      d[3] = v.w;
+    }
+    for (int64_t q = head + 4 * nv + threadIdx.x; q < n; q += blockDim.x) dst[q] = src[q];
+  }
+}
+
 // need[tile_adj_start[t]] = 1 for every tile t with a frontier entry.
 __global__ void mark_runs_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
                                  const int32_t* __restrict__ tile_adj_start,
@@ -236,6 +267,15 @@ cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, con
   if (cell_off && map)
     mark_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, map, flags, status);
   count_flags_kernel<<<256, 256, 0, st>>>(flags, n_flags, count);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_load_blocks(const int32_t* host_indices, const int64_t* e0, const int64_t* e1,
+                               const int2* jobs, int32_t njobs, int32_t* gbuf, int64_t epb,
+                               int num_sms, cudaStream_t st) {
+  if (njobs <= 0) return cudaSuccess;
+  const int grid = njobs < num_sms * 4 ? njobs : num_sms * 4;
+  load_blocks_kernel<<<grid, kThreads, 0, st>>>(host_indices, e0, e1, jobs, njobs, gbuf, epb);
   return cudaGetLastError();
 }
 

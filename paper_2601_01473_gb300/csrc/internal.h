@@ -173,6 +173,12 @@ cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, con
                               uint8_t* flags, int64_t n_flags, int64_t* count,
                               const int32_t* status, cudaStream_t st);
 
+// Copies physical blocks jobs[i].x (edges e0..e1 of host_indices, a device
+// view of pinned host memory) into graph-buffer slots jobs[i].y.
+cudaError_t launch_load_blocks(const int32_t* host_indices, const int64_t* e0, const int64_t* e1,
+                               const int2* jobs, int32_t njobs, int32_t* gbuf, int64_t epb,
+                               int num_sms, cudaStream_t st);
+
 // need[r] = 1 for every block run r whose tiles hold a frontier entry
 // (need is cleared first).
 cudaError_t launch_mark_runs(const int32_t* cell_off, int32_t T, int32_t H,

@@ -287,7 +287,7 @@ def test_streamed_topology_matches_oracle(cuda_device, a, b, c, bb, buf_blocks, 
     og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
     max_obj = 8 + 4 * int((off[1:] - off[:-1]).max())
     host_ind = ind.pin_memory()
-    buf = max(buf_blocks, -(-max_obj // bb) + 1) * bb
+    buf = max(buf_blocks, 2 * (-(-max_obj // bb)) + 2) * bb
     g = Graph(off.to(cuda_device), host_ind, feats.to(cuda_device), adj_block_bytes=bb,
               feat_block_bytes=4096, topology_on_host=True, graph_buffer_bytes=buf)
     for step in range(2):
