@@ -246,6 +246,12 @@ def main():
     ap.add_argument("--graph-buffer-gb", type=float, default=4.0)
     ap.add_argument("--stream", action="store_true",
                     help="features in pinned host memory, streamed block-wise per hyperbatch")
+    ap.add_argument("--feature-cache-gb", type=float, default=0.0,
+                    help="with --stream: HBM feature cache of the most requested blocks")
+    ap.add_argument("--feature-cache-threshold", type=int, default=0,
+                    help="with --stream: requests a block must exceed to be cached")
+    ap.add_argument("--feature-io", default="blocks", choices=["blocks", "rows"],
+                    help="with --stream: load whole feature blocks, or read requested rows in place")
     args = ap.parse_args()
 
     world, rank, local = dist_env()
@@ -297,7 +303,10 @@ def main():
             host_link = {"h2d_peak_GBps": pinned_h2d_peak(dev)}
     g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes, device=local,
               stream=stream, features_on_host=args.stream, topology_on_host=args.stream_topology,
-              graph_buffer_bytes=topo["graph_buffer_bytes"] if topo else 0)
+              graph_buffer_bytes=topo["graph_buffer_bytes"] if topo else 0,
+              feature_cache_bytes=int(args.feature_cache_gb * 2**30) if args.stream else 0,
+              feature_cache_threshold=args.feature_cache_threshold,
+              feature_io=args.feature_io if args.stream else "blocks")
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
@@ -404,6 +413,17 @@ def main():
                           "streamed_GBps": sb / (g_ms / 1e3) / 1e9 if g_ms else None})
         host_link["frac"] = (host_link["streamed_GBps"] / host_link["h2d_peak_GBps"]
                              if host_link["streamed_GBps"] else None)
+        if args.feature_cache_gb > 0:
+            c0, c1 = counters[0], counters[-1]
+            n = max(1, len(counters) - 1)
+            hits = (c1["fcache_hit_blocks"] - c0["fcache_hit_blocks"]) / n
+            loads = (c1["fcache_loaded_blocks"] - c0["fcache_loaded_blocks"]) / n
+            host_link["feature_cache"] = {
+                "bytes": int(args.feature_cache_gb * 2**30),
+                "threshold": args.feature_cache_threshold,
+                "hit_blocks_per_step": hits, "loaded_blocks_per_step": loads,
+                "hit_rate": hits / (hits + host_link["streamed_blocks_per_step"])
+                if hits + host_link["streamed_blocks_per_step"] else None}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -422,7 +442,10 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "int32",
             "data": "synthetic",
             "config": {"workload": f"{w.name}: {w.describe()}"
-                           + (" features streamed from pinned host memory" if args.stream else "")
+                           + (f" features in pinned host memory ({args.feature_io} I/O)"
+                              if args.stream else "")
+                           + (f", {args.feature_cache_gb:g} GB feature cache"
+                              if args.stream and args.feature_cache_gb > 0 else "")
                            + (f" topology in pinned host memory, {args.graph_buffer_gb:g} GB graph buffer"
                               if args.stream_topology else ""),
                        "graph": {"nodes": info["num_nodes"], "edges": info["num_edges"],
@@ -514,7 +537,8 @@ def run_reference(args, w, world, rank):
            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "int32", "data": "synthetic", "impl": "reference",
            "config": {"workload": f"{w.name}: {w.describe()}"
-                           + (" features streamed from pinned host memory" if args.stream else "")
+                           + (f" features in pinned host memory ({args.feature_io} I/O)"
+                              if args.stream else "")
                            + (f" topology in pinned host memory, {args.graph_buffer_gb:g} GB graph buffer"
                               if args.stream_topology else ""), "H": w.H, "B": w.B,
                       "fanouts": list(w.fanouts)},

@@ -77,9 +77,11 @@ typedef struct agnes_ctx agnes_ctx; /* opaque, owned by the library */
  * Host arrays are copied to device memory the library owns.  Device arrays
  * are borrowed: the caller keeps them alive and unchanged until
  * agnes_free.  With features_on_host = 1 the feature matrix stays in pinned
- * host memory (borrowed) and each hyperbatch streams the feature blocks it
- * needs into device staging slots on a side stream (the asynchronous
- * block I/O of Sec. 3.4 (4), with the host link standing in for the SSD).
+ * host memory (borrowed; 16-byte aligned, rows a multiple of 16 bytes) and
+ * each hyperbatch reads what it needs over the host link, which stands in
+ * for the SSD: whole feature blocks into device staging slots on a side
+ * stream (feature_io = AGNES_FEATURE_IO_BLOCKS, the asynchronous block I/O
+ * of Sec. 3.4 (4)), or only the requested rows (AGNES_FEATURE_IO_ROWS).
  * With topology_on_host = 1 the neighbour lists (indices, pinned host
  * memory, borrowed) stay on the host; offsets are still copied or borrowed
  * in device memory.  Each hop loads the topology blocks its frontier touches
@@ -87,7 +89,15 @@ typedef struct agnes_ctx agnes_ctx; /* opaque, owned by the library */
  * at least the largest object), reusing resident blocks and evicting the
  * least recently used unpinned ones; a block stays pinned until the hop has
  * sampled all its requests (Sec. 3.4 (1)).  When a hop's blocks do not fit,
- * the hop runs in waves of blocks in ascending order. */
+ * the hop runs in waves of blocks in ascending order.
+ * With features_on_host = 1 and feature_cache_bytes > 0, an HBM feature
+ * cache (Sec. 3.4 (2)) keeps the feature blocks whose cumulative request
+ * count (rows gathered from them, over all hyperbatches so far) exceeds
+ * feature_cache_threshold, hottest first, up to its capacity
+ * (feature_cache_bytes / feature block size blocks).  The set is re-picked
+ * after each hyperbatch; a newly admitted block is loaded into its cache
+ * slot the next time a hyperbatch touches it and read in place from then on.
+ * The cache holds whole feature blocks, the unit of host transfers. */
 typedef struct {
   int64_t num_nodes;
   int64_t num_edges;
@@ -102,7 +112,22 @@ typedef struct {
   int64_t feat_block_bytes;
   int32_t topology_on_host; /* 1: indices stay in pinned host memory (see below) */
   int64_t graph_buffer_bytes; /* HBM graph buffer for topology_on_host (0: whole topology) */
+  int64_t feature_cache_bytes;     /* features_on_host: HBM feature cache (0: none) */
+  int64_t feature_cache_threshold; /* cumulative requests a block must exceed to be cached */
+  int32_t feature_io;              /* features_on_host: AGNES_FEATURE_IO_BLOCKS or _ROWS */
 } agnes_graph_desc;
+
+/* How host-resident features reach the gather (features_on_host = 1).
+ * BLOCKS: every touched feature block is loaded whole into HBM, batch by
+ *   batch, overlapped with the gather (the block-wise I/O of Sec. 3.3 and the
+ *   asynchronous I/O of Sec. 3.4 (4)); 0, the default.
+ * ROWS: the gather reads each requested row in place from pinned host memory
+ *   over the host link (or from the feature cache), so only requested rows
+ *   cross the link.  Not in the paper: its storage is an SSD, where small
+ *   reads are slow; a cache-coherent host link serves row-sized reads at the
+ *   rate of bulk copies. */
+#define AGNES_FEATURE_IO_BLOCKS 0
+#define AGNES_FEATURE_IO_ROWS 1
 
 /* Loads a graph on `device` and builds its block tables: the object index
  * table T^g_obj of Sec. 3.2 (greedy in-order packing of objects of
@@ -205,12 +230,17 @@ typedef struct {
   int64_t rows;                     /* sum over minibatches of num_nodes */
   int64_t distinct_rows;            /* distinct node ids among all gathered rows */
   int64_t row_bytes;
-  int64_t streamed_bytes;           /* features_on_host: bytes copied host -> device */
-  int64_t streamed_blocks;          /* features_on_host: feature blocks copied */
+  int64_t streamed_bytes;           /* features_on_host: bytes read over the host link
+                                       (row mode: requested rows, before L2 reuse) */
+  int64_t streamed_blocks;          /* features_on_host: touched feature blocks not
+                                       served by the feature cache */
+  /* the rest are totals since agnes_load_graph, not per hyperbatch */
   int64_t topo_loaded_blocks;       /* topology_on_host: blocks copied into the graph buffer */
   int64_t topo_loaded_bytes;
   int64_t topo_hit_blocks;          /* needed blocks already resident */
   int64_t topo_waves;               /* fill launches over all hops */
+  int64_t fcache_hit_blocks;        /* feature blocks read in place from the feature cache */
+  int64_t fcache_loaded_blocks;     /* feature blocks copied into the feature cache */
 } agnes_counters;
 agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
 

@@ -19,6 +19,7 @@ MAX_HOPS = 8
 MAX_FANOUT = 1024
 
 F32, F16 = 0, 1
+FEATURE_IO = {"blocks": 0, "rows": 1}  # AGNES_FEATURE_IO_BLOCKS / _ROWS
 _DTYPES = {torch.float32: F32, torch.float16: F16}
 _TORCH_OF = {F32: torch.float32, F16: torch.float16}
 
@@ -48,6 +49,9 @@ class _GraphDesc(ctypes.Structure):
         ("feat_block_bytes", ctypes.c_int64),
         ("topology_on_host", ctypes.c_int32),
         ("graph_buffer_bytes", ctypes.c_int64),
+        ("feature_cache_bytes", ctypes.c_int64),
+        ("feature_cache_threshold", ctypes.c_int64),
+        ("feature_io", ctypes.c_int32),
     ]
 
 
@@ -93,6 +97,8 @@ class _Counters(ctypes.Structure):
         ("topo_loaded_bytes", ctypes.c_int64),
         ("topo_hit_blocks", ctypes.c_int64),
         ("topo_waves", ctypes.c_int64),
+        ("fcache_hit_blocks", ctypes.c_int64),
+        ("fcache_loaded_blocks", ctypes.c_int64),
     ]
 
 
@@ -233,7 +239,8 @@ class Graph:
     def __init__(self, offsets, indices, features, adj_block_bytes: int = 1 << 20,
                  feat_block_bytes: int | None = None, device: int = 0, stream=None,
                  features_on_host: bool = False, topology_on_host: bool = False,
-                 graph_buffer_bytes: int = 0):
+                 graph_buffer_bytes: int = 0, feature_cache_bytes: int = 0,
+                 feature_cache_threshold: int = 0, feature_io: str = "blocks"):
         if offsets.dtype not in (torch.int32, torch.int64):
             raise TypeError("offsets must be int32 or int64")
         if indices.dtype != torch.int32:
@@ -261,6 +268,11 @@ class Graph:
         d.feat_block_bytes = feat_block_bytes if feat_block_bytes is not None else adj_block_bytes
         d.topology_on_host = int(topology_on_host)
         d.graph_buffer_bytes = graph_buffer_bytes
+        d.feature_cache_bytes = feature_cache_bytes
+        d.feature_cache_threshold = feature_cache_threshold
+        if feature_io not in FEATURE_IO:
+            raise ValueError(f"feature_io must be one of {sorted(FEATURE_IO)}")
+        d.feature_io = FEATURE_IO[feature_io]
         ctx = ctypes.c_void_p()
         with torch.cuda.device(self.device):
             rc = lib().agnes_load_graph(ctypes.byref(d), device, _stream_handle(stream),
@@ -340,7 +352,9 @@ class Graph:
                 "rows": c.rows, "distinct_rows": c.distinct_rows, "row_bytes": c.row_bytes,
                 "streamed_bytes": c.streamed_bytes, "streamed_blocks": c.streamed_blocks,
                 "topo_loaded_blocks": c.topo_loaded_blocks, "topo_loaded_bytes": c.topo_loaded_bytes,
-                "topo_hit_blocks": c.topo_hit_blocks, "topo_waves": c.topo_waves}
+                "topo_hit_blocks": c.topo_hit_blocks, "topo_waves": c.topo_waves,
+                "fcache_hit_blocks": c.fcache_hit_blocks,
+                "fcache_loaded_blocks": c.fcache_loaded_blocks}
 
     def info(self) -> dict:
         g = _GraphInfo()

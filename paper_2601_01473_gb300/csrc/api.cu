@@ -15,6 +15,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <new>
 #include <vector>
 
@@ -93,6 +94,8 @@ struct agnes_ctx {
   int32_t feat_dtype = 0;
   int64_t feat_dim = 0, row_bytes = 0;
   int32_t features_on_host = 0;
+  int32_t feature_io = AGNES_FEATURE_IO_BLOCKS;
+  const char* features_dev = nullptr;  // device view of host-resident features
   int64_t adj_block_bytes = 0, feat_block_bytes = 0;
   BlockTables bt;
 
@@ -115,9 +118,28 @@ struct agnes_ctx {
   cudaEvent_t slot_copied[kStreamSlots] = {nullptr};
   cudaEvent_t slot_free[kStreamSlots] = {nullptr};
   bool slot_used[kStreamSlots] = {false};
-  uint8_t* h_flags = nullptr;    // pinned, one byte per feature block
+  int32_t* d_counts = nullptr;   // requests per feature block (this hyperbatch)
+  int32_t* h_counts = nullptr;   // pinned copy
   int32_t* h_touched = nullptr;  // pinned, touched feature blocks of the last hyperbatch
   int32_t* d_touched = nullptr;
+  unsigned long long* h_src = nullptr;  // pinned: device address of each touched block's copy
+  unsigned long long* d_src = nullptr;
+  int32_t* h_job_blk = nullptr;         // pinned: blocks to load this hyperbatch ...
+  int32_t* d_job_blk = nullptr;
+  unsigned long long* h_job_dst = nullptr;  // ... and where to
+  unsigned long long* d_job_dst = nullptr;
+  unsigned long long* h_addr = nullptr;  // row mode: current address of every feature block
+  unsigned long long* d_addr = nullptr;
+  cudaEvent_t gather_start = nullptr;
+  // feature cache C_f (Sec. 3.4 (2)): blocks whose cumulative request count
+  // reaches the threshold, hottest first, up to fcache_slots blocks
+  int64_t fcache_slots = 0, fcache_threshold = 0;
+  char* fcache = nullptr;
+  std::vector<int64_t> acc;          // cumulative requests per feature block
+  std::vector<int32_t> cslot_of;     // block -> cache slot, -1 if not admitted
+  std::vector<int32_t> cblock_of;    // cache slot -> block, -1 if free
+  std::vector<uint8_t> cresident;    // cache slot holds its block's rows
+  int64_t fcache_hits = 0, fcache_loads = 0;
   std::vector<int32_t> fblock_first_tile;
   int64_t streamed_bytes = 0, streamed_blocks = 0;
 
@@ -453,8 +475,19 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (ctx->copy_stream) cudaStreamDestroy(ctx->copy_stream);
   cudaFree(ctx->slots);
   cudaFree(ctx->d_touched);
-  if (ctx->h_flags) cudaFreeHost(ctx->h_flags);
+  cudaFree(ctx->d_counts);
+  cudaFree(ctx->d_src);
+  cudaFree(ctx->d_job_blk);
+  cudaFree(ctx->d_job_dst);
+  cudaFree(ctx->d_addr);
+  cudaFree(ctx->fcache);
+  if (ctx->gather_start) cudaEventDestroy(ctx->gather_start);
+  if (ctx->h_counts) cudaFreeHost(ctx->h_counts);
   if (ctx->h_touched) cudaFreeHost(ctx->h_touched);
+  if (ctx->h_src) cudaFreeHost(ctx->h_src);
+  if (ctx->h_job_blk) cudaFreeHost(ctx->h_job_blk);
+  if (ctx->h_job_dst) cudaFreeHost(ctx->h_job_dst);
+  if (ctx->h_addr) cudaFreeHost(ctx->h_addr);
   {
     agnes_ctx::Topo& tp = ctx->topo;
     if (tp.copy) cudaStreamDestroy(tp.copy);
@@ -489,22 +522,51 @@ static agnes_status adopt_or_copy(agnes_ctx* ctx, const void* src, size_t bytes,
   return AGNES_OK;
 }
 
-// Staging ring, copy stream and host tables for host-resident features.
-static agnes_status setup_streaming(agnes_ctx* ctx, cudaStream_t st) {
+// Staging ring (block mode), feature cache, copy stream and host tables for
+// host-resident features.
+static agnes_status setup_streaming(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStream_t st) {
   const int64_t nfb = ctx->bt.n_feat_blocks;
-  ctx->slot_bytes = (int64_t)kStreamBatchBlocks * ctx->bt.rows_per_feat_block * ctx->row_bytes;
+  const int64_t blk = ctx->bt.rows_per_feat_block * ctx->row_bytes;
+  {
+    void* dv = nullptr;
+    CK(ctx, cudaHostGetDevicePointer(&dv, ctx->features, 0));
+    ctx->features_dev = (const char*)dv;
+  }
   CK(ctx, cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking));
   for (int i = 0; i < kStreamSlots; ++i) {
     CK(ctx, cudaEventCreateWithFlags(&ctx->slot_copied[i], cudaEventDisableTiming));
     CK(ctx, cudaEventCreateWithFlags(&ctx->slot_free[i], cudaEventDisableTiming));
   }
-  CK(ctx, cudaMalloc((void**)&ctx->slots, (size_t)(ctx->slot_bytes * kStreamSlots)));
-  CK(ctx, cudaMalloc((void**)&ctx->d_touched, sizeof(int32_t) * (size_t)(nfb + 1)));
-  CK(ctx, cudaMallocHost((void**)&ctx->h_flags, (size_t)(nfb + 1)));
-  CK(ctx, cudaMallocHost((void**)&ctx->h_touched, sizeof(int32_t) * (size_t)(nfb + 1)));
-  ctx->fblock_first_tile.resize((size_t)(nfb + 1));
+  CK(ctx, cudaEventCreateWithFlags(&ctx->gather_start, cudaEventDisableTiming));
+  if (ctx->feature_io == AGNES_FEATURE_IO_BLOCKS) {
+    ctx->slot_bytes = (int64_t)kStreamBatchBlocks * blk;
+    CK(ctx, cudaMalloc((void**)&ctx->slots, (size_t)(ctx->slot_bytes * kStreamSlots)));
+  }
+  const size_t n1 = (size_t)(nfb + 1);
+  CK(ctx, cudaMalloc((void**)&ctx->d_touched, sizeof(int32_t) * n1));
+  CK(ctx, cudaMalloc((void**)&ctx->d_counts, sizeof(int32_t) * n1));
+  CK(ctx, cudaMalloc((void**)&ctx->d_src, sizeof(unsigned long long) * n1));
+  CK(ctx, cudaMalloc((void**)&ctx->d_job_blk, sizeof(int32_t) * n1));
+  CK(ctx, cudaMalloc((void**)&ctx->d_job_dst, sizeof(unsigned long long) * n1));
+  CK(ctx, cudaMalloc((void**)&ctx->d_addr, sizeof(unsigned long long) * n1));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_counts, sizeof(int32_t) * n1));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_touched, sizeof(int32_t) * n1));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_src, sizeof(unsigned long long) * n1));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_job_blk, sizeof(int32_t) * n1));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_job_dst, sizeof(unsigned long long) * n1));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_addr, sizeof(unsigned long long) * n1));
+  ctx->fblock_first_tile.resize(n1);
   CK(ctx, cudaMemcpyAsync(ctx->fblock_first_tile.data(), ctx->bt.fblock_first_tile,
-                          sizeof(int32_t) * (size_t)(nfb + 1), cudaMemcpyDeviceToHost, st));
+                          sizeof(int32_t) * n1, cudaMemcpyDeviceToHost, st));
+  ctx->fcache_slots = d->feature_cache_bytes > 0 ? d->feature_cache_bytes / blk : 0;
+  if (ctx->fcache_slots > nfb) ctx->fcache_slots = nfb;
+  ctx->fcache_threshold = d->feature_cache_threshold;
+  if (ctx->fcache_slots > 0)
+    CK(ctx, cudaMalloc((void**)&ctx->fcache, (size_t)(ctx->fcache_slots * blk)));
+  ctx->acc.assign((size_t)nfb, 0);
+  ctx->cslot_of.assign((size_t)nfb, -1);
+  ctx->cblock_of.assign((size_t)ctx->fcache_slots, -1);
+  ctx->cresident.assign((size_t)ctx->fcache_slots, 0);
   CK(ctx, cudaStreamSynchronize(st));
   return AGNES_OK;
 }
@@ -644,6 +706,20 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
     set_err(nullptr, "features_on_host needs feature rows of a multiple of 16 bytes");
     return AGNES_EINVAL;
   }
+  if (d->features_on_host && ((uintptr_t)d->features % 16) != 0) {
+    set_err(nullptr, "features_on_host needs a 16-byte aligned feature matrix");
+    return AGNES_EINVAL;
+  }
+  if (d->feature_io != AGNES_FEATURE_IO_BLOCKS && d->feature_io != AGNES_FEATURE_IO_ROWS) {
+    set_err(nullptr, "feature_io must be AGNES_FEATURE_IO_BLOCKS or AGNES_FEATURE_IO_ROWS");
+    return AGNES_EINVAL;
+  }
+  if (d->feature_cache_bytes < 0 || d->feature_cache_threshold < 0 ||
+      (d->feature_cache_bytes > 0 && !d->features_on_host)) {
+    set_err(nullptr, "feature_cache_bytes and feature_cache_threshold must be >= 0, and a "
+                     "feature cache needs features_on_host");
+    return AGNES_EINVAL;
+  }
   if (cudaSetDevice(device) != cudaSuccess) {
     cudaGetLastError();
     set_err(nullptr, "invalid device %d", device);
@@ -664,6 +740,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   ctx->feat_dim = d->feat_dim;
   ctx->row_bytes = row_bytes;
   ctx->features_on_host = d->features_on_host;
+  ctx->feature_io = d->feature_io;
   ctx->adj_block_bytes = d->adj_block_bytes;
   ctx->feat_block_bytes = d->feat_block_bytes;
   cudaStream_t st = (cudaStream_t)cuda_stream;
@@ -717,7 +794,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
                                        sizeof(ctx->err));
     if (e != cudaSuccess) rc = e == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;
   }
-  if (rc == AGNES_OK && d->features_on_host) rc = setup_streaming(ctx, st);
+  if (rc == AGNES_OK && d->features_on_host) rc = setup_streaming(ctx, d, st);
   if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0) rc = setup_topology(ctx, d, st);
   if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
     set_err(ctx, "cudaEventCreate failed");
@@ -830,55 +907,231 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
   return AGNES_OK;
 }
 
-// Gather with host-resident features (Sec. 3.4 (4) asynchronous I/O, the
-// host link standing in for the SSD): the touched feature blocks are read
-// back once, then copied batch by batch into the ring of HBM slots on the
-// side stream; each batch's gather waits for its slot's copy event and the
-// next copy into a slot waits for the gather that last read it.
-static agnes_status gather_streamed(agnes_ctx* ctx, int cur, cudaStream_t st) {
+// Bytes of feature block b (the last block of the matrix may be short).
+static int64_t feat_block_bytes_of(const agnes_ctx* ctx, int32_t b) {
+  const int64_t rpb = ctx->bt.rows_per_feat_block;
+  const int64_t r0 = (int64_t)b * rpb;
+  const int64_t r1 = r0 + rpb < ctx->N ? r0 + rpb : ctx->N;
+  return (r1 - r0) * ctx->row_bytes;
+}
+
+// Block mode (Sec. 3.3 block-wise I/O, Sec. 3.4 (4) asynchronous I/O, the
+// host link standing in for the SSD).  A touched block that is cached and
+// resident is read in place; one admitted to the cache but not yet loaded is
+// loaded into its cache slot; any other is loaded into the ring of HBM
+// staging slots.  Batch by batch, a loader kernel on the side stream reads
+// the batch's blocks over the host link; the batch's gather waits for it and
+// the next load into a slot waits for the gather that last read it.
+static agnes_status gather_blocks_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* bytes_out,
+                                     int64_t* hits_out, cudaStream_t st) {
   Workspace& w = ctx->ws;
-  const int64_t nfb = ctx->bt.n_feat_blocks;
   const int64_t rpb = ctx->bt.rows_per_feat_block;
   const int64_t rb = ctx->row_bytes;
+  const int64_t blk = rpb * rb;
   const int32_t H = w.H;
-  CK(ctx, cudaMemcpyAsync(ctx->h_flags, w.feat_flags, (size_t)nfb, cudaMemcpyDeviceToHost, st));
-  CK(ctx, cudaStreamSynchronize(st));
-  int32_t n = 0;
-  for (int64_t b = 0; b < nfb; ++b)
-    if (ctx->h_flags[b]) ctx->h_touched[n++] = (int32_t)b;
-  if (n > 0)
+  const int32_t nbatch = (n + kStreamBatchBlocks - 1) / kStreamBatchBlocks;
+  std::vector<int32_t> job0((size_t)nbatch + 1, 0);
+  int32_t nj = 0;
+  int64_t bytes = 0, hits = 0;
+  for (int32_t batch = 0; batch < nbatch; ++batch) {
+    const int32_t i0 = batch * kStreamBatchBlocks;
+    const int32_t i1 = i0 + kStreamBatchBlocks < n ? i0 + kStreamBatchBlocks : n;
+    char* slot = ctx->slots + (int64_t)(batch % kStreamSlots) * ctx->slot_bytes;
+    job0[(size_t)batch] = nj;
+    int32_t p = 0;
+    for (int32_t i = i0; i < i1; ++i) {
+      const int32_t b = ctx->h_touched[i];
+      const int32_t cs = ctx->fcache_slots ? ctx->cslot_of[(size_t)b] : -1;
+      unsigned long long a;
+      bool load = true;
+      if (cs >= 0) {
+        a = (unsigned long long)(uintptr_t)(ctx->fcache + (int64_t)cs * blk);
+        if (ctx->cresident[(size_t)cs]) {
+          load = false;
+          hits += 1;
+        } else {
+          ctx->cresident[(size_t)cs] = 1;
+          ctx->fcache_loads += 1;
+        }
+      } else {
+        a = (unsigned long long)(uintptr_t)(slot + (int64_t)p++ * blk);
+      }
+      ctx->h_src[i] = a;
+      if (load) {
+        ctx->h_job_blk[nj] = b;
+        ctx->h_job_dst[nj] = a;
+        ++nj;
+        bytes += feat_block_bytes_of(ctx, b);
+      }
+    }
+  }
+  job0[(size_t)nbatch] = nj;
+  if (n > 0) {
     CK(ctx, cudaMemcpyAsync(ctx->d_touched, ctx->h_touched, sizeof(int32_t) * n,
                             cudaMemcpyHostToDevice, st));
-  int64_t bytes = 0;
-  for (int32_t i0 = 0, batch = 0; i0 < n; i0 += kStreamBatchBlocks, ++batch) {
+    CK(ctx, cudaMemcpyAsync(ctx->d_src, ctx->h_src, sizeof(unsigned long long) * n,
+                            cudaMemcpyHostToDevice, st));
+  }
+  if (nj > 0) {
+    CK(ctx, cudaMemcpyAsync(ctx->d_job_blk, ctx->h_job_blk, sizeof(int32_t) * nj,
+                            cudaMemcpyHostToDevice, st));
+    CK(ctx, cudaMemcpyAsync(ctx->d_job_dst, ctx->h_job_dst, sizeof(unsigned long long) * nj,
+                            cudaMemcpyHostToDevice, st));
+  }
+  // the job tables are on the device, and cache slots are no longer read by
+  // earlier gathers, once st reaches this point
+  CK(ctx, cudaEventRecord(ctx->gather_start, st));
+  CK(ctx, cudaStreamWaitEvent(ctx->copy_stream, ctx->gather_start, 0));
+  for (int32_t batch = 0; batch < nbatch; ++batch) {
+    const int32_t i0 = batch * kStreamBatchBlocks;
     const int32_t nb = n - i0 < kStreamBatchBlocks ? n - i0 : kStreamBatchBlocks;
     const int s = batch % kStreamSlots;
-    char* slot = ctx->slots + (int64_t)s * ctx->slot_bytes;
     if (ctx->slot_used[s]) CK(ctx, cudaStreamWaitEvent(ctx->copy_stream, ctx->slot_free[s], 0));
-    for (int32_t p = 0; p < nb;) {  // one copy per run of consecutive blocks
-      int32_t q = p;
-      while (q + 1 < nb && ctx->h_touched[i0 + q + 1] == ctx->h_touched[i0 + q] + 1) ++q;
-      const int64_t r0 = (int64_t)ctx->h_touched[i0 + p] * rpb;
-      int64_t r1 = ((int64_t)ctx->h_touched[i0 + q] + 1) * rpb;
-      if (r1 > ctx->N) r1 = ctx->N;
-      const int64_t nbytes = (r1 - r0) * rb;
-      CK(ctx, cudaMemcpyAsync(slot + (int64_t)p * rpb * rb, (const char*)ctx->features + r0 * rb,
-                              (size_t)nbytes, cudaMemcpyHostToDevice, ctx->copy_stream));
-      bytes += nbytes;
-      p = q + 1;
-    }
+    const int32_t j0 = job0[(size_t)batch], j1 = job0[(size_t)batch + 1];
+    CK(ctx, launch_load_feat_blocks(ctx->features_dev, ctx->N * rb, ctx->d_job_blk + j0,
+                                    ctx->d_job_dst + j0, j1 - j0, blk, ctx->num_sms,
+                                    ctx->copy_stream));
     CK(ctx, cudaEventRecord(ctx->slot_copied[s], ctx->copy_stream));
     CK(ctx, cudaStreamWaitEvent(st, ctx->slot_copied[s], 0));
     const int64_t cell_lo = (int64_t)ctx->fblock_first_tile[ctx->h_touched[i0]] * H;
     const int64_t cell_hi = (int64_t)ctx->fblock_first_tile[ctx->h_touched[i0 + nb - 1] + 1] * H;
-    CK(ctx, launch_gather_staged(slot, rb, rpb, ctx->d_touched + i0, nb, w.fb_id[cur],
+    CK(ctx, launch_gather_staged(ctx->d_src + i0, rb, rpb, ctx->d_touched + i0, nb, w.fb_id[cur],
                                  w.fb_pos[cur], w.fcell_off[cur], cell_lo, cell_hi, w.feats_out,
                                  w.status, ctx->num_sms, st));
     CK(ctx, cudaEventRecord(ctx->slot_free[s], st));
     ctx->slot_used[s] = true;
   }
+  *bytes_out = bytes;
+  *hits_out = hits;
+  return AGNES_OK;
+}
+
+// Row mode: each gathered row is read where its block is -- in place from
+// pinned host memory over the host link (only the requested rows cross it),
+// or from the block's feature-cache slot.  Touched blocks admitted to the
+// cache but not yet loaded are loaded whole first (by the loader kernel, on
+// the caller's stream), then one gather walks the whole final bucket through
+// the per-block address table.
+static agnes_status gather_rows_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* bytes_out,
+                                   int64_t* hits_out, cudaStream_t st) {
+  Workspace& w = ctx->ws;
+  const int64_t nfb = ctx->bt.n_feat_blocks;
+  const int64_t rpb = ctx->bt.rows_per_feat_block;
+  const int64_t rb = ctx->row_bytes;
+  const int64_t blk = rpb * rb;
+  int32_t nj = 0;
+  int64_t bytes = 0, hits = 0;
+  for (int32_t i = 0; i < n; ++i) {
+    const int32_t b = ctx->h_touched[i];
+    const int32_t cs = ctx->fcache_slots ? ctx->cslot_of[(size_t)b] : -1;
+    if (cs < 0) {
+      bytes += (int64_t)ctx->h_counts[b] * rb;
+    } else if (ctx->cresident[(size_t)cs]) {
+      hits += 1;
+    } else {
+      ctx->h_job_blk[nj] = b;
+      ctx->h_job_dst[nj] = (unsigned long long)(uintptr_t)(ctx->fcache + (int64_t)cs * blk);
+      ++nj;
+      ctx->cresident[(size_t)cs] = 1;
+      ctx->fcache_loads += 1;
+      bytes += feat_block_bytes_of(ctx, b);
+    }
+  }
+  for (int64_t b = 0; b < nfb; ++b) {
+    const int32_t cs = ctx->fcache_slots ? ctx->cslot_of[(size_t)b] : -1;
+    ctx->h_addr[b] = (cs >= 0 && ctx->cresident[(size_t)cs])
+                         ? (unsigned long long)(uintptr_t)(ctx->fcache + (int64_t)cs * blk)
+                         : (unsigned long long)(uintptr_t)(ctx->features_dev + b * blk);
+  }
+  CK(ctx, cudaMemcpyAsync(ctx->d_addr, ctx->h_addr, sizeof(unsigned long long) * (size_t)nfb,
+                          cudaMemcpyHostToDevice, st));
+  if (nj > 0) {
+    CK(ctx, cudaMemcpyAsync(ctx->d_job_blk, ctx->h_job_blk, sizeof(int32_t) * nj,
+                            cudaMemcpyHostToDevice, st));
+    CK(ctx, cudaMemcpyAsync(ctx->d_job_dst, ctx->h_job_dst, sizeof(unsigned long long) * nj,
+                            cudaMemcpyHostToDevice, st));
+    CK(ctx, launch_load_feat_blocks(ctx->features_dev, ctx->N * rb, ctx->d_job_blk, ctx->d_job_dst,
+                                    nj, blk, ctx->num_sms, st));
+  }
+  const int64_t cells = (int64_t)ctx->bt.T * w.H;
+  CK(ctx, launch_gather_table(ctx->d_addr, rb, rpb, w.fb_id[cur], w.fb_pos[cur],
+                              w.fcell_off[cur] + cells, w.feats_out, w.status, ctx->num_sms, st));
+  *bytes_out = bytes;
+  *hits_out = hits;
+  return AGNES_OK;
+}
+
+// After a hyperbatch: add its requests to the cumulative counts and re-pick
+// the cached blocks -- those whose count exceeds the threshold, hottest
+// first, up to the cache's capacity.  Blocks that stay keep their slot and
+// rows; newly admitted blocks get a free slot and are loaded the next time a
+// hyperbatch touches them.  Feature rows are read-only, so a block that
+// leaves the cache needs no write-back.
+static void update_feature_cache(agnes_ctx* ctx, int32_t n_touched) {
+  for (int32_t i = 0; i < n_touched; ++i) {
+    const int32_t b = ctx->h_touched[i];
+    ctx->acc[(size_t)b] += ctx->h_counts[b];
+  }
+  const int64_t C = ctx->fcache_slots;
+  if (C == 0) return;
+  const int64_t nfb = (int64_t)ctx->acc.size();
+  std::vector<int32_t> cand;
+  cand.reserve((size_t)nfb);
+  for (int64_t b = 0; b < nfb; ++b)
+    if (ctx->acc[(size_t)b] > 0 && ctx->acc[(size_t)b] > ctx->fcache_threshold)
+      cand.push_back((int32_t)b);
+  if ((int64_t)cand.size() > C) {
+    std::nth_element(cand.begin(), cand.begin() + C, cand.end(), [&](int32_t x, int32_t y) {
+      return ctx->acc[(size_t)x] != ctx->acc[(size_t)y] ? ctx->acc[(size_t)x] > ctx->acc[(size_t)y]
+                                                        : x < y;
+    });
+    cand.resize((size_t)C);
+  }
+  std::vector<uint8_t> keep((size_t)nfb, 0);
+  for (int32_t b : cand) keep[(size_t)b] = 1;
+  for (int64_t sl = 0; sl < C; ++sl) {  // release slots of blocks that leave
+    const int32_t b = ctx->cblock_of[(size_t)sl];
+    if (b >= 0 && !keep[(size_t)b]) {
+      ctx->cslot_of[(size_t)b] = -1;
+      ctx->cblock_of[(size_t)sl] = -1;
+      ctx->cresident[(size_t)sl] = 0;
+    }
+  }
+  int64_t free_sl = 0;
+  for (int32_t b : cand) {  // admit the new ones into free slots
+    if (ctx->cslot_of[(size_t)b] >= 0) continue;
+    while (free_sl < C && ctx->cblock_of[(size_t)free_sl] >= 0) ++free_sl;
+    if (free_sl >= C) break;
+    ctx->cslot_of[(size_t)b] = (int32_t)free_sl;
+    ctx->cblock_of[(size_t)free_sl] = b;
+    ctx->cresident[(size_t)free_sl] = 0;
+  }
+}
+
+// Gather with host-resident features.  The request count of every feature
+// block (rows gathered from it, over all minibatches) is read back once; the
+// touched blocks are those with a request.  Then block mode or row mode runs
+// the gather, and the feature cache (Sec. 3.4 (2)) is re-picked.
+static agnes_status gather_streamed(agnes_ctx* ctx, int cur, cudaStream_t st) {
+  Workspace& w = ctx->ws;
+  const int64_t nfb = ctx->bt.n_feat_blocks;
+  CK(ctx, launch_count_feat_requests(w.fcell_off[cur], (int32_t)ctx->bt.T, w.H,
+                                     ctx->bt.tile_feat_block, ctx->d_counts, nfb, w.status, st));
+  CK(ctx, cudaMemcpyAsync(ctx->h_counts, ctx->d_counts, sizeof(int32_t) * (size_t)nfb,
+                          cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
+  int32_t n = 0;
+  for (int64_t b = 0; b < nfb; ++b)
+    if (ctx->h_counts[b]) ctx->h_touched[n++] = (int32_t)b;
+  int64_t bytes = 0, hits = 0;
+  const agnes_status rc = ctx->feature_io == AGNES_FEATURE_IO_ROWS
+                              ? gather_rows_io(ctx, cur, n, &bytes, &hits, st)
+                              : gather_blocks_io(ctx, cur, n, &bytes, &hits, st);
+  if (rc != AGNES_OK) return rc;
   ctx->streamed_bytes = bytes;
-  ctx->streamed_blocks = n;
+  ctx->streamed_blocks = n - hits;
+  ctx->fcache_hits += hits;
+  update_feature_cache(ctx, n);
   return AGNES_OK;
 }
 
@@ -1162,6 +1415,8 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
   out->topo_loaded_bytes = ctx->topo.loaded_bytes;
   out->topo_hit_blocks = ctx->topo.hits;
   out->topo_waves = ctx->topo.waves;
+  out->fcache_hit_blocks = ctx->fcache_hits;
+  out->fcache_loaded_blocks = ctx->fcache_loads;
   return AGNES_OK;
 }
 

@@ -84,12 +84,14 @@ gather_bytes_kernel(const uint8_t* __restrict__ feats, int64_t row_bytes,
   }
 }
 
-// Streaming variant: rows come from an HBM staging slot holding the batch's
-// feature blocks (copied from pinned host memory on the side stream).  LPR
-// lanes per row, each lane moving the row's 16-byte vectors l, l+LPR, ...
+// Streaming variant: rows come from HBM copies of their feature blocks (a
+// staging slot of the ring or the feature cache).  The batch's blocks are
+// touched[0 .. nb) (ascending) and block touched[p] starts at device address
+// src[p].  LPR lanes per row, each lane moving the row's 16-byte vectors
+// l, l+LPR, ...
 template <int LPR>
 __global__ void __launch_bounds__(kThreads)
-gather_staged_kernel(const uint4* __restrict__ slot, int64_t vecs, int64_t rpb,
+gather_staged_kernel(const unsigned long long* __restrict__ src, int64_t vecs, int64_t rpb,
                      const int32_t* __restrict__ touched, int32_t nb,
                      const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
                      const int32_t* __restrict__ cell_off, int64_t cell_lo, int64_t cell_hi,
@@ -110,9 +112,71 @@ gather_staged_kernel(const uint4* __restrict__ slot, int64_t vecs, int64_t rpb,
       const int32_t mid = (lo + hi) >> 1;
       if (__ldg(touched + mid) <= b) lo = mid; else hi = mid;
     }
-    const int64_t row = (int64_t)lo * rpb + (v - (int64_t)b * rpb);
+    const uint4* blk = (const uint4*)__ldg(src + lo);
+    const int64_t row = v - (int64_t)b * rpb;
     for (int64_t c = l; c < vecs; c += LPR)
-      __stcs(out + g * vecs + c, __ldg(slot + row * vecs + c));
+      __stcs(out + g * vecs + c, __ldg(blk + row * vecs + c));
+  }
+}
+
+// Row mode of host-resident features: every row is read from its feature
+// block's current address, addr[v / rpb] -- an HBM feature-cache slot, or the
+// block's pinned host memory read in place over the host link.  Walks the
+// whole final bucket; LPR lanes per row, lane l moving vectors l, l+LPR, ...
+// The row data is read with plain loads (it may be host memory).
+template <int LPR>
+__global__ void __launch_bounds__(kThreads)
+gather_table_kernel(const unsigned long long* __restrict__ addr, int64_t vecs, int32_t rpb,
+                    const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
+                    const int32_t* total_ptr, uint4* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  constexpr int kRowsPerWarp = 32 / LPR;
+  const int64_t total = *total_ptr;
+  const int lane = lane_id();
+  const int sub = lane / LPR, l = lane % LPR;
+  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = warp0 * kRowsPerWarp + sub; i < total; i += nwarps * kRowsPerWarp) {
+    const int32_t v = __ldg(fb_id + i);
+    const int64_t g = __ldg(fb_pos + i);
+    const int32_t b = v / rpb;
+    const uint4* src = (const uint4*)__ldg(addr + b) + (int64_t)(v - b * rpb) * vecs;
+    for (int64_t c = l; c < vecs; c += LPR) __stcs(out + g * vecs + c, src[c]);
+  }
+}
+
+// Copies whole feature blocks from pinned host memory, read in place over the
+// host link: job j copies block blk[j] (vpb 16-byte vectors) to device address
+// dst[j].  Vectors at or past host_vecs (the end of the matrix, inside its
+// last block) are skipped.  The jobs form one flat range of vectors, four in
+// flight per thread.
+__global__ void __launch_bounds__(kThreads)
+load_feat_blocks_kernel(const uint4* __restrict__ host, int64_t host_vecs,
+                        const int32_t* __restrict__ blk, const unsigned long long* __restrict__ dst,
+                        int32_t njobs, int64_t vpb) {
+  const int64_t total = (int64_t)njobs * vpb;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q0 < total; q0 += 4 * stride) {
+    uint4 v[4];
+    int64_t j[4], r[4];
+    bool ok[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t q = q0 + u * stride;
+      ok[u] = false;
+      if (q < total) {
+        j[u] = q / vpb;
+        r[u] = q - j[u] * vpb;
+        const int64_t s = (int64_t)__ldg(blk + j[u]) * vpb + r[u];
+        if (s < host_vecs) {
+          v[u] = host[s];
+          ok[u] = true;
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (ok[u]) ((uint4*)__ldg(dst + j[u]))[r[u]] = v[u];
   }
 }
 
@@ -124,6 +188,18 @@ __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < ncells;
        c += (int64_t)gridDim.x * blockDim.x)
     if (cell_off[c + 1] > cell_off[c]) flags[map[c / H]] = 1;
+}
+
+// Requests per feature block: counts[tile_feat_block[t]] += entries of tile t.
+__global__ void count_feat_requests_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
+                                           const int32_t* __restrict__ tile_feat_block,
+                                           int32_t* __restrict__ counts, const int32_t* status) {
+  if (failed(status)) return;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t n = cell_off[(t + 1) * H] - cell_off[t * H];
+    if (n) atomicAdd(counts + tile_feat_block[t], n);
+  }
 }
 
 // Copies the edge lists of physical blocks from pinned host memory (read in
@@ -238,19 +314,18 @@ cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* f
   return cudaGetLastError();
 }
 
-cudaError_t launch_gather_staged(const void* slot, int64_t row_bytes, int64_t rpb,
+cudaError_t launch_gather_staged(const unsigned long long* src, int64_t row_bytes, int64_t rpb,
                                  const int32_t* touched, int32_t nb, const int32_t* fb_id,
                                  const int32_t* fb_pos, const int32_t* cell_off, int64_t cell_lo,
                                  int64_t cell_hi, void* out, const int32_t* status, int num_sms,
                                  cudaStream_t st) {
   const int64_t vecs = row_bytes / 16;
-  const uint4* sl = (const uint4*)slot;
   uint4* o = (uint4*)out;
-#define AGNES_STAGED(LPR)                                                                    \
-  gather_staged_kernel<LPR><<<resident_grid((const void*)gather_staged_kernel<LPR>, kThreads, \
-                                            num_sms),                                        \
-                              kThreads, 0, st>>>(sl, vecs, rpb, touched, nb, fb_id, fb_pos,   \
-                                                 cell_off, cell_lo, cell_hi, o, status)
+  // four CTAs per SM, so the block loader on the copy stream can run beside it
+#define AGNES_STAGED(LPR)                                                                   \
+  gather_staged_kernel<LPR><<<num_sms * 4, kThreads, 0, st>>>(src, vecs, rpb, touched, nb,   \
+                                                               fb_id, fb_pos, cell_off, cell_lo, \
+                                                               cell_hi, o, status)
   if (vecs <= 8)
     AGNES_STAGED(8);
   else if (vecs <= 16)
@@ -261,12 +336,50 @@ cudaError_t launch_gather_staged(const void* slot, int64_t row_bytes, int64_t rp
   return cudaGetLastError();
 }
 
+cudaError_t launch_gather_table(const unsigned long long* addr, int64_t row_bytes, int64_t rpb,
+                                const int32_t* fb_id, const int32_t* fb_pos, const int32_t* total,
+                                void* out, const int32_t* status, int num_sms, cudaStream_t st) {
+  const int64_t vecs = row_bytes / 16;
+  uint4* o = (uint4*)out;
+#define AGNES_TABLE(LPR)                                                                    \
+  gather_table_kernel<LPR><<<resident_grid((const void*)gather_table_kernel<LPR>, kThreads,  \
+                                           num_sms),                                        \
+                             kThreads, 0, st>>>(addr, vecs, (int32_t)rpb, fb_id, fb_pos, total, \
+                                                o, status)
+  if (vecs <= 8)
+    AGNES_TABLE(8);
+  else if (vecs <= 16)
+    AGNES_TABLE(16);
+  else
+    AGNES_TABLE(32);
+#undef AGNES_TABLE
+  return cudaGetLastError();
+}
+
+cudaError_t launch_load_feat_blocks(const void* host_dev, int64_t host_bytes, const int32_t* blk,
+                                    const unsigned long long* dst, int32_t njobs,
+                                    int64_t block_bytes, int num_sms, cudaStream_t st) {
+  if (njobs <= 0) return cudaSuccess;
+  load_feat_blocks_kernel<<<num_sms, kThreads, 0, st>>>((const uint4*)host_dev, host_bytes / 16,
+                                                        blk, dst, njobs, block_bytes / 16);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, const int32_t* map,
                               uint8_t* flags, int64_t n_flags, int64_t* count,
                               const int32_t* status, cudaStream_t st) {
   if (cell_off && map)
     mark_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, map, flags, status);
   count_flags_kernel<<<256, 256, 0, st>>>(flags, n_flags, count);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_count_feat_requests(const int32_t* cell_off, int32_t T, int32_t H,
+                                       const int32_t* tile_feat_block, int32_t* counts,
+                                       int64_t nfb, const int32_t* status, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int32_t) * (size_t)nfb, st);
+  if (e != cudaSuccess) return e;
+  count_feat_requests_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, tile_feat_block, counts, status);
   return cudaGetLastError();
 }
 

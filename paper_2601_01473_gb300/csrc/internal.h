@@ -157,21 +157,42 @@ cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* f
                           const int32_t* fb_pos, const int32_t* total, void* out,
                           const int32_t* status, int num_sms, cudaStream_t st);
 
-// Gathers the rows of a batch of feature blocks staged in an HBM slot: the
-// batch's blocks are touched[0 .. nb) (ascending), packed in the slot one
-// block (rpb rows) after another; its bucket entries are those of cells
+// Gathers the rows of a batch of feature blocks held in HBM copies: the
+// batch's blocks are touched[0 .. nb) (ascending), block touched[p] starts at
+// device address src[p]; its bucket entries are those of cells
 // [cell_lo, cell_hi) of cell_off.  Rows must be a multiple of 16 bytes.
-cudaError_t launch_gather_staged(const void* slot, int64_t row_bytes, int64_t rpb,
+cudaError_t launch_gather_staged(const unsigned long long* src, int64_t row_bytes, int64_t rpb,
                                  const int32_t* touched, int32_t nb, const int32_t* fb_id,
                                  const int32_t* fb_pos, const int32_t* cell_off, int64_t cell_lo,
                                  int64_t cell_hi, void* out, const int32_t* status, int num_sms,
                                  cudaStream_t st);
+
+// Gathers every row of the final bucket from its feature block's address:
+// row v at (const uint4*)addr[v / rpb] + (v % rpb) * row_bytes / 16 (an HBM
+// cache slot or mapped pinned host memory).  Rows must be a multiple of 16
+// bytes.
+cudaError_t launch_gather_table(const unsigned long long* addr, int64_t row_bytes, int64_t rpb,
+                                const int32_t* fb_id, const int32_t* fb_pos, const int32_t* total,
+                                void* out, const int32_t* status, int num_sms, cudaStream_t st);
+
+// Copies feature blocks blk[0 .. njobs) (block_bytes each, the last block of
+// the matrix possibly shorter) from host_dev, the device view of pinned host
+// memory holding host_bytes bytes, to device addresses dst[0 .. njobs).
+// block_bytes, host_bytes and every address must be multiples of 16.
+cudaError_t launch_load_feat_blocks(const void* host_dev, int64_t host_bytes, const int32_t* blk,
+                                    const unsigned long long* dst, int32_t njobs,
+                                    int64_t block_bytes, int num_sms, cudaStream_t st);
 
 // Marks flags[map[t]] for every tile t whose cells (t, 0..H-1) in cell_off
 // hold an entry, then counts set flags into *count (int64).
 cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, const int32_t* map,
                               uint8_t* flags, int64_t n_flags, int64_t* count,
                               const int32_t* status, cudaStream_t st);
+
+// counts[b] = requests (bucket entries) for feature block b (cleared first).
+cudaError_t launch_count_feat_requests(const int32_t* cell_off, int32_t T, int32_t H,
+                                       const int32_t* tile_feat_block, int32_t* counts,
+                                       int64_t nfb, const int32_t* status, cudaStream_t st);
 
 // Copies physical blocks jobs[i].x (edges e0..e1 of host_indices, a device
 // view of pinned host memory) into graph-buffer slots jobs[i].y.

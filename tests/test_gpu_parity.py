@@ -223,28 +223,81 @@ def test_workload_parity_all_minibatches(cuda_device, name):
     g.close()
 
 
+@pytest.mark.parametrize("io", ["blocks", "rows"])
 @pytest.mark.parametrize("dtype,dim,fbb,H", [
     (torch.float32, 16, 1024, 6),     # ~1900 feature blocks: many batches, the slot ring wraps
     (torch.float16, 128, 4096, 3),
     (torch.float16, 128, 1 << 20, 1),  # one block per batch
+    (torch.float32, 12, 1008, 2),     # 48-byte rows, 21 rows per block: odd vector counts
 ])
-def test_streamed_features_match_oracle(cuda_device, dtype, dim, fbb, H):
-    """Features in pinned host memory, streamed block by block through the HBM
-    slot ring: same bytes as the oracle, over two hyperbatches in a row."""
+def test_streamed_features_match_oracle(cuda_device, dtype, dim, fbb, H, io):
+    """Features in pinned host memory, read over the host link block by block
+    through the HBM slot ring, or row by row: same bytes as the oracle, over
+    two hyperbatches in a row."""
     off, ind, feats = make(30000, 10, seed=dim + H, dtype=dtype, dim=dim)
     og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
     host_feats = feats.pin_memory()
     g = Graph(off.to(cuda_device), ind.to(cuda_device), host_feats, adj_block_bytes=8192,
-              feat_block_bytes=fbb, features_on_host=True)
+              feat_block_bytes=fbb, features_on_host=True, feature_io=io)
+    rb = dim * feats.element_size()
     for step in range(2):
         targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), H, 200, 7, step)
         g.prepare(targets.to(cuda_device), [8, 4], 21, 100 * step)
         compare(g, og, targets.numpy(), [8, 4], 21, 100 * step, 8192, fbb)
         c = g.counters()
         assert c["streamed_blocks"] == g.stats()[-1]
-        assert 0 < c["streamed_bytes"] <= c["streamed_blocks"] * (fbb // (dim * feats.element_size())) \
-            * dim * feats.element_size()
+        if io == "blocks":
+            assert 0 < c["streamed_bytes"] <= c["streamed_blocks"] * (fbb // rb) * rb
+        else:
+            assert c["streamed_bytes"] == c["rows"] * rb
     g.close()
+
+
+@pytest.mark.parametrize("io", ["blocks", "rows"])
+@pytest.mark.parametrize("cache_blocks,threshold", [
+    (200, 0),          # cache holds ~1/5 of the blocks: the hottest ones
+    (100000, 0),       # cache holds every block: from the third hyperbatch on, all hits
+    (300, 10**9),      # no block's count exceeds the threshold: nothing cached
+])
+def test_feature_cache_matches_oracle(cuda_device, cache_blocks, threshold, io):
+    """Streamed features with the access-count feature cache: same bytes as
+    the oracle over several hyperbatches, while cached blocks are read in
+    place instead of being copied again."""
+    n, dim, fbb = 30000, 64, 4096
+    off, ind, feats = make(n, 10, seed=5, dtype=torch.float16, dim=dim)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    g = Graph(off.to(cuda_device), ind.to(cuda_device), feats.pin_memory(), adj_block_bytes=8192,
+              feat_block_bytes=fbb, features_on_host=True, feature_cache_bytes=cache_blocks * fbb,
+              feature_cache_threshold=threshold, feature_io=io)
+    nfb = -(-n // (fbb // (dim * 2)))
+    prev_hits = prev_loads = 0
+    for step in range(4):
+        targets = synth.hyperbatch_targets(torch.arange(n, dtype=torch.int32), 3, 100, 11, step)
+        g.prepare(targets.to(cuda_device), [6, 3], 4, 50 * step)
+        compare(g, og, targets.numpy(), [6, 3], 4, 50 * step, 8192, fbb)
+        c = g.counters()
+        hits, loads = c["fcache_hit_blocks"] - prev_hits, c["fcache_loaded_blocks"] - prev_loads
+        prev_hits, prev_loads = c["fcache_hit_blocks"], c["fcache_loaded_blocks"]
+        assert c["streamed_blocks"] + hits == g.stats()[-1]
+        assert loads <= c["streamed_blocks"]
+        if step == 0 or threshold >= 10**9:
+            assert hits == 0 and loads == 0
+        if cache_blocks >= nfb and step >= 2:
+            assert hits > 0
+    if cache_blocks >= nfb:
+        assert prev_loads <= nfb  # nothing is evicted, so no block is loaded twice
+    if threshold < 10**9:
+        assert prev_loads > 0 and prev_hits > 0
+        assert prev_loads <= min(cache_blocks, nfb) * 3
+    g.close()
+
+
+def test_feature_cache_needs_host_features(cuda_device):
+    off, ind, feats = make(2000, 6, seed=4, dim=16)
+    with pytest.raises(AgnesError) as e:
+        Graph(off.to(cuda_device), ind.to(cuda_device), feats.to(cuda_device),
+              adj_block_bytes=4096, feat_block_bytes=4096, feature_cache_bytes=1 << 20)
+    assert e.value.status == 1
 
 
 def test_fetch_all_equals_per_minibatch_fetch(cuda_device):
