@@ -250,6 +250,9 @@ def main():
                     help="with --stream: HBM feature cache of the most requested blocks")
     ap.add_argument("--feature-cache-threshold", type=int, default=0,
                     help="with --stream: requests a block must exceed to be cached")
+    ap.add_argument("--ablation", action="store_true",
+                    help="AGNES-No (one minibatch per hyperbatch) vs AGNES-HB, three settings")
+    ap.add_argument("--ablation-hyperbatches", type=int, default=3)
     ap.add_argument("--feature-io", default="blocks", choices=["blocks", "rows"],
                     help="with --stream: load whole feature blocks, or read requested rows in place")
     args = ap.parse_args()
@@ -267,6 +270,8 @@ def main():
         return run_reference(args, w, world, rank)
     if args.sweep:
         return run_sweep(args, w)
+    if args.ablation:
+        return run_ablation(args, w)
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
@@ -509,6 +514,78 @@ def run_sweep(args, w):
                               "feat_blocks_touched": stats[-1],
                               "adj_blocks": info["adj_blocks"], "feat_blocks": info["feat_blocks"],
                               "block_io_bytes": (sum(stats[:-1]) + stats[-1]) * bb}), flush=True)
+        g.close()
+
+
+def run_ablation(args, w):
+    """AGNES-No against AGNES-HB (the paper's EQ2): the same minibatches
+    prepared one per hyperbatch (No) and H per hyperbatch (HB), with the graph
+    resident in HBM, with features in pinned host memory (block I/O) and with
+    topology in pinned host memory (4 GB graph buffer).  Both arms draw
+    identical samples (same seed and minibatch ids); one JSON line per setting."""
+    from paper_2601_01473_gb300 import Graph
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    offsets, indices, features = build_graph(w, dev)
+    pool = target_pool(w, dev)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream(dev)
+    fan = list(w.fanouts)
+    H = w.H
+    n_hb = max(1, args.ablation_hyperbatches)
+    steps = [targets_for_step(w, pool, s) for s in range(1 + n_hb)]
+    settings = [("resident", {}, 64), ("features_on_host", {"features_on_host": True}, 4),
+                ("topology_on_host", {"topology_on_host": True,
+                                      "graph_buffer_bytes": int(args.graph_buffer_gb * 2**30)}, 4)]
+    host_feats = host_ind = None
+    for name, kw, n_no in settings:
+        if kw.get("features_on_host") and host_feats is None:
+            host_feats = features.cpu().pin_memory()
+        if kw.get("topology_on_host") and host_ind is None:
+            host_ind = indices.cpu().pin_memory()
+        f = host_feats if kw.get("features_on_host") else features
+        ind = host_ind if kw.get("topology_on_host") else indices
+        torch.cuda.empty_cache()
+        g = Graph(offsets, ind, f, w.adj_block_bytes, w.feat_block_bytes, device=0, stream=stream,
+                  **kw)
+
+        def link_bytes():
+            c = g.counters()
+            return c["streamed_bytes"], c["topo_loaded_bytes"], c
+
+        def timed(calls):
+            torch.cuda.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            moved = 0
+            for t, gid0 in calls:
+                g.prepare(t, fan, w.seed, gid0, stream)
+                sb, _, _ = link_bytes() if kw.get("features_on_host") else (0, 0, None)
+                moved += sb
+            e1.record(stream)
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1), moved
+
+        # warm-up: one hyperbatch and one single-minibatch hyperbatch
+        g.prepare(steps[0], fan, w.seed, 0, stream)
+        g.prepare(steps[0][:1], fan, w.seed, 0, stream)
+        t0 = g.counters()["topo_loaded_bytes"]
+        hb_ms, hb_feat = timed([(steps[1 + s], (1 + s) * H) for s in range(n_hb)])
+        t1 = g.counters()["topo_loaded_bytes"]
+        no_calls = [(steps[1][j:j + 1], H + j) for j in range(min(n_no, H))]
+        no_ms, no_feat = timed(no_calls)
+        t2 = g.counters()["topo_loaded_bytes"]
+        hb_mbs = n_hb * H / (hb_ms / 1e3)
+        no_mbs = len(no_calls) / (no_ms / 1e3)
+        print(json.dumps({
+            "ablation": "AGNES-No vs AGNES-HB", "workload": w.name, "setting": name,
+            "H": H, "B": w.B, "fanouts": fan,
+            "hb": {"minibatches_per_s": hb_mbs, "minibatches": n_hb * H,
+                   "host_link_bytes_per_minibatch": (hb_feat + t1 - t0) / (n_hb * H)},
+            "no": {"minibatches_per_s": no_mbs, "minibatches": len(no_calls),
+                   "host_link_bytes_per_minibatch": (no_feat + t2 - t1) / len(no_calls)},
+            "hb_over_no": hb_mbs / no_mbs}), flush=True)
         g.close()
 
 
