@@ -22,6 +22,7 @@ import sys
 import tempfile
 import time
 
+import numpy as np
 import torch
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -126,11 +127,14 @@ class ClockSampler:
 
 
 def kernel_launches_per_step(K: int) -> int:
-    """Kernels libagnes launches per hyperbatch: target bucketing 6 (count,
-    3-kernel scan, scatter, sort) + 1 size fill; per hop 19 (count, 3 scan,
-    fill, hist, 3 scan, scatter, dedup count, 3 scan, size add, 3 scan,
-    emit); 1 gather; K+2 for the blocks-touched counts."""
-    return 7 + 19 * K + 1 + K + 2
+    """Kernels libagnes launches per hyperbatch with the graph in HBM (the
+    ncu launch list of profiles/step_rmat100m_traffic.md has 59 at K = 3):
+    target bucketing 5 (count, 2-kernel scan, scatter, sort); per hop 16
+    (count, 2-kernel scan, fill, 2-kernel scan, scatter, cells, big cells,
+    3-kernel column scan, 2-kernel scan, col fix-up, compaction); after the
+    last hop 3 (feature-block marks, their count, gather) and K counts of
+    touched topology blocks."""
+    return 5 + 16 * K + 3 + K
 
 
 def algorithmic_bytes(c: dict, off_bytes: int) -> dict:
@@ -253,6 +257,10 @@ def main():
     ap.add_argument("--ablation", action="store_true",
                     help="AGNES-No (one minibatch per hyperbatch) vs AGNES-HB, three settings")
     ap.add_argument("--ablation-hyperbatches", type=int, default=3)
+    ap.add_argument("--sage", action="store_true",
+                    help="time the GraphSAGE-mean consumer layer on a prepared hyperbatch")
+    ap.add_argument("--sage-d-out", type=int, default=128)
+    ap.add_argument("--sage-out", default="f32", choices=["f32", "f16"])
     ap.add_argument("--feature-io", default="blocks", choices=["blocks", "rows"],
                     help="with --stream: load whole feature blocks, or read requested rows in place")
     args = ap.parse_args()
@@ -272,6 +280,8 @@ def main():
         return run_sweep(args, w)
     if args.ablation:
         return run_ablation(args, w)
+    if args.sage:
+        return run_sage(args, w)
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
@@ -567,11 +577,12 @@ def run_ablation(args, w):
             torch.cuda.synchronize()
             return e0.elapsed_time(e1), moved
 
-        # warm-up: one hyperbatch and one single-minibatch hyperbatch
+        # each arm is warmed up right before it is timed (a change of H
+        # re-sizes the workspace, which must stay outside the timed region)
         g.prepare(steps[0], fan, w.seed, 0, stream)
-        g.prepare(steps[0][:1], fan, w.seed, 0, stream)
         t0 = g.counters()["topo_loaded_bytes"]
         hb_ms, hb_feat = timed([(steps[1 + s], (1 + s) * H) for s in range(n_hb)])
+        g.prepare(steps[0][:1], fan, w.seed, 0, stream)
         t1 = g.counters()["topo_loaded_bytes"]
         no_calls = [(steps[1][j:j + 1], H + j) for j in range(min(n_no, H))]
         no_ms, no_feat = timed(no_calls)
@@ -587,6 +598,75 @@ def run_ablation(args, w):
                    "host_link_bytes_per_minibatch": (no_feat + t2 - t1) / len(no_calls)},
             "hb_over_no": hb_mbs / no_mbs}), flush=True)
         g.close()
+
+
+def run_sage(args, w):
+    """The consumer: one GraphSAGE-mean layer (agnes_sage_mean_layer) over the
+    outermost hop of a prepared hyperbatch, fed by the gathered features.
+    Reports its time per launch against the HBM roofline (each src row read
+    once, the output written once) and its tensor-core rate."""
+    from paper_2601_01473_gb300 import Graph
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    offsets, indices, features = build_graph(w, dev)
+    pool = target_pool(w, dev)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream(dev)
+    fan = list(w.fanouts)
+    K = len(fan)
+    g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes, device=0,
+              stream=stream)
+    g.prepare(targets_for_step(w, pool, 0), fan, w.seed, 0, stream)
+    allv = g.fetch_all()
+    d_in, d_out = w.feat_dim, args.sage_d_out
+    out_dtype = torch.float16 if args.sage_out == "f16" else torch.float32
+    gen = torch.Generator().manual_seed(7)
+    wt = (torch.randn(d_out, 2 * d_in, generator=gen) / (2 * d_in) ** 0.5).to(torch.float16).to(dev)
+    bias = (torch.randn(d_out, generator=gen) * 0.1).to(dev)
+    x = allv.feats
+    for _ in range(args.warmup):
+        g.sage_mean_layer(K - 1, x, wt, bias, out_dtype=out_dtype, stream=stream)
+    times = []
+    with ClockSampler(0) as clk:
+        for _ in range(args.steps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g.sage_mean_layer(K - 1, x, wt, bias, out_dtype=out_dtype, stream=stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    nd = allv.node_size[K - 1].astype(np.int64)
+    ns = allv.node_size[K].astype(np.int64)
+    ne = allv.edges[K - 1].astype(np.int64)
+    rb = d_in * features.element_size()
+    ob = 2 if out_dtype == torch.float16 else 4
+    algo = int((ns * rb).sum() + (ne * 4).sum() + ((nd + 1) * 8).sum() + (nd * d_out * ob).sum()
+               + wt.numel() * 2)
+    flops = int((nd * 2 * 2 * d_in * d_out).sum())
+    hbm, peak_kind = measured_peak()
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            bf16 = float(json.load(f)["bf16_tflops"])
+    except Exception:
+        bf16 = None
+    gbs = algo / (ms / 1e3) / 1e9
+    print(json.dumps({
+        "sage": "GraphSAGE-mean layer over the outermost hop (agnes_sage_mean_layer)",
+        "workload": f"{w.name}: {w.describe()}", "d_in": d_in, "d_out": d_out,
+        "x_dtype": str(features.dtype).replace("torch.", ""), "out_dtype": args.sage_out,
+        "dst_rows": int(nd.sum()), "edges": int(ne.sum()), "src_rows": int(ns.sum()),
+        "ms_per_launch": ms, "dst_rows_per_s": float(nd.sum()) / (ms / 1e3),
+        "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
+                     "frac": gbs / hbm if hbm else None, "algorithmic_bytes_per_launch": algo,
+                     "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"},
+        "tensor": {"tflops": flops / (ms / 1e3) / 1e12, "flops_per_launch": flops,
+                   "fp16_dense_peak_tflops": bf16,
+                   "peak_source": "measured bf16 burst (MEASURED_PEAKS.json bf16_tflops); "
+                                  "fp16 has the same nominal rate"},
+        "clocks": clk.summary()}), flush=True)
+    g.close()
 
 
 def run_reference(args, w, world, rank):

@@ -274,6 +274,39 @@ agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable);
 agnes_status agnes_phase_times(agnes_ctx* ctx, int32_t ago, float* ms, int32_t n,
                                int32_t* n_out);
 
+/* A GraphSAGE-mean layer over hop `hop` of every minibatch of the last
+ * hyperbatch: the consumer of the prepared blocks.  It is an instance of
+ * eq. (1) (Sec. 3.1), with the mean of the in-neighbours' rows as the
+ * aggregation and a fully connected layer with ReLU as the update:
+ *   out_i = ReLU(W_self x_i + W_neigh mean_{e in row i} x_{col[e]} + b)
+ * for every dst row i of the hop (dst_h is a prefix of src_h, so x_i is row
+ * i of x).  Layers stack from the outermost hop in: hop K-1 takes the
+ * gathered features (x = feats of agnes_fetch_hyperbatch, x_stride_rows =
+ * feats_stride_rows) and its output rows are src_{K-2}, the input of hop K-2.
+ *  x      device, minibatch j's src_h rows at x + (j*x_stride_rows + r)*d_in
+ *         elements of x_dtype (AGNES_F32 or AGNES_F16); x_stride_rows >= the
+ *         largest |src_h|.
+ *  w      device, d_out x 2*d_in IEEE fp16, row-major: columns [0, d_in)
+ *         multiply x_i (W_self), [d_in, 2*d_in) the mean (W_neigh).
+ *  bias   device, d_out floats, or NULL for none.
+ *  out    device, minibatch j's dst_h rows at out + (j*out_stride_rows + i)*
+ *         d_out elements of out_dtype; out_stride_rows >= the largest |dst_h|.
+ * Arithmetic: the mean is summed and divided in fp32, the update's inputs
+ * are rounded to fp16, and the products are accumulated in fp32 on the
+ * tensor cores (tcgen05).  d_in is a multiple of 8, d_out a multiple of 32
+ * in [32, 256], and the two operands must fit shared memory:
+ * 512*d_in + 4*d_in*d_out + 17440 <= AGNES_SAGE_MAX_SMEM bytes (ERANGE
+ * otherwise).  x, w and out are 16-byte aligned.  Waits for the hyperbatch
+ * like agnes_fetch_hyperbatch, runs on cuda_stream and waits for it.
+ * Errors: EINVAL, ERANGE, ESTATE, ECUDA, ETIMEOUT (a tensor-core completion
+ * wait ran out; the layer's output is then undefined). */
+#define AGNES_SAGE_MAX_SMEM 232448
+agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const void* x, int32_t x_dtype,
+                                   int64_t x_stride_rows, int64_t d_in, const void* w,
+                                   const float* bias, int32_t d_out, void* out,
+                                   int32_t out_dtype, int64_t out_stride_rows,
+                                   void* cuda_stream);
+
 /* Allocation-free variant of one step of the path: for a node list (for
  * example one minibatch's frontier), the per-node edge counts of one hop's
  * sampling, min(deg(v), fanout), and their prefix sum -- the indptr that

@@ -128,6 +128,9 @@ SIGNATURES = {
     "agnes_phase_times": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)],
                           ctypes.c_int),
     "agnes_hop_indptr_noalloc": ([_P, _P, ctypes.c_int64, ctypes.c_int32, _P, _P], ctypes.c_int),
+    "agnes_sage_mean_layer": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int64,
+                               ctypes.c_int64, _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
+                               ctypes.c_int64, _P], ctypes.c_int),
     "agnes_free": ([_P], ctypes.c_int),
     "agnes_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "agnes_last_error": ([_P], ctypes.c_char_p),
@@ -332,6 +335,31 @@ class Graph:
         v = _HyperbatchView()
         _check(lib().agnes_fetch_hyperbatch(self._ctx, ctypes.byref(v)), self._ctx)
         return HyperbatchView(v, self.device)
+
+    def sage_mean_layer(self, hop: int, x: torch.Tensor, w: torch.Tensor, bias=None,
+                        out_dtype: torch.dtype = torch.float32, stream=None) -> torch.Tensor:
+        """One GraphSAGE-mean layer (agnes_sage_mean_layer) over hop ``hop`` of
+        every minibatch of the last hyperbatch.  ``x`` is [H, rows, d_in]
+        (minibatch j's src_hop rows first), ``w`` is [d_out, 2 d_in] fp16
+        ([W_self | W_neigh]), ``bias`` [d_out] fp32 or None.  Returns
+        [H, max |dst_hop|, d_out]; rows past a minibatch's |dst_hop| are
+        unspecified."""
+        if x.dim() != 3 or x.dtype not in _DTYPES or not x.is_contiguous():
+            raise TypeError("x must be a contiguous [H, rows, d_in] float32/float16 tensor")
+        if w.dtype != torch.float16 or w.dim() != 2 or not w.is_contiguous():
+            raise TypeError("w must be a contiguous [d_out, 2*d_in] float16 tensor")
+        if bias is not None and (bias.dtype != torch.float32 or not bias.is_contiguous()):
+            raise TypeError("bias must be a contiguous float32 tensor")
+        H, rows, d_in = x.shape
+        d_out = w.shape[0]
+        sizes = self.fetch_all().node_size
+        max_dst = int(sizes[hop].max()) if 0 <= hop < sizes.shape[0] - 1 else 0
+        out = torch.empty((H, max(max_dst, 1), d_out), dtype=out_dtype, device=x.device)
+        _check(lib().agnes_sage_mean_layer(
+            self._ctx, hop, x.data_ptr(), _DTYPES[x.dtype], rows, d_in, w.data_ptr(),
+            bias.data_ptr() if bias is not None else None, d_out, out.data_ptr(),
+            _DTYPES[out_dtype], out.shape[1], _stream_handle(stream)), self._ctx)
+        return out
 
     def sizes(self, j: int) -> dict:
         """Host-side sizes of minibatch j (no device data touched)."""

@@ -94,6 +94,10 @@ struct agnes_ctx {
   int32_t feat_dtype = 0;
   int64_t feat_dim = 0, row_bytes = 0;
   int32_t features_on_host = 0;
+  void* scratch = nullptr;  // ctx_scratch
+  size_t scratch_bytes = 0;
+  void* pinned = nullptr;   // ctx_pinned
+  size_t pinned_bytes = 0;
   int32_t feature_io = AGNES_FEATURE_IO_BLOCKS;
   const char* features_dev = nullptr;  // device view of host-resident features
   int64_t adj_block_bytes = 0, feat_block_bytes = 0;
@@ -188,9 +192,36 @@ static void set_err(agnes_ctx* ctx, const char* fmt, ...) {
 
 void ctx_graph_view(const agnes_ctx* ctx, agnes::GraphView* out) {
   out->device = ctx->device;
+  out->num_sms = ctx->num_sms;
   out->offsets = ctx->offsets;
   out->offsets_bits = ctx->offsets_bits;
   out->N = ctx->N;
+}
+
+cudaError_t ctx_scratch(agnes_ctx* ctx, size_t bytes, void** out) {
+  if (ctx->scratch_bytes < bytes) {
+    cudaFree(ctx->scratch);
+    ctx->scratch = nullptr;
+    ctx->scratch_bytes = 0;
+    const cudaError_t e = cudaMalloc(&ctx->scratch, bytes);
+    if (e != cudaSuccess) return e;
+    ctx->scratch_bytes = bytes;
+  }
+  *out = ctx->scratch;
+  return cudaSuccess;
+}
+
+cudaError_t ctx_pinned(agnes_ctx* ctx, size_t bytes, void** out) {
+  if (ctx->pinned_bytes < bytes) {
+    if (ctx->pinned) cudaFreeHost(ctx->pinned);
+    ctx->pinned = nullptr;
+    ctx->pinned_bytes = 0;
+    const cudaError_t e = cudaMallocHost(&ctx->pinned, bytes);
+    if (e != cudaSuccess) return e;
+    ctx->pinned_bytes = bytes;
+  }
+  *out = ctx->pinned;
+  return cudaSuccess;
 }
 
 void ctx_set_error(agnes_ctx* ctx, const char* fmt, ...) {
@@ -477,6 +508,8 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   cudaFree(ctx->d_touched);
   cudaFree(ctx->d_counts);
   cudaFree(ctx->d_src);
+  cudaFree(ctx->scratch);
+  if (ctx->pinned) cudaFreeHost(ctx->pinned);
   cudaFree(ctx->d_job_blk);
   cudaFree(ctx->d_job_dst);
   cudaFree(ctx->d_addr);

@@ -213,6 +213,7 @@ cudaError_t launch_distinct_rows(const int32_t* fb_id, const int32_t* cell_off,
 // ---- api.cu: read-only view of a loaded graph for other translation units --
 struct GraphView {
   int device;
+  int num_sms;
   const void* offsets;
   int offsets_bits;
   int64_t N;
@@ -223,3 +224,8 @@ struct GraphView {
 struct agnes_ctx;
 void ctx_graph_view(const agnes_ctx* ctx, agnes::GraphView* out);
 void ctx_set_error(agnes_ctx* ctx, const char* fmt, ...);
+// A device buffer owned by ctx of at least `bytes` (grown on demand, freed by
+// agnes_free); its contents do not outlive the call that asked for it.
+cudaError_t ctx_scratch(agnes_ctx* ctx, size_t bytes, void** out);
+// The same for pinned host memory (staging for small host <-> device copies).
+cudaError_t ctx_pinned(agnes_ctx* ctx, size_t bytes, void** out);
