@@ -52,7 +52,11 @@ class _OrcMinibatch(ctypes.Structure):
         ("nodes", ctypes.c_void_p),
         ("num_nodes", ctypes.c_int64),
         ("feats", ctypes.c_void_p),
+        ("dst", ctypes.c_void_p * MAX_HOPS),
     ]
+
+
+FRONTIER = {"src": 0, "sampled": 1}  # ORC_FRONTIER_SRC / ORC_FRONTIER_SAMPLED
 
 
 def lib() -> ctypes.CDLL:
@@ -78,6 +82,11 @@ def lib() -> ctypes.CDLL:
             ctypes.c_int32, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int,
             ctypes.POINTER(_OrcMinibatch)]
         L.orc_sample_minibatch.restype = ctypes.c_int
+        L.orc_sample_minibatch_mode.argtypes = [
+            ctypes.POINTER(_OrcGraph), ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p,
+            ctypes.c_int32, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int, ctypes.c_int32,
+            ctypes.POINTER(_OrcMinibatch)]
+        L.orc_sample_minibatch_mode.restype = ctypes.c_int
         L.orc_free_minibatch.argtypes = [ctypes.POINTER(_OrcMinibatch)]
         L.orc_free_minibatch.restype = None
         L.orc_hyperbatch_stats.argtypes = [
@@ -195,6 +204,7 @@ def _to_dict(mb: _OrcMinibatch, row_bytes: int, feat_dtype, feat_shape_tail):
             "indptr": _copy(mb.indptr[h], nd + 1, np.int64),
             "nbr": _copy(mb.nbr[h], ne, np.int32),
             "col": _copy(mb.col[h], ne, np.int32),
+            "dst": _copy(mb.dst[h], nd, np.int32),
         })
     n = int(mb.num_nodes)
     out = {"hops": hops, "nodes": _copy(mb.nodes, n, np.int32), "num_nodes": n}
@@ -210,13 +220,17 @@ def _feat_meta(graph: Graph):
     return graph.features.dtype, tuple(graph.features.shape[1:])
 
 
-def sample_minibatch(graph: Graph, targets, fanouts, seed: int, gid: int, gather: bool = True):
-    """Samples + gathers one minibatch with global id ``gid`` (see module doc)."""
+def sample_minibatch(graph: Graph, targets, fanouts, seed: int, gid: int, gather: bool = True,
+                     frontier: str = "src"):
+    """Samples + gathers one minibatch with global id ``gid`` (see module doc).
+    ``frontier`` = "src" (dst_{h+1} = src_h) or "sampled" (dst_{h+1} = the
+    distinct ids sampled at hop h: Algorithm 1's N_in <- N_out)."""
     t = np.ascontiguousarray(targets, dtype=np.int32)
     f = np.ascontiguousarray(fanouts, dtype=np.int32)
     mb = _OrcMinibatch()
-    rc = lib().orc_sample_minibatch(ctypes.byref(graph._struct), _ptr(t), t.shape[0], _ptr(f),
-                                    f.shape[0], seed, gid, int(gather), ctypes.byref(mb))
+    rc = lib().orc_sample_minibatch_mode(ctypes.byref(graph._struct), _ptr(t), t.shape[0],
+                                         _ptr(f), f.shape[0], seed, gid, int(gather),
+                                         FRONTIER[frontier], ctypes.byref(mb))
     if rc != 0:
         raise OracleError(f"orc_sample_minibatch failed ({rc})")
     try:
@@ -227,7 +241,8 @@ def sample_minibatch(graph: Graph, targets, fanouts, seed: int, gid: int, gather
 
 
 def hyperbatch(graph: Graph, targets, fanouts, seed: int, first_gid: int, gather: bool,
-               adj_block_bytes: int, feat_block_bytes: int, threads: int = 1):
+               adj_block_bytes: int, feat_block_bytes: int, threads: int = 1,
+               frontier: str = "src"):
     """Runs every minibatch of a hyperbatch (targets: [H, B]) and the
     blocks-touched statistics.  Returns (list of per-minibatch dicts, stats
     list of K+1 ints).  threads > 1 runs independent minibatches on host
@@ -239,9 +254,9 @@ def hyperbatch(graph: Graph, targets, fanouts, seed: int, first_gid: int, gather
     status = [None] * H
 
     def run(j):
-        status[j] = lib().orc_sample_minibatch(
+        status[j] = lib().orc_sample_minibatch_mode(
             ctypes.byref(graph._struct), _ptr(t[j]), t.shape[1], _ptr(f), f.shape[0],
-            seed, first_gid + j, int(gather), ctypes.byref(arr[j]))
+            seed, first_gid + j, int(gather), FRONTIER[frontier], ctypes.byref(arr[j]))
 
     try:
         if threads > 1:

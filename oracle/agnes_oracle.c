@@ -213,9 +213,11 @@ void orc_free_minibatch(orc_minibatch* mb) {
     free(mb->indptr[h]);
     free(mb->nbr[h]);
     free(mb->col[h]);
+    free(mb->dst[h]);
     mb->indptr[h] = NULL;
     mb->nbr[h] = NULL;
     mb->col[h] = NULL;
+    mb->dst[h] = NULL;
   }
   free(mb->nodes);
   free(mb->feats);
@@ -227,8 +229,17 @@ int orc_sample_minibatch(const orc_graph* g, const int32_t* targets,
                          int32_t B, const int32_t* fanouts, int32_t K,
                          uint64_t seed, uint64_t gid, int do_gather,
                          orc_minibatch* out) {
+  return orc_sample_minibatch_mode(g, targets, B, fanouts, K, seed, gid, do_gather,
+                                   ORC_FRONTIER_SRC, out);
+}
+
+int orc_sample_minibatch_mode(const orc_graph* g, const int32_t* targets,
+                              int32_t B, const int32_t* fanouts, int32_t K,
+                              uint64_t seed, uint64_t gid, int do_gather,
+                              int32_t frontier_mode, orc_minibatch* out) {
   if (orc_check_graph(g) != ORC_OK || !out || !fanouts || B < 0 || K < 1 ||
-      K > ORC_MAX_HOPS || (B > 0 && !targets))
+      K > ORC_MAX_HOPS || (B > 0 && !targets) ||
+      (frontier_mode != ORC_FRONTIER_SRC && frontier_mode != ORC_FRONTIER_SAMPLED))
     return ORC_EINVAL;
   memset(out, 0, sizeof(*out));
   out->K = K;
@@ -265,6 +276,9 @@ int orc_sample_minibatch(const orc_graph* g, const int32_t* targets,
     const int32_t k = fanouts[h];
     const int64_t nd = n_nodes; /* dst_h = nodes[0 .. nd) */
     out->num_dst[h] = nd;
+    out->dst[h] = (int32_t*)malloc(sizeof(int32_t) * (size_t)(nd > 0 ? nd : 1));
+    if (!out->dst[h]) goto fail;
+    memcpy(out->dst[h], nodes, sizeof(int32_t) * (size_t)nd);
 
     /* Sample: indptr over dst positions, neighbour ids in slot order. */
     int64_t* indptr = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nd + 1));
@@ -350,6 +364,20 @@ int orc_sample_minibatch(const orc_graph* g, const int32_t* targets,
     }
     free(dsorted);
     free(uniq);
+
+    /* Algorithm 1 read literally: the next frontier is N_out, the distinct
+     * ids sampled at this hop, ascending (the last hop keeps src). */
+    if (frontier_mode == ORC_FRONTIER_SAMPLED && h + 1 < K) {
+      int32_t* sorted = (int32_t*)malloc(sizeof(int32_t) * (size_t)(ne > 0 ? ne : 1));
+      if (!sorted) goto fail;
+      memcpy(sorted, nbr, sizeof(int32_t) * (size_t)ne);
+      qsort(sorted, (size_t)ne, sizeof(int32_t), orc_cmp_i32);
+      int64_t n_out = 0; /* N_out is a subset of src_h, so it fits in nodes */
+      for (int64_t e = 0; e < ne; ++e)
+        if (e == 0 || sorted[e] != sorted[e - 1]) nodes[n_out++] = sorted[e];
+      free(sorted);
+      n_nodes = n_out;
+    }
   }
 
   out->nodes = nodes;
@@ -408,7 +436,7 @@ int orc_hyperbatch_stats(const orc_graph* g, const orc_minibatch* mbs,
     int64_t count = 0;
     for (int32_t j = 0; j < H; ++j) {
       for (int64_t i = 0; i < mbs[j].num_dst[h]; ++i) {
-        int32_t b = node_block[mbs[j].nodes[i]];
+        int32_t b = node_block[mbs[j].dst[h][i]];
         if (!mark[b]) {
           mark[b] = 1;
           ++count;

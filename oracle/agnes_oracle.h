@@ -62,7 +62,18 @@ typedef struct {
   int32_t* nodes;
   int64_t num_nodes;
   uint8_t* feats;
+  int32_t* dst[ORC_MAX_HOPS]; /* dst_h (num_dst[h] ids) of every hop */
 } orc_minibatch;
+
+/* Which nodes form the next hop's frontier.
+ * ORC_FRONTIER_SRC: dst_{h+1} = src_h = dst_h ++ new_h (every node reached so
+ *   far, so eq. (1) has an embedding for every dst at every layer).
+ * ORC_FRONTIER_SAMPLED: dst_{h+1} = N_out, the distinct ids sampled at hop h
+ *   in ascending order (Algorithm 1 read literally: N_in <- N_out).
+ * Blocks (src_h = dst_h ++ new_h, col into src_h) and the gathered src_{K-1}
+ * are defined the same way in both. */
+#define ORC_FRONTIER_SRC 0
+#define ORC_FRONTIER_SAMPLED 1
 
 /* Philox4x32 with 10 rounds (Salmon, Moraes, Dror, Shaw, SC'11). */
 void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2],
@@ -86,17 +97,24 @@ int orc_build_adj_blocks(const orc_graph* g, int64_t block_bytes,
                          int32_t* node_block, int64_t* num_blocks);
 
 /* Samples and gathers one minibatch (global id g).  targets: B distinct
- * node ids.  fanouts: K entries (fanouts[0] applies to the targets). */
+ * node ids.  fanouts: K entries (fanouts[0] applies to the targets).
+ * The frontier is ORC_FRONTIER_SRC. */
 int orc_sample_minibatch(const orc_graph* g, const int32_t* targets,
                          int32_t B, const int32_t* fanouts, int32_t K,
                          uint64_t seed, uint64_t gid, int do_gather,
                          orc_minibatch* out);
 
+/* The same with the frontier rule chosen by frontier_mode. */
+int orc_sample_minibatch_mode(const orc_graph* g, const int32_t* targets,
+                              int32_t B, const int32_t* fanouts, int32_t K,
+                              uint64_t seed, uint64_t gid, int do_gather,
+                              int32_t frontier_mode, orc_minibatch* out);
+
 void orc_free_minibatch(orc_minibatch* mb);
 
 /* Blocks-touched statistics for a hyperbatch of H already-sampled
  * minibatches: out[h] (h < K) = number of distinct adjacency blocks that
- * hold a node of dst_{h+1} of any minibatch; out[K] = number of distinct
+ * hold a node of dst_h (the frontier of hop h + 1) of any minibatch; out[K] = number of distinct
  * feature blocks (feat_rows_per_block rows each) that hold a node of src_K
  * of any minibatch. */
 int orc_hyperbatch_stats(const orc_graph* g, const orc_minibatch* mbs,
