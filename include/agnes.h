@@ -157,10 +157,24 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
                                       uint64_t seed, uint64_t first_minibatch_id,
                                       void* cuda_stream);
 
+/* Which nodes form each next hop's frontier (set per ctx; takes effect at
+ * the next agnes_prepare_hyperbatch).
+ * AGNES_FRONTIER_SRC (default): dst_{h+1} = src_h = dst_h ++ new_h, every
+ *   node reached so far, so the layer of eq. (1) over each hop has an input
+ *   row for each of its src nodes from the layer below.
+ * AGNES_FRONTIER_SAMPLED: dst_{h+1} = N_out, the distinct ids sampled at hop
+ *   h in ascending order (Algorithm 1 read literally: N_in <- N_out).
+ * In both, hop h's block has src_h = dst_h ++ new_h (new_h = the sampled ids
+ * not in dst_h, ascending) and col indexes src_h; the gathered rows are
+ * src_{K-1}.  Errors: EINVAL. */
+#define AGNES_FRONTIER_SRC 0
+#define AGNES_FRONTIER_SAMPLED 1
+agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode);
+
 /* View of minibatch j of the last prepared hyperbatch.  Per hop h (0-based
- * index, hop number h+1): the bipartite block has num_dst[h] dst nodes
- * (= nodes[0 .. num_dst[h])) and num_src[h] src nodes
- * (= nodes[0 .. num_src[h])); indptr[h] (num_dst[h]+1 int64, device) groups
+ * index, hop number h+1): the bipartite block has num_dst[h] dst nodes and
+ * num_src[h] src nodes, dst_h being the first num_dst[h] of src_h (with the
+ * default frontier, both are prefixes of nodes); indptr[h] (num_dst[h]+1 int64, device) groups
  * the num_edges[h] edges by dst; col[h] (num_edges[h] int32, device) gives
  * each edge's src index.  nodes (num_nodes int32, device) = src_K in global
  * ids; feats (num_nodes x feat_dim of feat_dtype, device, row-major) their
@@ -194,9 +208,10 @@ agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_vi
  *   col[h] + j*col_stride[h]         num_edges = edges[h*H + j]
  *   nodes + j*nodes_stride           num_nodes = node_size[K*H + j]
  *   feats + j*feats_stride_rows*row_bytes
- * node_size[h*H + j] (0 <= h <= K) is |dst_{h+1}| = |src_h| of minibatch j
- * (node_size[0..H) = B); edges is K x H.  node_size and edges are host
- * memory owned by ctx.  Everything stays valid until the next prepare or
+ * node_size[h*H + j] is |dst_h| of minibatch j for h < K (node_size[0..H)
+ * = B) and num_nodes = |src_{K-1}| for h = K; src_size[h*H + j] is |src_h|
+ * (equal to node_size[(h+1)*H + j] with the default frontier); edges is
+ * K x H.  node_size, src_size and edges are host memory owned by ctx.  Everything stays valid until the next prepare or
  * free.  Errors as agnes_fetch_minibatch. */
 typedef struct {
   int32_t K, H;
@@ -212,6 +227,7 @@ typedef struct {
   int64_t feat_dim;
   const int32_t* node_size;
   const int32_t* edges;
+  const int32_t* src_size;  /* K x H: |src_h| of minibatch j at h*H + j */
 } agnes_hyperbatch_view;
 agnes_status agnes_fetch_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out);
 

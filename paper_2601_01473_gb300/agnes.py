@@ -20,6 +20,7 @@ MAX_FANOUT = 1024
 
 F32, F16 = 0, 1
 FEATURE_IO = {"blocks": 0, "rows": 1}  # AGNES_FEATURE_IO_BLOCKS / _ROWS
+FRONTIER = {"src": 0, "sampled": 1}    # AGNES_FRONTIER_SRC / _SAMPLED
 _DTYPES = {torch.float32: F32, torch.float16: F16}
 _TORCH_OF = {F32: torch.float32, F16: torch.float16}
 
@@ -80,6 +81,7 @@ class _HyperbatchView(ctypes.Structure):
         ("feats", ctypes.c_void_p), ("feats_stride_rows", ctypes.c_int64),
         ("feat_dtype", ctypes.c_int32), ("feat_dim", ctypes.c_int64),
         ("node_size", ctypes.c_void_p), ("edges", ctypes.c_void_p),
+        ("src_size", ctypes.c_void_p),
     ]
 
 
@@ -128,6 +130,7 @@ SIGNATURES = {
     "agnes_phase_times": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)],
                           ctypes.c_int),
     "agnes_hop_indptr_noalloc": ([_P, _P, ctypes.c_int64, ctypes.c_int32, _P, _P], ctypes.c_int),
+    "agnes_set_frontier_mode": ([_P, ctypes.c_int32], ctypes.c_int),
     "agnes_sage_mean_layer": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int64,
                                ctypes.c_int64, _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
                                ctypes.c_int64, _P], ctypes.c_int),
@@ -219,7 +222,9 @@ class HyperbatchView:
                                    shape=((K + 1) * H,)).reshape(K + 1, H).copy()
         ed = np.ctypeslib.as_array(ctypes.cast(v.edges, ctypes.POINTER(ctypes.c_int32)),
                                    shape=(K * H,)).reshape(K, H).copy()
-        self.node_size, self.edges = sz, ed
+        ss = np.ctypeslib.as_array(ctypes.cast(v.src_size, ctypes.POINTER(ctypes.c_int32)),
+                                   shape=(K * H,)).reshape(K, H).copy()
+        self.node_size, self.edges, self.src_size = sz, ed, ss
         self.indptr = [_wrap(v.indptr[h], (H, v.indptr_stride[h]), torch.int64, device)
                        for h in range(K)]
         self.col = [_wrap(v.col[h], (H, v.col_stride[h]), torch.int32, device) for h in range(K)]
@@ -230,7 +235,7 @@ class HyperbatchView:
     def view(self, j: int) -> "MinibatchView":
         hops = []
         for h in range(self.K):
-            nd, ns, ne = int(self.node_size[h, j]), int(self.node_size[h + 1, j]), int(self.edges[h, j])
+            nd, ns, ne = int(self.node_size[h, j]), int(self.src_size[h, j]), int(self.edges[h, j])
             hops.append(Hop(nd, ns, ne, self.indptr[h][j, :nd + 1], self.col[h][j, :ne]))
         n = int(self.node_size[self.K, j])
         return MinibatchView(hops, self.nodes[j, :n], self.feats[j, :n])
@@ -335,6 +340,14 @@ class Graph:
         v = _HyperbatchView()
         _check(lib().agnes_fetch_hyperbatch(self._ctx, ctypes.byref(v)), self._ctx)
         return HyperbatchView(v, self.device)
+
+    def set_frontier(self, mode: str) -> None:
+        """"src" (dst_{h+1} = src_h, the default) or "sampled" (dst_{h+1} =
+        the distinct ids sampled at hop h: Algorithm 1's N_in <- N_out);
+        applies from the next prepare."""
+        if mode not in FRONTIER:
+            raise ValueError(f"frontier must be one of {sorted(FRONTIER)}")
+        _check(lib().agnes_set_frontier_mode(self._ctx, FRONTIER[mode]), self._ctx)
 
     def sage_mean_layer(self, hop: int, x: torch.Tensor, w: torch.Tensor, bias=None,
                         out_dtype: torch.dtype = torch.float32, stream=None) -> torch.Tensor:

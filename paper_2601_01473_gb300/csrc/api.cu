@@ -51,7 +51,9 @@ struct Workspace {
   int32_t* nfcnt = nullptr;
   int32_t* newcnt = nullptr;
   int32_t* newbase = nullptr;
-  int32_t* nsz = nullptr;   // (K+1) x H
+  int32_t* nsz = nullptr;   // (K+1) x H: |dst_h| (h < K), |src_{K-1}| (h = K)
+  int32_t* srcsz = nullptr; // K x H: |src_h|
+  int32_t* noutbase = nullptr;  // T*H: sampled frontier: per-minibatch scan of next-frontier counts
   int32_t* ecnt = nullptr;  // K x H
   int64_t* indptr[AGNES_MAX_HOPS] = {nullptr};
   int32_t* col[AGNES_MAX_HOPS] = {nullptr};
@@ -73,7 +75,7 @@ struct Workspace {
   int32_t* status = nullptr;
   unsigned long long* distinct = nullptr;
 
-  // pinned host readback: [status][nsz (K+1)H][ecnt KH] then int64 stats (K+1)
+  // pinned host readback: [status][nsz (K+1)H][ecnt KH][srcsz KH] then int64 stats (K+1)
   void* h_back = nullptr;
   size_t h_back_bytes = 0;
 };
@@ -99,6 +101,7 @@ struct agnes_ctx {
   void* pinned = nullptr;   // ctx_pinned
   size_t pinned_bytes = 0;
   int32_t feature_io = AGNES_FEATURE_IO_BLOCKS;
+  int32_t frontier_mode = AGNES_FRONTIER_SRC;
   const char* features_dev = nullptr;  // device view of host-resident features
   int64_t adj_block_bytes = 0, feat_block_bytes = 0;
   BlockTables bt;
@@ -280,6 +283,8 @@ static void free_workspace(Workspace* w) {
   cudaFree(w->newcnt);
   cudaFree(w->newbase);
   cudaFree(w->nsz);
+  cudaFree(w->srcsz);
+  cudaFree(w->noutbase);
   cudaFree(w->ecnt);
   for (int h = 0; h < AGNES_MAX_HOPS; ++h) {
     cudaFree(w->indptr[h]);
@@ -369,6 +374,8 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.newcnt, cells);
   WA(w.newbase, cells);
   WA(w.nsz, (int64_t)(K + 1) * H);
+  WA(w.srcsz, (int64_t)K * H);
+  WA(w.noutbase, cells);
   WA(w.ecnt, (int64_t)K * H);
   for (int h = 0; h < K; ++h) {
     WA(w.indptr[h], (int64_t)H * (cap[h] + 1));
@@ -396,7 +403,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.status, 1);
   WA(w.distinct, 1);
 #undef WA
-  w.h_back_bytes = sizeof(int32_t) * (1 + (size_t)(K + 1) * H + (size_t)K * H + 1) +
+  w.h_back_bytes = sizeof(int32_t) * (1 + (size_t)(K + 1) * H + 2 * (size_t)K * H + 1) +
                    sizeof(int64_t) * (K + 2);
   if (cudaMallocHost(&w.h_back, w.h_back_bytes) != cudaSuccess) {
     cudaGetLastError();
@@ -421,6 +428,7 @@ struct Back {
   int32_t* status;
   int32_t* nsz;
   int32_t* ecnt;
+  int32_t* srcsz;
   int64_t* stats;
 };
 
@@ -430,7 +438,8 @@ static Back back_of(Workspace& w) {
   b.status = p;
   b.nsz = p + 1;
   b.ecnt = b.nsz + (size_t)(w.K + 1) * w.H;
-  size_t off32 = 1 + (size_t)(w.K + 1) * w.H + (size_t)w.K * w.H + 1;
+  b.srcsz = b.ecnt + (size_t)w.K * w.H;
+  size_t off32 = 1 + (size_t)(w.K + 1) * w.H + 2 * (size_t)w.K * w.H + 1;
   b.stats = (int64_t*)((char*)w.h_back + ((off32 * sizeof(int32_t) + 7) & ~(size_t)7));
   return b;
 }
@@ -1310,6 +1319,9 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     d.nfb_pos = w.fb_pos[1 - cur];
     d.nsz_prev = nsz_prev;
     d.nsz_next = w.nsz + (int64_t)(h + 1) * H;
+    d.srcsz = w.srcsz + (int64_t)h * H;
+    d.noutbase = w.noutbase;
+    d.frontier_sampled = ctx->frontier_mode == AGNES_FRONTIER_SAMPLED && h + 1 < K;
     d.nodes = w.nodes;
     d.col = w.col[h];
     d.tile_adj_block = ctx->bt.tile_adj_block;
@@ -1337,6 +1349,7 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   CK(ctx, cudaMemcpyAsync(b.status, w.status, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.nsz, w.nsz, sizeof(int32_t) * (K + 1) * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.ecnt, w.ecnt, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaMemcpyAsync(b.srcsz, w.srcsz, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.stats, w.stats, sizeof(int64_t) * (K + 1), cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaEventRecord(ctx->done, st));
   ctx->n_phases[ring] = ctx->profiling ? ph - 1 : 0;
@@ -1363,7 +1376,7 @@ agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_vi
   out->K = w.K;
   for (int h = 0; h < w.K; ++h) {
     out->num_dst[h] = b.nsz[(size_t)h * w.H + j];
-    out->num_src[h] = b.nsz[(size_t)(h + 1) * w.H + j];
+    out->num_src[h] = b.srcsz[(size_t)h * w.H + j];
     out->num_edges[h] = b.ecnt[(size_t)h * w.H + j];
     out->indptr[h] = w.indptr[h] + (int64_t)j * (w.cap[h] + 1);
     out->col[h] = w.col[h] + (int64_t)j * w.cap[h] * w.fan[h];
@@ -1373,6 +1386,16 @@ agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_vi
   out->feats = (const char*)w.feats_out + (int64_t)j * w.capK * ctx->row_bytes;
   out->feat_dtype = ctx->feat_dtype;
   out->feat_dim = ctx->feat_dim;
+  return AGNES_OK;
+}
+
+agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode) {
+  if (!ctx) return AGNES_EINVAL;
+  if (mode != AGNES_FRONTIER_SRC && mode != AGNES_FRONTIER_SAMPLED) {
+    set_err(ctx, "frontier mode must be AGNES_FRONTIER_SRC or AGNES_FRONTIER_SAMPLED");
+    return AGNES_EINVAL;
+  }
+  ctx->frontier_mode = mode;
   return AGNES_OK;
 }
 
@@ -1402,6 +1425,7 @@ agnes_status agnes_fetch_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out) 
   out->feat_dim = ctx->feat_dim;
   out->node_size = b.nsz;
   out->edges = b.ecnt;
+  out->src_size = b.srcsz;
   return AGNES_OK;
 }
 

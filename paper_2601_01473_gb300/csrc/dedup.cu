@@ -58,6 +58,7 @@ struct CellArgs {
   int32_t* col;              // H x ecap: final col, or -(1 + local new rank)
   int32_t* big_list;         // cells with more than kDedupSmallMax entries
   int32_t* big_n;
+  bool sampled;              // next frontier = the cell's distinct sampled ids
   const int32_t* status;
 };
 
@@ -101,7 +102,7 @@ constexpr int kSlotCap = 1024;
 constexpr int kSmallMax = kDedupSmallMax;
 constexpr int kRoundFill = kSlotCap - kSmallMax;  // a cell starting below this fits
 
-enum : uint8_t { kSlotF = 1, kSlotLeader = 2, kSlotInD = 4 };
+enum : uint8_t { kSlotF = 1, kSlotLeader = 2, kSlotInD = 4, kSlotFirst = 8 };
 
 struct GroupSmem {
   int32_t fn[kGroupCells];
@@ -139,7 +140,7 @@ __global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
         a.big_list[atomicAdd(a.big_n, 1)] = (int32_t)my_cell;
       } else if (c.sn == 0) {
         a.newcnt[my_cell] = 0;
-        a.nfcnt[my_cell] = c.fn;
+        a.nfcnt[my_cell] = a.sampled ? 0 : c.fn;
       }
     }
     const int32_t ns = staged ? n : 0;
@@ -207,13 +208,15 @@ __global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
           if (sm.id[mid] < id) lo2 = mid + 1; else hi2 = mid;
         }
         uint8_t fl = 0;
-        if (lo2 < fe && sm.id[lo2] == id) {
+        const bool inD = lo2 < fe && sm.id[lo2] == id;
+        if (inD) {
           fl = kSlotInD;
           sm.fidx[sl] = (int16_t)lo2;
-        } else {
+        }
+        if (!inD || a.sampled) {  // first occurrence among the cell's samples
           bool dup = false;
           for (int32_t q = fe; q < sl; ++q) dup |= sm.id[q] == id;
-          if (!dup) fl = kSlotLeader;
+          if (!dup) fl |= (inD ? 0 : kSlotLeader) | (a.sampled ? kSlotFirst : 0);
         }
         sm.flag[sl] = fl;
       }
@@ -221,10 +224,13 @@ __global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
       // the owner counts its cell's new ids
       if (mine_in_round) {
         const int32_t fs = sm.ps[tid] - rbase;
-        int32_t cnt = 0;
-        for (int32_t q = fs + c.fn; q < fs + n; ++q) cnt += (sm.flag[q] & kSlotLeader) != 0;
+        int32_t cnt = 0, first = 0;
+        for (int32_t q = fs + c.fn; q < fs + n; ++q) {
+          cnt += (sm.flag[q] & kSlotLeader) != 0;
+          first += (sm.flag[q] & kSlotFirst) != 0;
+        }
         a.newcnt[my_cell] = cnt;
-        a.nfcnt[my_cell] = c.fn + cnt;
+        a.nfcnt[my_cell] = a.sampled ? first : c.fn + cnt;
       }
       // phase 2: local ranks, col, next-frontier entries
       for (int32_t sl = tid; sl < used; sl += kCellThreads) {
@@ -236,8 +242,13 @@ __global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
         for (int32_t q = fe; q < se; ++q) lessN += (sm.flag[q] & kSlotLeader) && sm.id[q] < id;
         const int32_t tb = sm.tb[l];
         if (fl & kSlotF) {
-          put_tmp(a, tb + (sl - fs) + lessN, id, sm.x[sl]);
+          if (!a.sampled) put_tmp(a, tb + (sl - fs) + lessN, id, sm.x[sl]);
           continue;
+        }
+        if (fl & kSlotFirst) {  // sampled frontier: the cell's distinct samples, ascending
+          int32_t lessS = 0;
+          for (int32_t q = fe; q < se; ++q) lessS += (sm.flag[q] & kSlotFirst) && sm.id[q] < id;
+          put_tmp(a, tb + lessS, id, 0);
         }
         const int64_t jrow = (int64_t)sm.j[l] * a.ecap;
         if (fl & kSlotInD) {
@@ -245,7 +256,7 @@ __global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
           continue;
         }
         a.col[jrow + sm.x[sl]] = -1 - lessN;
-        if (fl & kSlotLeader) {
+        if ((fl & kSlotLeader) && !a.sampled) {
           int32_t lo2 = fs, hi2 = fe;  // frontier ids smaller than id
           while (lo2 < hi2) {
             const int32_t mid = (lo2 + hi2) >> 1;
@@ -308,7 +319,7 @@ __global__ void __launch_bounds__(kThreads) dedup_big_kernel(CellArgs a) {
     if (c.sn == 0) {  // nothing sampled: the compaction copies the frontier cell
       if (lane == 0) {
         a.newcnt[cell] = 0;
-        a.nfcnt[cell] = c.fn;
+        a.nfcnt[cell] = a.sampled ? 0 : c.fn;
       }
       continue;
     }
@@ -316,19 +327,23 @@ __global__ void __launch_bounds__(kThreads) dedup_big_kernel(CellArgs a) {
     const int32_t words = (a.tm.tile_first[c.t + 1] - base + 31) >> 5;
     mark_bits(a, c, D, Nw, base, words);
     // new = S & ~D; per-word exclusive ranks of D and new
-    uint32_t dw[4], nw[4];
-    int32_t sd = 0, snw = 0;
+    uint32_t dw[4], nw[4], sw[4];
+    int32_t sd = 0, snw = 0, ssw = 0;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int w = lane * 4 + q;
       dw[q] = w < words ? D[w] : 0u;
-      nw[q] = w < words ? (Nw[w] & ~dw[q]) : 0u;
+      sw[q] = w < words ? Nw[w] : 0u;
+      nw[q] = sw[q] & ~dw[q];
       sd += __popc(dw[q]);
       snw += __popc(nw[q]);
+      ssw += __popc(sw[q]);
     }
     const int32_t tot_new = warp_sum(snw);
+    const int32_t tot_s = warp_sum(ssw);
     int32_t rd = warp_incl_scan(sd) - sd;
     int32_t rn = warp_incl_scan(snw) - snw;
+    int32_t rs = warp_incl_scan(ssw) - ssw;
     __syncwarp();
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -342,7 +357,7 @@ __global__ void __launch_bounds__(kThreads) dedup_big_kernel(CellArgs a) {
     __syncwarp();
     if (lane == 0) {
       a.newcnt[cell] = tot_new;
-      a.nfcnt[cell] = c.fn + tot_new;
+      a.nfcnt[cell] = a.sampled ? tot_s : c.fn + tot_new;
     }
     const int64_t jcap = (int64_t)c.j * a.capK;
     int32_t* col = a.col + (int64_t)c.j * a.ecap;
@@ -355,6 +370,21 @@ __global__ void __launch_bounds__(kThreads) dedup_big_kernel(CellArgs a) {
                                : -1 - (pN[w] + __popc(Nw[w] & below));
     }
     const int32_t tb = c.fo + c.so;
+    if (a.sampled) {  // the tile's distinct sampled ids, ascending
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int w = lane * 4 + q;
+        uint32_t rest = w < words ? sw[q] : 0u;
+        while (rest) {
+          const int bb = __ffs(rest) - 1;
+          rest &= rest - 1u;
+          put_tmp(a, tb + rs + __popc(sw[q] & ((1u << bb) - 1u)), base + w * 32 + bb, 0);
+        }
+        rs += __popc(sw[q]);
+      }
+      __syncwarp();
+      continue;
+    }
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int w = lane * 4 + q;
@@ -409,6 +439,8 @@ struct CompactArgs {
   const int32_t* nfcell_off;
   const int32_t* newbase;
   const int32_t* nsz_prev;
+  const int32_t* noutbase;   // sampled frontier: rows are positions among the distinct samples
+  bool sampled;
   int32_t* nfb_id;
   int32_t* nfb_pos;
   int32_t* nodes;
@@ -436,8 +468,9 @@ __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs
       const int32_t sn = a.soff[cell + 1] - so;
       const int32_t j = (int32_t)(cell % a.H);
       s_nfo[tid] = a.nfcell_off[cell];
-      s_src[tid] = sn == 0 ? fo : ~(fo + so);
-      s_row[tid] = (int32_t)((int64_t)j * a.capK + a.nsz_prev[j] + a.newbase[cell]);
+      s_src[tid] = sn == 0 && !a.sampled ? fo : ~(fo + so);
+      s_row[tid] = (int32_t)((int64_t)j * a.capK +
+                             (a.sampled ? a.noutbase[cell] : a.nsz_prev[j] + a.newbase[cell]));
     }
     if (tid == 0) s_nfo[last - c0] = a.nfcell_off[last];
     __syncthreads();
@@ -458,7 +491,10 @@ __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs
         const int2 e = a.tmp[~src + r];
         id = e.x;
         pos = e.y;
-        if (pos < 0) {
+        if (a.sampled) {
+          pos = s_row[lo] + r;
+          a.nodes[pos] = id;
+        } else if (pos < 0) {
           pos = s_row[lo] + (-1 - pos);
           a.nodes[pos] = id;
         }
@@ -505,6 +541,7 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   c.col = d.col;
   c.big_list = d.big_list;
   c.big_n = d.big_n;
+  c.sampled = d.frontier_sampled;
   c.status = a.status;
   dedup_cells_kernel<<<resident_grid((const void*)dedup_cells_kernel, kCellThreads, num_sms),
                        kCellThreads, 0, st>>>(c);
@@ -512,8 +549,15 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
                      st>>>(c);
   // per-minibatch offsets of the new ids: scan down the tiles of the
   // tile-major [T x H] count matrix; totals give the next frontier sizes
-  e = col_scan(d.newcnt, d.newbase, a.T, a.H, d.nsz_prev, d.nsz_next, d.scan_scratch, a.status,
-               st);
+  // |src_h| = |dst_h| + new ids; the next frontier is src_h, or (sampled
+  // frontier) the distinct sampled ids, numbered by their own column scan
+  e = col_scan(d.newcnt, d.newbase, a.T, a.H, d.nsz_prev, d.srcsz, d.scan_scratch, a.status, st);
+  if (e != cudaSuccess) return e;
+  if (d.frontier_sampled)
+    e = col_scan(d.nfcnt, d.noutbase, a.T, a.H, nullptr, d.nsz_next, d.scan_scratch, a.status,
+                 st);
+  else
+    e = cudaMemcpyAsync(d.nsz_next, d.srcsz, sizeof(int32_t) * a.H, cudaMemcpyDeviceToDevice, st);
   if (e != cudaSuccess) return e;
   e = seg_scan<int32_t, int32_t>(d.nfcnt, 0, d.nfcell_off, 0, nullptr, ncells, 1, ncells, true,
                                  nullptr, d.scan_scratch, a.status, st);
@@ -532,6 +576,8 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   k.nfcell_off = d.nfcell_off;
   k.newbase = d.newbase;
   k.nsz_prev = d.nsz_prev;
+  k.noutbase = d.noutbase;
+  k.sampled = d.frontier_sampled;
   k.nfb_id = d.nfb_id;
   k.nfb_pos = d.nfb_pos;
   k.nodes = d.nodes;

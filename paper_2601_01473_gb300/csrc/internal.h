@@ -142,7 +142,10 @@ struct DedupBufs {
   int32_t* nfb_id;          // next frontier bucket
   int32_t* nfb_pos;
   const int32_t* nsz_prev;  // H frontier sizes
-  int32_t* nsz_next;        // H
+  int32_t* nsz_next;        // H: next frontier sizes
+  int32_t* srcsz;           // H: |src_h| = |dst_h| + new ids
+  int32_t* noutbase;        // T*H (frontier_sampled): per-minibatch scan of nfcnt over tiles
+  bool frontier_sampled;    // next frontier = distinct sampled ids (Algorithm 1's N_out)
   int32_t* nodes;           // H x capK
   int32_t* col;             // H x ecap
   const int32_t* tile_adj_block;

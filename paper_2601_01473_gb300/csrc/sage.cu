@@ -467,7 +467,7 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
   int64_t tiles = 0;
   for (int j = 0; j < H; ++j) {
     const int64_t nd = v.node_size[(size_t)hop * H + j];
-    const int64_t ns = v.node_size[(size_t)(hop + 1) * H + j];
+    const int64_t ns = v.src_size[(size_t)hop * H + j];
     max_dst = nd > max_dst ? nd : max_dst;
     max_src = ns > max_src ? ns : max_src;
     tabs[j] = (int32_t)tiles;

@@ -23,16 +23,18 @@ def _bytes(t: torch.Tensor) -> np.ndarray:
 
 
 def compare(g: Graph, og: oracle.Graph, targets: np.ndarray, fanouts, seed, gid0, adj_bb, feat_bb,
-            check_stats=True, only=None):
+            check_stats=True, only=None, frontier="src"):
     """Compares every (or the listed) minibatch of g's last hyperbatch with
     the oracle."""
     H = targets.shape[0]
     js = range(H) if only is None else only
     if check_stats:
-        ref, ref_stats = oracle.hyperbatch(og, targets, fanouts, seed, gid0, True, adj_bb, feat_bb)
+        ref, ref_stats = oracle.hyperbatch(og, targets, fanouts, seed, gid0, True, adj_bb, feat_bb,
+                                           frontier=frontier)
         assert g.stats() == ref_stats
     else:
-        ref = {j: oracle.sample_minibatch(og, targets[j], fanouts, seed, gid0 + j) for j in js}
+        ref = {j: oracle.sample_minibatch(og, targets[j], fanouts, seed, gid0 + j,
+                                          frontier=frontier) for j in js}
     for j in js:
         v, r = g.fetch(j), ref[j]
         assert np.array_equal(v.nodes.cpu().numpy(), r["nodes"]), f"nodes of minibatch {j}"
@@ -298,6 +300,35 @@ def test_feature_cache_needs_host_features(cuda_device):
         Graph(off.to(cuda_device), ind.to(cuda_device), feats.to(cuda_device),
               adj_block_bytes=4096, feat_block_bytes=4096, feature_cache_bytes=1 << 20)
     assert e.value.status == 1
+
+
+@pytest.mark.parametrize("bb,fan,H,B", [
+    (8192, [8, 4, 2], 4, 200),       # small cells (short tiles)
+    (1 << 20, [15, 10, 5], 3, 300),  # 4096-id tiles: cells of hundreds of entries
+    (4096, [5, 5], 6, 100),
+])
+def test_sampled_frontier_matches_oracle(cuda_device, bb, fan, H, B):
+    """Algorithm 1's literal frontier (N_in <- N_out): bit-exact blocks, node
+    lists, features and blocks-touched statistics, then the default frontier
+    again on the same ctx."""
+    off, ind, feats = make(30000, 12, seed=bb % 97 + len(fan))
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    g = load(off, ind, feats, bb, bb)
+    targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), H, B, 5, 0)
+    g.set_frontier("sampled")
+    g.prepare(targets.to(cuda_device), fan, 13, 7)
+    compare(g, og, targets.numpy(), fan, 13, 7, bb, bb, frontier="sampled")
+    allv = g.fetch_all()
+    if len(fan) > 1:  # the sampled frontier is a strict subset of src somewhere
+        assert (allv.node_size[1] < allv.src_size[0]).any()
+    g.set_frontier("src")
+    g.prepare(targets.to(cuda_device), fan, 13, 7)
+    compare(g, og, targets.numpy(), fan, 13, 7, bb, bb, frontier="src")
+    allv = g.fetch_all()
+    assert np.array_equal(allv.node_size[1:len(fan)], allv.src_size[:len(fan) - 1])
+    with pytest.raises(ValueError):
+        g.set_frontier("bogus")
+    g.close()
 
 
 def test_fetch_all_equals_per_minibatch_fetch(cuda_device):

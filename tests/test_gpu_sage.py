@@ -38,7 +38,7 @@ def _check_layer(allv, hop, x, w, b, out, x_f16, out_f16):
     worst = 0.0
     for j in range(allv.H):
         nd = int(allv.node_size[hop, j])
-        ns = int(allv.node_size[hop + 1, j])
+        ns = int(allv.src_size[hop, j])
         ne = int(allv.edges[hop, j])
         indptr = allv.indptr[hop][j, :nd + 1].cpu().numpy()
         col = allv.col[hop][j, :ne].cpu().numpy()
