@@ -153,9 +153,11 @@ def algorithmic_bytes(c: dict, off_bytes: int) -> dict:
     return {"sampling": hop, "gather": gather, "total": hop + gather}
 
 
-def gather_traffic_from_profile():
+def gather_traffic_from_profile(workload: str):
     """Per-launch DRAM traffic of the gather kernel from the committed ncu
-    summary, if it was taken on the current gather source."""
+    summary, if it was taken on the current gather source and this workload."""
+    if workload != "rmat100m":
+        return None
     path = os.path.join(ROOT, "profiles", "gather_rmat100m.md")
     src = os.path.join(ROOT, "paper_2601_01473_gb300", "csrc", "gather.cu")
     try:
@@ -400,7 +402,7 @@ def main():
                 "frac": achieved / peak if achieved else None,
                 "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
                 if peak_kind == "measured" else "fallback 6.8 TB/s",
-                "traffic": gather_traffic_from_profile(),
+                "traffic": gather_traffic_from_profile(w.name),
                 "algorithmic_bytes_per_launch": gather_bytes,
                 "avg_launch_ms": g_ms,
                 "path_algorithmic_bytes_per_step": total_bytes,

@@ -48,6 +48,39 @@ __device__ __forceinline__ int64_t block_excl_scan(int64_t v, int64_t* total) {
   return out;
 }
 
+// In-place exclusive scan of n int64 values at p (element i at p[i * stride])
+// by one CTA: each pass loads kItems consecutive values per thread before
+// scanning them, so a pass costs one memory round trip.  Returns the total.
+__device__ __forceinline__ int64_t cta_scan_inplace(int64_t* p, int64_t n, int64_t stride,
+                                                   bool volatile_loads) {
+  int64_t carry = 0;
+  for (int64_t base = 0; base < n; base += (int64_t)kThreads * kItems) {
+    const int64_t i0 = base + (int64_t)threadIdx.x * kItems;
+    int64_t v[kItems];
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t i = i0 + k;
+      v[k] = i < n ? (volatile_loads ? *(volatile int64_t*)(p + i * stride) : p[i * stride]) : 0;
+    }
+    int64_t run = 0;
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t x = v[k];
+      v[k] = run;
+      run += x;
+    }
+    int64_t tot;
+    const int64_t ex = block_excl_scan(run, &tot);
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t i = i0 + k;
+      if (i < n) p[i * stride] = carry + ex + v[k];
+    }
+    carry += tot;
+  }
+  return carry;
+}
+
 // Chunk sums; the last chunk of a segment to finish (atomic ticket after a
 // fence, no waiting) then scans the segment's chunk sums in place, writes
 // the segment total, and resets the ticket for the next scan.
@@ -63,10 +96,16 @@ scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t*
   const int64_t len = seg_len(d_len, const_len, s);
   const int64_t begin = c * kChunk;
   int64_t sum = 0;
-  if (begin < len) {
+  if (begin < len) {  // all of the thread's loads in flight at once
     const InT* p = in + (int64_t)s * in_stride;
-    const int64_t end = min(len, begin + kChunk);
-    for (int64_t i = begin + threadIdx.x; i < end; i += kThreads) sum += (int64_t)p[i];
+    InT v[kItems];
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t i = begin + k * kThreads + threadIdx.x;
+      v[k] = i < len ? p[i] : (InT)0;
+    }
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) sum += (int64_t)v[k];
   }
   __shared__ int64_t wsum[kThreads / 32];
   __shared__ bool last;
@@ -85,16 +124,7 @@ scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t*
   __syncthreads();
   if (!last) return;
   __threadfence();
-  int64_t* ps = partial + (int64_t)s * chunks;
-  int64_t carry = 0;
-  for (int64_t base = 0; base < chunks; base += kThreads) {
-    const int64_t i = base + threadIdx.x;
-    const int64_t v = i < chunks ? *(volatile int64_t*)(ps + i) : 0;
-    int64_t tot;
-    const int64_t ex = block_excl_scan(v, &tot);
-    if (i < chunks) ps[i] = carry + ex;
-    carry += tot;
-  }
+  const int64_t carry = cta_scan_inplace(partial + (int64_t)s * chunks, chunks, 1, true);
   if (threadIdx.x == 0) {
     if (write_end) out[(int64_t)s * out_stride + len] = (OutT)carry;
     if (seg_total) seg_total[s] = (int32_t)carry;
@@ -119,6 +149,7 @@ scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict
   const int64_t wbase = begin + (int64_t)warp * (32 * kItems);
   const InT* p = in + (int64_t)s * in_stride;
   OutT* q = out + (int64_t)s * out_stride;
+  const int64_t chunk_off = partial[(int64_t)s * chunks + c];  // issued with the loads below
   int64_t v[kItems];
 #pragma unroll
   for (int k = 0; k < kItems; ++k) {
@@ -142,7 +173,7 @@ scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict
     if (lane < kThreads / 32) wtot[lane] = wi - w;
   }
   __syncthreads();
-  const int64_t off = partial[(int64_t)s * chunks + c] + wtot[warp];
+  const int64_t off = chunk_off + wtot[warp];
 #pragma unroll
   for (int k = 0; k < kItems; ++k) {
     const int64_t i = wbase + k * 32 + lane;
@@ -151,7 +182,7 @@ scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict
 }
 
 // ---- column scan of a row-major [rows x cols] matrix ----------------------------
-constexpr int kColRows = 64;  // rows per chunk
+constexpr int kColRows = 16;  // rows per chunk
 
 __global__ void __launch_bounds__(128)
 col_reduce_kernel(const int32_t* __restrict__ in, int64_t rows, int32_t cols,
@@ -161,9 +192,12 @@ col_reduce_kernel(const int32_t* __restrict__ in, int64_t rows, int32_t cols,
   if (c >= cols) return;
   const int64_t r0 = (int64_t)blockIdx.x * kColRows;
   const int64_t r1 = min(rows, r0 + kColRows);
+  int32_t v[kColRows];
+#pragma unroll
+  for (int k = 0; k < kColRows; ++k) v[k] = r0 + k < r1 ? in[(r0 + k) * cols + c] : 0;
   int64_t sum = 0;
-#pragma unroll 8
-  for (int64_t r = r0; r < r1; ++r) sum += in[r * cols + c];
+#pragma unroll
+  for (int k = 0; k < kColRows; ++k) sum += v[k];
   partial[(int64_t)blockIdx.x * cols + c] = sum;
 }
 
@@ -174,15 +208,7 @@ col_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, int32_t cols,
                     const int32_t* status) {
   if (status && failed(status)) return;
   const int32_t c = blockIdx.x;
-  int64_t carry = 0;
-  for (int64_t base = 0; base < chunks; base += kThreads) {
-    const int64_t i = base + threadIdx.x;
-    const int64_t v = i < chunks ? partial[i * cols + c] : 0;
-    int64_t tot;
-    const int64_t ex = block_excl_scan(v, &tot);
-    if (i < chunks) partial[i * cols + c] = carry + ex;
-    carry += tot;
-  }
+  const int64_t carry = cta_scan_inplace(partial + c, chunks, cols, false);
   if (threadIdx.x == 0 && total_out)
     total_out[c] = (int32_t)carry + (add_in ? add_in[c] : 0);
 }
@@ -196,11 +222,13 @@ col_down_kernel(const int32_t* __restrict__ in, int32_t* __restrict__ out, int64
   const int64_t r0 = (int64_t)blockIdx.x * kColRows;
   const int64_t r1 = min(rows, r0 + kColRows);
   int64_t run = partial[(int64_t)blockIdx.x * cols + c];
-#pragma unroll 8
-  for (int64_t r = r0; r < r1; ++r) {
-    const int32_t v = in[r * cols + c];
-    out[r * cols + c] = (int32_t)run;
-    run += v;
+  int32_t v[kColRows];
+#pragma unroll
+  for (int k = 0; k < kColRows; ++k) v[k] = r0 + k < r1 ? in[(r0 + k) * cols + c] : 0;
+#pragma unroll
+  for (int k = 0; k < kColRows; ++k) {
+    if (r0 + k < r1) out[(r0 + k) * cols + c] = (int32_t)run;
+    run += v[k];
   }
 }
 
