@@ -310,9 +310,10 @@ agnes_status agnes_phase_times(agnes_ctx* ctx, int32_t ago, float* ms, int32_t n
  * Arithmetic: the mean is summed and divided in fp32, the update's inputs
  * are rounded to fp16, and the products are accumulated in fp32 on the
  * tensor cores (tcgen05).  d_in is a multiple of 8, d_out a multiple of 32
- * in [32, 256], and the two operands must fit shared memory:
- * 512*d_in + 4*d_in*d_out + 17440 <= AGNES_SAGE_MAX_SMEM bytes (ERANGE
- * otherwise).  x, w and out are 16-byte aligned.  Waits for the hyperbatch
+ * in [32, 256], and W plus one 128-row tile of [x_i | mean_i] must fit
+ * shared memory: 512*d_in + 4*d_in*d_out + 128 <= AGNES_SAGE_MAX_SMEM bytes
+ * (ERANGE otherwise).  Scratch: the layer keeps [x_i | mean_i] of every dst
+ * row (4*d_in bytes each) in device memory owned by ctx.  x, w and out are 16-byte aligned.  Waits for the hyperbatch
  * like agnes_fetch_hyperbatch, runs on cuda_stream and waits for it.
  * Errors: EINVAL, ERANGE, ESTATE, ECUDA, ETIMEOUT (a tensor-core completion
  * wait ran out; the layer's output is then undefined). */

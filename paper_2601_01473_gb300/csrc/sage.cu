@@ -5,24 +5,24 @@
 //
 //   out_i = ReLU(W_self x_i + W_neigh mean_{(i,u) in hop} x_u + b).
 //
-// One persistent CTA per SM takes tiles of 128 dst rows of one minibatch.
-// Its 16 warps aggregate the tile into shared memory as the update's input
-// A = [x_dst | agg] (128 x 2 d_in, fp16, in the K-major no-swizzle layout of
-// tcgen05 shared-memory operands: 8-row x 16-byte core matrices, the 16 row
-// groups of a 16-byte K slice stored one after another).  One thread then
-// issues the tile's chain of tcgen05.mma (M = 128, N = d_out, K = 16 each)
-// against W (loaded into shared memory once per CTA, same layout) with the
-// fp32 accumulator in tensor memory, and commits it to an mbarrier.  Every
-// warp reads a 32-row x d_out/4 slice of the accumulator back with
-// tcgen05.ld, adds the bias, applies ReLU and stores it.
-//
-// The aggregation reads ~(1 + deg) rows per dst row from HBM and the
-// contraction is 2 * 128 * 2 d_in * d_out flops per tile, so for the sampled
-// degrees the layer is bound by HBM, with the tensor cores keeping the
-// update off the critical path.
+// Two kernels.  The dst rows of minibatch j form ceil(|dst_h| / 128) tiles of
+// 128 rows (the MMA's M).
+//  1. sage_agg_kernel (HBM-bound gather): for every row, the mean of its
+//     neighbours' rows in fp32, written with the row itself as the update's
+//     input A = [x_i | mean_i] in fp16 -- each tile as the exact image of a
+//     tcgen05 K-major, no-swizzle shared-memory operand (8-row x 16-byte core
+//     matrices, the 16 row groups of one 16-byte K slice after one another).
+//     No shared memory and no barriers, so it runs at full occupancy.
+//  2. sage_gemm_kernel (persistent, warp-specialised, one CTA per SM): W is
+//     loaded into shared memory once; a producer lane moves A tiles into a
+//     ring of shared-memory stages with cp.async.bulk (mbarrier transaction
+//     counts); an MMA lane issues each tile's tcgen05.mma chain (M = 128,
+//     N = d_out, K = 16 each) into one of two TMEM accumulators; four
+//     epilogue warps read the accumulator back with tcgen05.ld, add the bias,
+//     apply ReLU and store -- overlapped with the next tile's copy and MMA.
+// Every mbarrier wait is bounded; on timeout the kernel records an error,
+// frees its tensor memory and returns.
 #include <cuda_fp16.h>
-
-#include <vector>
 
 #include "../../include/agnes.h"
 #include "common.cuh"
@@ -32,16 +32,16 @@ namespace agnes {
 
 namespace {
 
-constexpr int kM = 128;          // dst rows per tile (the MMA's M)
-constexpr int kSageThreads = 512;
-constexpr int kSageWarps = kSageThreads / 32;
+constexpr int kM = 128;              // dst rows per tile (the MMA's M)
 constexpr int kWaitIters = 1 << 24;  // mbarrier polls before giving up (~1 s)
-constexpr int kIpSlots = kM + 2;     // staged indptr entries (kM + 1, padded to 16 bytes)
-constexpr int kColCap = 4096;        // staged columns per tile (fanouts up to 32)
-constexpr size_t kStageBytes = kIpSlots * 8 + kColCap * 4 + 16;  // + mbarrier, TMEM slot
+constexpr int kAggThreads = 256;
+constexpr int kGemmThreads = 256;    // warp 0 producer, warp 1 MMA, warps 4-7 epilogue
+constexpr int kBarBytes = 128;       // mbarriers + TMEM address slot
+// Every GEMM CTA asks for at least this much shared memory, so no two CTAs
+// share an SM (and its 512 tensor-memory columns).
+constexpr size_t kSageMinSmem = 120 * 1024;
 
-// error word bits
-constexpr int32_t kSageTimeout = 1;
+constexpr int32_t kSageTimeout = 1;  // error word bits
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
@@ -49,7 +49,7 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 
 // Byte offset of element (r, k) in a K-major no-swizzle operand of `rows`
 // rows: core matrix (r / 8, k / 8) at ((k / 8) * rows / 8 + r / 8) * 128.
-__device__ __forceinline__ uint32_t kmajor_off(int r, int k, int rows) {
+__host__ __device__ __forceinline__ uint32_t kmajor_off(int r, int k, int rows) {
   return (uint32_t)((((k >> 3) * (rows >> 3)) + (r >> 3)) * 128 + (r & 7) * 16 + (k & 7) * 2);
 }
 
@@ -79,6 +79,27 @@ __device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t a, uint64_t b,
       : "memory");
 }
 
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+// Waits for the phase with the given parity to complete; false after
+// kWaitIters polls.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   for (int it = 0; it < kWaitIters; ++it) {
     uint32_t done;
@@ -95,47 +116,19 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   return false;
 }
 
-struct SageArgs {
-  const void* x;              // minibatch j's src rows at x + (j * x_stride + r) * d_in
-  int64_t x_stride;
-  const int64_t* indptr;      // minibatch j at indptr + j * indptr_stride
-  int64_t indptr_stride;
-  const int32_t* col;
-  int64_t col_stride;
-  const int32_t* tile_start;  // H + 1: first tile of each minibatch
-  const int32_t* num_dst;     // host-computed per minibatch dst sizes (device copy)
-  int32_t H;
-  int32_t d_in, d_out;
-  const __half* w;            // d_out x 2 d_in
-  const float* bias;          // d_out or null
-  void* out;                  // minibatch j's dst rows at out + (j * out_stride + i) * d_out
-  int64_t out_stride;
-  int32_t* err;
-};
-
-// 8 consecutive features of row r as fp16 (fp32 inputs are rounded).
-template <typename T>
-__device__ __forceinline__ uint4 load8_h(const T* row, int c);
-
-template <>
-__device__ __forceinline__ uint4 load8_h<__half>(const __half* row, int c) {
-  return __ldg((const uint4*)row + c);
-}
-
-template <>
-__device__ __forceinline__ uint4 load8_h<float>(const float* row, int c) {
-  const float4 a = __ldg((const float4*)row + 2 * c), b = __ldg((const float4*)row + 2 * c + 1);
-  uint4 r;
-  __half2 h;
-  h = __floats2half2_rn(a.x, a.y); r.x = *(uint32_t*)&h;
-  h = __floats2half2_rn(a.z, a.w); r.y = *(uint32_t*)&h;
-  h = __floats2half2_rn(b.x, b.y); r.z = *(uint32_t*)&h;
-  h = __floats2half2_rn(b.z, b.w); r.w = *(uint32_t*)&h;
-  return r;
+// Bulk copy of `bytes` (a multiple of 16, both addresses 16-byte aligned)
+// from global memory into shared memory, completing a transaction on bar.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
 }
 
 // 8 consecutive features of a row as raw 16-byte vectors (one for fp16, two
-// for fp32), loaded before they are summed so that many are in flight.
+// for fp32).
 template <typename T>
 struct Chunk {
   uint4 v[sizeof(T) / 2];
@@ -166,19 +159,162 @@ __device__ __forceinline__ void add_chunk(const Chunk<float>& ch, float* acc) {
   for (int q = 0; q < 8; ++q) acc[q] += f[q];
 }
 
-template <typename T, typename OutT>
-__global__ void __launch_bounds__(kSageThreads, 1) sage_mean_kernel(SageArgs a) {
+__device__ __forceinline__ uint4 to_half8(const float* f) {
+  uint4 o;
+  __half2 h;
+  h = __floats2half2_rn(f[0], f[1]); o.x = *(uint32_t*)&h;
+  h = __floats2half2_rn(f[2], f[3]); o.y = *(uint32_t*)&h;
+  h = __floats2half2_rn(f[4], f[5]); o.z = *(uint32_t*)&h;
+  h = __floats2half2_rn(f[6], f[7]); o.w = *(uint32_t*)&h;
+  return o;
+}
+
+struct SageArgs {
+  const void* x;              // minibatch j's src rows at x + (j * x_stride + r) * d_in
+  int64_t x_stride;
+  const int64_t* indptr;      // minibatch j at indptr + j * indptr_stride
+  int64_t indptr_stride;
+  const int32_t* col;
+  int64_t col_stride;
+  const int32_t* tile_start;  // H + 1: first tile of each minibatch
+  const int32_t* num_dst;     // H: |dst_h| per minibatch
+  const int32_t* tile_mb;     // per tile: its minibatch
+  int32_t H;
+  int32_t d_in, d_out;
+  uint8_t* A;                 // tiles x (kM x 2 d_in fp16), each tile a shared-memory image
+  const __half* w;            // d_out x 2 d_in
+  const float* bias;          // d_out or null
+  void* out;                  // minibatch j's dst rows at out + (j * out_stride + i) * d_out
+  int64_t out_stride;
+  int32_t stages;             // A stages in the GEMM's shared memory
+  int32_t* err;
+};
+
+
+// Items (R, c): row R of the tile space, 8-feature chunk c of x; each
+// thread takes kAggU items kAggThreads apart at a time, every load stage
+// issued for all of them before the next.  Writes the chunk of x_i and of
+// mean_i into the row's A tile (zeros past |dst_h|).
+constexpr int kAggU = 1;
+
+template <typename T>
+__global__ void __launch_bounds__(kAggThreads, 5) sage_agg_kernel(SageArgs a, int64_t rows_total) {
+  constexpr int kER = sizeof(T) == 2 ? 8 : 4;  // edges in flight per item and round
+  constexpr int U = kAggU;
+  const int chunks = a.d_in / 8;
+  const int64_t items = rows_total * chunks;
+  const size_t tile_bytes = (size_t)kM * 2 * a.d_in * 2;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q0 = blockIdx.x * (int64_t)blockDim.x * U + threadIdx.x; q0 < items;
+       q0 += stride * U) {
+    int c[U], tile[U], r[U];
+    bool row_ok[U];
+    const T* x[U];
+    const int32_t* cl[U];
+    int64_t e0[U], e1[U], span = 0;
+    Chunk<T> sc[U];
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int64_t q = q0 + (int64_t)k * blockDim.x;
+      const int64_t R = q < items ? q / chunks : 0;
+      c[k] = (int)(q - R * chunks);
+      tile[k] = (int)(R / kM);
+      r[k] = (int)(R - (int64_t)tile[k] * kM);
+      row_ok[k] = false;
+      e0[k] = e1[k] = 0;
+      if (q < items) {
+        const int j = __ldg(a.tile_mb + tile[k]);
+        const int i = (tile[k] - __ldg(a.tile_start + j)) * kM + r[k];
+        if (i < __ldg(a.num_dst + j)) {
+          row_ok[k] = true;
+          x[k] = (const T*)a.x + (size_t)j * a.x_stride * a.d_in;
+          cl[k] = a.col + (size_t)j * a.col_stride;
+          const int64_t* ip = a.indptr + (size_t)j * a.indptr_stride;
+          sc[k] = load_chunk<T>(x[k] + (size_t)i * a.d_in, c[k]);
+          e0[k] = __ldg(ip + i);
+          e1[k] = __ldg(ip + i + 1);
+          span = e1[k] - e0[k] > span ? e1[k] - e0[k] : span;
+        }
+      }
+    }
+    float acc[U][8];
+#pragma unroll
+    for (int k = 0; k < U; ++k)
+#pragma unroll
+      for (int z = 0; z < 8; ++z) acc[k][z] = 0.f;
+    for (int64_t base = 0; base < span; base += kER) {
+      int32_t idx[U][kER];
+#pragma unroll
+      for (int k = 0; k < U; ++k)
+#pragma unroll
+        for (int u = 0; u < kER; ++u)
+          idx[k][u] = e0[k] + base + u < e1[k] ? __ldg(cl[k] + e0[k] + base + u) : -1;
+      Chunk<T> val[U][kER];
+#pragma unroll
+      for (int k = 0; k < U; ++k)
+#pragma unroll
+        for (int u = 0; u < kER; ++u) {
+          if (idx[k][u] >= 0) {
+            val[k][u] = load_chunk<T>(x[k] + (size_t)idx[k][u] * a.d_in, c[k]);
+          } else {
+#pragma unroll
+            for (int z = 0; z < (int)(sizeof(T) / 2); ++z)
+              val[k][u].v[z] = make_uint4(0, 0, 0, 0);
+          }
+        }
+#pragma unroll
+      for (int k = 0; k < U; ++k)
+#pragma unroll
+        for (int u = 0; u < kER; ++u) add_chunk(val[k][u], acc[k]);
+    }
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int64_t q = q0 + (int64_t)k * blockDim.x;
+      if (q >= items) continue;
+      uint4 self = make_uint4(0, 0, 0, 0), mean = make_uint4(0, 0, 0, 0);
+      if (row_ok[k]) {
+        if constexpr (sizeof(T) == 2) {
+          self = sc[k].v[0];
+        } else {
+          const float* f = (const float*)&sc[k].v[0];
+          float g[8];
+#pragma unroll
+          for (int z = 0; z < 8; ++z) g[z] = f[z];
+          self = to_half8(g);
+        }
+        if (e1[k] > e0[k]) {
+          const float deg = (float)(e1[k] - e0[k]);
+#pragma unroll
+          for (int z = 0; z < 8; ++z) acc[k][z] /= deg;
+          mean = to_half8(acc[k]);
+        }
+      }
+      uint8_t* At = a.A + (size_t)tile[k] * tile_bytes;
+      *(uint4*)(At + kmajor_off(r[k], c[k] * 8, kM)) = self;
+      *(uint4*)(At + kmajor_off(r[k], a.d_in + c[k] * 8, kM)) = mean;
+    }
+  }
+}
+
+template <typename OutT>
+__global__ void __launch_bounds__(kGemmThreads, 1) sage_gemm_kernel(SageArgs a) {
   extern __shared__ __align__(1024) uint8_t smem[];
-  const int KT = 2 * a.d_in;        // the update's K
+  const int KT = 2 * a.d_in;
   const int N = a.d_out;
-  uint8_t* sA = smem;                                   // kM x KT fp16
-  uint8_t* sW = smem + (size_t)kM * KT * 2;             // N x KT fp16
-  int64_t* s_ip = (int64_t*)(sW + (size_t)N * KT * 2);  // kM + 1 (padded to kIpSlots)
-  int32_t* s_col = (int32_t*)(s_ip + kIpSlots);          // kColCap
-  uint64_t* bar = (uint64_t*)(s_col + kColCap);
-  uint32_t* tmem_slot = (uint32_t*)(bar + 1);
+  const int S = a.stages;
+  const uint32_t tile_bytes = (uint32_t)kM * KT * 2;
+  uint8_t* sW = smem;                                 // N x KT fp16
+  uint8_t* sA = smem + (size_t)N * KT * 2;            // S stages of kM x KT fp16
+  uint64_t* bars = (uint64_t*)(sA + (size_t)S * tile_bytes);
+  // full[0..S), empty[4..4+S), dfull[8..10), dempty[10..12), then the TMEM slot
+  const uint32_t bar0 = smem_u32(bars);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const uint32_t ncols = N <= 32 ? 32 : (N <= 64 ? 64 : (N <= 128 ? 128 : 256));
+  const uint32_t ncols = 2 * N <= 64 ? 64 : (2 * N <= 128 ? 128 : (2 * N <= 256 ? 256 : 512));
+  uint32_t* tmem_slot = (uint32_t*)(bars + 12);
+#define AGNES_FULL(s) (bar0 + 8u * (uint32_t)(s))
+#define AGNES_EMPTY(s) (bar0 + 8u * (uint32_t)(4 + (s)))
+#define AGNES_DFULL(d) (bar0 + 8u * (uint32_t)(8 + (d)))
+#define AGNES_DEMPTY(d) (bar0 + 8u * (uint32_t)(10 + (d)))
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -188,12 +324,19 @@ __global__ void __launch_bounds__(kSageThreads, 1) sage_mean_kernel(SageArgs a) 
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   if (tid == 0) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bar)) : "memory");
+    for (int s = 0; s < S; ++s) {
+      mbar_init(AGNES_FULL(s), 1);
+      mbar_init(AGNES_EMPTY(s), 1);
+    }
+    for (int d = 0; d < 2; ++d) {
+      mbar_init(AGNES_DFULL(d), 1);
+      mbar_init(AGNES_DEMPTY(d), 4);  // one arrival per epilogue warp
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   // W into its K-major layout: 16-byte chunk (n, kc) = W[n][8 kc .. 8 kc + 7]
   const int kchunks = KT / 8;
-  for (int q = tid; q < N * kchunks; q += kSageThreads) {
+  for (int q = tid; q < N * kchunks; q += kGemmThreads) {
     const int n = q / kchunks, kc = q - n * kchunks;
     *(uint4*)(sW + kmajor_off(n, kc * 8, N)) = __ldg((const uint4*)(a.w + (size_t)n * KT) + kc);
   }
@@ -202,175 +345,112 @@ __global__ void __launch_bounds__(kSageThreads, 1) sage_mean_kernel(SageArgs a) 
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
-  const uint32_t idesc = idesc_f16(kM, N);
-  const uint32_t a_addr = smem_u32(sA), w_addr = smem_u32(sW);
   const int total_tiles = __ldg(a.tile_start + a.H);
-  const int chunks = a.d_in / 8;  // 16-byte fp16 chunks per half of A's row
-  uint32_t phase = 0;
   bool ok = true;
 
-  for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
-    int lo = 0, hi = a.H;  // minibatch of this tile: last j with tile_start[j] <= tile
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (__ldg(a.tile_start + mid) <= tile) lo = mid; else hi = mid;
-    }
-    const int j = lo;
-    const int row0 = (tile - __ldg(a.tile_start + j)) * kM;
-    const int nd = __ldg(a.num_dst + j);
-    const T* x = (const T*)a.x + (size_t)j * a.x_stride * a.d_in;
-    const int64_t* ip = a.indptr + (size_t)j * a.indptr_stride;
-    const int32_t* cl = a.col + (size_t)j * a.col_stride;
-
-    // stage the tile's indptr (rows past nd get empty ranges) and, when they
-    // fit, its edges' columns in shared memory with coalesced loads, so the
-    // row loads below do not wait on an indptr -> col chain per item
-    const int rows = nd - row0 < kM ? nd - row0 : kM;
-    if (tid <= kM) s_ip[tid] = __ldg(ip + row0 + (tid < rows ? tid : rows));
-    __syncthreads();
-    const int64_t eb = s_ip[0], ne_t = s_ip[kM] - eb;
-    const bool staged = ne_t <= kColCap;
-    if (staged)
-      for (int64_t e = tid; e < ne_t; e += kSageThreads) s_col[e] = __ldg(cl + eb + e);
-    __syncthreads();
-    // aggregation: item (r, c) = row r's 8-feature chunk c; two items per
-    // thread at a time, kER edges of each in flight per round
-    constexpr int kER = sizeof(T) == 2 ? 8 : 4;
-    for (int q0 = tid; q0 < kM * chunks; q0 += 2 * kSageThreads) {
-      int r[2], c[2];
-      int64_t e0[2], e1[2];
-      uint4 self[2];
-      float acc[2][8];
-      int64_t span = 0;
-#pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int q = q0 + k * kSageThreads;
-        r[k] = q / chunks;
-        c[k] = q - r[k] * chunks;
-        self[k] = make_uint4(0, 0, 0, 0);
-        e0[k] = e1[k] = 0;
-        if (q < kM * chunks && r[k] < rows) {
-          self[k] = load8_h<T>(x + (size_t)(row0 + r[k]) * a.d_in, c[k]);
-          e0[k] = s_ip[r[k]] - eb;
-          e1[k] = s_ip[r[k] + 1] - eb;
+  if (warp == 0) {
+    // producer: A tile k of this CTA into stage k % S
+    if (lane == 0) {
+      int k = 0;
+      for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x, ++k) {
+        const int s = k % S;
+        if (k >= S && !mbar_wait(AGNES_EMPTY(s), (uint32_t)((k / S - 1) & 1))) {
+          ok = false;
+          break;
         }
-        span = e1[k] - e0[k] > span ? e1[k] - e0[k] : span;
-#pragma unroll
-        for (int f = 0; f < 8; ++f) acc[k][f] = 0.f;
-      }
-      for (int64_t base = 0; base < span; base += kER) {
-        // indices first, then every row load, then the sums: the loads of a
-        // round are independent and all in flight together
-        int32_t idx[2][kER];
-#pragma unroll
-        for (int k = 0; k < 2; ++k)
-#pragma unroll
-          for (int u = 0; u < kER; ++u) {
-            const int64_t e = e0[k] + base + u;
-            idx[k][u] = e < e1[k] ? (staged ? s_col[e] : __ldg(cl + eb + e)) : -1;
-          }
-        Chunk<T> val[2][kER];
-#pragma unroll
-        for (int k = 0; k < 2; ++k)
-#pragma unroll
-          for (int u = 0; u < kER; ++u) {
-            if (idx[k][u] >= 0) {
-              val[k][u] = load_chunk<T>(x + (size_t)idx[k][u] * a.d_in, c[k]);
-            } else {
-#pragma unroll
-              for (int q = 0; q < (int)(sizeof(T) / 2); ++q) val[k][u].v[q] = make_uint4(0, 0, 0, 0);
-            }
-          }
-#pragma unroll
-        for (int k = 0; k < 2; ++k)
-#pragma unroll
-          for (int u = 0; u < kER; ++u) add_chunk(val[k][u], acc[k]);
-      }
-#pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        if (q0 + k * kSageThreads >= kM * chunks) continue;
-        uint4 mean = make_uint4(0, 0, 0, 0);
-        if (e1[k] > e0[k]) {
-          const float deg = (float)(e1[k] - e0[k]);
-          __half2 h;
-          h = __floats2half2_rn(acc[k][0] / deg, acc[k][1] / deg); mean.x = *(uint32_t*)&h;
-          h = __floats2half2_rn(acc[k][2] / deg, acc[k][3] / deg); mean.y = *(uint32_t*)&h;
-          h = __floats2half2_rn(acc[k][4] / deg, acc[k][5] / deg); mean.z = *(uint32_t*)&h;
-          h = __floats2half2_rn(acc[k][6] / deg, acc[k][7] / deg); mean.w = *(uint32_t*)&h;
-        }
-        *(uint4*)(sA + kmajor_off(r[k], c[k] * 8, kM)) = self[k];
-        *(uint4*)(sA + kmajor_off(r[k], a.d_in + c[k] * 8, kM)) = mean;
+        mbar_arrive_tx(AGNES_FULL(s), tile_bytes);
+        bulk_g2s(smem_u32(sA + (size_t)s * tile_bytes), a.A + (size_t)tile * tile_bytes,
+                 tile_bytes, AGNES_FULL(s));
       }
     }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
-    if (tid == 0) {
+  } else if (warp == 1) {
+    // MMA issuer: tile k from stage k % S into accumulator k % 2
+    if (lane == 0) {
+      const uint32_t idesc = idesc_f16(kM, N);
+      const uint32_t w_addr = smem_u32(sW);
+      int k = 0;
+      for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x, ++k) {
+        const int s = k % S, d = k & 1;
+        if (!mbar_wait(AGNES_FULL(s), (uint32_t)((k / S) & 1)) ||
+            (k >= 2 && !mbar_wait(AGNES_DEMPTY(d), (uint32_t)((k / 2 - 1) & 1)))) {
+          ok = false;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t a_addr = smem_u32(sA + (size_t)s * tile_bytes);
+        const uint32_t dcol = tmem + (uint32_t)(d * N);
+        // K step t covers K columns [16 t, 16 t + 16): core-matrix columns 2t, 2t+1
+        for (int t = 0; t < KT / 16; ++t) {
+          const uint64_t da = smem_desc(a_addr + (uint32_t)(2 * t) * (kM / 8) * 128,
+                                        (kM / 8) * 128, 128);
+          const uint64_t dw = smem_desc(w_addr + (uint32_t)(2 * t) * (uint32_t)(N / 8) * 128,
+                                        (uint32_t)(N / 8) * 128, 128);
+          mma_f16(dcol, da, dw, idesc, t > 0 ? 1u : 0u);
+        }
+        mma_commit(AGNES_EMPTY(s));  // the stage is free once these MMAs have read it
+        mma_commit(AGNES_DFULL(d));  // and the accumulator is complete
+      }
+    }
+  } else if (warp >= 4) {
+    // epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 (its rows)
+    const int quad = warp & 3;
+    int k = 0;
+    for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x, ++k) {
+      const int d = k & 1;
+      if (!mbar_wait(AGNES_DFULL(d), (uint32_t)((k / 2) & 1))) {
+        ok = false;
+        break;
+      }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      // K step s covers K columns [16 s, 16 s + 16): core-matrix columns 2s, 2s+1
-      for (int s = 0; s < KT / 16; ++s) {
-        const uint64_t da = smem_desc(a_addr + (uint32_t)(2 * s) * (kM / 8) * 128,
-                                      (kM / 8) * 128, 128);
-        const uint64_t dw = smem_desc(w_addr + (uint32_t)(2 * s) * (uint32_t)(N / 8) * 128,
-                                      (uint32_t)(N / 8) * 128, 128);
-        mma_f16(tmem, da, dw, idesc, s > 0 ? 1u : 0u);
-      }
-      asm volatile(
-          "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-              smem_u32(bar))
-          : "memory");
-    }
-    const bool done = mbar_wait(smem_u32(bar), phase);
-    phase ^= 1u;
-    if (__syncthreads_or(!done)) {
-      ok = false;
-      break;
-    }
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    // epilogue: warp w reads lanes 32 (w % 4) .. +31 (its rows) and the
-    // column quarter w / 4, eight columns per tcgen05.ld
-    {
-      const int quad = warp & 3, part = warp >> 2;
-      const int r = quad * 32 + lane;
-      const int i = row0 + r;
-      const int cols = N / 4;
+      const int j = __ldg(a.tile_mb + tile);
+      const int i = (tile - __ldg(a.tile_start + j)) * kM + quad * 32 + lane;
+      const bool valid = i < __ldg(a.num_dst + j);
       OutT* orow = (OutT*)a.out + ((size_t)j * a.out_stride + i) * N;
-      for (int c0 = part * cols; c0 < (part + 1) * cols; c0 += 8) {
-        uint32_t v[8];
-        const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)c0;
+      for (int c0 = 0; c0 < N; c0 += 32) {  // 32 columns per tcgen05.ld, one wait
+        uint32_t v[32];
+        const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(d * N + c0);
         asm volatile(
-            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+            "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, "
+            "%10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, "
+            "%26, %27, %28, %29, %30, %31}, [%32];"
             : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]),
-              "=r"(v[6]), "=r"(v[7])
+              "=r"(v[6]), "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]),
+              "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]),
+              "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+              "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]),
+              "=r"(v[30]), "=r"(v[31])
             : "r"(taddr)
             : "memory");
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-        if (i < nd) {
-          float f[8];
+        if (valid) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            f[q] = __uint_as_float(v[q]) + (a.bias ? __ldg(a.bias + c0 + q) : 0.f);
-            f[q] = f[q] > 0.f ? f[q] : 0.f;
-          }
-          if constexpr (sizeof(OutT) == 4) {
-            ((float4*)(orow + c0))[0] = make_float4(f[0], f[1], f[2], f[3]);
-            ((float4*)(orow + c0))[1] = make_float4(f[4], f[5], f[6], f[7]);
-          } else {
-            uint4 o;
-            __half2 h;
-            h = __floats2half2_rn(f[0], f[1]); o.x = *(uint32_t*)&h;
-            h = __floats2half2_rn(f[2], f[3]); o.y = *(uint32_t*)&h;
-            h = __floats2half2_rn(f[4], f[5]); o.z = *(uint32_t*)&h;
-            h = __floats2half2_rn(f[6], f[7]); o.w = *(uint32_t*)&h;
-            *(uint4*)(orow + c0) = o;
+          for (int g = 0; g < 4; ++g) {
+            float f[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const int cc = c0 + 8 * g + q;
+              f[q] = __uint_as_float(v[8 * g + q]) + (a.bias ? __ldg(a.bias + cc) : 0.f);
+              f[q] = f[q] > 0.f ? f[q] : 0.f;
+            }
+            if constexpr (sizeof(OutT) == 4) {
+              ((float4*)(orow + c0 + 8 * g))[0] = make_float4(f[0], f[1], f[2], f[3]);
+              ((float4*)(orow + c0 + 8 * g))[1] = make_float4(f[4], f[5], f[6], f[7]);
+            } else {
+              *(uint4*)(orow + c0 + 8 * g) = to_half8(f);
+            }
           }
         }
       }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(AGNES_DEMPTY(d));
     }
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
   }
-  if (!ok && tid == 0) atomicOr(a.err, kSageTimeout);
+#undef AGNES_FULL
+#undef AGNES_EMPTY
+#undef AGNES_DFULL
+#undef AGNES_DEMPTY
+  if (!ok) atomicOr(a.err, kSageTimeout);
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 0) {
@@ -380,8 +460,9 @@ __global__ void __launch_bounds__(kSageThreads, 1) sage_mean_kernel(SageArgs a) 
   }
 }
 
-size_t sage_smem_bytes(int64_t d_in, int64_t d_out) {
-  return (size_t)kM * 2 * d_in * 2 + (size_t)d_out * 2 * d_in * 2 + kStageBytes;
+// Shared memory of the GEMM kernel with `stages` A stages.
+size_t gemm_smem_bytes(int64_t d_in, int64_t d_out, int stages) {
+  return (size_t)d_out * 2 * d_in * 2 + (size_t)stages * kM * 2 * d_in * 2 + kBarBytes;
 }
 
 bool is_device_ptr(const void* p) {
@@ -393,19 +474,21 @@ bool is_device_ptr(const void* p) {
   return attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged;
 }
 
-static_assert(kStageBytes == 17440, "the header's shared-memory formula");
-
-// Every CTA asks for at least this much shared memory, so no two CTAs share
-// an SM (and its 512 tensor-memory columns).
-constexpr size_t kSageMinSmem = 120 * 1024;
-
 template <typename T, typename OutT>
-cudaError_t launch_sage(const SageArgs& a, int grid, size_t smem, cudaStream_t st) {
+cudaError_t launch_sage(const SageArgs& a, int64_t tiles, int num_sms, cudaStream_t st) {
+  const int64_t rows = tiles * kM;
+  const int64_t items = rows * (a.d_in / 8);
+  int64_t agg_grid = resident_grid((const void*)sage_agg_kernel<T>, kAggThreads, num_sms);
+  const int64_t per_cta = (int64_t)kAggThreads * kAggU;
+  if (agg_grid * per_cta > items) agg_grid = (items + per_cta - 1) / per_cta;
+  sage_agg_kernel<T><<<(unsigned)agg_grid, kAggThreads, 0, st>>>(a, rows);
+  size_t smem = gemm_smem_bytes(a.d_in, a.d_out, a.stages);
   if (smem < kSageMinSmem) smem = kSageMinSmem;
-  cudaError_t e = cudaFuncSetAttribute(sage_mean_kernel<T, OutT>,
+  cudaError_t e = cudaFuncSetAttribute(sage_gemm_kernel<OutT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  sage_mean_kernel<T, OutT><<<grid, kSageThreads, smem, st>>>(a);
+  const int grid = (int)(tiles < num_sms ? tiles : num_sms);
+  sage_gemm_kernel<OutT><<<grid, kGemmThreads, smem, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -441,10 +524,11 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
                        "[32, 256]");
     return AGNES_EINVAL;
   }
-  const size_t smem = sage_smem_bytes(d_in, d_out);
-  if (smem > AGNES_SAGE_MAX_SMEM) {
+  int stages = 2;
+  if (gemm_smem_bytes(d_in, d_out, stages) > AGNES_SAGE_MAX_SMEM) stages = 1;
+  if (gemm_smem_bytes(d_in, d_out, stages) > AGNES_SAGE_MAX_SMEM) {
     ctx_set_error(ctx, "d_in %lld with d_out %d needs %zu bytes of shared memory (limit %d)",
-                  (long long)d_in, d_out, smem, AGNES_SAGE_MAX_SMEM);
+                  (long long)d_in, d_out, gemm_smem_bytes(d_in, d_out, 1), AGNES_SAGE_MAX_SMEM);
     return AGNES_ERANGE;
   }
   if (((uintptr_t)x | (uintptr_t)w | (uintptr_t)out) % 16 != 0 ||
@@ -454,8 +538,11 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
   }
   const int H = v.H;
   int64_t max_src = 0, max_dst = 0;
-  // pinned staging: error word (16 bytes), then tile_start (H + 1), num_dst (H)
-  const size_t tab_bytes = sizeof(int32_t) * ((size_t)2 * H + 1);
+  // pinned staging: error word (16 bytes), then tile_start (H + 1), num_dst
+  // (H), tile_mb (one per tile)
+  int64_t tiles = 0;
+  for (int j = 0; j < H; ++j) tiles += ((int64_t)v.node_size[(size_t)hop * H + j] + kM - 1) / kM;
+  const size_t tab_bytes = sizeof(int32_t) * ((size_t)2 * H + 1 + (size_t)tiles);
   void* hp = nullptr;
   cudaError_t e = ctx_pinned(ctx, 16 + tab_bytes, &hp);
   if (e != cudaSuccess) {
@@ -464,7 +551,7 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
   }
   int32_t* h_err = (int32_t*)hp;
   int32_t* tabs = (int32_t*)((char*)hp + 16);
-  int64_t tiles = 0;
+  tiles = 0;
   for (int j = 0; j < H; ++j) {
     const int64_t nd = v.node_size[(size_t)hop * H + j];
     const int64_t ns = v.src_size[(size_t)hop * H + j];
@@ -472,6 +559,7 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
     max_src = ns > max_src ? ns : max_src;
     tabs[j] = (int32_t)tiles;
     tabs[H + 1 + j] = (int32_t)nd;
+    for (int64_t t = tiles; t < tiles + (nd + kM - 1) / kM; ++t) tabs[2 * H + 1 + t] = j;
     tiles += (nd + kM - 1) / kM;
   }
   tabs[H] = (int32_t)tiles;
@@ -488,8 +576,11 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
   GraphView g;
   ctx_graph_view(ctx, &g);
   cudaStream_t st = (cudaStream_t)cuda_stream;
+  // device scratch: error word and tables, then (256-byte aligned) the A tiles
+  const size_t a_off = (16 + tab_bytes + 255) & ~(size_t)255;
+  const size_t a_bytes = (size_t)tiles * kM * 2 * (size_t)d_in * 2;
   void* scratch = nullptr;
-  e = ctx_scratch(ctx, 16 + tab_bytes, &scratch);
+  e = ctx_scratch(ctx, a_off + a_bytes, &scratch);
   int32_t* err = (int32_t*)scratch;
   int32_t* d_tabs = (int32_t*)((char*)scratch + 16);
   if (e == cudaSuccess) e = cudaMemsetAsync(err, 0, sizeof(int32_t), st);
@@ -504,21 +595,23 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
     a.col_stride = v.col_stride[hop];
     a.tile_start = d_tabs;
     a.num_dst = d_tabs + H + 1;
+    a.tile_mb = d_tabs + 2 * H + 1;
     a.H = H;
     a.d_in = (int32_t)d_in;
     a.d_out = d_out;
+    a.A = (uint8_t*)scratch + a_off;
     a.w = (const __half*)w;
     a.bias = bias;
     a.out = out;
     a.out_stride = out_stride_rows;
+    a.stages = stages;
     a.err = err;
-    const int grid = (int)(tiles < g.num_sms ? tiles : g.num_sms);
     if (x_dtype == AGNES_F16)
-      e = out_dtype == AGNES_F32 ? launch_sage<__half, float>(a, grid, smem, st)
-                                 : launch_sage<__half, __half>(a, grid, smem, st);
+      e = out_dtype == AGNES_F32 ? launch_sage<__half, float>(a, tiles, g.num_sms, st)
+                                 : launch_sage<__half, __half>(a, tiles, g.num_sms, st);
     else
-      e = out_dtype == AGNES_F32 ? launch_sage<float, float>(a, grid, smem, st)
-                                 : launch_sage<float, __half>(a, grid, smem, st);
+      e = out_dtype == AGNES_F32 ? launch_sage<float, float>(a, tiles, g.num_sms, st)
+                                 : launch_sage<float, __half>(a, tiles, g.num_sms, st);
   }
   *h_err = 0;
   if (e == cudaSuccess)
@@ -529,7 +622,7 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
     return e == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;
   }
   if (*h_err & kSageTimeout) {
-    ctx_set_error(ctx, "agnes_sage_mean_layer: the tensor-core wait ran out");
+    ctx_set_error(ctx, "agnes_sage_mean_layer: a tensor-core or copy wait ran out");
     return AGNES_ETIMEOUT;
   }
   return AGNES_OK;
