@@ -69,6 +69,10 @@ WORKLOADS = {
     # (~6 entries) with ~4 GB on the device
     "prof5m": Workload("prof5m", 5_000_000, 16, 0.57, 0.19, 0.19, "int64", "float16", 128,
                        MB, MB, 128, 64, (15, 10, 5), 0.05, 3),
+    # profiling stand-in for the dedup kernels: rmat100m's hop-3 cell density (~5 entries per
+    # (tile, minibatch) cell) over 1.5M cells, 16-wide features, a few GB on the device
+    "prof_cells": Workload("prof_cells", 10_000_000, 16, 0.57, 0.19, 0.19, "int64", "float16", 16,
+                           MB, MB, 512, 100, (15, 10, 5), 0.05, 4),
     "mini_skew": Workload("mini_skew", 1_000_000, 28, 0.6, 0.2, 0.15, "int64", "float16", 256,
                           MB, MB, 8, 1024, (25, 10), None, 2),
 }
