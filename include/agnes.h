@@ -121,9 +121,12 @@ typedef struct {
  * BLOCKS: every touched feature block is loaded whole into HBM, batch by
  *   batch, overlapped with the gather (the block-wise I/O of Sec. 3.3 and the
  *   asynchronous I/O of Sec. 3.4 (4)); 0, the default.
- * ROWS: the gather reads each requested row in place from pinned host memory
- *   over the host link (or from the feature cache), so only requested rows
- *   cross the link.  Not in the paper: its storage is an SSD, where small
+ * ROWS: only requested rows cross the host link, read in place from pinned
+ *   host memory by the GPU.  Without a feature cache, each distinct requested
+ *   row of the hyperbatch crosses once into an HBM staging area that serves
+ *   every request; with a cache, every row is read where its block is (cache
+ *   slot or host memory), since the rows several minibatches request are
+ *   then mostly in the cache.  Not in the paper: its storage is an SSD, where small
  *   reads are slow; a cache-coherent host link serves row-sized reads at the
  *   rate of bulk copies. */
 #define AGNES_FEATURE_IO_BLOCKS 0
@@ -247,7 +250,9 @@ typedef struct {
   int64_t distinct_rows;            /* distinct node ids among all gathered rows */
   int64_t row_bytes;
   int64_t streamed_bytes;           /* features_on_host: bytes read over the host link
-                                       (row mode: requested rows, before L2 reuse) */
+                                       (row mode: distinct rows without a cache, every
+                                       request of an uncached block with one; plus
+                                       blocks loaded into the cache) */
   int64_t streamed_blocks;          /* features_on_host: touched feature blocks not
                                        served by the feature cache */
   /* the rest are totals since agnes_load_graph, not per hyperbatch */

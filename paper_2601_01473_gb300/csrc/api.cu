@@ -137,6 +137,17 @@ struct agnes_ctx {
   unsigned long long* d_job_dst = nullptr;
   unsigned long long* h_addr = nullptr;  // row mode: current address of every feature block
   unsigned long long* d_addr = nullptr;
+  // row mode: requested-id bitmaps per tile, their word prefixes and counts,
+  // the scan of the counts, the staging rows, and the rows read from host
+  uint32_t* rm_bitmap = nullptr;
+  uint16_t* rm_wpref = nullptr;
+  int32_t* rm_dcnt = nullptr;
+  int32_t* rm_doff = nullptr;
+  char* rm_staging = nullptr;
+  int64_t rm_staging_rows = 0;
+  unsigned long long* d_host_rows = nullptr;
+  int64_t* h_rm = nullptr;  // pinned: [0] distinct rows, [1] rows read from host memory
+  int64_t cache_load_bytes = 0;
   cudaEvent_t gather_start = nullptr;
   // feature cache C_f (Sec. 3.4 (2)): blocks whose cumulative request count
   // reaches the threshold, hottest first, up to fcache_slots blocks
@@ -522,6 +533,13 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   cudaFree(ctx->d_job_blk);
   cudaFree(ctx->d_job_dst);
   cudaFree(ctx->d_addr);
+  cudaFree(ctx->rm_bitmap);
+  cudaFree(ctx->rm_wpref);
+  cudaFree(ctx->rm_dcnt);
+  cudaFree(ctx->rm_doff);
+  cudaFree(ctx->rm_staging);
+  cudaFree(ctx->d_host_rows);
+  if (ctx->h_rm) cudaFreeHost(ctx->h_rm);
   cudaFree(ctx->fcache);
   if (ctx->gather_start) cudaEventDestroy(ctx->gather_start);
   if (ctx->h_counts) cudaFreeHost(ctx->h_counts);
@@ -583,6 +601,15 @@ static agnes_status setup_streaming(agnes_ctx* ctx, const agnes_graph_desc* d, c
   if (ctx->feature_io == AGNES_FEATURE_IO_BLOCKS) {
     ctx->slot_bytes = (int64_t)kStreamBatchBlocks * blk;
     CK(ctx, cudaMalloc((void**)&ctx->slots, (size_t)(ctx->slot_bytes * kStreamSlots)));
+  } else {
+    const size_t T = (size_t)ctx->bt.T;
+    CK(ctx, cudaMalloc((void**)&ctx->rm_bitmap, sizeof(uint32_t) * T * kTileWords));
+    CK(ctx, cudaMalloc((void**)&ctx->rm_wpref, sizeof(uint16_t) * T * kTileWords));
+    CK(ctx, cudaMalloc((void**)&ctx->rm_dcnt, sizeof(int32_t) * T));
+    CK(ctx, cudaMalloc((void**)&ctx->rm_doff, sizeof(int32_t) * (T + 1)));
+    CK(ctx, cudaMalloc((void**)&ctx->d_host_rows, sizeof(unsigned long long)));
+    CK(ctx, cudaMallocHost((void**)&ctx->h_rm, sizeof(int64_t) * 2));
+    ctx->h_rm[0] = ctx->h_rm[1] = 0;
   }
   const size_t n1 = (size_t)(nfb + 1);
   CK(ctx, cudaMalloc((void**)&ctx->d_touched, sizeof(int32_t) * n1));
@@ -1048,12 +1075,16 @@ static agnes_status gather_blocks_io(agnes_ctx* ctx, int cur, int32_t n, int64_t
   return AGNES_OK;
 }
 
-// Row mode: each gathered row is read where its block is -- in place from
-// pinned host memory over the host link (only the requested rows cross it),
-// or from the block's feature-cache slot.  Touched blocks admitted to the
-// cache but not yet loaded are loaded whole first (by the loader kernel, on
-// the caller's stream), then one gather walks the whole final bucket through
-// the per-block address table.
+// Row mode: only the requested rows cross the host link.  Touched blocks
+// admitted to the cache but not yet loaded are loaded whole first.
+//  - Without a feature cache, each distinct requested row crosses once: the
+//    tiles' bitmaps of requested ids give every distinct row a staging row in
+//    HBM, a loader reads them over the link, and the gather serves every
+//    request from staging.
+//  - With a feature cache the hot rows, the ones several minibatches request,
+//    sit in HBM, and the link carries mostly rows requested once; the gather
+//    then reads every row where its block is (cache slot or host memory),
+//    so the cached reads overlap the host reads in one pass.
 static agnes_status gather_rows_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* bytes_out,
                                    int64_t* hits_out, cudaStream_t st) {
   Workspace& w = ctx->ws;
@@ -1061,13 +1092,16 @@ static agnes_status gather_rows_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* 
   const int64_t rpb = ctx->bt.rows_per_feat_block;
   const int64_t rb = ctx->row_bytes;
   const int64_t blk = rpb * rb;
+  const int32_t T = (int32_t)ctx->bt.T;
+  const int64_t cells = (int64_t)T * w.H;
+  const bool dedup = ctx->fcache_slots == 0;
   int32_t nj = 0;
-  int64_t bytes = 0, hits = 0;
+  int64_t bytes = 0, hits = 0, requested_host = 0;
   for (int32_t i = 0; i < n; ++i) {
     const int32_t b = ctx->h_touched[i];
     const int32_t cs = ctx->fcache_slots ? ctx->cslot_of[(size_t)b] : -1;
     if (cs < 0) {
-      bytes += (int64_t)ctx->h_counts[b] * rb;
+      requested_host += ctx->h_counts[b];
     } else if (ctx->cresident[(size_t)cs]) {
       hits += 1;
     } else {
@@ -1095,10 +1129,45 @@ static agnes_status gather_rows_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* 
     CK(ctx, launch_load_feat_blocks(ctx->features_dev, ctx->N * rb, ctx->d_job_blk, ctx->d_job_dst,
                                     nj, blk, ctx->num_sms, st));
   }
-  const int64_t cells = (int64_t)ctx->bt.T * w.H;
-  CK(ctx, launch_gather_table(ctx->d_addr, rb, rpb, w.fb_id[cur], w.fb_pos[cur],
-                              w.fcell_off[cur] + cells, w.feats_out, w.status, ctx->num_sms, st));
-  *bytes_out = bytes;
+  ctx->cache_load_bytes = bytes;
+  if (!dedup) {
+    CK(ctx, launch_gather_table(ctx->d_addr, rb, rpb, w.fb_id[cur], w.fb_pos[cur],
+                                w.fcell_off[cur] + cells, w.feats_out, w.status, ctx->num_sms, st));
+    ctx->h_rm[1] = requested_host;  // every request of an uncached block crosses the link
+    *bytes_out = bytes + requested_host * rb;
+    *hits_out = hits;
+    return AGNES_OK;
+  }
+  // distinct requested rows per tile, and their total (for the staging size)
+  CK(ctx, launch_tile_bitmaps(w.fb_id[cur], w.fcell_off[cur], ctx->bt.tile_first, T, w.H,
+                              ctx->rm_bitmap, ctx->rm_wpref, ctx->rm_dcnt, w.status, st));
+  CK(ctx, (seg_scan<int32_t, int32_t>(ctx->rm_dcnt, 0, ctx->rm_doff, 0, nullptr, T, 1, T, true,
+                                      nullptr, w.scan_scratch, w.status, st)));
+  int32_t* h_total = (int32_t*)ctx->h_rm;
+  CK(ctx, cudaMemcpyAsync(h_total, ctx->rm_doff + T, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
+  const int64_t distinct = *h_total;
+  if (distinct > ctx->rm_staging_rows) {
+    cudaFree(ctx->rm_staging);
+    ctx->rm_staging = nullptr;
+    ctx->rm_staging_rows = 0;
+    const int64_t rows = distinct + distinct / 8 + 1024;
+    CK(ctx, cudaMalloc((void**)&ctx->rm_staging, (size_t)(rows * rb)));
+    ctx->rm_staging_rows = rows;
+  }
+  CK(ctx, cudaMemsetAsync(ctx->d_host_rows, 0, sizeof(unsigned long long), st));
+  CK(ctx, launch_load_distinct_rows(ctx->d_addr, rb, rpb, ctx->rm_bitmap, ctx->rm_wpref,
+                                    ctx->rm_doff, T, ctx->bt.tile_first, ctx->rm_staging, 0, 0,
+                                    ctx->d_host_rows, w.status, ctx->num_sms, st));
+  CK(ctx, launch_gather_staged_rows(ctx->rm_staging, rb, w.fb_id[cur], w.fb_pos[cur],
+                                    w.fcell_off[cur] + cells, ctx->bt.tile_first,
+                                    ctx->bt.chunk_tile, T, ctx->rm_bitmap, ctx->rm_wpref,
+                                    ctx->rm_doff, ctx->d_addr, rpb, 0, 0, 0, 0, w.feats_out,
+                                    w.status, ctx->num_sms, st));
+  // rows read over the link, for the counters (read after the hyperbatch is done)
+  CK(ctx, cudaMemcpyAsync(ctx->h_rm + 1, ctx->d_host_rows, sizeof(int64_t),
+                          cudaMemcpyDeviceToHost, st));
+  *bytes_out = bytes + distinct * rb;
   *hits_out = hits;
   return AGNES_OK;
 }
@@ -1466,7 +1535,10 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
                                (int32_t)ctx->bt.T, w.H, w.distinct, nullptr));
   CK(ctx, cudaMemcpy(&distinct, w.distinct, sizeof(distinct), cudaMemcpyDeviceToHost));
   out->distinct_rows = (int64_t)distinct;
-  out->streamed_bytes = ctx->features_on_host ? ctx->streamed_bytes : 0;
+  out->streamed_bytes = !ctx->features_on_host ? 0
+                        : ctx->feature_io == AGNES_FEATURE_IO_ROWS
+                            ? ctx->cache_load_bytes + ctx->h_rm[1] * ctx->row_bytes
+                            : ctx->streamed_bytes;
   out->streamed_blocks = ctx->features_on_host ? ctx->streamed_blocks : 0;
   out->topo_loaded_blocks = ctx->topo.loaded_blocks;
   out->topo_loaded_bytes = ctx->topo.loaded_bytes;

@@ -281,6 +281,196 @@ distinct_rows_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restric
   }
 }
 
+// Row mode, de-duplicated: each distinct row of the hyperbatch crosses the
+// host link once.  tile_bitmap_kernel (one warp per tile) records which ids
+// of the tile any minibatch requests (bits), the exclusive prefix of set bits
+// per 32-id word (wpref) and the count (dcnt); after a scan of dcnt into doff,
+// load_distinct_rows_kernel copies distinct row d of tile t to staging row
+// doff[t] + d, and gather_staged_rows_kernel serves every request from there.
+__global__ void __launch_bounds__(kThreads)
+tile_bitmap_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict__ cell_off,
+                   const int32_t* __restrict__ tile_first, int32_t T, int32_t H,
+                   uint32_t* __restrict__ bitmap, uint16_t* __restrict__ wpref,
+                   int32_t* __restrict__ dcnt, const int32_t* status) {
+  if (failed(status)) return;
+  __shared__ uint32_t bits_s[kWarps][kTileWords];
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  uint32_t* bits = bits_s[warp];
+  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+  for (int64_t t = blockIdx.x * (int64_t)kWarps + warp; t < T; t += nwarps) {
+    const int32_t base = tile_first[t];
+    for (int w = lane; w < kTileWords; w += 32) bits[w] = 0;
+    __syncwarp();
+    const int32_t o = cell_off[t * H], e = cell_off[(t + 1) * H];
+    for (int32_t i = o + lane; i < e; i += 32) {
+      const int32_t lu = fb_id[i] - base;
+      atomicOr(&bits[lu >> 5], 1u << (lu & 31));
+    }
+    __syncwarp();
+    // lane l owns words 4l .. 4l+3
+    uint32_t wv[4];
+    int cnt = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      wv[q] = bits[lane * 4 + q];
+      cnt += __popc(wv[q]);
+    }
+    int run = warp_incl_scan(cnt) - cnt;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      bitmap[t * kTileWords + lane * 4 + q] = wv[q];
+      wpref[t * kTileWords + lane * 4 + q] = (uint16_t)run;
+      run += __popc(wv[q]);
+    }
+    if (lane == 31) dcnt[t] = run;
+    __syncwarp();
+  }
+}
+
+// Rank of id (in tile t, base = tile_first[t]) among the tile's requested ids.
+__device__ __forceinline__ int32_t tile_rank(const uint32_t* __restrict__ bitmap,
+                                             const uint16_t* __restrict__ wpref, int64_t t,
+                                             int32_t lu) {
+  const int64_t w = t * kTileWords + (lu >> 5);
+  return (int32_t)__ldg(wpref + w) + __popc(__ldg(bitmap + w) & ((1u << (lu & 31)) - 1u));
+}
+
+// Distinct row d (of doff[T]): tile t = last with doff[t] <= d; the row is
+// the (d - doff[t])-th requested id of the tile, copied from its feature
+// block's address in host memory (over the link; counted in *host_rows) to
+// staging row d.  Rows of blocks in the feature cache, [cache_lo, cache_hi),
+// are not staged: the gather reads them in place.  LPR lanes per row.
+template <int LPR>
+__global__ void __launch_bounds__(kThreads)
+load_distinct_rows_kernel(const unsigned long long* __restrict__ addr, int64_t vecs, int32_t rpb,
+                          const uint32_t* __restrict__ bitmap, const uint16_t* __restrict__ wpref,
+                          const int32_t* __restrict__ doff, int32_t T,
+                          const int32_t* __restrict__ tile_first, uint4* __restrict__ staging,
+                          unsigned long long cache_lo, unsigned long long cache_hi,
+                          unsigned long long* host_rows, const int32_t* status) {
+  if (failed(status)) return;
+  constexpr int kRowsPerWarp = 32 / LPR;
+  const int64_t total = __ldg(doff + T);
+  const int lane = lane_id();
+  const int sub = lane / LPR, l = lane % LPR;
+  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  uint32_t from_host = 0;
+  for (int64_t d = warp0 * kRowsPerWarp + sub; d < total; d += nwarps * kRowsPerWarp) {
+    int32_t lo = 0, hi = T;  // tile: last t with doff[t] <= d
+    while (hi - lo > 1) {
+      const int32_t mid = (lo + hi) >> 1;
+      if (__ldg(doff + mid) <= d) lo = mid; else hi = mid;
+    }
+    const int32_t t = lo, r = (int32_t)(d - __ldg(doff + t));
+    int32_t wl = 0, wh = kTileWords;  // word: last w with wpref[w] <= r
+    while (wh - wl > 1) {
+      const int32_t mid = (wl + wh) >> 1;
+      if ((int32_t)__ldg(wpref + (int64_t)t * kTileWords + mid) <= r) wl = mid; else wh = mid;
+    }
+    const uint32_t bits = __ldg(bitmap + (int64_t)t * kTileWords + wl);
+    const int32_t k = r - (int32_t)__ldg(wpref + (int64_t)t * kTileWords + wl);
+    const int32_t id = __ldg(tile_first + t) + wl * 32 + (int32_t)__fns(bits, 0, k + 1);
+    const int32_t b = id / rpb;
+    const unsigned long long a = __ldg(addr + b);
+    if (a >= cache_lo && a < cache_hi) continue;
+    const uint4* src = (const uint4*)a + (int64_t)(id - b * rpb) * vecs;
+    for (int64_t c = l; c < vecs; c += LPR) staging[d * vecs + c] = src[c];
+    if (l == 0) ++from_host;
+  }
+  from_host = warp_sum(from_host);
+  if (lane == 0 && from_host) atomicAdd(host_rows, (unsigned long long)from_host);
+}
+
+// Source of row id: in place in the feature cache when its block is there,
+// else its staging row.
+__device__ __forceinline__ const uint4* staged_row_src(
+    const uint4* __restrict__ staging, int64_t vecs, const unsigned long long* __restrict__ addr,
+    int32_t rpb, unsigned long long cache_lo, unsigned long long cache_hi, TileMap tm,
+    const uint32_t* __restrict__ bitmap, const uint16_t* __restrict__ wpref,
+    const int32_t* __restrict__ doff, int32_t id) {
+  const int32_t b = id / rpb;
+  const unsigned long long a = __ldg(addr + b);
+  if (a >= cache_lo && a < cache_hi) return (const uint4*)a + (int64_t)(id - b * rpb) * vecs;
+  const int32_t t = tile_of(tm, id);
+  const int64_t srow =
+      (int64_t)__ldg(doff + t) + tile_rank(bitmap, wpref, t, id - __ldg(tm.tile_first + t));
+  return staging + srow * vecs;
+}
+
+// Every entry of the final bucket from the staging row of its id (or the
+// feature cache).  which = 0: every entry; 1: only entries whose block is in
+// the feature cache; 2: only the others.
+template <int LPR, int U>
+__global__ void __launch_bounds__(kThreads)
+gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __restrict__ fb_id,
+                          const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
+                          TileMap tm, const uint32_t* __restrict__ bitmap,
+                          const uint16_t* __restrict__ wpref, const int32_t* __restrict__ doff,
+                          const unsigned long long* __restrict__ addr, int32_t rpb,
+                          unsigned long long cache_lo, unsigned long long cache_hi, int which,
+                          uint4* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  constexpr int kRowsPerWarp = 32 / LPR;
+  constexpr int kStep = kRowsPerWarp * U;
+  const int64_t total = *total_ptr;
+  const int lane = lane_id();
+  const int sub = lane / LPR, l = lane % LPR;
+  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t r0 = warp0 * kStep; r0 < total; r0 += nwarps * kStep) {
+    uint4 v[U];
+    int32_t g[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t i = r0 + u * kRowsPerWarp + sub;
+      g[u] = -1;
+      if (i < total) {
+        const int32_t id = __ldg(fb_id + i);
+        if (which != 0) {
+          const unsigned long long a = __ldg(addr + id / rpb);
+          if ((a >= cache_lo && a < cache_hi) != (which == 1)) continue;
+        }
+        g[u] = __ldg(fb_pos + i);
+        v[u] = __ldg(staged_row_src(staging, LPR, addr, rpb, cache_lo, cache_hi, tm, bitmap, wpref,
+                                    doff, id) +
+                     l);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (g[u] >= 0) __stcs(out + (int64_t)g[u] * LPR + l, v[u]);
+  }
+}
+
+// Rows of any multiple of 16 bytes: one warp per row.
+__global__ void __launch_bounds__(kThreads)
+gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
+                               const int32_t* __restrict__ fb_id,
+                               const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
+                               TileMap tm, const uint32_t* __restrict__ bitmap,
+                               const uint16_t* __restrict__ wpref,
+                               const int32_t* __restrict__ doff,
+                               const unsigned long long* __restrict__ addr, int32_t rpb,
+                               unsigned long long cache_lo, unsigned long long cache_hi, int which,
+                               uint4* __restrict__ out, const int32_t* status) {
+  if (failed(status)) return;
+  const int64_t total = *total_ptr;
+  const int lane = lane_id();
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
+    const int32_t id = __ldg(fb_id + i);
+    if (which != 0) {
+      const unsigned long long a = __ldg(addr + id / rpb);
+      if ((a >= cache_lo && a < cache_hi) != (which == 1)) continue;
+    }
+    const int64_t g = __ldg(fb_pos + i);
+    const uint4* src = staged_row_src(staging, vecs, addr, rpb, cache_lo, cache_hi, tm, bitmap,
+                                      wpref, doff, id);
+    for (int64_t c = lane; c < vecs; c += 32) __stcs(out + g * vecs + c, __ldg(src + c));
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
@@ -362,6 +552,77 @@ cudaError_t launch_load_feat_blocks(const void* host_dev, int64_t host_bytes, co
   if (njobs <= 0) return cudaSuccess;
   load_feat_blocks_kernel<<<num_sms, kThreads, 0, st>>>((const uint4*)host_dev, host_bytes / 16,
                                                         blk, dst, njobs, block_bytes / 16);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tile_bitmaps(const int32_t* fb_id, const int32_t* cell_off,
+                                const int32_t* tile_first, int32_t T, int32_t H, uint32_t* bitmap,
+                                uint16_t* wpref, int32_t* dcnt, const int32_t* status,
+                                cudaStream_t st) {
+  tile_bitmap_kernel<<<1184, kThreads, 0, st>>>(fb_id, cell_off, tile_first, T, H, bitmap, wpref,
+                                                dcnt, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_load_distinct_rows(const unsigned long long* addr, int64_t row_bytes,
+                                      int64_t rpb, const uint32_t* bitmap, const uint16_t* wpref,
+                                      const int32_t* doff, int32_t T, const int32_t* tile_first,
+                                      void* staging, unsigned long long cache_lo,
+                                      unsigned long long cache_hi, unsigned long long* host_rows,
+                                      const int32_t* status, int num_sms, cudaStream_t st) {
+  const int64_t vecs = row_bytes / 16;
+  uint4* sg = (uint4*)staging;
+#define AGNES_LOADD(LPR)                                                                      \
+  load_distinct_rows_kernel<LPR><<<resident_grid((const void*)load_distinct_rows_kernel<LPR>, \
+                                                 kThreads, num_sms),                          \
+                                   kThreads, 0, st>>>(addr, vecs, (int32_t)rpb, bitmap, wpref, \
+                                                      doff, T, tile_first, sg, cache_lo,       \
+                                                      cache_hi, host_rows, status)
+  if (vecs <= 8)
+    AGNES_LOADD(8);
+  else if (vecs <= 16)
+    AGNES_LOADD(16);
+  else
+    AGNES_LOADD(32);
+#undef AGNES_LOADD
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, const int32_t* fb_id,
+                                      const int32_t* fb_pos, const int32_t* total,
+                                      const int32_t* tile_first, const int32_t* chunk_tile,
+                                      int32_t T, const uint32_t* bitmap, const uint16_t* wpref,
+                                      const int32_t* doff, const unsigned long long* addr,
+                                      int64_t rpb, unsigned long long cache_lo,
+                                      unsigned long long cache_hi, int which, int grid_less,
+                                      void* out, const int32_t* status, int num_sms,
+                                      cudaStream_t st) {
+  const int64_t vecs = row_bytes / 16;
+  const uint4* sg = (const uint4*)staging;
+  uint4* o = (uint4*)out;
+  const TileMap tm{tile_first, chunk_tile, T};
+  // grid_less CTAs per SM are left free (for a kernel running beside this one)
+  auto grid_of = [&](const void* k) {
+    const int g = resident_grid(k, kThreads, num_sms) - grid_less * num_sms;
+    return g > num_sms ? g : num_sms;
+  };
+#define AGNES_GSR(LPR)                                                                          \
+  gather_staged_rows_kernel<LPR, 4><<<grid_of((const void*)gather_staged_rows_kernel<LPR, 4>),  \
+                                      kThreads, 0, st>>>(sg, fb_id, fb_pos, total, tm, bitmap,  \
+                                                         wpref, doff, addr, (int32_t)rpb,       \
+                                                         cache_lo, cache_hi, which, o, status)
+  if (vecs == 8)
+    AGNES_GSR(8);
+  else if (vecs == 16)
+    AGNES_GSR(16);
+  else if (vecs == 32)
+    AGNES_GSR(32);
+  else
+    gather_staged_rows_wide_kernel<<<grid_of((const void*)gather_staged_rows_wide_kernel),
+                                     kThreads, 0, st>>>(sg, vecs, fb_id, fb_pos, total, tm, bitmap,
+                                                        wpref, doff, addr, (int32_t)rpb, cache_lo,
+                                                        cache_hi, which, o, status);
+#undef AGNES_GSR
   return cudaGetLastError();
 }
 

@@ -178,6 +178,37 @@ cudaError_t launch_gather_table(const unsigned long long* addr, int64_t row_byte
                                 const int32_t* fb_id, const int32_t* fb_pos, const int32_t* total,
                                 void* out, const int32_t* status, int num_sms, cudaStream_t st);
 
+// Row mode, de-duplicated (see gather.cu): per tile t, the bitmap of requested
+// ids (kTileWords words at bitmap + t * kTileWords), the exclusive prefix of
+// set bits per word (wpref) and their count (dcnt[t]).
+cudaError_t launch_tile_bitmaps(const int32_t* fb_id, const int32_t* cell_off,
+                                const int32_t* tile_first, int32_t T, int32_t H, uint32_t* bitmap,
+                                uint16_t* wpref, int32_t* dcnt, const int32_t* status,
+                                cudaStream_t st);
+// Copies every distinct requested row (doff = exclusive scan of dcnt, T + 1
+// entries) of a block outside the feature cache [cache_lo, cache_hi) from its
+// block's address to staging, counting them in *host_rows.
+cudaError_t launch_load_distinct_rows(const unsigned long long* addr, int64_t row_bytes,
+                                      int64_t rpb, const uint32_t* bitmap, const uint16_t* wpref,
+                                      const int32_t* doff, int32_t T, const int32_t* tile_first,
+                                      void* staging, unsigned long long cache_lo,
+                                      unsigned long long cache_hi, unsigned long long* host_rows,
+                                      const int32_t* status, int num_sms, cudaStream_t st);
+// Gathers entries of the final bucket from the staging row of their id, or
+// in place from the feature cache when their block's address (addr, one per
+// feature block of rpb rows) lies in [cache_lo, cache_hi).  which = 0: every
+// entry, 1: cached blocks only, 2: the others.  The grid leaves grid_less CTAs
+// per SM free.
+cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, const int32_t* fb_id,
+                                      const int32_t* fb_pos, const int32_t* total,
+                                      const int32_t* tile_first, const int32_t* chunk_tile,
+                                      int32_t T, const uint32_t* bitmap, const uint16_t* wpref,
+                                      const int32_t* doff, const unsigned long long* addr,
+                                      int64_t rpb, unsigned long long cache_lo,
+                                      unsigned long long cache_hi, int which, int grid_less,
+                                      void* out, const int32_t* status, int num_sms,
+                                      cudaStream_t st);
+
 // Copies feature blocks blk[0 .. njobs) (block_bytes each, the last block of
 // the matrix possibly shorter) from host_dev, the device view of pinned host
 // memory holding host_bytes bytes, to device addresses dst[0 .. njobs).
