@@ -250,6 +250,9 @@ def main():
     ap.add_argument("--stream-topology", action="store_true",
                     help="neighbour lists in pinned host memory, loaded into an HBM graph buffer")
     ap.add_argument("--graph-buffer-gb", type=float, default=4.0)
+    ap.add_argument("--topology-io", default="blocks", choices=["blocks", "rows"],
+                    help="with --stream-topology: load whole blocks into the graph buffer, or "
+                         "read sampled neighbour entries in place")
     ap.add_argument("--stream", action="store_true",
                     help="features in pinned host memory, streamed block-wise per hyperbatch")
     ap.add_argument("--feature-cache-gb", type=float, default=0.0,
@@ -321,6 +324,7 @@ def main():
     g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes, device=local,
               stream=stream, features_on_host=args.stream, topology_on_host=args.stream_topology,
               graph_buffer_bytes=topo["graph_buffer_bytes"] if topo else 0,
+              topology_io=args.topology_io if args.stream_topology else "blocks",
               feature_cache_bytes=int(args.feature_cache_gb * 2**30) if args.stream else 0,
               feature_cache_threshold=args.feature_cache_threshold,
               feature_io=args.feature_io if args.stream else "blocks")
@@ -463,7 +467,9 @@ def main():
                               if args.stream else "")
                            + (f", {args.feature_cache_gb:g} GB feature cache"
                               if args.stream and args.feature_cache_gb > 0 else "")
-                           + (f" topology in pinned host memory, {args.graph_buffer_gb:g} GB graph buffer"
+                           + ((f" topology in pinned host memory, {args.graph_buffer_gb:g} GB graph buffer"
+                               if args.topology_io == "blocks" else
+                               " topology in pinned host memory (rows I/O)")
                               if args.stream_topology else ""),
                        "graph": {"nodes": info["num_nodes"], "edges": info["num_edges"],
                                  "adj_blocks": info["adj_blocks"], "tiles": info["tiles"],

@@ -115,7 +115,17 @@ typedef struct {
   int64_t feature_cache_bytes;     /* features_on_host: HBM feature cache (0: none) */
   int64_t feature_cache_threshold; /* cumulative requests a block must exceed to be cached */
   int32_t feature_io;              /* features_on_host: AGNES_FEATURE_IO_BLOCKS or _ROWS */
+  int32_t topology_io;             /* topology_on_host: AGNES_TOPOLOGY_IO_BLOCKS or _ROWS */
 } agnes_graph_desc;
+
+/* How host-resident neighbour lists reach the sampler (topology_on_host = 1).
+ * BLOCKS: the blocks a hop's frontier touches are loaded whole into the HBM
+ *   graph buffer (LRU + pinning, Sec. 3.4 (1)); 0, the default.
+ * ROWS: the sampler reads each sampled neighbour entry in place from pinned
+ *   host memory over the host link; no graph buffer (graph_buffer_bytes is
+ *   ignored).  Not in the paper, for the reason given for feature rows. */
+#define AGNES_TOPOLOGY_IO_BLOCKS 0
+#define AGNES_TOPOLOGY_IO_ROWS 1
 
 /* How host-resident features reach the gather (features_on_host = 1).
  * BLOCKS: every touched feature block is loaded whole into HBM, batch by

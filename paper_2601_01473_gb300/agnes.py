@@ -19,7 +19,7 @@ MAX_HOPS = 8
 MAX_FANOUT = 1024
 
 F32, F16 = 0, 1
-FEATURE_IO = {"blocks": 0, "rows": 1}  # AGNES_FEATURE_IO_BLOCKS / _ROWS
+FEATURE_IO = {"blocks": 0, "rows": 1}  # AGNES_FEATURE_IO_* and AGNES_TOPOLOGY_IO_* values
 FRONTIER = {"src": 0, "sampled": 1}    # AGNES_FRONTIER_SRC / _SAMPLED
 _DTYPES = {torch.float32: F32, torch.float16: F16}
 _TORCH_OF = {F32: torch.float32, F16: torch.float16}
@@ -53,6 +53,7 @@ class _GraphDesc(ctypes.Structure):
         ("feature_cache_bytes", ctypes.c_int64),
         ("feature_cache_threshold", ctypes.c_int64),
         ("feature_io", ctypes.c_int32),
+        ("topology_io", ctypes.c_int32),
     ]
 
 
@@ -248,7 +249,8 @@ class Graph:
                  feat_block_bytes: int | None = None, device: int = 0, stream=None,
                  features_on_host: bool = False, topology_on_host: bool = False,
                  graph_buffer_bytes: int = 0, feature_cache_bytes: int = 0,
-                 feature_cache_threshold: int = 0, feature_io: str = "blocks"):
+                 feature_cache_threshold: int = 0, feature_io: str = "blocks",
+                 topology_io: str = "blocks"):
         if offsets.dtype not in (torch.int32, torch.int64):
             raise TypeError("offsets must be int32 or int64")
         if indices.dtype != torch.int32:
@@ -281,6 +283,9 @@ class Graph:
         if feature_io not in FEATURE_IO:
             raise ValueError(f"feature_io must be one of {sorted(FEATURE_IO)}")
         d.feature_io = FEATURE_IO[feature_io]
+        if topology_io not in FEATURE_IO:
+            raise ValueError(f"topology_io must be one of {sorted(FEATURE_IO)}")
+        d.topology_io = FEATURE_IO[topology_io]
         ctx = ctypes.c_void_p()
         with torch.cuda.device(self.device):
             rc = lib().agnes_load_graph(ctypes.byref(d), device, _stream_handle(stream),

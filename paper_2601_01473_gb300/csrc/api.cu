@@ -779,6 +779,10 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
     set_err(nullptr, "features_on_host needs a 16-byte aligned feature matrix");
     return AGNES_EINVAL;
   }
+  if (d->topology_io != AGNES_TOPOLOGY_IO_BLOCKS && d->topology_io != AGNES_TOPOLOGY_IO_ROWS) {
+    set_err(nullptr, "topology_io must be AGNES_TOPOLOGY_IO_BLOCKS or AGNES_TOPOLOGY_IO_ROWS");
+    return AGNES_EINVAL;
+  }
   if (d->feature_io != AGNES_FEATURE_IO_BLOCKS && d->feature_io != AGNES_FEATURE_IO_ROWS) {
     set_err(nullptr, "feature_io must be AGNES_FEATURE_IO_BLOCKS or AGNES_FEATURE_IO_ROWS");
     return AGNES_EINVAL;
@@ -820,6 +824,19 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   if (rc == AGNES_OK && d->num_edges > 0 && !d->topology_on_host)
     rc = adopt_or_copy(ctx, d->indices, (size_t)d->num_edges * 4, (void**)&ctx->indices,
                        &ctx->own_indices, st);
+  if (rc == AGNES_OK && d->num_edges > 0 && d->topology_on_host &&
+      d->topology_io == AGNES_TOPOLOGY_IO_ROWS) {
+    // the sampler reads neighbour entries in place, through the device view
+    void* dv = nullptr;
+    if (cudaHostGetDevicePointer(&dv, const_cast<int32_t*>(d->indices), 0) != cudaSuccess) {
+      cudaGetLastError();
+      set_err(ctx, "cudaHostGetDevicePointer failed for the host neighbour lists");
+      rc = AGNES_ECUDA;
+    } else {
+      ctx->indices = (int32_t*)dv;
+      ctx->own_indices = false;
+    }
+  }
   if (rc == AGNES_OK) {
     if (d->features_on_host) {
       ctx->features = const_cast<void*>(d->features);
@@ -864,7 +881,9 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
     if (e != cudaSuccess) rc = e == cudaErrorMemoryAllocation ? AGNES_ENOMEM : AGNES_ECUDA;
   }
   if (rc == AGNES_OK && d->features_on_host) rc = setup_streaming(ctx, d, st);
-  if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0) rc = setup_topology(ctx, d, st);
+  if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0 &&
+      d->topology_io == AGNES_TOPOLOGY_IO_BLOCKS)
+    rc = setup_topology(ctx, d, st);
   if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
     set_err(ctx, "cudaEventCreate failed");
     rc = AGNES_ECUDA;

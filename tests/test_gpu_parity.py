@@ -385,6 +385,28 @@ def test_streamed_topology_matches_oracle(cuda_device, a, b, c, bb, buf_blocks, 
     g.close()
 
 
+@pytest.mark.parametrize("a,b,c,fan", [
+    (0.57, 0.19, 0.19, [8, 4]),
+    (0.6, 0.2, 0.15, [25, 10]),      # skewed: hubs with neighbour lists of many blocks
+    (0.57, 0.19, 0.19, [6, 4, 2]),
+])
+def test_topology_read_in_place_matches_oracle(cuda_device, a, b, c, fan):
+    """Neighbour lists in pinned host memory, read in place over the host
+    link (AGNES_TOPOLOGY_IO_ROWS): same samples as the oracle."""
+    off, ind = synth.rmat_csr(30000, 14, a, b, c, seed=len(fan) * 7, offsets_dtype=torch.int64)
+    feats = synth.normal_features(30000, 32, torch.float16, 6)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    g = Graph(off.to(cuda_device), ind.pin_memory(), feats.to(cuda_device), adj_block_bytes=4096,
+              feat_block_bytes=4096, topology_on_host=True, topology_io="rows")
+    for step in range(2):
+        targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), 4, 150, 9, step)
+        g.prepare(targets.to(cuda_device), fan, 77, 10 * step)
+        compare(g, og, targets.numpy(), fan, 77, 10 * step, 4096, 4096)
+    cnt = g.counters()
+    assert cnt["topo_loaded_blocks"] == 0 and cnt["topo_waves"] == 0
+    g.close()
+
+
 def test_graph_buffer_smaller_than_an_object_is_rejected(cuda_device):
     off, ind = synth.rmat_csr(5000, 30, 0.6, 0.2, 0.15, seed=1)
     feats = synth.normal_features(5000, 8, torch.float32, 2)
