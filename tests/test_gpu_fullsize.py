@@ -65,3 +65,52 @@ def test_fullsize_parity(cuda_device, name, sample):
                                      w.adj_block_bytes, w.feat_block_bytes,
                                      threads=os.cpu_count() or 1)
     assert got_stats == ref_stats
+
+
+@pytest.mark.timeout(1200)
+def test_config5_variants_parity(cuda_device):
+    """Config 5 at full size: rmat100m's graph as a sweep point (256 KB blocks,
+    H = 16), with its features in pinned host memory (row I/O through a 4 GB
+    feature cache, then block I/O), and with its neighbour lists read in place
+    from pinned host memory.  Sampled minibatches bit-exact against the oracle."""
+    w = WORKLOADS["rmat100m"]
+    offsets, indices, features = build_graph(w, cuda_device)
+    pool = target_pool(w, cuda_device)
+    ws = w.with_(H=16, adj_block_bytes=256 * 1024, feat_block_bytes=256 * 1024)
+    targets = targets_for_step(ws, pool, 3)
+    fan = list(w.fanouts)
+    sample = (0, 9, 15)
+    host_feats = features.cpu().pin_memory()
+    host_ind = indices.cpu().pin_memory()
+    got = {}
+    variants = {
+        "sweep": dict(offsets=offsets, indices=indices, features=features),
+        "rows+cache": dict(offsets=offsets, indices=indices, features=host_feats,
+                           features_on_host=True, feature_io="rows",
+                           feature_cache_bytes=4 << 30),
+        "blocks": dict(offsets=offsets, indices=indices, features=host_feats,
+                       features_on_host=True),
+        "topology rows": dict(offsets=offsets, indices=host_ind, features=features,
+                              topology_on_host=True, topology_io="rows"),
+    }
+    for name, kw in variants.items():
+        g = Graph(adj_block_bytes=ws.adj_block_bytes, feat_block_bytes=ws.feat_block_bytes, **kw)
+        for step in range(3):  # blocks admitted after the first load in the second; hits from the third
+            g.prepare(targets, fan, w.seed, 500)
+        got[name] = {j: (g.fetch(j).nodes.cpu().numpy(),
+                         [(h.indptr.cpu().numpy(), h.col.cpu().numpy()) for h in g.fetch(j).hops],
+                         _bytes(g.fetch(j).feats)) for j in sample}
+        if name == "rows+cache":
+            assert g.counters()["fcache_hit_blocks"] > 0
+        g.close()
+    og = oracle.Graph(offsets.cpu().numpy(), host_ind.numpy(), host_feats.numpy())
+    t = targets.cpu().numpy()
+    for j in sample:
+        r = oracle.sample_minibatch(og, t[j], fan, w.seed, 500 + j)
+        for name in variants:
+            nodes, hops, feats = got[name][j]
+            assert np.array_equal(nodes, r["nodes"]), f"{name}: nodes of minibatch {j}"
+            for h, (ip, col) in enumerate(hops):
+                assert np.array_equal(ip, r["hops"][h]["indptr"]), f"{name}: indptr {h} mb {j}"
+                assert np.array_equal(col, r["hops"][h]["col"]), f"{name}: col {h} mb {j}"
+            assert np.array_equal(feats, r["feats"].view(np.uint8).reshape(-1)), f"{name}: feats {j}"
