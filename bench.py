@@ -159,7 +159,7 @@ def gather_traffic_from_profile(workload: str):
     if workload != "rmat100m":
         return None
     path = os.path.join(ROOT, "profiles", "gather_rmat100m.md")
-    src = os.path.join(ROOT, "paper_2601_01473_gb300", "csrc", "gather.cu")
+    src = os.path.join(ROOT, "paper_2601_01473_gb300", "csrc", "gather_hbm.cu")
     try:
         sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
         vals = {}
@@ -167,7 +167,7 @@ def gather_traffic_from_profile(workload: str):
             if ":" in line and line.strip().startswith("- "):
                 k, v = line.strip()[2:].split(":", 1)
                 vals[k.strip()] = v.strip()
-        if vals.get("gather.cu sha256 prefix") != sha:
+        if vals.get("gather_hbm.cu sha256 prefix") != sha:
             return None
         return float(vals["dram bytes per launch (full workload)"])
     except Exception:

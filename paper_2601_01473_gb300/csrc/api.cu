@@ -1181,7 +1181,7 @@ static agnes_status gather_rows_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* 
   CK(ctx, launch_gather_staged_rows(ctx->rm_staging, rb, w.fb_id[cur], w.fb_pos[cur],
                                     w.fcell_off[cur] + cells, ctx->bt.tile_first,
                                     ctx->bt.chunk_tile, T, ctx->rm_bitmap, ctx->rm_wpref,
-                                    ctx->rm_doff, ctx->d_addr, rpb, 0, 0, 0, 0, w.feats_out,
+                                    ctx->rm_doff, ctx->d_addr, rpb, 0, 0, w.feats_out,
                                     w.status, ctx->num_sms, st));
   // rows read over the link, for the counters (read after the hyperbatch is done)
   CK(ctx, cudaMemcpyAsync(ctx->h_rm + 1, ctx->d_host_rows, sizeof(int64_t),

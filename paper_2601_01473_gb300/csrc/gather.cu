@@ -1,14 +1,10 @@
-// gather.cu -- block-wise feature gathering (Algorithm 1's gathering loop,
-// Sec. 3.4 (2)) and the bookkeeping kernels for blocks-touched statistics.
-//
-// The final frontier bucket lists every gathered node once per minibatch, in
-// (tile, minibatch, id) order, with its output row.  Tiles never straddle a
-// feature block, so walking the bucket in order visits each feature block
-// once for all minibatches: a row requested by several minibatches is read
-// from HBM once and served from L2 afterwards.  Rows are copied as 16-byte
-// vectors (bit-exact, no float conversion); a group of row_bytes/16 lanes
-// moves one row, each lane keeping U rows in flight; output stores are
-// streaming (evict-first) so they do not push the feature rows out of L2.
+// gather.cu -- feature gathering from host-resident features (staged
+// blocks, the feature cache, row reads over the host link), the topology
+// block loader, and the bookkeeping kernels for blocks-touched statistics.
+// The gather from HBM-resident features is in gather_hbm.cu.  Every gather
+// walks the final bucket, which lists each gathered node once per minibatch
+// in (tile, minibatch, id) order with its output row, and copies rows as
+// 16-byte vectors (bit-exact).
 #include "common.cuh"
 #include "internal.h"
 
@@ -18,71 +14,6 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-
-// LPR lanes per row, row = LPR 16-byte vectors, U rows in flight per lane.
-template <int LPR, int U>
-__global__ void __launch_bounds__(kThreads)
-gather_vec_kernel(const uint4* __restrict__ feats, const int32_t* __restrict__ fb_id,
-                  const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
-                  uint4* __restrict__ out, const int32_t* status) {
-  if (failed(status)) return;
-  constexpr int kRowsPerWarp = 32 / LPR;
-  constexpr int kStep = kRowsPerWarp * U;
-  const int64_t total = *total_ptr;
-  const int lane = lane_id();
-  const int sub = lane / LPR, l = lane % LPR;
-  const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t r0 = warp0 * kStep; r0 < total; r0 += nwarps * kStep) {
-    uint4 v[U];
-    int32_t g[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t i = r0 + u * kRowsPerWarp + sub;
-      g[u] = -1;
-      if (i < total) {
-        const int32_t id = __ldg(fb_id + i);
-        g[u] = __ldg(fb_pos + i);
-        v[u] = __ldg(feats + (int64_t)id * LPR + l);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (g[u] >= 0) __stcs(out + (int64_t)g[u] * LPR + l, v[u]);
-  }
-}
-
-// Any row size that is a multiple of 16 bytes: one warp per row.
-__global__ void __launch_bounds__(kThreads)
-gather_rows_kernel(const uint4* __restrict__ feats, int64_t vecs, const int32_t* __restrict__ fb_id,
-                   const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
-                   uint4* __restrict__ out, const int32_t* status) {
-  if (failed(status)) return;
-  const int64_t total = *total_ptr;
-  const int lane = lane_id();
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
-    const int64_t src = (int64_t)__ldg(fb_id + i) * vecs;
-    const int64_t dst = (int64_t)__ldg(fb_pos + i) * vecs;
-    for (int64_t c = lane; c < vecs; c += 32) __stcs(out + dst + c, __ldg(feats + src + c));
-  }
-}
-
-// Rows whose size is not a multiple of 16 bytes: byte copy, one warp per row.
-__global__ void __launch_bounds__(kThreads)
-gather_bytes_kernel(const uint8_t* __restrict__ feats, int64_t row_bytes,
-                    const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
-                    const int32_t* total_ptr, uint8_t* __restrict__ out, const int32_t* status) {
-  if (failed(status)) return;
-  const int64_t total = *total_ptr;
-  const int lane = lane_id();
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
-    const int64_t src = (int64_t)__ldg(fb_id + i) * row_bytes;
-    const int64_t dst = (int64_t)__ldg(fb_pos + i) * row_bytes;
-    for (int64_t c = lane; c < row_bytes; c += 32) out[dst + c] = __ldg(feats + src + c);
-  }
-}
 
 // Streaming variant: rows come from HBM copies of their feature blocks (a
 // staging slot of the ring or the feature cache).  The batch's blocks are
@@ -399,8 +330,7 @@ __device__ __forceinline__ const uint4* staged_row_src(
 }
 
 // Every entry of the final bucket from the staging row of its id (or the
-// feature cache).  which = 0: every entry; 1: only entries whose block is in
-// the feature cache; 2: only the others.
+// feature cache).
 template <int LPR, int U>
 __global__ void __launch_bounds__(kThreads)
 gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __restrict__ fb_id,
@@ -408,7 +338,7 @@ gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __re
                           TileMap tm, const uint32_t* __restrict__ bitmap,
                           const uint16_t* __restrict__ wpref, const int32_t* __restrict__ doff,
                           const unsigned long long* __restrict__ addr, int32_t rpb,
-                          unsigned long long cache_lo, unsigned long long cache_hi, int which,
+                          unsigned long long cache_lo, unsigned long long cache_hi,
                           uint4* __restrict__ out, const int32_t* status) {
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
@@ -427,10 +357,6 @@ gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __re
       g[u] = -1;
       if (i < total) {
         const int32_t id = __ldg(fb_id + i);
-        if (which != 0) {
-          const unsigned long long a = __ldg(addr + id / rpb);
-          if ((a >= cache_lo && a < cache_hi) != (which == 1)) continue;
-        }
         g[u] = __ldg(fb_pos + i);
         v[u] = __ldg(staged_row_src(staging, LPR, addr, rpb, cache_lo, cache_hi, tm, bitmap, wpref,
                                     doff, id) +
@@ -452,7 +378,7 @@ gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
                                const uint16_t* __restrict__ wpref,
                                const int32_t* __restrict__ doff,
                                const unsigned long long* __restrict__ addr, int32_t rpb,
-                               unsigned long long cache_lo, unsigned long long cache_hi, int which,
+                               unsigned long long cache_lo, unsigned long long cache_hi,
                                uint4* __restrict__ out, const int32_t* status) {
   if (failed(status)) return;
   const int64_t total = *total_ptr;
@@ -460,10 +386,6 @@ gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
     const int32_t id = __ldg(fb_id + i);
-    if (which != 0) {
-      const unsigned long long a = __ldg(addr + id / rpb);
-      if ((a >= cache_lo && a < cache_hi) != (which == 1)) continue;
-    }
     const int64_t g = __ldg(fb_pos + i);
     const uint4* src = staged_row_src(staging, vecs, addr, rpb, cache_lo, cache_hi, tm, bitmap,
                                       wpref, doff, id);
@@ -472,37 +394,6 @@ gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
 }
 
 }  // namespace
-
-cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
-                          const int32_t* fb_pos, const int32_t* total, void* out,
-                          const int32_t* status, int num_sms, cudaStream_t st) {
-  const bool aligned = (row_bytes % 16 == 0) && ((uintptr_t)feats % 16 == 0) &&
-                       ((uintptr_t)out % 16 == 0);
-  if (aligned) {
-    const int64_t vecs = row_bytes / 16;
-    const uint4* f = (const uint4*)feats;
-    uint4* o = (uint4*)out;
-#define AGNES_GRID(KERNEL) resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st
-    if (vecs == 8)
-      gather_vec_kernel<8, 4><<<AGNES_GRID((gather_vec_kernel<8, 4>))>>>(f, fb_id, fb_pos, total, o,
-                                                                         status);
-    else if (vecs == 16)
-      gather_vec_kernel<16, 4><<<AGNES_GRID((gather_vec_kernel<16, 4>))>>>(f, fb_id, fb_pos, total,
-                                                                           o, status);
-    else if (vecs == 32)
-      gather_vec_kernel<32, 4><<<AGNES_GRID((gather_vec_kernel<32, 4>))>>>(f, fb_id, fb_pos, total,
-                                                                           o, status);
-    else
-      gather_rows_kernel<<<AGNES_GRID(gather_rows_kernel)>>>(f, vecs, fb_id, fb_pos, total, o,
-                                                             status);
-  } else {
-    gather_bytes_kernel<<<AGNES_GRID(gather_bytes_kernel)>>>((const uint8_t*)feats, row_bytes,
-                                                             fb_id, fb_pos, total, (uint8_t*)out,
-                                                             status);
-  }
-#undef AGNES_GRID
-  return cudaGetLastError();
-}
 
 cudaError_t launch_gather_staged(const unsigned long long* src, int64_t row_bytes, int64_t rpb,
                                  const int32_t* touched, int32_t nb, const int32_t* fb_id,
@@ -594,23 +485,19 @@ cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, co
                                       int32_t T, const uint32_t* bitmap, const uint16_t* wpref,
                                       const int32_t* doff, const unsigned long long* addr,
                                       int64_t rpb, unsigned long long cache_lo,
-                                      unsigned long long cache_hi, int which, int grid_less,
-                                      void* out, const int32_t* status, int num_sms,
-                                      cudaStream_t st) {
+                                      unsigned long long cache_hi, void* out,
+                                      const int32_t* status, int num_sms, cudaStream_t st) {
   const int64_t vecs = row_bytes / 16;
   const uint4* sg = (const uint4*)staging;
   uint4* o = (uint4*)out;
   const TileMap tm{tile_first, chunk_tile, T};
-  // grid_less CTAs per SM are left free (for a kernel running beside this one)
-  auto grid_of = [&](const void* k) {
-    const int g = resident_grid(k, kThreads, num_sms) - grid_less * num_sms;
-    return g > num_sms ? g : num_sms;
-  };
 #define AGNES_GSR(LPR)                                                                          \
-  gather_staged_rows_kernel<LPR, 4><<<grid_of((const void*)gather_staged_rows_kernel<LPR, 4>),  \
+  gather_staged_rows_kernel<LPR, 4><<<resident_grid(                                            \
+                                          (const void*)gather_staged_rows_kernel<LPR, 4>,        \
+                                          kThreads, num_sms),                                   \
                                       kThreads, 0, st>>>(sg, fb_id, fb_pos, total, tm, bitmap,  \
                                                          wpref, doff, addr, (int32_t)rpb,       \
-                                                         cache_lo, cache_hi, which, o, status)
+                                                         cache_lo, cache_hi, o, status)
   if (vecs == 8)
     AGNES_GSR(8);
   else if (vecs == 16)
@@ -618,10 +505,11 @@ cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, co
   else if (vecs == 32)
     AGNES_GSR(32);
   else
-    gather_staged_rows_wide_kernel<<<grid_of((const void*)gather_staged_rows_wide_kernel),
+    gather_staged_rows_wide_kernel<<<resident_grid((const void*)gather_staged_rows_wide_kernel,
+                                                   kThreads, num_sms),
                                      kThreads, 0, st>>>(sg, vecs, fb_id, fb_pos, total, tm, bitmap,
                                                         wpref, doff, addr, (int32_t)rpb, cache_lo,
-                                                        cache_hi, which, o, status);
+                                                        cache_hi, o, status);
 #undef AGNES_GSR
   return cudaGetLastError();
 }

@@ -194,20 +194,17 @@ cudaError_t launch_load_distinct_rows(const unsigned long long* addr, int64_t ro
                                       void* staging, unsigned long long cache_lo,
                                       unsigned long long cache_hi, unsigned long long* host_rows,
                                       const int32_t* status, int num_sms, cudaStream_t st);
-// Gathers entries of the final bucket from the staging row of their id, or
-// in place from the feature cache when their block's address (addr, one per
-// feature block of rpb rows) lies in [cache_lo, cache_hi).  which = 0: every
-// entry, 1: cached blocks only, 2: the others.  The grid leaves grid_less CTAs
-// per SM free.
+// Gathers every entry of the final bucket from the staging row of its id,
+// or in place from the feature cache when its block's address (addr, one per
+// feature block of rpb rows) lies in [cache_lo, cache_hi).
 cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, const int32_t* fb_id,
                                       const int32_t* fb_pos, const int32_t* total,
                                       const int32_t* tile_first, const int32_t* chunk_tile,
                                       int32_t T, const uint32_t* bitmap, const uint16_t* wpref,
                                       const int32_t* doff, const unsigned long long* addr,
                                       int64_t rpb, unsigned long long cache_lo,
-                                      unsigned long long cache_hi, int which, int grid_less,
-                                      void* out, const int32_t* status, int num_sms,
-                                      cudaStream_t st);
+                                      unsigned long long cache_hi, void* out,
+                                      const int32_t* status, int num_sms, cudaStream_t st);
 
 // Copies feature blocks blk[0 .. njobs) (block_bytes each, the last block of
 // the matrix possibly shorter) from host_dev, the device view of pinned host
