@@ -81,6 +81,33 @@ def test_golden_fixture(cuda_device):
     g.close()
 
 
+@pytest.mark.parametrize("fanouts,H,B", [
+    ((1024,), 3, 40),          # the largest fanout: 32 chunks of the wide sampler
+    ((100, 3), 4, 60),         # several chunks, then a small hop
+    ((2,) * 8, 3, 50),         # the most hops
+])
+def test_parity_extreme_fanouts_and_hops(cuda_device, fanouts, H, B):
+    """Skewed graph whose hubs have far more than 1024 neighbours."""
+    off, ind = synth.rmat_csr(20000, 60, 0.6, 0.2, 0.15, 13, offsets_dtype=torch.int64)
+    assert int((off[1:] - off[:-1]).max()) > 2 * max(fanouts)
+    feats = synth.normal_features(20000, 16, torch.float32, 14)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    # targets include the highest-degree nodes
+    deg = off[1:] - off[:-1]
+    hubs = torch.argsort(deg, descending=True)[:H * B // 4].to(torch.int32)
+    rest = synth.hyperbatch_targets(torch.arange(20000, dtype=torch.int32), H, B, 2, 0)
+    targets = rest.clone()
+    for j in range(H):  # put hubs into every minibatch, keeping the targets distinct
+        row = targets[j].tolist()
+        extra = [h for h in hubs.tolist() if h not in row][:B // 4]
+        targets[j, :len(extra)] = torch.tensor(extra, dtype=torch.int32)
+        assert len(set(targets[j].tolist())) == B
+    g = load(off, ind, feats, 16384, 16384)
+    g.prepare(targets.to(cuda_device), list(fanouts), 99, 7)
+    compare(g, og, targets.numpy(), list(fanouts), 99, 7, 16384, 16384)
+    g.close()
+
+
 @pytest.mark.parametrize("bits,dtype,fanouts", [
     (32, torch.float32, (10, 5)),
     (64, torch.float16, (15, 10, 5)),
