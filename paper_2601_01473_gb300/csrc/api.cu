@@ -188,6 +188,7 @@ struct agnes_ctx {
     cudaEvent_t uploaded = nullptr, wave_done[2] = {nullptr, nullptr};
     bool uploaded_used = false;
     int64_t loaded_blocks = 0, loaded_bytes = 0, hits = 0, waves = 0;
+    uint64_t sweeps = 0;  // hops sampled so far (sets the sweep direction)
   } topo;
 
   char err[512] = {0};
@@ -917,9 +918,14 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
                            st));
   CK(ctx, cudaMemcpyAsync(tp.h_need, tp.d_need, (size_t)ns, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaStreamSynchronize(st));
-  int64_t r = 0;
-  while (r < ns && !tp.h_need[r]) ++r;
-  while (r < ns) {
+  // Hops sweep their block runs in alternating directions, so each hop
+  // starts on the blocks the previous one used last -- the ones LRU kept.
+  // (The order of a hop's blocks does not change any result.)
+  const int64_t step = (tp.sweeps++ & 1) ? -1 : 1;
+  auto inside = [&](int64_t x) { return x >= 0 && x < ns; };
+  int64_t r = step > 0 ? 0 : ns - 1;
+  while (inside(r) && !tp.h_need[r]) r += step;
+  while (inside(r)) {
     // the staging buffers (jobs, slot table) are rewritten below: wait until
     // the previous wave's upload and loads have consumed them
     if (tp.uploaded_used) CK(ctx, cudaEventSynchronize(tp.uploaded));
@@ -927,11 +933,10 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
     const uint32_t wave = tp.wave;
     int64_t pinned_now = 0;
     int32_t njobs = 0;
-    const int64_t r_first = r;
-    int64_t r_last = r;
-    while (r < ns) {
+    int64_t r_lo = r, r_hi = r;  // the wave's runs, [r_lo, r_hi]
+    while (inside(r)) {
       if (!tp.h_need[r]) {
-        ++r;
+        r += step;
         continue;
       }
       const int32_t b0 = tp.start_block[(size_t)r], b1 = tp.start_block[(size_t)r + 1];
@@ -960,8 +965,9 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
         lru_touch(tp, sl);
         ++pinned_now;
       }
-      r_last = r;
-      ++r;
+      r_lo = r < r_lo ? r : r_lo;
+      r_hi = r > r_hi ? r : r_hi;
+      r += step;
     }
     // the slots taken now were last read by wave - 2 at the latest
     CK(ctx, cudaStreamWaitEvent(tp.copy, tp.wave_done[wave & 1], 0));
@@ -978,8 +984,8 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
     tp.uploaded_used = true;
     CK(ctx, cudaStreamWaitEvent(st, tp.uploaded, 0));
     FillRange fr;
-    fr.cell_lo = (int64_t)tp.run_first_tile[(size_t)r_first] * H;
-    fr.cell_hi = (int64_t)tp.run_first_tile[(size_t)r_last + 1] * H;
+    fr.cell_lo = (int64_t)tp.run_first_tile[(size_t)r_lo] * H;
+    fr.cell_hi = (int64_t)tp.run_first_tile[(size_t)r_hi + 1] * H;
     fr.tile_adj_block = ctx->bt.tile_adj_block;
     fr.blk_slot = tp.d_slot;
     fr.blk_e0 = ctx->bt.blk_e0;
@@ -990,7 +996,7 @@ static agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int
                                w.scnt, w.scell, w.srank, fr, ctx->num_sms, st));
     CK(ctx, cudaEventRecord(tp.wave_done[wave & 1], st));
     tp.waves += 1;
-    while (r < ns && !tp.h_need[r]) ++r;
+    while (inside(r) && !tp.h_need[r]) r += step;
   }
   return AGNES_OK;
 }
