@@ -127,14 +127,14 @@ class ClockSampler:
 
 
 def kernel_launches_per_step(K: int) -> int:
-    """Kernels libagnes launches per hyperbatch with the graph in HBM (the
-    ncu launch list of profiles/step_rmat100m_traffic.md has 59 at K = 3):
-    target bucketing 5 (count, 2-kernel scan, scatter, sort); per hop 16
+    """Kernels libagnes launches per hyperbatch with the graph in HBM (61 at
+    K = 3): the sampling-key write and the dst-size fill 2; target bucketing 5
+    (count, 2-kernel scan, scatter, sort); per hop 16
     (count, 2-kernel scan, fill, 2-kernel scan, scatter, cells, big cells,
     3-kernel column scan, 2-kernel scan, col fix-up, compaction); after the
     last hop 3 (feature-block marks, their count, gather) and K counts of
     touched topology blocks."""
-    return 5 + 16 * K + 3 + K
+    return 2 + 5 + 16 * K + 3 + K
 
 
 def algorithmic_bytes(c: dict, off_bytes: int) -> dict:

@@ -160,7 +160,13 @@ agnes_status agnes_load_graph(const agnes_graph_desc* desc, int device, void* cu
  *  fanouts   K host int32 values, fanouts[0] for the targets' hop;
  *            1 <= fanouts[h] <= AGNES_MAX_FANOUT, 1 <= K <= AGNES_MAX_HOPS.
  *  seed, first_minibatch_id  key the random draws (see above).
- * Stream-ordered: returns once the work is enqueued.  Element-wise checks of
+ * Stream-ordered: returns once the work is enqueued, after the ctx's previous
+ * prepare (on whatever stream) and before anything later on cuda_stream.
+ * Issued while cuda_stream is being captured into the caller's own CUDA
+ * graph, the work is recorded into that graph instead of run: fetch and
+ * stats describe it only once the caller has launched the graph and waited
+ * for it, the caller orders those launches with the ctx's other prepares,
+ * and no phase times are recorded.  Element-wise checks of
  * targets (range, distinctness) run on the device and are reported by the
  * next agnes_fetch_minibatch / agnes_hyperbatch_stats call as EINVAL.
  * Errors here: EINVAL (bad scalar args), ERANGE (H * capacity >= 2^31 output
@@ -183,6 +189,20 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
 #define AGNES_FRONTIER_SRC 0
 #define AGNES_FRONTIER_SAMPLED 1
 agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode);
+
+/* How agnes_prepare_hyperbatch issues its work when features and topology
+ * are resident in HBM.  enabled = 1 (default): the hyperbatch's launch
+ * sequence (memsets, ~60 kernels, the size read-back) is captured into a
+ * CUDA graph on a private stream the first time a shape is seen (H, B,
+ * fanouts, frontier mode, profiling) and replayed as one graph launch on the
+ * caller's stream for every later hyperbatch of that shape; the targets copy
+ * and the sampling key {seed, first_minibatch_id} are written to device
+ * memory ahead of it.  enabled = 0: every call launches the sequence
+ * directly.  Results are identical either way.  A caller stream that is
+ * itself being captured, and the host-resident modes (whose calls read sizes
+ * back mid-sequence), always take the direct path.  Takes effect at the next
+ * prepare.  Errors: EINVAL (enabled not 0 or 1). */
+agnes_status agnes_set_graph_mode(agnes_ctx* ctx, int32_t enabled);
 
 /* View of minibatch j of the last prepared hyperbatch.  Per hop h (0-based
  * index, hop number h+1): the bipartite block has num_dst[h] dst nodes and
@@ -272,6 +292,8 @@ typedef struct {
   int64_t topo_waves;               /* fill launches over all hops */
   int64_t fcache_hit_blocks;        /* feature blocks read in place from the feature cache */
   int64_t fcache_loaded_blocks;     /* feature blocks copied into the feature cache */
+  int64_t graph_captures;           /* launch sequences captured (agnes_set_graph_mode) */
+  int64_t graph_launches;           /* prepares issued as one graph launch */
 } agnes_counters;
 agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
 

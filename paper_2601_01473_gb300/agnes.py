@@ -102,6 +102,7 @@ class _Counters(ctypes.Structure):
         ("topo_waves", ctypes.c_int64),
         ("fcache_hit_blocks", ctypes.c_int64),
         ("fcache_loaded_blocks", ctypes.c_int64),
+        ("graph_captures", ctypes.c_int64), ("graph_launches", ctypes.c_int64),
     ]
 
 
@@ -132,6 +133,7 @@ SIGNATURES = {
                           ctypes.c_int),
     "agnes_hop_indptr_noalloc": ([_P, _P, ctypes.c_int64, ctypes.c_int32, _P, _P], ctypes.c_int),
     "agnes_set_frontier_mode": ([_P, ctypes.c_int32], ctypes.c_int),
+    "agnes_set_graph_mode": ([_P, ctypes.c_int32], ctypes.c_int),
     "agnes_sage_mean_layer": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int64,
                                ctypes.c_int64, _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
                                ctypes.c_int64, _P], ctypes.c_int),
@@ -354,6 +356,12 @@ class Graph:
             raise ValueError(f"frontier must be one of {sorted(FRONTIER)}")
         _check(lib().agnes_set_frontier_mode(self._ctx, FRONTIER[mode]), self._ctx)
 
+    def set_graph_mode(self, enabled: bool) -> None:
+        """Replay the resident path's launch sequence as one captured CUDA
+        graph per hyperbatch shape (True, the default), or launch it directly
+        on every prepare (False); the results are the same."""
+        _check(lib().agnes_set_graph_mode(self._ctx, 1 if enabled else 0), self._ctx)
+
     def sage_mean_layer(self, hop: int, x: torch.Tensor, w: torch.Tensor, bias=None,
                         out_dtype: torch.dtype = torch.float32, stream=None) -> torch.Tensor:
         """One GraphSAGE-mean layer (agnes_sage_mean_layer) over hop ``hop`` of
@@ -400,7 +408,8 @@ class Graph:
                 "topo_loaded_blocks": c.topo_loaded_blocks, "topo_loaded_bytes": c.topo_loaded_bytes,
                 "topo_hit_blocks": c.topo_hit_blocks, "topo_waves": c.topo_waves,
                 "fcache_hit_blocks": c.fcache_hit_blocks,
-                "fcache_loaded_blocks": c.fcache_loaded_blocks}
+                "fcache_loaded_blocks": c.fcache_loaded_blocks,
+                "graph_captures": c.graph_captures, "graph_launches": c.graph_launches}
 
     def info(self) -> dict:
         g = _GraphInfo()

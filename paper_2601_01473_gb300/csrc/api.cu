@@ -74,6 +74,7 @@ struct Workspace {
   int64_t* scan_scratch = nullptr;
   int32_t* status = nullptr;
   unsigned long long* distinct = nullptr;
+  uint64_t* key = nullptr;  // sampling key {seed, first minibatch id}
 
   // pinned host readback: [status][nsz (K+1)H][ecnt KH][srcsz KH] then int64 stats (K+1)
   void* h_back = nullptr;
@@ -117,6 +118,24 @@ struct agnes_ctx {
   int n_phases[kEventRing] = {0};          // per ring slot; 0 = not profiled
   cudaEvent_t ev[kEventRing][kMaxPhases + 1] = {{nullptr}};
   bool ev_created = false;
+  uint64_t ws_gen = 0;  // bumped whenever the workspace is reallocated
+
+  // The resident path's launch sequence, captured once per hyperbatch shape
+  // and replayed as one CUDA graph launch (agnes_set_graph_mode).
+  struct LaunchGraph {
+    bool enabled = true;
+    cudaStream_t cap = nullptr;  // private stream the sequence is captured on
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    // what the capture depends on
+    int32_t H = 0, B = 0, K = 0, fan[AGNES_MAX_HOPS] = {0}, frontier_mode = 0;
+    bool profiling = false;
+    uint64_t ws_gen = 0;
+    // phase-event nodes, re-pointed at each launch's ring slot
+    cudaGraphNode_t phase_node[kMaxPhases + 1] = {nullptr};
+    int n_marks = 0;
+    int64_t captures = 0, launches = 0;
+  } lg;
 
   // streaming of host-resident features (features_on_host)
   cudaStream_t copy_stream = nullptr;
@@ -275,11 +294,15 @@ static bool is_pinned_host_ptr(const void* p) {
   return attr.type == cudaMemoryTypeHost;
 }
 
-__global__ static void fill_i32_kernel(int32_t* p, int64_t n, int32_t v) {
+namespace agnes {
+namespace {
+__global__ void fill_i32_kernel(int32_t* p, int64_t n, int32_t v) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
     p[i] = v;
 }
+}  // namespace
+}  // namespace agnes
 
 static void free_workspace(Workspace* w) {
   cudaFree(w->nodes);
@@ -319,6 +342,7 @@ static void free_workspace(Workspace* w) {
   cudaFree(w->scan_scratch);
   cudaFree(w->status);
   cudaFree(w->distinct);
+  cudaFree(w->key);
   if (w->h_back) cudaFreeHost(w->h_back);
   *w = Workspace();
 }
@@ -336,6 +360,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   if (same) return AGNES_OK;
   cudaDeviceSynchronize();
   free_workspace(&w);
+  ctx->ws_gen += 1;  // launch sequences captured over the old buffers are stale
   w.H = H;
   w.B = B;
   w.K = K;
@@ -414,6 +439,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.scan_scratch, scratch);
   WA(w.status, 1);
   WA(w.distinct, 1);
+  WA(w.key, 2);
 #undef WA
   w.h_back_bytes = sizeof(int32_t) * (1 + (size_t)(K + 1) * H + 2 * (size_t)K * H + 1) +
                    sizeof(int64_t) * (K + 2);
@@ -492,6 +518,14 @@ static agnes_status wait_prepared(agnes_ctx* ctx) {
 // Public API
 // ============================================================================
 
+static void drop_launch_graph(agnes_ctx::LaunchGraph* g) {
+  if (g->exec) cudaGraphExecDestroy(g->exec);
+  if (g->graph) cudaGraphDestroy(g->graph);
+  g->exec = nullptr;
+  g->graph = nullptr;
+  g->n_marks = 0;
+}
+
 extern "C" {
 
 const char* agnes_status_string(agnes_status s) {
@@ -514,6 +548,8 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (!ctx) return AGNES_OK;
   cudaSetDevice(ctx->device);
   cudaDeviceSynchronize();
+  drop_launch_graph(&ctx->lg);
+  if (ctx->lg.cap) cudaStreamDestroy(ctx->lg.cap);
   free_workspace(&ctx->ws);
   free_block_tables(&ctx->bt);
   if (ctx->own_offsets) cudaFree(ctx->offsets);
@@ -1271,73 +1307,24 @@ static agnes_status gather_streamed(agnes_ctx* ctx, int cur, cudaStream_t st) {
   return AGNES_OK;
 }
 
-agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, int32_t H,
-                                      int32_t B, const int32_t* fanouts, int32_t K,
-                                      uint64_t seed, uint64_t first_minibatch_id,
-                                      void* cuda_stream) {
-  if (!ctx) {
-    set_err(nullptr, "ctx is NULL");
-    return AGNES_EINVAL;
-  }
-  if (!targets || !fanouts) {
-    set_err(ctx, "targets and fanouts must be non-NULL");
-    return AGNES_EINVAL;
-  }
-  if (H < 1 || H > 65535 || B < 1 || K < 1 || K > AGNES_MAX_HOPS) {
-    set_err(ctx, "need 1 <= H <= 65535, B >= 1, 1 <= K <= %d", AGNES_MAX_HOPS);
-    return AGNES_EINVAL;
-  }
-  if (B > ctx->N) {
-    set_err(ctx, "B = %d distinct targets exceed N = %lld", B, (long long)ctx->N);
-    return AGNES_EINVAL;
-  }
-  int64_t cap[AGNES_MAX_HOPS + 1];
-  cap[0] = B;
-  for (int h = 0; h < K; ++h) {
-    if (fanouts[h] < 1 || fanouts[h] > AGNES_MAX_FANOUT) {
-      set_err(ctx, "fanouts[%d] = %d outside [1, %d]", h, fanouts[h], AGNES_MAX_FANOUT);
-      return AGNES_EINVAL;
-    }
-    const int64_t grown = cap[h] * (1 + (int64_t)fanouts[h]);
-    cap[h + 1] = grown < ctx->N ? grown : ctx->N;
-  }
-  const int64_t lim = ((int64_t)1 << 31) - 1;
-  for (int h = 0; h < K; ++h) {
-    if ((int64_t)H * cap[h] * fanouts[h] > lim) {
-      set_err(ctx, "H x edge capacity of hop %d exceeds 2^31", h + 1);
-      return AGNES_ERANGE;
-    }
-  }
-  if ((int64_t)H * cap[K] > lim) {
-    set_err(ctx, "H x node capacity (%lld) exceeds 2^31", (long long)(H * cap[K]));
-    return AGNES_ERANGE;
-  }
-  if (cudaSetDevice(ctx->device) != cudaSuccess) {
-    cudaGetLastError();
-    set_err(ctx, "cudaSetDevice failed");
-    return AGNES_ECUDA;
-  }
-  agnes_status rc = ensure_workspace(ctx, H, B, fanouts, K, cap);
-  if (rc != AGNES_OK) return rc;
-
+// Enqueues one hyperbatch on st whose targets are already in w.nodes and whose
+// sampling key is in w.key: the bucketing of the targets, K hops of sampling
+// and dedup, the feature gather, the statistics and the size read-back.
+// mark_flags is cudaEventRecordExternal while the sequence is being captured,
+// so the phase events become event-record nodes of the graph; *n_marks gets
+// the number of phase events recorded.
+static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, int32_t K,
+                                       const int64_t* cap, int ring, unsigned mark_flags,
+                                       cudaStream_t st, int* n_marks) {
+  agnes_status rc = AGNES_OK;
   Workspace& w = ctx->ws;
-  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const int32_t H = w.H, B = w.B;
   const int32_t T = (int32_t)ctx->bt.T;
   const int64_t cells = (int64_t)T * H;
   const int nsm = ctx->num_sms;
-  ctx->prepared = false;
-  ctx->synced = false;
-
-  if (ctx->profiling && !ctx->ev_created) {
-    for (int r = 0; r < kEventRing; ++r)
-      for (int i = 0; i <= kMaxPhases; ++i) CK(ctx, cudaEventCreate(&ctx->ev[r][i]));
-    ctx->ev_created = true;
-  }
-  const int ring = (int)(ctx->n_prepared % kEventRing);
-  ctx->n_phases[ring] = 0;
   int ph = 0;
   auto mark = [&]() {
-    if (ctx->profiling) cudaEventRecord(ctx->ev[ring][ph++], st);
+    if (ctx->profiling) cudaEventRecordWithFlags(ctx->ev[ring][ph++], st, mark_flags);
   };
 
   mark();
@@ -1346,8 +1333,6 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   CK(ctx, cudaMemsetAsync(w.adj_flags, 0, (size_t)K * ctx->bt.n_blocks, st));
   CK(ctx, cudaMemsetAsync(w.feat_flags, 0, (size_t)ctx->bt.n_feat_blocks, st));
   CK(ctx, cudaMemsetAsync(w.stats, 0, sizeof(int64_t) * (K + 1), st));
-  CK(ctx, cudaMemcpy2DAsync(w.nodes, sizeof(int32_t) * w.capK, targets, sizeof(int32_t) * B,
-                            sizeof(int32_t) * B, H, cudaMemcpyDefault, st));
   fill_i32_kernel<<<(H + 255) / 256, 256, 0, st>>>(w.nsz, H, B);
   CK(ctx, cudaGetLastError());
   CK(ctx, launch_bucket_targets(w.nodes, w.capK, H, B, (int32_t)ctx->N, ctx->bt.tile_first,
@@ -1370,8 +1355,7 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     a.ecap = cap[h] * fanouts[h];
     a.k = fanouts[h];
     a.hop = h + 1;
-    a.seed = seed;
-    a.first_gid = first_minibatch_id;
+    a.key = w.key;
     a.status = w.status;
     int32_t* nsz_prev = w.nsz + (int64_t)h * H;
     int32_t* ecnt = w.ecnt + (int64_t)h * H;
@@ -1445,13 +1429,181 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   CK(ctx, cudaMemcpyAsync(b.ecnt, w.ecnt, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.srcsz, w.srcsz, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.stats, w.stats, sizeof(int64_t) * (K + 1), cudaMemcpyDeviceToHost, st));
-  CK(ctx, cudaEventRecord(ctx->done, st));
-  ctx->n_phases[ring] = ctx->profiling ? ph - 1 : 0;
+  *n_marks = ph;
+  return AGNES_OK;
+}
+
+
+// Whether work enqueued on st is being captured (by the caller's own graph
+// capture); an unknown state counts as captured, so the sequence is enqueued
+// as it is.
+static bool stream_capturing(cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    return true;
+  }
+  return cs != cudaStreamCaptureStatusNone;
+}
+
+// The resident path as one graph launch.  The launch sequence is captured on
+// a private stream the first time a hyperbatch shape (H, B, fanouts, frontier
+// mode, profiling, workspace) is seen, and replayed for every later hyperbatch
+// of that shape: everything that varies between them (the targets, the seed,
+// the minibatch ids) is in device memory by then.  With profiling on, the
+// captured phase-event nodes are pointed at this prepare's ring slot.
+static agnes_status launch_graphed(agnes_ctx* ctx, const int32_t* fanouts, int32_t K,
+                                   const int64_t* cap, int ring, cudaStream_t st,
+                                   int* n_marks) {
+  agnes_ctx::LaunchGraph& g = ctx->lg;
+  const Workspace& w = ctx->ws;
+  bool same = g.exec && g.H == w.H && g.B == w.B && g.K == K &&
+              g.frontier_mode == ctx->frontier_mode && g.profiling == ctx->profiling &&
+              g.ws_gen == ctx->ws_gen;
+  for (int h = 0; same && h < K; ++h) same = g.fan[h] == fanouts[h];
+  if (!same) {
+    drop_launch_graph(&g);
+    if (!g.cap) CK(ctx, cudaStreamCreateWithFlags(&g.cap, cudaStreamNonBlocking));
+    CK(ctx, cudaStreamBeginCapture(g.cap, cudaStreamCaptureModeRelaxed));
+    int nm = 0;
+    const agnes_status rc =
+        enqueue_hyperbatch(ctx, fanouts, K, cap, ring, cudaEventRecordExternal, g.cap, &nm);
+    cudaGraph_t graph = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(g.cap, &graph);
+    if (rc != AGNES_OK || e != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      cudaGetLastError();
+      if (rc != AGNES_OK) return rc;
+      set_err(ctx, "capturing the launch sequence failed: %s", cudaGetErrorString(e));
+      return AGNES_ECUDA;
+    }
+    g.graph = graph;
+    CK(ctx, cudaGraphInstantiate(&g.exec, graph, 0));
+    if (ctx->profiling) {
+      size_t n = 0;
+      CK(ctx, cudaGraphGetNodes(graph, nullptr, &n));
+      std::vector<cudaGraphNode_t> nodes(n);
+      CK(ctx, cudaGraphGetNodes(graph, nodes.data(), &n));
+      for (int i = 0; i < nm; ++i) g.phase_node[i] = nullptr;
+      for (cudaGraphNode_t nd : nodes) {
+        cudaGraphNodeType t;
+        CK(ctx, cudaGraphNodeGetType(nd, &t));
+        if (t != cudaGraphNodeTypeEventRecord) continue;
+        cudaEvent_t ev = nullptr;
+        CK(ctx, cudaGraphEventRecordNodeGetEvent(nd, &ev));
+        for (int i = 0; i < nm; ++i)
+          if (ctx->ev[ring][i] == ev) g.phase_node[i] = nd;
+      }
+      for (int i = 0; i < nm; ++i) {
+        if (!g.phase_node[i]) {
+          drop_launch_graph(&g);
+          set_err(ctx, "phase event %d is missing from the captured launch sequence", i);
+          return AGNES_ECUDA;
+        }
+      }
+    }
+    g.n_marks = nm;
+    g.H = w.H;
+    g.B = w.B;
+    g.K = K;
+    for (int h = 0; h < K; ++h) g.fan[h] = fanouts[h];
+    g.frontier_mode = ctx->frontier_mode;
+    g.profiling = ctx->profiling;
+    g.ws_gen = ctx->ws_gen;
+    g.captures += 1;
+  }
+  if (g.profiling)
+    for (int i = 0; i < g.n_marks; ++i)
+      CK(ctx, cudaGraphExecEventRecordNodeSetEvent(g.exec, g.phase_node[i], ctx->ev[ring][i]));
+  CK(ctx, cudaGraphLaunch(g.exec, st));
+  g.launches += 1;
+  *n_marks = g.n_marks;
+  return AGNES_OK;
+}
+
+agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, int32_t H,
+                                      int32_t B, const int32_t* fanouts, int32_t K,
+                                      uint64_t seed, uint64_t first_minibatch_id,
+                                      void* cuda_stream) {
+  if (!ctx) {
+    set_err(nullptr, "ctx is NULL");
+    return AGNES_EINVAL;
+  }
+  if (!targets || !fanouts) {
+    set_err(ctx, "targets and fanouts must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  if (H < 1 || H > 65535 || B < 1 || K < 1 || K > AGNES_MAX_HOPS) {
+    set_err(ctx, "need 1 <= H <= 65535, B >= 1, 1 <= K <= %d", AGNES_MAX_HOPS);
+    return AGNES_EINVAL;
+  }
+  if (B > ctx->N) {
+    set_err(ctx, "B = %d distinct targets exceed N = %lld", B, (long long)ctx->N);
+    return AGNES_EINVAL;
+  }
+  int64_t cap[AGNES_MAX_HOPS + 1];
+  cap[0] = B;
+  for (int h = 0; h < K; ++h) {
+    if (fanouts[h] < 1 || fanouts[h] > AGNES_MAX_FANOUT) {
+      set_err(ctx, "fanouts[%d] = %d outside [1, %d]", h, fanouts[h], AGNES_MAX_FANOUT);
+      return AGNES_EINVAL;
+    }
+    const int64_t grown = cap[h] * (1 + (int64_t)fanouts[h]);
+    cap[h + 1] = grown < ctx->N ? grown : ctx->N;
+  }
+  const int64_t lim = ((int64_t)1 << 31) - 1;
+  for (int h = 0; h < K; ++h) {
+    if ((int64_t)H * cap[h] * fanouts[h] > lim) {
+      set_err(ctx, "H x edge capacity of hop %d exceeds 2^31", h + 1);
+      return AGNES_ERANGE;
+    }
+  }
+  if ((int64_t)H * cap[K] > lim) {
+    set_err(ctx, "H x node capacity (%lld) exceeds 2^31", (long long)(H * cap[K]));
+    return AGNES_ERANGE;
+  }
+  if (cudaSetDevice(ctx->device) != cudaSuccess) {
+    cudaGetLastError();
+    set_err(ctx, "cudaSetDevice failed");
+    return AGNES_ECUDA;
+  }
+  agnes_status rc = ensure_workspace(ctx, H, B, fanouts, K, cap);
+  if (rc != AGNES_OK) return rc;
+  Workspace& w = ctx->ws;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  ctx->prepared = false;
+  ctx->synced = false;
+  if (ctx->profiling && !ctx->ev_created) {
+    for (int r = 0; r < kEventRing; ++r)
+      for (int i = 0; i <= kMaxPhases; ++i) CK(ctx, cudaEventCreate(&ctx->ev[r][i]));
+    ctx->ev_created = true;
+  }
+  const int ring = (int)(ctx->n_prepared % kEventRing);
+  ctx->n_phases[ring] = 0;
+  // a prepare on another stream than the last one still runs after it: both
+  // use the ctx's buffers (a caller's own capture orders its replays itself)
+  const bool capturing = stream_capturing(st);
+  if (ctx->n_prepared > 0 && !capturing) CK(ctx, cudaStreamWaitEvent(st, ctx->done, 0));
+  CK(ctx, cudaMemcpy2DAsync(w.nodes, sizeof(int32_t) * w.capK, targets, sizeof(int32_t) * B,
+                            sizeof(int32_t) * B, H, cudaMemcpyDefault, st));
+  CK(ctx, launch_set_key(w.key, seed, first_minibatch_id, st));
+  int n_marks = 0;
+  const bool resident = !ctx->features_on_host && !ctx->topo.on;
+  if (resident && ctx->lg.enabled && !capturing)
+    rc = launch_graphed(ctx, fanouts, K, cap, ring, st, &n_marks);
+  else
+    rc = enqueue_hyperbatch(ctx, fanouts, K, cap, ring, cudaEventRecordDefault, st, &n_marks);
+  if (rc != AGNES_OK) return rc;
+  // inside a caller's capture nothing has run yet: the caller orders its
+  // replays, and there are no phase times to read
+  if (!capturing) CK(ctx, cudaEventRecord(ctx->done, st));
+  ctx->n_phases[ring] = ctx->profiling && !capturing ? n_marks - 1 : 0;
   ctx->n_prepared += 1;
-  ctx->cur = cur;
+  ctx->cur = K & 1;  // the frontier buffers swap once per hop
   ctx->prepared = true;
   return AGNES_OK;
 }
+
 
 agnes_status agnes_fetch_minibatch(agnes_ctx* ctx, int32_t j, agnes_minibatch_view* out) {
   if (!ctx || !out) {
@@ -1490,6 +1642,16 @@ agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode) {
     return AGNES_EINVAL;
   }
   ctx->frontier_mode = mode;
+  return AGNES_OK;
+}
+
+agnes_status agnes_set_graph_mode(agnes_ctx* ctx, int32_t enabled) {
+  if (!ctx) return AGNES_EINVAL;
+  if (enabled != 0 && enabled != 1) {
+    set_err(ctx, "graph mode must be 0 or 1");
+    return AGNES_EINVAL;
+  }
+  ctx->lg.enabled = enabled == 1;
   return AGNES_OK;
 }
 
@@ -1571,6 +1733,8 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
   out->topo_waves = ctx->topo.waves;
   out->fcache_hit_blocks = ctx->fcache_hits;
   out->fcache_loaded_blocks = ctx->fcache_loads;
+  out->graph_captures = ctx->lg.captures;
+  out->graph_launches = ctx->lg.launches;
   return AGNES_OK;
 }
 

@@ -80,10 +80,13 @@ struct HopArgs {
   int64_t ecap;      // edge capacity per minibatch at this hop
   int32_t k;         // fanout
   int32_t hop;       // 1-based
-  uint64_t seed;
-  uint64_t first_gid;
+  const uint64_t* key;  // device: {seed, first minibatch id} (launch_set_key)
   int32_t* status;
 };
+
+// Writes the sampling key {seed, first minibatch id} to device memory ahead
+// of a hyperbatch (one 1-thread kernel: the arguments travel with the launch).
+cudaError_t launch_set_key(uint64_t* key, uint64_t seed, uint64_t first_gid, cudaStream_t st);
 
 cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32_t B, int32_t N,
                                   const int32_t* tile_first, const int32_t* chunk_tile, int32_t T,

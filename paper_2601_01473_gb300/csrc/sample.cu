@@ -206,10 +206,21 @@ struct FillArgs {
   int32_t* nbr;
   int64_t capK, cap_prev, ecap;
   int32_t k, hop;
-  uint32_t key_lo, key_hi;
-  uint64_t first_gid;
+  const uint64_t* key;  // device: {seed, first minibatch id}
   int32_t* status;
 };
+
+// The sampling key, read from device memory once per thread, so that one
+// captured launch sequence serves every seed and minibatch id.
+struct Key {
+  uint32_t lo, hi;
+  uint64_t gid0;
+};
+
+__device__ __forceinline__ Key load_key(const uint64_t* key) {
+  const uint64_t seed = __ldg(key);
+  return Key{(uint32_t)seed, (uint32_t)(seed >> 32), __ldg(key + 1)};
+}
 
 // Neighbour at position pos of node v (edges off_v .. off_v + deg).  With
 // streamed topology the edge sits in the graph-buffer slot of its physical
@@ -229,12 +240,12 @@ __device__ __forceinline__ int32_t edge_at(const FillArgs& a, int32_t v, int64_t
   return __ldg(a.gbuf + (int64_t)slot * a.epb + (off_v + pos - __ldg(a.blk_e0 + b)));
 }
 
-__device__ __forceinline__ int64_t draw(const FillArgs& a, int32_t v, int32_t s, uint64_t gid,
-                                        int64_t J) {
+__device__ __forceinline__ int64_t draw(const FillArgs& a, const Key& key, int32_t v, int32_t s,
+                                        uint64_t gid, int64_t J) {
   const uint4 x = philox4x32_10(
       make_uint4((uint32_t)v, ((uint32_t)a.hop << 24) | (uint32_t)s, (uint32_t)gid,
                  (uint32_t)(gid >> 32)),
-      make_uint2(a.key_lo, a.key_hi));
+      make_uint2(key.lo, key.hi));
   const uint64_t r = ((uint64_t)x.y << 32) | (uint64_t)x.x;
   return (int64_t)__umul64hi(r, (uint64_t)(J + 1));
 }
@@ -261,6 +272,7 @@ template <typename OffT, int G, bool kStreamed>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
   if (failed(a.status)) return;
+  const Key key = load_key(a.key);
   const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
   constexpr int kGroups = 32 / G;
   const int lane = lane_id();
@@ -290,7 +302,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
         }
       } else {
         const int64_t J = d - a.k + s;
-        const int64_t t = s < a.k ? draw(a, v, s, a.first_gid + j, J) : -1;
+        const int64_t t = s < a.k ? draw(a, key, v, s, key.gid0 + j, J) : -1;
         bool collided = false;
         for (int q = 0; q < a.k; ++q) {
           const int64_t mine = collided ? J : t;
@@ -317,6 +329,7 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
   __shared__ int32_t chosen_s[kWarps][kMaxFanout];
   const int warp = threadIdx.x >> 5, lane = lane_id();
   int32_t* chosen = chosen_s[warp];
+  const Key key = load_key(a.key);
   const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
   const uint32_t capk32 = (uint32_t)a.capK;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -341,7 +354,7 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
       const int s = c0 + lane;
       const bool valid = s < a.k;
       const int64_t J = d - a.k + s;
-      const int64_t t = valid ? draw(a, v, s, a.first_gid + j, J) : -1;
+      const int64_t t = valid ? draw(a, key, v, s, key.gid0 + j, J) : -1;
       bool collided = false;
       for (int q = 0; q < c0; ++q) collided |= (chosen[q] == t);
       const int m = min(32, a.k - c0);
@@ -379,6 +392,16 @@ cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32
   targets_sort_kernel<<<resident_grid((const void*)targets_sort_kernel, kThreads, num_sms),
                         kThreads, 0, st>>>(fcell_off, ncells, H, tm, tmp_id, tmp_pos,
                                                  fb_id, fb_pos, status);
+  return cudaGetLastError();
+}
+
+static __global__ void set_key_kernel(uint64_t* key, uint64_t seed, uint64_t first_gid) {
+  key[0] = seed;
+  key[1] = first_gid;
+}
+
+cudaError_t launch_set_key(uint64_t* key, uint64_t seed, uint64_t first_gid, cudaStream_t st) {
+  set_key_kernel<<<1, 1, 0, st>>>(key, seed, first_gid);
   return cudaGetLastError();
 }
 
@@ -447,9 +470,7 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.ecap = a.ecap;
   f.k = a.k;
   f.hop = a.hop;
-  f.key_lo = (uint32_t)a.seed;
-  f.key_hi = (uint32_t)(a.seed >> 32);
-  f.first_gid = a.first_gid;
+  f.key = a.key;
   f.status = a.status;
   const bool streamed = r.gbuf != nullptr;
   if (a.offsets_bits == 32) {
