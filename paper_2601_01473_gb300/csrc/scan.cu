@@ -22,6 +22,7 @@ constexpr int kChunk = kThreads * kItems;  // elements per block and chunk
 // kMaxSegments) first, kept at zero between scans, then the chunk sums.
 constexpr int64_t kMaxSegments = 65536;
 constexpr int64_t kTicketElems = kMaxSegments / 2;  // int64 slots holding the uint32 tickets
+constexpr int64_t kGridBlocks = 2048;  // blocks of a segmented scan (at least one per segment)
 
 __device__ __forceinline__ int64_t seg_len(const int32_t* d_len, int64_t const_len, int s) {
   return d_len ? (int64_t)d_len[s] : const_len;
@@ -83,7 +84,11 @@ __device__ __forceinline__ int64_t cta_scan_inplace(int64_t* p, int64_t n, int64
 
 // Chunk sums; the last chunk of a segment to finish (atomic ticket after a
 // fence, no waiting) then scans the segment's chunk sums in place, writes
-// the segment total, and resets the ticket for the next scan.
+// the segment total, and resets the ticket for the next scan.  Only the
+// chunks that hold elements of the segment take part (at least one, which
+// writes the total of an empty segment); a block takes chunks blockIdx.x,
+// blockIdx.x + gridDim.x, ... so the grid need not cover a segment's whole
+// capacity.
 template <typename InT, typename OutT>
 __global__ void __launch_bounds__(kThreads)
 scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t* d_len,
@@ -92,43 +97,48 @@ scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t*
                    bool write_end, int32_t* seg_total, const int32_t* status) {
   if (status && failed(status)) return;
   const int s = blockIdx.y;
-  const int64_t c = blockIdx.x;
   const int64_t len = seg_len(d_len, const_len, s);
-  const int64_t begin = c * kChunk;
-  int64_t sum = 0;
-  if (begin < len) {  // all of the thread's loads in flight at once
-    const InT* p = in + (int64_t)s * in_stride;
-    InT v[kItems];
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-      const int64_t i = begin + k * kThreads + threadIdx.x;
-      v[k] = i < len ? p[i] : (InT)0;
-    }
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) sum += (int64_t)v[k];
-  }
+  int64_t nvalid = len > 0 ? (len + kChunk - 1) / kChunk : 1;
+  if (nvalid > chunks) nvalid = chunks;
   __shared__ int64_t wsum[kThreads / 32];
   __shared__ bool last;
-  sum = warp_sum(sum);
-  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = sum;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    int64_t v = threadIdx.x < kThreads / 32 ? wsum[threadIdx.x] : 0;
-    v = warp_sum(v);
-    if (threadIdx.x == 0) {
-      partial[(int64_t)s * chunks + c] = v;
-      __threadfence();
-      last = atomicAdd(tickets + s, 1u) == (unsigned)(chunks - 1);
+  for (int64_t c = blockIdx.x; c < nvalid; c += gridDim.x) {
+    const int64_t begin = c * kChunk;
+    int64_t sum = 0;
+    if (begin < len) {  // all of the thread's loads in flight at once
+      const InT* p = in + (int64_t)s * in_stride;
+      InT v[kItems];
+#pragma unroll
+      for (int k = 0; k < kItems; ++k) {
+        const int64_t i = begin + k * kThreads + threadIdx.x;
+        v[k] = i < len ? p[i] : (InT)0;
+      }
+#pragma unroll
+      for (int k = 0; k < kItems; ++k) sum += (int64_t)v[k];
     }
-  }
-  __syncthreads();
-  if (!last) return;
-  __threadfence();
-  const int64_t carry = cta_scan_inplace(partial + (int64_t)s * chunks, chunks, 1, true);
-  if (threadIdx.x == 0) {
-    if (write_end) out[(int64_t)s * out_stride + len] = (OutT)carry;
-    if (seg_total) seg_total[s] = (int32_t)carry;
-    tickets[s] = 0;
+    sum = warp_sum(sum);
+    if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = sum;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      int64_t v = threadIdx.x < kThreads / 32 ? wsum[threadIdx.x] : 0;
+      v = warp_sum(v);
+      if (threadIdx.x == 0) {
+        partial[(int64_t)s * chunks + c] = v;
+        __threadfence();
+        last = atomicAdd(tickets + s, 1u) == (unsigned)(nvalid - 1);
+      }
+    }
+    __syncthreads();
+    if (last) {  // the segment's final chunk: no later chunk of this block remains
+      __threadfence();
+      const int64_t carry = cta_scan_inplace(partial + (int64_t)s * chunks, nvalid, 1, true);
+      if (threadIdx.x == 0) {
+        if (write_end) out[(int64_t)s * out_stride + len] = (OutT)carry;
+        if (seg_total) seg_total[s] = (int32_t)carry;
+        tickets[s] = 0;
+      }
+    }
+    __syncthreads();  // wsum and last are rewritten by the next chunk
   }
 }
 
@@ -141,43 +151,43 @@ scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict
                  const int64_t* __restrict__ partial, const int32_t* status) {
   if (status && failed(status)) return;
   const int s = blockIdx.y;
-  const int64_t c = blockIdx.x;
   const int64_t len = seg_len(d_len, const_len, s);
-  const int64_t begin = c * kChunk;
-  if (begin >= len) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t wbase = begin + (int64_t)warp * (32 * kItems);
   const InT* p = in + (int64_t)s * in_stride;
   OutT* q = out + (int64_t)s * out_stride;
-  const int64_t chunk_off = partial[(int64_t)s * chunks + c];  // issued with the loads below
-  int64_t v[kItems];
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    const int64_t i = wbase + k * 32 + lane;
-    v[k] = i < len ? (int64_t)p[i] : 0;
-  }
-  int64_t carry = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    const int64_t inc = warp_incl_scan(v[k]);
-    const int64_t x = v[k];
-    v[k] = carry + inc - x;
-    carry += __shfl_sync(0xffffffffu, inc, 31);
-  }
   __shared__ int64_t wtot[kThreads / 32];
-  if (lane == 0) wtot[warp] = carry;
-  __syncthreads();
-  if (warp == 0) {
-    const int64_t w = lane < kThreads / 32 ? wtot[lane] : 0;
-    const int64_t wi = warp_incl_scan(w);
-    if (lane < kThreads / 32) wtot[lane] = wi - w;
-  }
-  __syncthreads();
-  const int64_t off = chunk_off + wtot[warp];
+  for (int64_t c = blockIdx.x; c * kChunk < len; c += gridDim.x) {
+    const int64_t wbase = c * kChunk + (int64_t)warp * (32 * kItems);
+    const int64_t chunk_off = partial[(int64_t)s * chunks + c];  // issued with the loads below
+    int64_t v[kItems];
 #pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    const int64_t i = wbase + k * 32 + lane;
-    if (i < len) q[i] = (OutT)(off + v[k]);
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t i = wbase + k * 32 + lane;
+      v[k] = i < len ? (int64_t)p[i] : 0;
+    }
+    int64_t carry = 0;
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t inc = warp_incl_scan(v[k]);
+      const int64_t x = v[k];
+      v[k] = carry + inc - x;
+      carry += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    if (lane == 0) wtot[warp] = carry;
+    __syncthreads();
+    if (warp == 0) {
+      const int64_t w = lane < kThreads / 32 ? wtot[lane] : 0;
+      const int64_t wi = warp_incl_scan(w);
+      if (lane < kThreads / 32) wtot[lane] = wi - w;
+    }
+    __syncthreads();
+    const int64_t off = chunk_off + wtot[warp];
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t i = wbase + k * 32 + lane;
+      if (i < len) q[i] = (OutT)(off + v[k]);
+    }
+    __syncthreads();  // wtot is rewritten by the next chunk
   }
 }
 
@@ -287,7 +297,13 @@ cudaError_t seg_scan(const InT* in, int64_t in_stride, OutT* out, int64_t out_st
   if (nseg <= 0) return cudaSuccess;
   int64_t chunks = (max_len + kChunk - 1) / kChunk;
   if (chunks < 1) chunks = 1;
-  const dim3 grid((unsigned)chunks, (unsigned)nseg);
+  // Segments of a per-minibatch scan are usually far shorter than their
+  // capacity max_len: about kGridBlocks blocks in all, each looping over its
+  // segment's chunks, instead of a block per chunk of capacity.
+  int64_t gx = kGridBlocks / nseg;
+  if (gx < 1) gx = 1;
+  if (gx > chunks) gx = chunks;
+  const dim3 grid((unsigned)gx, (unsigned)nseg);
   if (nseg > kMaxSegments) return cudaErrorInvalidValue;
   unsigned int* tickets = (unsigned int*)scratch;
   int64_t* partial = scratch + kTicketElems;
