@@ -266,6 +266,9 @@ def main():
                     help="time the GraphSAGE-mean consumer layer on a prepared hyperbatch")
     ap.add_argument("--sage-d-out", type=int, default=128)
     ap.add_argument("--sage-out", default="f32", choices=["f32", "f16"])
+    ap.add_argument("--launch-mode", default="graph_pdl", choices=["direct", "graph", "graph_pdl"],
+                    help="resident path: direct launches, one CUDA graph per hyperbatch shape, "
+                         "or the graph with programmatic kernel edges")
     ap.add_argument("--feature-io", default="blocks", choices=["blocks", "rows"],
                     help="with --stream: load whole feature blocks, or read requested rows in place")
     args = ap.parse_args()
@@ -328,6 +331,7 @@ def main():
               feature_cache_bytes=int(args.feature_cache_gb * 2**30) if args.stream else 0,
               feature_cache_threshold=args.feature_cache_threshold,
               feature_io=args.feature_io if args.stream else "blocks")
+    g.set_launch_mode(args.launch_mode)
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
@@ -475,6 +479,7 @@ def main():
                                  "adj_blocks": info["adj_blocks"], "tiles": info["tiles"],
                                  "feat_blocks": info["feat_blocks"]},
                        "H": w.H, "B": w.B, "fanouts": fan, "parallelism": f"replicas{world}",
+                       "launch_mode": args.launch_mode,
                        "l2": "inputs larger than L2 (graph ~%.0f GB vs 129 MB L2), no flush"
                              % ((offsets.numel() * offsets.element_size()
                                  + indices.numel() * 4

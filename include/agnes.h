@@ -191,18 +191,27 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
 agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode);
 
 /* How agnes_prepare_hyperbatch issues its work when features and topology
- * are resident in HBM.  enabled = 1 (default): the hyperbatch's launch
- * sequence (memsets, ~60 kernels, the size read-back) is captured into a
- * CUDA graph on a private stream the first time a shape is seen (H, B,
- * fanouts, frontier mode, profiling) and replayed as one graph launch on the
- * caller's stream for every later hyperbatch of that shape; the targets copy
- * and the sampling key {seed, first_minibatch_id} are written to device
- * memory ahead of it.  enabled = 0: every call launches the sequence
- * directly.  Results are identical either way.  A caller stream that is
- * itself being captured, and the host-resident modes (whose calls read sizes
- * back mid-sequence), always take the direct path.  Takes effect at the next
- * prepare.  Errors: EINVAL (enabled not 0 or 1). */
-agnes_status agnes_set_graph_mode(agnes_ctx* ctx, int32_t enabled);
+ * are resident in HBM (set per ctx; takes effect at the next prepare).
+ * AGNES_LAUNCH_DIRECT: every call launches the sequence (memsets, ~60
+ *   kernels, the size read-back) on the caller's stream.
+ * AGNES_LAUNCH_GRAPH: the sequence is captured into a CUDA graph on a
+ *   private stream the first time a hyperbatch shape is seen (H, B, fanouts,
+ *   frontier mode, profiling) and replayed as one graph launch on the
+ *   caller's stream for every later hyperbatch of that shape; the targets
+ *   copy and the sampling key {seed, first_minibatch_id} are written to
+ *   device memory ahead of it.
+ * AGNES_LAUNCH_GRAPH_PDL (default): as AGNES_LAUNCH_GRAPH, with each
+ *   kernel-to-kernel edge of the graph made programmatic (programmatic
+ *   dependent launch: a kernel is launched once every block of the previous
+ *   one has exited, and first waits for its writes to become visible), so
+ *   each launch overlaps the previous kernel's completion.
+ * Results are identical in every mode.  A caller stream that is itself being
+ * captured, and the host-resident modes (whose calls read sizes back
+ * mid-sequence), always take the direct path.  Errors: EINVAL. */
+#define AGNES_LAUNCH_DIRECT 0
+#define AGNES_LAUNCH_GRAPH 1
+#define AGNES_LAUNCH_GRAPH_PDL 2
+agnes_status agnes_set_launch_mode(agnes_ctx* ctx, int32_t mode);
 
 /* View of minibatch j of the last prepared hyperbatch.  Per hop h (0-based
  * index, hop number h+1): the bipartite block has num_dst[h] dst nodes and
@@ -292,8 +301,9 @@ typedef struct {
   int64_t topo_waves;               /* fill launches over all hops */
   int64_t fcache_hit_blocks;        /* feature blocks read in place from the feature cache */
   int64_t fcache_loaded_blocks;     /* feature blocks copied into the feature cache */
-  int64_t graph_captures;           /* launch sequences captured (agnes_set_graph_mode) */
+  int64_t graph_captures;           /* launch sequences captured (agnes_set_launch_mode) */
   int64_t graph_launches;           /* prepares issued as one graph launch */
+  int64_t graph_programmatic_edges; /* programmatic kernel edges of the current graph */
 } agnes_counters;
 agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
 

@@ -21,6 +21,7 @@ MAX_FANOUT = 1024
 F32, F16 = 0, 1
 FEATURE_IO = {"blocks": 0, "rows": 1}  # AGNES_FEATURE_IO_* and AGNES_TOPOLOGY_IO_* values
 FRONTIER = {"src": 0, "sampled": 1}    # AGNES_FRONTIER_SRC / _SAMPLED
+LAUNCH = {"direct": 0, "graph": 1, "graph_pdl": 2}  # AGNES_LAUNCH_DIRECT / _GRAPH / _GRAPH_PDL
 _DTYPES = {torch.float32: F32, torch.float16: F16}
 _TORCH_OF = {F32: torch.float32, F16: torch.float16}
 
@@ -103,6 +104,7 @@ class _Counters(ctypes.Structure):
         ("fcache_hit_blocks", ctypes.c_int64),
         ("fcache_loaded_blocks", ctypes.c_int64),
         ("graph_captures", ctypes.c_int64), ("graph_launches", ctypes.c_int64),
+        ("graph_programmatic_edges", ctypes.c_int64),
     ]
 
 
@@ -133,7 +135,7 @@ SIGNATURES = {
                           ctypes.c_int),
     "agnes_hop_indptr_noalloc": ([_P, _P, ctypes.c_int64, ctypes.c_int32, _P, _P], ctypes.c_int),
     "agnes_set_frontier_mode": ([_P, ctypes.c_int32], ctypes.c_int),
-    "agnes_set_graph_mode": ([_P, ctypes.c_int32], ctypes.c_int),
+    "agnes_set_launch_mode": ([_P, ctypes.c_int32], ctypes.c_int),
     "agnes_sage_mean_layer": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int64,
                                ctypes.c_int64, _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
                                ctypes.c_int64, _P], ctypes.c_int),
@@ -356,11 +358,14 @@ class Graph:
             raise ValueError(f"frontier must be one of {sorted(FRONTIER)}")
         _check(lib().agnes_set_frontier_mode(self._ctx, FRONTIER[mode]), self._ctx)
 
-    def set_graph_mode(self, enabled: bool) -> None:
-        """Replay the resident path's launch sequence as one captured CUDA
-        graph per hyperbatch shape (True, the default), or launch it directly
-        on every prepare (False); the results are the same."""
-        _check(lib().agnes_set_graph_mode(self._ctx, 1 if enabled else 0), self._ctx)
+    def set_launch_mode(self, mode: str) -> None:
+        """How the resident path is issued: "direct" (every kernel launched by
+        each prepare), "graph" (captured once per hyperbatch shape, replayed as
+        one CUDA graph launch) or "graph_pdl" (the default: the graph with
+        programmatic kernel-to-kernel edges); the results are the same."""
+        if mode not in LAUNCH:
+            raise ValueError(f"launch mode must be one of {sorted(LAUNCH)}")
+        _check(lib().agnes_set_launch_mode(self._ctx, LAUNCH[mode]), self._ctx)
 
     def sage_mean_layer(self, hop: int, x: torch.Tensor, w: torch.Tensor, bias=None,
                         out_dtype: torch.dtype = torch.float32, stream=None) -> torch.Tensor:
@@ -409,7 +414,8 @@ class Graph:
                 "topo_hit_blocks": c.topo_hit_blocks, "topo_waves": c.topo_waves,
                 "fcache_hit_blocks": c.fcache_hit_blocks,
                 "fcache_loaded_blocks": c.fcache_loaded_blocks,
-                "graph_captures": c.graph_captures, "graph_launches": c.graph_launches}
+                "graph_captures": c.graph_captures, "graph_launches": c.graph_launches,
+                "graph_programmatic_edges": c.graph_programmatic_edges}
 
     def info(self) -> dict:
         g = _GraphInfo()

@@ -121,20 +121,20 @@ struct agnes_ctx {
   uint64_t ws_gen = 0;  // bumped whenever the workspace is reallocated
 
   // The resident path's launch sequence, captured once per hyperbatch shape
-  // and replayed as one CUDA graph launch (agnes_set_graph_mode).
+  // and replayed as one CUDA graph launch (agnes_set_launch_mode).
   struct LaunchGraph {
-    bool enabled = true;
+    int32_t mode = AGNES_LAUNCH_GRAPH_PDL;
     cudaStream_t cap = nullptr;  // private stream the sequence is captured on
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
     // what the capture depends on
-    int32_t H = 0, B = 0, K = 0, fan[AGNES_MAX_HOPS] = {0}, frontier_mode = 0;
+    int32_t H = 0, B = 0, K = 0, fan[AGNES_MAX_HOPS] = {0}, frontier_mode = 0, built_mode = 0;
     bool profiling = false;
     uint64_t ws_gen = 0;
     // phase-event nodes, re-pointed at each launch's ring slot
     cudaGraphNode_t phase_node[kMaxPhases + 1] = {nullptr};
     int n_marks = 0;
-    int64_t captures = 0, launches = 0;
+    int64_t captures = 0, launches = 0, programmatic_edges = 0;
   } lg;
 
   // streaming of host-resident features (features_on_host)
@@ -297,6 +297,7 @@ static bool is_pinned_host_ptr(const void* p) {
 namespace agnes {
 namespace {
 __global__ void fill_i32_kernel(int32_t* p, int64_t n, int32_t v) {
+  grid_dep_wait();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
     p[i] = v;
@@ -1446,6 +1447,42 @@ static bool stream_capturing(cudaStream_t st) {
   return cs != cudaStreamCaptureStatusNone;
 }
 
+// Turns every kernel-to-kernel edge of the captured sequence into a
+// programmatic one from the programmatic port: the kernels trigger nothing
+// early, so the next kernel is launched as soon as every block of its
+// predecessor has exited, and its blocks wait at their first statement
+// (grid_dep_wait) for the predecessor's writes to become visible; the launch
+// overlaps the predecessor's completion instead of following it.  (Launching
+// once all predecessor blocks had merely started was measured slower: the
+// waiting blocks took SM slots from the running kernel's tail.)  Edges
+// touching other nodes (memsets, copies, event records) keep full
+// serialisation.
+static cudaError_t make_programmatic(cudaGraph_t graph, int64_t* converted) {
+  size_t n = 0;
+  cudaError_t e = cudaGraphGetEdges(graph, nullptr, nullptr, nullptr, &n);
+  if (e != cudaSuccess || n == 0) return e;
+  std::vector<cudaGraphNode_t> from(n), to(n);
+  std::vector<cudaGraphEdgeData> data(n);
+  e = cudaGraphGetEdges(graph, from.data(), to.data(), data.data(), &n);
+  if (e != cudaSuccess) return e;
+  for (size_t i = 0; i < n; ++i) {
+    cudaGraphNodeType tf, tt;
+    if ((e = cudaGraphNodeGetType(from[i], &tf)) != cudaSuccess) return e;
+    if ((e = cudaGraphNodeGetType(to[i], &tt)) != cudaSuccess) return e;
+    if (tf != cudaGraphNodeTypeKernel || tt != cudaGraphNodeTypeKernel) continue;
+    if (data[i].type != cudaGraphDependencyTypeDefault || data[i].from_port != 0) continue;
+    if ((e = cudaGraphRemoveDependencies(graph, &from[i], &to[i], &data[i], 1)) != cudaSuccess)
+      return e;
+    cudaGraphEdgeData p;
+    memset(&p, 0, sizeof(p));
+    p.from_port = cudaGraphKernelNodePortProgrammatic;
+    p.type = cudaGraphDependencyTypeProgrammatic;
+    if ((e = cudaGraphAddDependencies(graph, &from[i], &to[i], &p, 1)) != cudaSuccess) return e;
+    *converted += 1;
+  }
+  return cudaSuccess;
+}
+
 // The resident path as one graph launch.  The launch sequence is captured on
 // a private stream the first time a hyperbatch shape (H, B, fanouts, frontier
 // mode, profiling, workspace) is seen, and replayed for every later hyperbatch
@@ -1459,7 +1496,7 @@ static agnes_status launch_graphed(agnes_ctx* ctx, const int32_t* fanouts, int32
   const Workspace& w = ctx->ws;
   bool same = g.exec && g.H == w.H && g.B == w.B && g.K == K &&
               g.frontier_mode == ctx->frontier_mode && g.profiling == ctx->profiling &&
-              g.ws_gen == ctx->ws_gen;
+              g.ws_gen == ctx->ws_gen && g.built_mode == g.mode;
   for (int h = 0; same && h < K; ++h) same = g.fan[h] == fanouts[h];
   if (!same) {
     drop_launch_graph(&g);
@@ -1478,6 +1515,8 @@ static agnes_status launch_graphed(agnes_ctx* ctx, const int32_t* fanouts, int32
       return AGNES_ECUDA;
     }
     g.graph = graph;
+    g.programmatic_edges = 0;
+    if (g.mode == AGNES_LAUNCH_GRAPH_PDL) CK(ctx, make_programmatic(graph, &g.programmatic_edges));
     CK(ctx, cudaGraphInstantiate(&g.exec, graph, 0));
     if (ctx->profiling) {
       size_t n = 0;
@@ -1508,6 +1547,7 @@ static agnes_status launch_graphed(agnes_ctx* ctx, const int32_t* fanouts, int32
     g.K = K;
     for (int h = 0; h < K; ++h) g.fan[h] = fanouts[h];
     g.frontier_mode = ctx->frontier_mode;
+    g.built_mode = g.mode;
     g.profiling = ctx->profiling;
     g.ws_gen = ctx->ws_gen;
     g.captures += 1;
@@ -1589,7 +1629,7 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   CK(ctx, launch_set_key(w.key, seed, first_minibatch_id, st));
   int n_marks = 0;
   const bool resident = !ctx->features_on_host && !ctx->topo.on;
-  if (resident && ctx->lg.enabled && !capturing)
+  if (resident && ctx->lg.mode != AGNES_LAUNCH_DIRECT && !capturing)
     rc = launch_graphed(ctx, fanouts, K, cap, ring, st, &n_marks);
   else
     rc = enqueue_hyperbatch(ctx, fanouts, K, cap, ring, cudaEventRecordDefault, st, &n_marks);
@@ -1645,13 +1685,13 @@ agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode) {
   return AGNES_OK;
 }
 
-agnes_status agnes_set_graph_mode(agnes_ctx* ctx, int32_t enabled) {
+agnes_status agnes_set_launch_mode(agnes_ctx* ctx, int32_t mode) {
   if (!ctx) return AGNES_EINVAL;
-  if (enabled != 0 && enabled != 1) {
-    set_err(ctx, "graph mode must be 0 or 1");
+  if (mode != AGNES_LAUNCH_DIRECT && mode != AGNES_LAUNCH_GRAPH && mode != AGNES_LAUNCH_GRAPH_PDL) {
+    set_err(ctx, "launch mode must be AGNES_LAUNCH_DIRECT, _GRAPH or _GRAPH_PDL");
     return AGNES_EINVAL;
   }
-  ctx->lg.enabled = enabled == 1;
+  ctx->lg.mode = mode;
   return AGNES_OK;
 }
 
@@ -1735,6 +1775,7 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
   out->fcache_loaded_blocks = ctx->fcache_loads;
   out->graph_captures = ctx->lg.captures;
   out->graph_launches = ctx->lg.launches;
+  out->graph_programmatic_edges = ctx->lg.programmatic_edges;
   return AGNES_OK;
 }
 

@@ -118,4 +118,11 @@ __device__ __forceinline__ bool failed(const int32_t* status) {
   return *(volatile const int32_t*)status != 0;
 }
 
+// Programmatic dependent launch: a kernel launched ahead of its predecessor's
+// completion (a programmatic graph edge) waits here until the predecessor has
+// finished and its writes are visible.  Every kernel of the hyperbatch path
+// calls it first, unconditionally, so completion stays transitive along the
+// chain; without a programmatic dependency it returns at once.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 }  // namespace agnes

@@ -29,6 +29,7 @@ dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict_
                      int64_t ecap, const int32_t* __restrict__ scell,
                      const int32_t* __restrict__ srank, const int32_t* __restrict__ soff,
                      int2* __restrict__ sb, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int32_t j = blockIdx.y;
   const int64_t E = ecnt[j];
@@ -122,6 +123,7 @@ __device__ __forceinline__ void put_tmp(const CellArgs& a, int32_t at, int32_t i
 }
 
 __global__ void __launch_bounds__(kCellThreads) dedup_cells_kernel(CellArgs a) {
+  grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ GroupSmem sm;
   const int tid = threadIdx.x, lane = lane_id(), warp = tid >> 5;
@@ -300,6 +302,7 @@ __device__ __forceinline__ void mark_bits(const CellArgs& a, const Cell& c, uint
 }
 
 __global__ void __launch_bounds__(kThreads) dedup_big_kernel(CellArgs a) {
+  grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ uint32_t D_s[kWarps][kTileWords];
   __shared__ uint32_t N_s[kWarps][kTileWords];
@@ -415,6 +418,7 @@ __global__ void __launch_bounds__(kThreads)
 dedup_fix_col_kernel(int32_t* __restrict__ col, const int32_t* __restrict__ ecnt, int64_t ecap,
                      const int32_t* __restrict__ scell, const int32_t* __restrict__ newbase,
                      const int32_t* __restrict__ nsz_prev, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int32_t j = blockIdx.y;
   const int64_t E = ecnt[j];
@@ -452,6 +456,7 @@ struct CompactArgs {
 // node (x = -(1 + r)) gets its output row j * capK + |dst_h| + newbase + r and
 // its id is appended to the minibatch's node list.
 __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs a) {
+  grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ int32_t s_nfo[kGroupCells + 1];
   __shared__ int32_t s_src[kGroupCells];   // source base in fb (>= 0) or ~base in tmp

@@ -27,6 +27,7 @@ gather_staged_kernel(const unsigned long long* __restrict__ src, int64_t vecs, i
                      const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
                      const int32_t* __restrict__ cell_off, int64_t cell_lo, int64_t cell_hi,
                      uint4* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
   const int64_t e0 = cell_off[cell_lo], e1 = cell_off[cell_hi];
@@ -60,6 +61,7 @@ __global__ void __launch_bounds__(kThreads)
 gather_table_kernel(const unsigned long long* __restrict__ addr, int64_t vecs, int32_t rpb,
                     const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
                     const int32_t* total_ptr, uint4* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
   const int64_t total = *total_ptr;
@@ -85,6 +87,7 @@ __global__ void __launch_bounds__(kThreads)
 load_feat_blocks_kernel(const uint4* __restrict__ host, int64_t host_vecs,
                         const int32_t* __restrict__ blk, const unsigned long long* __restrict__ dst,
                         int32_t njobs, int64_t vpb) {
+  grid_dep_wait();
   const int64_t total = (int64_t)njobs * vpb;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t q0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q0 < total; q0 += 4 * stride) {
@@ -114,6 +117,7 @@ load_feat_blocks_kernel(const uint4* __restrict__ host, int64_t host_vecs,
 __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
                             const int32_t* __restrict__ map, uint8_t* __restrict__ flags,
                             const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int64_t ncells = (int64_t)T * H;
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < ncells;
@@ -125,6 +129,7 @@ __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int
 __global__ void count_feat_requests_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
                                            const int32_t* __restrict__ tile_feat_block,
                                            int32_t* __restrict__ counts, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
        t += (int64_t)gridDim.x * blockDim.x) {
@@ -141,6 +146,7 @@ __global__ void __launch_bounds__(kThreads)
 load_blocks_kernel(const int32_t* __restrict__ host_indices, const int64_t* __restrict__ e0,
                    const int64_t* __restrict__ e1, const int2* __restrict__ jobs, int32_t njobs,
                    int32_t* __restrict__ gbuf, int64_t epb) {
+  grid_dep_wait();
   for (int32_t i = blockIdx.x; i < njobs; i += gridDim.x) {
     const int2 jb = jobs[i];
     const int64_t a = e0[jb.x], n = e1[jb.x] - a;
@@ -168,6 +174,7 @@ load_blocks_kernel(const int32_t* __restrict__ host_indices, const int64_t* __re
 __global__ void mark_runs_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
                                  const int32_t* __restrict__ tile_adj_start,
                                  uint8_t* __restrict__ need, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
        t += (int64_t)gridDim.x * blockDim.x)
@@ -176,6 +183,7 @@ __global__ void mark_runs_kernel(const int32_t* __restrict__ cell_off, int32_t T
 
 __global__ void count_flags_kernel(const uint8_t* __restrict__ flags, int64_t n,
                                    int64_t* __restrict__ count) {
+  grid_dep_wait();
   int64_t local = 0;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
@@ -189,6 +197,7 @@ __global__ void __launch_bounds__(kThreads)
 distinct_rows_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict__ cell_off,
                      const int32_t* __restrict__ tile_first, int32_t T, int32_t H,
                      unsigned long long* count) {
+  grid_dep_wait();
   __shared__ uint32_t bits_s[kWarps][kTileWords];
   const int warp = threadIdx.x >> 5, lane = lane_id();
   uint32_t* bits = bits_s[warp];
@@ -223,6 +232,7 @@ tile_bitmap_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict_
                    const int32_t* __restrict__ tile_first, int32_t T, int32_t H,
                    uint32_t* __restrict__ bitmap, uint16_t* __restrict__ wpref,
                    int32_t* __restrict__ dcnt, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   __shared__ uint32_t bits_s[kWarps][kTileWords];
   const int warp = threadIdx.x >> 5, lane = lane_id();
@@ -279,6 +289,7 @@ load_distinct_rows_kernel(const unsigned long long* __restrict__ addr, int64_t v
                           const int32_t* __restrict__ tile_first, uint4* __restrict__ staging,
                           unsigned long long cache_lo, unsigned long long cache_hi,
                           unsigned long long* host_rows, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
   const int64_t total = __ldg(doff + T);
@@ -340,6 +351,7 @@ gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __re
                           const unsigned long long* __restrict__ addr, int32_t rpb,
                           unsigned long long cache_lo, unsigned long long cache_hi,
                           uint4* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
   constexpr int kStep = kRowsPerWarp * U;
@@ -380,6 +392,7 @@ gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
                                const unsigned long long* __restrict__ addr, int32_t rpb,
                                unsigned long long cache_lo, unsigned long long cache_hi,
                                uint4* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int64_t total = *total_ptr;
   const int lane = lane_id();

@@ -24,6 +24,7 @@ __global__ void __launch_bounds__(kThreads)
 gather_vec_kernel(const uint4* __restrict__ feats, const int32_t* __restrict__ fb_id,
                   const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
                   uint4* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
   constexpr int kStep = kRowsPerWarp * U;
@@ -56,6 +57,7 @@ __global__ void __launch_bounds__(kThreads)
 gather_rows_kernel(const uint4* __restrict__ feats, int64_t vecs, const int32_t* __restrict__ fb_id,
                    const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
                    uint4* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int64_t total = *total_ptr;
   const int lane = lane_id();
@@ -72,6 +74,7 @@ __global__ void __launch_bounds__(kThreads)
 gather_bytes_kernel(const uint8_t* __restrict__ feats, int64_t row_bytes,
                     const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
                     const int32_t* total_ptr, uint8_t* __restrict__ out, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int64_t total = *total_ptr;
   const int lane = lane_id();

@@ -29,6 +29,7 @@ constexpr int kWarps = kThreads / 32;
 __global__ void __launch_bounds__(kThreads)
 targets_count_kernel(const int32_t* __restrict__ nodes, int64_t capK, int32_t H, int32_t B,
                      int32_t N, TileMap tm, int32_t* __restrict__ fcnt, int32_t* status) {
+  grid_dep_wait();
   const int64_t total = (int64_t)H * B;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) & ~31ll; i0 < total;
@@ -55,6 +56,7 @@ targets_scatter_kernel(const int32_t* __restrict__ nodes, int64_t capK, int32_t 
                        int32_t N, TileMap tm, int32_t* __restrict__ fcnt,
                        const int32_t* __restrict__ fcell_off, int32_t* __restrict__ tmp_id,
                        int32_t* __restrict__ tmp_pos, const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int64_t total = (int64_t)H * B;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -87,6 +89,7 @@ __global__ void __launch_bounds__(kThreads)
 targets_sort_kernel(const int32_t* __restrict__ fcell_off, int64_t ncells, int32_t H, TileMap tm,
                     const int32_t* __restrict__ tmp_id, const int32_t* __restrict__ tmp_pos,
                     int32_t* __restrict__ fb_id, int32_t* __restrict__ fb_pos, int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   __shared__ uint32_t bits_s[kWarps][kTileWords];
   __shared__ int32_t pref_s[kWarps][kTileWords];
@@ -169,6 +172,7 @@ sample_count_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict
                     const int32_t* total_ptr, const OffT* __restrict__ off, int64_t capK,
                     int64_t cap_prev, int32_t k, int32_t* __restrict__ cnt,
                     const int32_t* status) {
+  grid_dep_wait();
   if (failed(status)) return;
   const int64_t total = *total_ptr;
   const uint32_t capk32 = (uint32_t)capK;
@@ -271,6 +275,7 @@ __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t 
 template <typename OffT, int G, bool kStreamed>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
+  grid_dep_wait();
   if (failed(a.status)) return;
   const Key key = load_key(a.key);
   const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
@@ -325,6 +330,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
 template <typename OffT, bool kStreamed>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
+  grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ int32_t chosen_s[kWarps][kMaxFanout];
   const int warp = threadIdx.x >> 5, lane = lane_id();
@@ -396,6 +402,7 @@ cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32
 }
 
 static __global__ void set_key_kernel(uint64_t* key, uint64_t seed, uint64_t first_gid) {
+  grid_dep_wait();
   key[0] = seed;
   key[1] = first_gid;
 }

@@ -95,6 +95,7 @@ scan_reduce_kernel(const InT* __restrict__ in, int64_t in_stride, const int32_t*
                    int64_t const_len, int64_t chunks, int64_t* __restrict__ partial,
                    unsigned int* __restrict__ tickets, OutT* __restrict__ out, int64_t out_stride,
                    bool write_end, int32_t* seg_total, const int32_t* status) {
+  grid_dep_wait();
   if (status && failed(status)) return;
   const int s = blockIdx.y;
   const int64_t len = seg_len(d_len, const_len, s);
@@ -149,6 +150,7 @@ __global__ void __launch_bounds__(kThreads)
 scan_down_kernel(const InT* __restrict__ in, int64_t in_stride, OutT* __restrict__ out,
                  int64_t out_stride, const int32_t* d_len, int64_t const_len, int64_t chunks,
                  const int64_t* __restrict__ partial, const int32_t* status) {
+  grid_dep_wait();
   if (status && failed(status)) return;
   const int s = blockIdx.y;
   const int64_t len = seg_len(d_len, const_len, s);
@@ -197,6 +199,7 @@ constexpr int kColRows = 16;  // rows per chunk
 __global__ void __launch_bounds__(128)
 col_reduce_kernel(const int32_t* __restrict__ in, int64_t rows, int32_t cols,
                   int64_t* __restrict__ partial, const int32_t* status) {
+  grid_dep_wait();
   if (status && failed(status)) return;
   const int32_t c = blockIdx.y * 128 + threadIdx.x;
   if (c >= cols) return;
@@ -216,6 +219,7 @@ __global__ void __launch_bounds__(kThreads)
 col_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, int32_t cols,
                     const int32_t* __restrict__ add_in, int32_t* __restrict__ total_out,
                     const int32_t* status) {
+  grid_dep_wait();
   if (status && failed(status)) return;
   const int32_t c = blockIdx.x;
   const int64_t carry = cta_scan_inplace(partial + c, chunks, cols, false);
@@ -226,6 +230,7 @@ col_partials_kernel(int64_t* __restrict__ partial, int64_t chunks, int32_t cols,
 __global__ void __launch_bounds__(128)
 col_down_kernel(const int32_t* __restrict__ in, int32_t* __restrict__ out, int64_t rows,
                 int32_t cols, const int64_t* __restrict__ partial, const int32_t* status) {
+  grid_dep_wait();
   if (status && failed(status)) return;
   const int32_t c = blockIdx.y * 128 + threadIdx.x;
   if (c >= cols) return;

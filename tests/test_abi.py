@@ -47,7 +47,7 @@ def test_null_arguments_are_rejected_without_a_device(L):
     fan = (ctypes.c_int32 * 1)(5)
     assert L.agnes_prepare_hyperbatch(None, None, 1, 1, fan, 1, 0, 0, None) == 1
     assert L.agnes_fetch_minibatch(None, 0, None) == 1
-    assert L.agnes_set_graph_mode(None, 1) == 1
+    assert L.agnes_set_launch_mode(None, 1) == 1
     assert L.agnes_free(None) == 0
 
 

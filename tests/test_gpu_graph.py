@@ -55,9 +55,12 @@ def _same(a, b):
 def test_graph_replays_match_the_oracle_and_direct_launches(cuda_device):
     off, ind, feats = make(30000, 10, seed=5, dim=32)
     og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    pdl = load(off, ind, feats, ADJ, FEAT)  # the default launch mode
     graphed = load(off, ind, feats, ADJ, FEAT)
+    graphed.set_launch_mode("graph")
     direct = load(off, ind, feats, ADJ, FEAT)
-    direct.set_graph_mode(False)
+    direct.set_launch_mode("direct")
+    ctxs = (pdl, graphed, direct)
     pool = torch.arange(30000, dtype=torch.int32)
     # (H, fanouts, seed, first minibatch id, frontier, profiling)
     seq = [(6, [6, 4, 3], 1, 0, "src", False),
@@ -69,22 +72,27 @@ def test_graph_replays_match_the_oracle_and_direct_launches(cuda_device):
            (6, [6, 4, 3], 3, 24, "src", True)]      # replay, phase events re-pointed
     for step, (H, fan, seed, gid, frontier, prof) in enumerate(seq):
         targets = synth.hyperbatch_targets(pool, H, 150, 3, step)
-        for g in (graphed, direct):
+        for g in ctxs:
             g.set_frontier(frontier)
             g.set_profiling(prof)
             g.prepare(targets.to(cuda_device), fan, seed, gid)
-        compare(graphed, og, targets.numpy(), fan, seed, gid, ADJ, FEAT, frontier=frontier)
-        _same(_snapshot(graphed), _snapshot(direct))
+        compare(pdl, og, targets.numpy(), fan, seed, gid, ADJ, FEAT, frontier=frontier)
+        ref = _snapshot(pdl)
+        for g in ctxs[1:]:
+            _same(ref, _snapshot(g))
         if prof:
-            for g in (graphed, direct):
+            for g in ctxs:
                 t = g.phase_times(0)
                 assert len(t) == 2 + 3 * len(fan) and all(x >= 0 for x in t)
-    c = graphed.counters()
-    assert c["graph_captures"] == 4 and c["graph_launches"] == len(seq)
+    for g in ctxs[:2]:
+        c = g.counters()
+        assert c["graph_captures"] == 4 and c["graph_launches"] == len(seq)
+    assert pdl.counters()["graph_programmatic_edges"] > 20
+    assert graphed.counters()["graph_programmatic_edges"] == 0
     d = direct.counters()
     assert d["graph_captures"] == 0 and d["graph_launches"] == 0
-    graphed.close()
-    direct.close()
+    for g in ctxs:
+        g.close()
 
 
 def test_prepare_inside_a_callers_capture(cuda_device):
