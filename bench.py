@@ -429,6 +429,11 @@ def main():
             "topology_bytes": indices.numel() * 4})
         hb, lb = topo["hit_blocks_per_step"], topo["loaded_blocks_per_step"]
         topo["hit_rate"] = hb / (hb + lb) if hb + lb else None
+        if args.topology_io == "rows":  # graph buffer = topology cache; hits are requests
+            req = statistics.mean(sum(c["frontier"]) for c in counters[1:]) if n > 0 else 0
+            cr = (c1["topo_cached_requests"] - c0["topo_cached_requests"]) / n
+            topo.update({"requests_per_step": req, "cached_requests_per_step": cr,
+                         "hit_rate": cr / req if req else None})
         topo["load_GBps_over_step"] = topo["loaded_bytes_per_step"] / (elapsed_ms / args.steps / 1e3) / 1e9
     if host_link is not None and args.stream:
         sb = statistics.mean(c["streamed_bytes"] for c in counters)

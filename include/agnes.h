@@ -111,7 +111,8 @@ typedef struct {
   int64_t adj_block_bytes;
   int64_t feat_block_bytes;
   int32_t topology_on_host; /* 1: indices stay in pinned host memory (see below) */
-  int64_t graph_buffer_bytes; /* HBM graph buffer for topology_on_host (0: whole topology) */
+  int64_t graph_buffer_bytes; /* topology_on_host: HBM graph buffer (blocks I/O; 0: whole
+                                 topology) or topology cache (rows I/O; 0: none) */
   int64_t feature_cache_bytes;     /* features_on_host: HBM feature cache (0: none) */
   int64_t feature_cache_threshold; /* cumulative requests a block must exceed to be cached */
   int32_t feature_io;              /* features_on_host: AGNES_FEATURE_IO_BLOCKS or _ROWS */
@@ -122,8 +123,15 @@ typedef struct {
  * BLOCKS: the blocks a hop's frontier touches are loaded whole into the HBM
  *   graph buffer (LRU + pinning, Sec. 3.4 (1)); 0, the default.
  * ROWS: the sampler reads each sampled neighbour entry in place from pinned
- *   host memory over the host link; no graph buffer (graph_buffer_bytes is
- *   ignored).  Not in the paper, for the reason given for feature rows. */
+ *   host memory over the host link.  Not in the paper, for the reason given
+ *   for feature rows.  With graph_buffer_bytes > 0 the buffer is a topology
+ *   cache instead: the block runs (a block start and its continuation
+ *   blocks) with the most frontier requests since load are kept in it,
+ *   hottest first, up to its capacity, in the spirit of the count-based
+ *   feature cache of Sec. 3.4 (2); the sampler reads a cached block from HBM
+ *   and any other in place.  The set is picked before the 2nd hyperbatch and
+ *   re-picked every 8 hyperbatches after; a prepare that re-picks first waits
+ *   for the previous hyperbatch. */
 #define AGNES_TOPOLOGY_IO_BLOCKS 0
 #define AGNES_TOPOLOGY_IO_ROWS 1
 
@@ -295,15 +303,18 @@ typedef struct {
   int64_t streamed_blocks;          /* features_on_host: touched feature blocks not
                                        served by the feature cache */
   /* the rest are totals since agnes_load_graph, not per hyperbatch */
-  int64_t topo_loaded_blocks;       /* topology_on_host: blocks copied into the graph buffer */
+  int64_t topo_loaded_blocks;       /* topology_on_host: blocks copied into the graph buffer
+                                       or the topology cache */
   int64_t topo_loaded_bytes;
-  int64_t topo_hit_blocks;          /* needed blocks already resident */
+  int64_t topo_hit_blocks;          /* needed blocks already resident (blocks I/O) */
   int64_t topo_waves;               /* fill launches over all hops */
   int64_t fcache_hit_blocks;        /* feature blocks read in place from the feature cache */
   int64_t fcache_loaded_blocks;     /* feature blocks copied into the feature cache */
   int64_t graph_captures;           /* launch sequences captured (agnes_set_launch_mode) */
   int64_t graph_launches;           /* prepares issued as one graph launch */
   int64_t graph_programmatic_edges; /* programmatic kernel edges of the current graph */
+  int64_t topo_cached_requests;     /* rows I/O with a topology cache: frontier entries
+                                       whose topology block was cached */
 } agnes_counters;
 agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out);
 

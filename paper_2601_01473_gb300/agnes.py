@@ -105,6 +105,7 @@ class _Counters(ctypes.Structure):
         ("fcache_loaded_blocks", ctypes.c_int64),
         ("graph_captures", ctypes.c_int64), ("graph_launches", ctypes.c_int64),
         ("graph_programmatic_edges", ctypes.c_int64),
+        ("topo_cached_requests", ctypes.c_int64),
     ]
 
 
@@ -415,7 +416,8 @@ class Graph:
                 "fcache_hit_blocks": c.fcache_hit_blocks,
                 "fcache_loaded_blocks": c.fcache_loaded_blocks,
                 "graph_captures": c.graph_captures, "graph_launches": c.graph_launches,
-                "graph_programmatic_edges": c.graph_programmatic_edges}
+                "graph_programmatic_edges": c.graph_programmatic_edges,
+                "topo_cached_requests": c.topo_cached_requests}
 
     def info(self) -> dict:
         g = _GraphInfo()

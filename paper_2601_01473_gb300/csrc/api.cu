@@ -33,6 +33,9 @@ constexpr int kEventRing = 64;  // prepares whose phase times stay readable
 // holding a batch of up to kStreamBatchBlocks touched feature blocks.
 constexpr int kStreamSlots = 4;
 constexpr int kStreamBatchBlocks = 64;
+// In-place topology reads with a topology cache: hyperbatches between re-picks
+// of the cached block runs.
+constexpr int64_t kTopoRepickEvery = 8;
 
 struct Workspace {
   int32_t H = 0, B = 0, K = 0;
@@ -208,6 +211,14 @@ struct agnes_ctx {
     bool uploaded_used = false;
     int64_t loaded_blocks = 0, loaded_bytes = 0, hits = 0, waves = 0;
     uint64_t sweeps = 0;  // hops sampled so far (sets the sweep direction)
+    // in-place reads (AGNES_TOPOLOGY_IO_ROWS) with a topology cache: gbuf holds
+    // the most requested block runs, the sampler reads the rest in place
+    bool cache = false;
+    unsigned long long* d_acc = nullptr;   // n_starts: frontier entries per run since load
+    unsigned long long* h_acc = nullptr;   // pinned read-back of d_acc (at re-picks)
+    unsigned long long* d_cached = nullptr;  // frontier entries on cached blocks since load
+    unsigned long long* h_cached = nullptr;  // pinned, read back after every hyperbatch
+    std::vector<int32_t> run_of;        // n_blocks: block run of each physical block
   } topo;
 
   char err[512] = {0};
@@ -599,6 +610,10 @@ agnes_status agnes_free(agnes_ctx* ctx) {
     cudaFree(tp.d_need);
     if (tp.h_slot_stage) cudaFreeHost(tp.h_slot_stage);
     if (tp.h_need) cudaFreeHost(tp.h_need);
+    cudaFree(tp.d_acc);
+    cudaFree(tp.d_cached);
+    if (tp.h_acc) cudaFreeHost(tp.h_acc);
+    if (tp.h_cached) cudaFreeHost(tp.h_cached);
   }
   if (ctx->ev_created)
     for (int r = 0; r < kEventRing; ++r)
@@ -679,10 +694,12 @@ static agnes_status setup_streaming(agnes_ctx* ctx, const agnes_graph_desc* d, c
 }
 
 // Graph buffer, tables and copy stream for topology in pinned host memory.
-static agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStream_t st) {
+// Host copies of the block tables the topology modes plan with: the edge
+// range of every physical block and the blocks of every block run.
+static agnes_status topology_host_tables(agnes_ctx* ctx, const agnes_graph_desc* d,
+                                         cudaStream_t st) {
   agnes_ctx::Topo& tp = ctx->topo;
   const int64_t nb = ctx->bt.n_blocks, ns = ctx->bt.n_starts;
-  tp.on = true;
   tp.host_indices = d->indices;
   tp.epb = d->adj_block_bytes / 4;
   tp.e0.resize((size_t)nb);
@@ -699,6 +716,53 @@ static agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cu
                           sizeof(int32_t) * (ns + 1), cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaStreamSynchronize(st));
   tp.start_block[(size_t)ns] = (int32_t)nb;
+  return AGNES_OK;
+}
+
+// A topology cache for in-place reads: graph_buffer_bytes / adj_block_bytes
+// slots, filled between hyperbatches with the block runs the frontiers
+// requested most (update_topology_cache).
+static agnes_status setup_topology_cache(agnes_ctx* ctx, const agnes_graph_desc* d,
+                                         cudaStream_t st) {
+  agnes_ctx::Topo& tp = ctx->topo;
+  agnes_status rc = topology_host_tables(ctx, d, st);
+  if (rc != AGNES_OK) return rc;
+  const int64_t nb = ctx->bt.n_blocks, ns = ctx->bt.n_starts;
+  tp.slots = d->graph_buffer_bytes / d->adj_block_bytes;
+  if (tp.slots > nb) tp.slots = nb;
+  if (tp.slots < 1) return AGNES_OK;
+  tp.cache = true;
+  tp.dev_view = ctx->indices;  // the device view of the host neighbour lists
+  CK(ctx, cudaMalloc((void**)&tp.gbuf, sizeof(int32_t) * (size_t)(tp.slots * tp.epb)));
+  CK(ctx, cudaMalloc((void**)&tp.d_slot, sizeof(int32_t) * (size_t)nb));
+  CK(ctx, cudaMallocHost((void**)&tp.h_slot_stage, sizeof(int32_t) * (size_t)nb));
+  CK(ctx, cudaMemsetAsync(tp.d_slot, 0xff, sizeof(int32_t) * (size_t)nb, st));
+  CK(ctx, cudaMalloc((void**)&tp.d_acc, sizeof(unsigned long long) * (size_t)ns));
+  CK(ctx, cudaMallocHost((void**)&tp.h_acc, sizeof(unsigned long long) * (size_t)ns));
+  CK(ctx, cudaMalloc((void**)&tp.d_cached, sizeof(unsigned long long)));
+  CK(ctx, cudaMallocHost((void**)&tp.h_cached, sizeof(unsigned long long)));
+  CK(ctx, cudaMemsetAsync(tp.d_acc, 0, sizeof(unsigned long long) * (size_t)ns, st));
+  CK(ctx, cudaMemsetAsync(tp.d_cached, 0, sizeof(unsigned long long), st));
+  *tp.h_cached = 0;
+  tp.jobs_cap = (int32_t)tp.slots;
+  CK(ctx, cudaMalloc((void**)&tp.d_jobs, sizeof(int2) * (size_t)tp.jobs_cap));
+  CK(ctx, cudaMallocHost((void**)&tp.h_jobs, sizeof(int2) * (size_t)tp.jobs_cap));
+  tp.slot_of.assign((size_t)nb, -1);
+  tp.block_of.assign((size_t)tp.slots, -1);
+  tp.run_of.resize((size_t)nb);
+  for (int64_t r = 0; r < ns; ++r)
+    for (int32_t b = tp.start_block[(size_t)r]; b < tp.start_block[(size_t)r + 1]; ++b)
+      tp.run_of[(size_t)b] = (int32_t)r;
+  CK(ctx, cudaStreamSynchronize(st));
+  return AGNES_OK;
+}
+
+static agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStream_t st) {
+  agnes_ctx::Topo& tp = ctx->topo;
+  const int64_t nb = ctx->bt.n_blocks, ns = ctx->bt.n_starts;
+  agnes_status rc = topology_host_tables(ctx, d, st);
+  if (rc != AGNES_OK) return rc;
+  tp.on = true;
   int64_t longest = 1;
   for (int64_t r = 0; r < ns; ++r) {
     const int64_t m = tp.start_block[(size_t)r + 1] - tp.start_block[(size_t)r];
@@ -922,6 +986,9 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0 &&
       d->topology_io == AGNES_TOPOLOGY_IO_BLOCKS)
     rc = setup_topology(ctx, d, st);
+  if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0 &&
+      d->topology_io == AGNES_TOPOLOGY_IO_ROWS && d->graph_buffer_bytes > 0)
+    rc = setup_topology_cache(ctx, d, st);
   if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
     set_err(ctx, "cudaEventCreate failed");
     rc = AGNES_ECUDA;
@@ -1288,8 +1355,8 @@ static void update_feature_cache(agnes_ctx* ctx, int32_t n_touched) {
 static agnes_status gather_streamed(agnes_ctx* ctx, int cur, cudaStream_t st) {
   Workspace& w = ctx->ws;
   const int64_t nfb = ctx->bt.n_feat_blocks;
-  CK(ctx, launch_count_feat_requests(w.fcell_off[cur], (int32_t)ctx->bt.T, w.H,
-                                     ctx->bt.tile_feat_block, ctx->d_counts, nfb, w.status, st));
+  CK(ctx, launch_count_requests(w.fcell_off[cur], (int32_t)ctx->bt.T, w.H,
+                                ctx->bt.tile_feat_block, ctx->d_counts, nfb, true, w.status, st));
   CK(ctx, cudaMemcpyAsync(ctx->h_counts, ctx->d_counts, sizeof(int32_t) * (size_t)nfb,
                           cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaStreamSynchronize(st));
@@ -1305,6 +1372,75 @@ static agnes_status gather_streamed(agnes_ctx* ctx, int cur, cudaStream_t st) {
   ctx->streamed_blocks = n - hits;
   ctx->fcache_hits += hits;
   update_feature_cache(ctx, n);
+  return AGNES_OK;
+}
+
+// Before hyperbatches 2, 2 + R, 2 + 2R, ... (R = kTopoRepickEvery) with a
+// topology cache: waits for the previous hyperbatch, reads back the request
+// count of every block run since load, and re-picks the cached runs -- most
+// requested first, whole runs, up to the cache's capacity.  Runs that stay
+// keep their slots; the blocks of newly admitted runs are copied into free
+// slots (loader kernel over the host link) and the slot table is uploaded,
+// all on st ahead of the hyperbatch.  Re-picking only every R hyperbatches
+// keeps the wait (an idle GPU while the host plans) and the churn rare.
+static agnes_status update_topology_cache(agnes_ctx* ctx, cudaStream_t st) {
+  agnes_ctx::Topo& tp = ctx->topo;
+  const int64_t n = ctx->n_prepared;
+  if (!tp.cache || n < 1 || (n - 1) % kTopoRepickEvery != 0) return AGNES_OK;
+  const int64_t ns = ctx->bt.n_starts, nb = ctx->bt.n_blocks, C = tp.slots;
+  CK(ctx, cudaEventSynchronize(ctx->done));  // also: nothing reads the cache while it changes
+  CK(ctx, cudaMemcpyAsync(tp.h_acc, tp.d_acc, sizeof(unsigned long long) * (size_t)ns,
+                          cudaMemcpyDeviceToHost, st));
+  CK(ctx, cudaStreamSynchronize(st));
+  const unsigned long long* acc = tp.h_acc;
+  std::vector<int32_t> cand;
+  for (int64_t r = 0; r < ns; ++r)
+    if (acc[r] > 0) cand.push_back((int32_t)r);
+  std::sort(cand.begin(), cand.end(),
+            [&](int32_t x, int32_t y) { return acc[x] != acc[y] ? acc[x] > acc[y] : x < y; });
+  std::vector<uint8_t> keep((size_t)ns, 0);
+  int64_t used = 0;
+  for (int32_t r : cand) {
+    const int64_t m = tp.start_block[(size_t)r + 1] - tp.start_block[(size_t)r];
+    if (used + m > C) continue;  // a run too big for what is left; smaller ones may fit
+    keep[(size_t)r] = 1;
+    used += m;
+  }
+  std::vector<int32_t> free_slots;
+  for (int64_t sl = 0; sl < C; ++sl) {
+    const int32_t b = tp.block_of[(size_t)sl];
+    if (b >= 0 && keep[(size_t)tp.run_of[(size_t)b]]) continue;
+    if (b >= 0) tp.slot_of[(size_t)b] = -1;
+    tp.block_of[(size_t)sl] = -1;
+    free_slots.push_back((int32_t)sl);
+  }
+  int32_t njobs = 0;
+  for (int32_t r : cand) {
+    if (!keep[(size_t)r]) continue;
+    for (int32_t b = tp.start_block[(size_t)r]; b < tp.start_block[(size_t)r + 1]; ++b) {
+      if (tp.slot_of[(size_t)b] >= 0) continue;
+      if (free_slots.empty()) {  // cannot happen: the kept runs fit in C slots
+        set_err(ctx, "topology cache out of slots");
+        return AGNES_EKERNEL;
+      }
+      const int32_t sl = free_slots.back();
+      free_slots.pop_back();
+      tp.slot_of[(size_t)b] = sl;
+      tp.block_of[(size_t)sl] = b;
+      tp.h_jobs[njobs++] = make_int2(b, sl);
+      tp.loaded_blocks += 1;
+      tp.loaded_bytes += sizeof(int32_t) * (tp.e1[(size_t)b] - tp.e0[(size_t)b]);
+    }
+  }
+  if (njobs > 0) {
+    CK(ctx, cudaMemcpyAsync(tp.d_jobs, tp.h_jobs, sizeof(int2) * (size_t)njobs,
+                            cudaMemcpyHostToDevice, st));
+    CK(ctx, launch_load_blocks(tp.dev_view, ctx->bt.blk_e0, ctx->bt.blk_e1, tp.d_jobs, njobs,
+                               tp.gbuf, tp.epb, ctx->num_sms, st));
+  }
+  memcpy(tp.h_slot_stage, tp.slot_of.data(), sizeof(int32_t) * (size_t)nb);
+  CK(ctx, cudaMemcpyAsync(tp.d_slot, tp.h_slot_stage, sizeof(int32_t) * (size_t)nb,
+                          cudaMemcpyHostToDevice, st));
   return AGNES_OK;
 }
 
@@ -1372,6 +1508,19 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
       FillRange r;
       r.cell_lo = 0;
       r.cell_hi = cells;
+      const agnes_ctx::Topo& tp = ctx->topo;
+      if (tp.cache) {  // requests per block run, then cached blocks from HBM, others in place
+        CK(ctx, launch_count_cache_requests(w.fcell_off[cur], T, H, ctx->bt.tile_adj_start,
+                                            ctx->bt.tile_adj_block, tp.d_slot, tp.d_acc,
+                                            tp.d_cached, w.status, st));
+        r.tile_adj_block = ctx->bt.tile_adj_block;
+        r.blk_slot = tp.d_slot;
+        r.blk_e0 = ctx->bt.blk_e0;
+        r.gbuf = tp.gbuf;
+        r.epb = tp.epb;
+        r.bb = ctx->adj_block_bytes;
+        r.in_place_fallback = true;
+      }
       CK(ctx, launch_sample_fill(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.indptr[h],
                                  w.nbr, w.scnt, w.scell, w.srank, r, nsm, st));
     }
@@ -1430,6 +1579,9 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
   CK(ctx, cudaMemcpyAsync(b.ecnt, w.ecnt, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.srcsz, w.srcsz, sizeof(int32_t) * K * H, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.stats, w.stats, sizeof(int64_t) * (K + 1), cudaMemcpyDeviceToHost, st));
+  if (ctx->topo.cache)
+    CK(ctx, cudaMemcpyAsync(ctx->topo.h_cached, ctx->topo.d_cached, sizeof(unsigned long long),
+                            cudaMemcpyDeviceToHost, st));
   *n_marks = ph;
   return AGNES_OK;
 }
@@ -1624,6 +1776,10 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   // use the ctx's buffers (a caller's own capture orders its replays itself)
   const bool capturing = stream_capturing(st);
   if (ctx->n_prepared > 0 && !capturing) CK(ctx, cudaStreamWaitEvent(st, ctx->done, 0));
+  if (!capturing) {
+    rc = update_topology_cache(ctx, st);
+    if (rc != AGNES_OK) return rc;
+  }
   CK(ctx, cudaMemcpy2DAsync(w.nodes, sizeof(int32_t) * w.capK, targets, sizeof(int32_t) * B,
                             sizeof(int32_t) * B, H, cudaMemcpyDefault, st));
   CK(ctx, launch_set_key(w.key, seed, first_minibatch_id, st));
@@ -1770,6 +1926,7 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
   out->topo_loaded_blocks = ctx->topo.loaded_blocks;
   out->topo_loaded_bytes = ctx->topo.loaded_bytes;
   out->topo_hit_blocks = ctx->topo.hits;
+  out->topo_cached_requests = ctx->topo.cache ? (int64_t)*ctx->topo.h_cached : 0;
   out->topo_waves = ctx->topo.waves;
   out->fcache_hit_blocks = ctx->fcache_hits;
   out->fcache_loaded_blocks = ctx->fcache_loads;

@@ -126,16 +126,39 @@ __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int
 }
 
 // Requests per feature block: counts[tile_feat_block[t]] += entries of tile t.
-__global__ void count_feat_requests_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
-                                           const int32_t* __restrict__ tile_feat_block,
-                                           int32_t* __restrict__ counts, const int32_t* status) {
+__global__ void count_requests_kernel(const int32_t* __restrict__ cell_off, int32_t T, int32_t H,
+                                      const int32_t* __restrict__ tile_map,
+                                      int32_t* __restrict__ counts, const int32_t* status) {
   grid_dep_wait();
   if (failed(status)) return;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
        t += (int64_t)gridDim.x * blockDim.x) {
     const int32_t n = cell_off[(t + 1) * H] - cell_off[t * H];
-    if (n) atomicAdd(counts + tile_feat_block[t], n);
+    if (n) atomicAdd(counts + tile_map[t], n);
   }
+}
+
+// Topology cache bookkeeping, per tile with frontier entries: acc[run of the
+// tile] += entries, and cached += entries when the tile's block has a slot.
+__global__ void count_cache_requests_kernel(const int32_t* __restrict__ cell_off, int32_t T,
+                                            int32_t H, const int32_t* __restrict__ tile_adj_start,
+                                            const int32_t* __restrict__ tile_adj_block,
+                                            const int32_t* __restrict__ blk_slot,
+                                            unsigned long long* __restrict__ acc,
+                                            unsigned long long* __restrict__ cached,
+                                            const int32_t* status) {
+  grid_dep_wait();
+  if (failed(status)) return;
+  unsigned long long hit = 0;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t n = cell_off[(t + 1) * H] - cell_off[t * H];
+    if (!n) continue;
+    atomicAdd(acc + tile_adj_start[t], (unsigned long long)n);
+    if (blk_slot[tile_adj_block[t]] >= 0) hit += (unsigned long long)n;
+  }
+  hit = warp_sum(hit);
+  if (lane_id() == 0 && hit) atomicAdd(cached, hit);
 }
 
 // Copies the edge lists of physical blocks from pinned host memory (read in
@@ -536,12 +559,24 @@ cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, con
   return cudaGetLastError();
 }
 
-cudaError_t launch_count_feat_requests(const int32_t* cell_off, int32_t T, int32_t H,
-                                       const int32_t* tile_feat_block, int32_t* counts,
-                                       int64_t nfb, const int32_t* status, cudaStream_t st) {
-  cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int32_t) * (size_t)nfb, st);
-  if (e != cudaSuccess) return e;
-  count_feat_requests_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, tile_feat_block, counts, status);
+cudaError_t launch_count_requests(const int32_t* cell_off, int32_t T, int32_t H,
+                                  const int32_t* tile_map, int32_t* counts, int64_t n,
+                                  bool zero_first, const int32_t* status, cudaStream_t st) {
+  if (zero_first) {
+    const cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int32_t) * (size_t)n, st);
+    if (e != cudaSuccess) return e;
+  }
+  count_requests_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, tile_map, counts, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_count_cache_requests(const int32_t* cell_off, int32_t T, int32_t H,
+                                        const int32_t* tile_adj_start,
+                                        const int32_t* tile_adj_block, const int32_t* blk_slot,
+                                        unsigned long long* acc, unsigned long long* cached,
+                                        const int32_t* status, cudaStream_t st) {
+  count_cache_requests_kernel<<<1184, 256, 0, st>>>(cell_off, T, H, tile_adj_start,
+                                                    tile_adj_block, blk_slot, acc, cached, status);
   return cudaGetLastError();
 }
 

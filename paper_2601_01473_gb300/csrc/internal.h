@@ -108,6 +108,9 @@ struct FillRange {
   const int64_t* blk_e0 = nullptr;
   const int32_t* gbuf = nullptr;
   int64_t epb = 0, bb = 0;
+  // gbuf is a topology cache: a block without a slot is read in place from
+  // HopArgs::indices (otherwise every needed block must have a slot)
+  bool in_place_fallback = false;
 };
 
 // Samples the frontier entries of cells [r.cell_lo, r.cell_hi) and records,
@@ -223,10 +226,21 @@ cudaError_t launch_mark_count(const int32_t* cell_off, int32_t T, int32_t H, con
                               uint8_t* flags, int64_t n_flags, int64_t* count,
                               const int32_t* status, cudaStream_t st);
 
-// counts[b] = requests (bucket entries) for feature block b (cleared first).
-cudaError_t launch_count_feat_requests(const int32_t* cell_off, int32_t T, int32_t H,
-                                       const int32_t* tile_feat_block, int32_t* counts,
-                                       int64_t nfb, const int32_t* status, cudaStream_t st);
+// Topology cache bookkeeping for one hop's frontier bucket: acc[run] +=
+// requests of the block run's tiles; cached += requests on tiles whose
+// topology block has a cache slot.  Both accumulate since load.
+cudaError_t launch_count_cache_requests(const int32_t* cell_off, int32_t T, int32_t H,
+                                        const int32_t* tile_adj_start,
+                                        const int32_t* tile_adj_block, const int32_t* blk_slot,
+                                        unsigned long long* acc, unsigned long long* cached,
+                                        const int32_t* status, cudaStream_t st);
+
+// counts[tile_map[t]] += requests (bucket entries) of tile t, for every tile:
+// per feature block (tile_feat_block) or per topology block run
+// (tile_adj_start).  zero_first clears the n counts first.
+cudaError_t launch_count_requests(const int32_t* cell_off, int32_t T, int32_t H,
+                                  const int32_t* tile_map, int32_t* counts, int64_t n,
+                                  bool zero_first, const int32_t* status, cudaStream_t st);
 
 // Copies physical blocks jobs[i].x (edges e0..e1 of host_indices, a device
 // view of pinned host memory) into graph-buffer slots jobs[i].y.

@@ -226,19 +226,27 @@ __device__ __forceinline__ Key load_key(const uint64_t* key) {
   return Key{(uint32_t)seed, (uint32_t)(seed >> 32), __ldg(key + 1)};
 }
 
-// Neighbour at position pos of node v (edges off_v .. off_v + deg).  With
-// streamed topology the edge sits in the graph-buffer slot of its physical
-// block: v's first block, plus, for an object larger than a block, the block
-// its byte offset (after the header) falls in.
-template <bool kStreamed>
+// Where the sampler reads neighbour entries.
+enum EdgeSrc : int {
+  kEdgesInPlace = 0,  // a.indices (HBM, or the device view of pinned host memory)
+  kEdgesBuffer = 1,   // the graph buffer: every needed block is resident
+  kEdgesCached = 2,   // the topology cache where the block is cached, else in place
+};
+
+// Neighbour at position pos of node v (edges off_v .. off_v + deg).  In the
+// graph buffer or the topology cache the edge sits in the slot of its
+// physical block: v's first block, plus, for an object larger than a block,
+// the block its byte offset (after the header) falls in.
+template <int kSrc>
 __device__ __forceinline__ int32_t edge_at(const FillArgs& a, int32_t v, int64_t off_v,
                                            int64_t deg, int64_t pos) {
-  if (!kStreamed) return __ldg(a.indices + off_v + pos);
+  if (kSrc == kEdgesInPlace) return __ldg(a.indices + off_v + pos);
   int64_t b = __ldg(a.tile_adj_block + tile_of(a.tm, v));
   if (a.hdr + 4 * deg > a.bb) b += (a.hdr + 4 * pos) / a.bb;
   const int32_t slot = __ldg(a.blk_slot + b);
-  if (slot < 0) {  // cannot happen: the host made every needed block resident
-    atomicOr(a.status, kErrInternal);
+  if (slot < 0) {
+    if (kSrc == kEdgesCached) return __ldg(a.indices + off_v + pos);
+    atomicOr(a.status, kErrInternal);  // cannot happen: the host made every needed block resident
     return 0;
   }
   return __ldg(a.gbuf + (int64_t)slot * a.epb + (off_v + pos - __ldg(a.blk_e0 + b)));
@@ -272,7 +280,7 @@ __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t 
 }
 
 // G lanes per frontier node, k <= G.
-template <typename OffT, int G, bool kStreamed>
+template <typename OffT, int G, int kSrc>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
   grid_dep_wait();
@@ -302,7 +310,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
       eidx = a.indptr[j * (a.cap_prev + 1) + pos] + s;
       if (d <= a.k) {
         if (s < d) {
-          u = edge_at<kStreamed>(a, v, base, d, s);
+          u = edge_at<kSrc>(a, v, base, d, s);
           has = true;
         }
       } else {
@@ -315,7 +323,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
           if (s > q && t == cq) collided = true;
         }
         if (s < a.k) {
-          u = edge_at<kStreamed>(a, v, base, d, collided ? J : t);
+          u = edge_at<kSrc>(a, v, base, d, collided ? J : t);
           has = true;
         }
       }
@@ -327,7 +335,7 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
 // One warp per frontier node for fanouts above 32: slots are drawn 32 at a
 // time; each candidate is checked against the choices of earlier chunks (kept
 // in shared memory) and then resolved within its chunk by shuffles.
-template <typename OffT, bool kStreamed>
+template <typename OffT, int kSrc>
 __global__ void __launch_bounds__(kThreads)
 sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
   grid_dep_wait();
@@ -352,7 +360,7 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
       for (int64_t q0 = 0; q0 < d; q0 += 32) {
         const int64_t q = q0 + lane;
         const bool has = q < d;
-        emit_edges(a, has, has ? edge_at<kStreamed>(a, v, base, d, q) : 0, j, ebase + q);
+        emit_edges(a, has, has ? edge_at<kSrc>(a, v, base, d, q) : 0, j, ebase + q);
       }
       continue;
     }
@@ -371,7 +379,7 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
       }
       const int64_t c = collided ? J : t;
       if (valid) chosen[s] = (int32_t)c;
-      emit_edges(a, valid, valid ? edge_at<kStreamed>(a, v, base, d, c) : 0, j, ebase + s);
+      emit_edges(a, valid, valid ? edge_at<kSrc>(a, v, base, d, c) : 0, j, ebase + s);
       __syncwarp();
     }
   }
@@ -429,21 +437,21 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
   return cudaGetLastError();
 }
 
-template <typename OffT, bool kStreamed>
+template <typename OffT, int kSrc>
 static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int num_sms,
                               cudaStream_t st) {
 #define AGNES_FILL(KERNEL)                                                                   \
   KERNEL<<<resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st>>>(f, off)
   if (k <= 4)
-    AGNES_FILL((sample_fill_kernel<OffT, 4, kStreamed>));
+    AGNES_FILL((sample_fill_kernel<OffT, 4, kSrc>));
   else if (k <= 8)
-    AGNES_FILL((sample_fill_kernel<OffT, 8, kStreamed>));
+    AGNES_FILL((sample_fill_kernel<OffT, 8, kSrc>));
   else if (k <= 16)
-    AGNES_FILL((sample_fill_kernel<OffT, 16, kStreamed>));
+    AGNES_FILL((sample_fill_kernel<OffT, 16, kSrc>));
   else if (k <= 32)
-    AGNES_FILL((sample_fill_kernel<OffT, 32, kStreamed>));
+    AGNES_FILL((sample_fill_kernel<OffT, 32, kSrc>));
   else
-    AGNES_FILL((sample_fill_wide_kernel<OffT, kStreamed>));
+    AGNES_FILL((sample_fill_wide_kernel<OffT, kSrc>));
 #undef AGNES_FILL
 }
 
@@ -479,18 +487,23 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.hop = a.hop;
   f.key = a.key;
   f.status = a.status;
-  const bool streamed = r.gbuf != nullptr;
-  if (a.offsets_bits == 32) {
-    if (streamed)
-      launch_fill_typed<int32_t, true>(f, (const int32_t*)a.offsets, a.k, num_sms, st);
-    else
-      launch_fill_typed<int32_t, false>(f, (const int32_t*)a.offsets, a.k, num_sms, st);
-  } else {
-    if (streamed)
-      launch_fill_typed<int64_t, true>(f, (const int64_t*)a.offsets, a.k, num_sms, st);
-    else
-      launch_fill_typed<int64_t, false>(f, (const int64_t*)a.offsets, a.k, num_sms, st);
-  }
+  const int src = r.gbuf == nullptr ? kEdgesInPlace : r.in_place_fallback ? kEdgesCached
+                                                                            : kEdgesBuffer;
+#define AGNES_FILL_SRC(OFF)                                                                  \
+  do {                                                                                      \
+    const OFF* off = (const OFF*)a.offsets;                                                 \
+    if (src == kEdgesInPlace)                                                               \
+      launch_fill_typed<OFF, kEdgesInPlace>(f, off, a.k, num_sms, st);                      \
+    else if (src == kEdgesBuffer)                                                           \
+      launch_fill_typed<OFF, kEdgesBuffer>(f, off, a.k, num_sms, st);                       \
+    else                                                                                    \
+      launch_fill_typed<OFF, kEdgesCached>(f, off, a.k, num_sms, st);                       \
+  } while (0)
+  if (a.offsets_bits == 32)
+    AGNES_FILL_SRC(int32_t);
+  else
+    AGNES_FILL_SRC(int64_t);
+#undef AGNES_FILL_SRC
   return cudaGetLastError();
 }
 

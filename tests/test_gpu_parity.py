@@ -434,6 +434,37 @@ def test_topology_read_in_place_matches_oracle(cuda_device, a, b, c, fan):
     g.close()
 
 
+@pytest.mark.parametrize("cache_bytes,mode", [(128 << 10, "graph_pdl"), (128 << 10, "direct"),
+                                              (4096, "graph_pdl"), (64 << 20, "graph_pdl")])
+def test_topology_cache_matches_oracle(cuda_device, cache_bytes, mode):
+    """In-place neighbour reads with a topology cache (graph_buffer_bytes in
+    rows mode): the hottest block runs are copied into HBM between
+    hyperbatches and read there, the rest in place; samples match the oracle
+    whatever is cached (a 1-slot cache, a partial one, one larger than the
+    topology), in graph and direct launch modes."""
+    off, ind = synth.rmat_csr(30000, 14, 0.6, 0.2, 0.15, seed=31, offsets_dtype=torch.int64)
+    feats = synth.normal_features(30000, 32, torch.float16, 6)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    g = Graph(off.to(cuda_device), ind.pin_memory(), feats.to(cuda_device), adj_block_bytes=4096,
+              feat_block_bytes=4096, topology_on_host=True, topology_io="rows",
+              graph_buffer_bytes=cache_bytes)
+    g.set_launch_mode(mode)
+    fan = [8, 5, 3]
+    slots = cache_bytes // 4096
+    for step in range(11):  # picks before hyperbatches 1 and 9 (0-based)
+        targets = synth.hyperbatch_targets(torch.arange(30000, dtype=torch.int32), 4, 150, 9, step)
+        g.prepare(targets.to(cuda_device), fan, 5, 10 * step)
+        compare(g, og, targets.numpy(), fan, 5, 10 * step, 4096, 4096)
+        cnt = g.counters()
+        if step == 0:
+            assert cnt["topo_loaded_blocks"] == 0 and cnt["topo_cached_requests"] == 0
+        if step == 1:
+            assert 0 < cnt["topo_loaded_blocks"] <= slots and cnt["topo_cached_requests"] > 0
+    assert cnt["topo_loaded_blocks"] <= 2 * slots
+    assert cnt["topo_hit_blocks"] == 0 and cnt["topo_waves"] == 0
+    g.close()
+
+
 def test_graph_buffer_smaller_than_an_object_is_rejected(cuda_device):
     off, ind = synth.rmat_csr(5000, 30, 0.6, 0.2, 0.15, seed=1)
     feats = synth.normal_features(5000, 8, torch.float32, 2)
