@@ -10,7 +10,7 @@ import pytest
 
 CSRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
                     "paper_2601_01473_gb300", "csrc")
-GRAPH_FILES = ["api.cu", "sample.cu", "dedup.cu", "scan.cu", "gather.cu", "gather_hbm.cu"]
+GRAPH_FILES = ["prepare.cu", "sample.cu", "dedup.cu", "scan.cu", "gather.cu", "gather_hbm.cu"]
 
 
 def _kernel_bodies(text):
