@@ -165,6 +165,8 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (ctx->h_rm) cudaFreeHost(ctx->h_rm);
   cudaFree(ctx->fcache);
   if (ctx->gather_start) cudaEventDestroy(ctx->gather_start);
+  for (int i = 0; i < kRowChunks; ++i)
+    if (ctx->rows_loaded[i]) cudaEventDestroy(ctx->rows_loaded[i]);
   if (ctx->h_counts) cudaFreeHost(ctx->h_counts);
   if (ctx->h_touched) cudaFreeHost(ctx->h_touched);
   if (ctx->h_src) cudaFreeHost(ctx->h_src);

@@ -23,6 +23,9 @@ constexpr int kEventRing = 64;  // prepares whose phase times stay readable
 // holding a batch of up to kStreamBatchBlocks touched feature blocks.
 constexpr int kStreamSlots = 4;
 constexpr int kStreamBatchBlocks = 64;
+// Row I/O of host-resident features: the distinct rows are loaded in this many
+// tile ranges, each range's gather starting once its rows are in.
+constexpr int kRowChunks = 8;
 // In-place topology reads with a topology cache: hyperbatches between re-picks
 // of the cached block runs.
 constexpr int64_t kTopoRepickEvery = 8;
@@ -182,6 +185,7 @@ struct agnes_ctx {
   int64_t* h_rm = nullptr;  // pinned: [0] distinct rows, [1] rows read from host memory
   int64_t cache_load_bytes = 0;
   cudaEvent_t gather_start = nullptr;
+  cudaEvent_t rows_loaded[agnes::kRowChunks] = {nullptr};  // row I/O: per tile range
   // feature cache C_f (Sec. 3.4 (2)): blocks whose cumulative request count
   // reaches the threshold, hottest first, up to fcache_slots blocks
   int64_t fcache_slots = 0, fcache_threshold = 0;

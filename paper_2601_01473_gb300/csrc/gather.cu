@@ -5,6 +5,8 @@
 // walks the final bucket, which lists each gathered node once per minibatch
 // in (tile, minibatch, id) order with its output row, and copies rows as
 // 16-byte vectors (bit-exact).
+#include <algorithm>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -299,30 +301,31 @@ __device__ __forceinline__ int32_t tile_rank(const uint32_t* __restrict__ bitmap
   return (int32_t)__ldg(wpref + w) + __popc(__ldg(bitmap + w) & ((1u << (lu & 31)) - 1u));
 }
 
-// Distinct row d (of doff[T]): tile t = last with doff[t] <= d; the row is
-// the (d - doff[t])-th requested id of the tile, copied from its feature
-// block's address in host memory (over the link; counted in *host_rows) to
-// staging row d.  Rows of blocks in the feature cache, [cache_lo, cache_hi),
-// are not staged: the gather reads them in place.  LPR lanes per row.
+// Distinct rows d of tiles [t_lo, t_hi) (d in [doff[t_lo], doff[t_hi])):
+// tile t = last with doff[t] <= d; the row is the (d - doff[t])-th requested
+// id of the tile, copied from its feature block's address in host memory
+// (over the link; counted in *host_rows) to staging row d.  Rows of blocks in
+// the feature cache, [cache_lo, cache_hi), are not staged: the gather reads
+// them in place.  LPR lanes per row.
 template <int LPR>
 __global__ void __launch_bounds__(kThreads)
 load_distinct_rows_kernel(const unsigned long long* __restrict__ addr, int64_t vecs, int32_t rpb,
                           const uint32_t* __restrict__ bitmap, const uint16_t* __restrict__ wpref,
-                          const int32_t* __restrict__ doff, int32_t T,
+                          const int32_t* __restrict__ doff, int32_t t_lo, int32_t t_hi,
                           const int32_t* __restrict__ tile_first, uint4* __restrict__ staging,
                           unsigned long long cache_lo, unsigned long long cache_hi,
                           unsigned long long* host_rows, const int32_t* status) {
   grid_dep_wait();
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
-  const int64_t total = __ldg(doff + T);
+  const int64_t d_lo = __ldg(doff + t_lo), d_hi = __ldg(doff + t_hi);
   const int lane = lane_id();
   const int sub = lane / LPR, l = lane % LPR;
   const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   uint32_t from_host = 0;
-  for (int64_t d = warp0 * kRowsPerWarp + sub; d < total; d += nwarps * kRowsPerWarp) {
-    int32_t lo = 0, hi = T;  // tile: last t with doff[t] <= d
+  for (int64_t d = d_lo + warp0 * kRowsPerWarp + sub; d < d_hi; d += nwarps * kRowsPerWarp) {
+    int32_t lo = t_lo, hi = t_hi;  // tile: last t with doff[t] <= d
     while (hi - lo > 1) {
       const int32_t mid = (lo + hi) >> 1;
       if (__ldg(doff + mid) <= d) lo = mid; else hi = mid;
@@ -368,7 +371,8 @@ __device__ __forceinline__ const uint4* staged_row_src(
 template <int LPR, int U>
 __global__ void __launch_bounds__(kThreads)
 gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __restrict__ fb_id,
-                          const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
+                          const int32_t* __restrict__ fb_pos, const int32_t* lo_ptr,
+                          const int32_t* hi_ptr,
                           TileMap tm, const uint32_t* __restrict__ bitmap,
                           const uint16_t* __restrict__ wpref, const int32_t* __restrict__ doff,
                           const unsigned long long* __restrict__ addr, int32_t rpb,
@@ -378,12 +382,12 @@ gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __re
   if (failed(status)) return;
   constexpr int kRowsPerWarp = 32 / LPR;
   constexpr int kStep = kRowsPerWarp * U;
-  const int64_t total = *total_ptr;
+  const int64_t total = *hi_ptr;
   const int lane = lane_id();
   const int sub = lane / LPR, l = lane % LPR;
   const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t r0 = warp0 * kStep; r0 < total; r0 += nwarps * kStep) {
+  for (int64_t r0 = *lo_ptr + warp0 * kStep; r0 < total; r0 += nwarps * kStep) {
     uint4 v[U];
     int32_t g[U];
 #pragma unroll
@@ -408,8 +412,9 @@ gather_staged_rows_kernel(const uint4* __restrict__ staging, const int32_t* __re
 __global__ void __launch_bounds__(kThreads)
 gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
                                const int32_t* __restrict__ fb_id,
-                               const int32_t* __restrict__ fb_pos, const int32_t* total_ptr,
-                               TileMap tm, const uint32_t* __restrict__ bitmap,
+                               const int32_t* __restrict__ fb_pos, const int32_t* lo_ptr,
+                               const int32_t* hi_ptr, TileMap tm,
+                               const uint32_t* __restrict__ bitmap,
                                const uint16_t* __restrict__ wpref,
                                const int32_t* __restrict__ doff,
                                const unsigned long long* __restrict__ addr, int32_t rpb,
@@ -417,10 +422,11 @@ gather_staged_rows_wide_kernel(const uint4* __restrict__ staging, int64_t vecs,
                                uint4* __restrict__ out, const int32_t* status) {
   grid_dep_wait();
   if (failed(status)) return;
-  const int64_t total = *total_ptr;
+  const int64_t total = *hi_ptr;
   const int lane = lane_id();
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < total; i += nwarps) {
+  for (int64_t i = *lo_ptr + ((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5); i < total;
+       i += nwarps) {
     const int32_t id = __ldg(fb_id + i);
     const int64_t g = __ldg(fb_pos + i);
     const uint4* src = staged_row_src(staging, vecs, addr, rpb, cache_lo, cache_hi, tm, bitmap,
@@ -493,18 +499,21 @@ cudaError_t launch_tile_bitmaps(const int32_t* fb_id, const int32_t* cell_off,
 
 cudaError_t launch_load_distinct_rows(const unsigned long long* addr, int64_t row_bytes,
                                       int64_t rpb, const uint32_t* bitmap, const uint16_t* wpref,
-                                      const int32_t* doff, int32_t T, const int32_t* tile_first,
-                                      void* staging, unsigned long long cache_lo,
-                                      unsigned long long cache_hi, unsigned long long* host_rows,
-                                      const int32_t* status, int num_sms, cudaStream_t st) {
+                                      const int32_t* doff, int32_t t_lo, int32_t t_hi,
+                                      const int32_t* tile_first, void* staging,
+                                      unsigned long long cache_lo, unsigned long long cache_hi,
+                                      unsigned long long* host_rows, const int32_t* status,
+                                      int max_blocks, int num_sms, cudaStream_t st) {
   const int64_t vecs = row_bytes / 16;
   uint4* sg = (uint4*)staging;
+  if (t_hi <= t_lo) return cudaSuccess;
 #define AGNES_LOADD(LPR)                                                                      \
-  load_distinct_rows_kernel<LPR><<<resident_grid((const void*)load_distinct_rows_kernel<LPR>, \
-                                                 kThreads, num_sms),                          \
+  load_distinct_rows_kernel<LPR><<<std::min(max_blocks, resident_grid(                        \
+                                       (const void*)load_distinct_rows_kernel<LPR>, kThreads,  \
+                                       num_sms)),                                              \
                                    kThreads, 0, st>>>(addr, vecs, (int32_t)rpb, bitmap, wpref, \
-                                                      doff, T, tile_first, sg, cache_lo,       \
-                                                      cache_hi, host_rows, status)
+                                                      doff, t_lo, t_hi, tile_first, sg,        \
+                                                      cache_lo, cache_hi, host_rows, status)
   if (vecs <= 8)
     AGNES_LOADD(8);
   else if (vecs <= 16)
@@ -516,7 +525,7 @@ cudaError_t launch_load_distinct_rows(const unsigned long long* addr, int64_t ro
 }
 
 cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, const int32_t* fb_id,
-                                      const int32_t* fb_pos, const int32_t* total,
+                                      const int32_t* fb_pos, const int32_t* lo, const int32_t* hi,
                                       const int32_t* tile_first, const int32_t* chunk_tile,
                                       int32_t T, const uint32_t* bitmap, const uint16_t* wpref,
                                       const int32_t* doff, const unsigned long long* addr,
@@ -531,7 +540,7 @@ cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, co
   gather_staged_rows_kernel<LPR, 4><<<resident_grid(                                            \
                                           (const void*)gather_staged_rows_kernel<LPR, 4>,        \
                                           kThreads, num_sms),                                   \
-                                      kThreads, 0, st>>>(sg, fb_id, fb_pos, total, tm, bitmap,  \
+                                      kThreads, 0, st>>>(sg, fb_id, fb_pos, lo, hi, tm, bitmap, \
                                                          wpref, doff, addr, (int32_t)rpb,       \
                                                          cache_lo, cache_hi, o, status)
   if (vecs == 8)
@@ -543,7 +552,7 @@ cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, co
   else
     gather_staged_rows_wide_kernel<<<resident_grid((const void*)gather_staged_rows_wide_kernel,
                                                    kThreads, num_sms),
-                                     kThreads, 0, st>>>(sg, vecs, fb_id, fb_pos, total, tm, bitmap,
+                                     kThreads, 0, st>>>(sg, vecs, fb_id, fb_pos, lo, hi, tm, bitmap,
                                                         wpref, doff, addr, (int32_t)rpb, cache_lo,
                                                         cache_hi, o, status);
 #undef AGNES_GSR

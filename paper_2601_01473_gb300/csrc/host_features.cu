@@ -27,6 +27,8 @@ agnes_status setup_streaming(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStre
     CK(ctx, cudaEventCreateWithFlags(&ctx->slot_free[i], cudaEventDisableTiming));
   }
   CK(ctx, cudaEventCreateWithFlags(&ctx->gather_start, cudaEventDisableTiming));
+  for (int i = 0; i < kRowChunks; ++i)
+    CK(ctx, cudaEventCreateWithFlags(&ctx->rows_loaded[i], cudaEventDisableTiming));
   if (ctx->feature_io == AGNES_FEATURE_IO_BLOCKS) {
     ctx->slot_bytes = (int64_t)kStreamBatchBlocks * blk;
     CK(ctx, cudaMalloc((void**)&ctx->slots, (size_t)(ctx->slot_bytes * kStreamSlots)));
@@ -249,14 +251,31 @@ static agnes_status gather_rows_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* 
     ctx->rm_staging_rows = rows;
   }
   CK(ctx, cudaMemsetAsync(ctx->d_host_rows, 0, sizeof(unsigned long long), st));
-  CK(ctx, launch_load_distinct_rows(ctx->d_addr, rb, rpb, ctx->rm_bitmap, ctx->rm_wpref,
-                                    ctx->rm_doff, T, ctx->bt.tile_first, ctx->rm_staging, 0, 0,
-                                    ctx->d_host_rows, w.status, ctx->num_sms, st));
-  CK(ctx, launch_gather_staged_rows(ctx->rm_staging, rb, w.fb_id[cur], w.fb_pos[cur],
-                                    w.fcell_off[cur] + cells, ctx->bt.tile_first,
-                                    ctx->bt.chunk_tile, T, ctx->rm_bitmap, ctx->rm_wpref,
-                                    ctx->rm_doff, ctx->d_addr, rpb, 0, 0, w.feats_out,
-                                    w.status, ctx->num_sms, st));
+  // The rows are loaded on the copy stream in kRowChunks tile ranges, and each
+  // range's gather (HBM-bound) runs on st once its rows are in, overlapping
+  // the next range's load (bound by the host link).  The loads start when st
+  // gets here: the bitmaps are built, and the previous hyperbatch's gathers
+  // no longer read the staging rows.  The loader is held to four CTAs per SM,
+  // enough rows in flight for the link, so the gathers find room beside it.
+  CK(ctx, cudaEventRecord(ctx->gather_start, st));
+  CK(ctx, cudaStreamWaitEvent(ctx->copy_stream, ctx->gather_start, 0));
+  for (int c = 0; c < kRowChunks; ++c) {
+    const int32_t t_lo = (int32_t)((int64_t)T * c / kRowChunks);
+    const int32_t t_hi = (int32_t)((int64_t)T * (c + 1) / kRowChunks);
+    if (t_hi <= t_lo) continue;
+    CK(ctx, launch_load_distinct_rows(ctx->d_addr, rb, rpb, ctx->rm_bitmap, ctx->rm_wpref,
+                                      ctx->rm_doff, t_lo, t_hi, ctx->bt.tile_first,
+                                      ctx->rm_staging, 0, 0, ctx->d_host_rows, w.status,
+                                      4 * ctx->num_sms, ctx->num_sms, ctx->copy_stream));
+    CK(ctx, cudaEventRecord(ctx->rows_loaded[c], ctx->copy_stream));
+    CK(ctx, cudaStreamWaitEvent(st, ctx->rows_loaded[c], 0));
+    CK(ctx, launch_gather_staged_rows(ctx->rm_staging, rb, w.fb_id[cur], w.fb_pos[cur],
+                                      w.fcell_off[cur] + (int64_t)t_lo * w.H,
+                                      w.fcell_off[cur] + (int64_t)t_hi * w.H, ctx->bt.tile_first,
+                                      ctx->bt.chunk_tile, T, ctx->rm_bitmap, ctx->rm_wpref,
+                                      ctx->rm_doff, ctx->d_addr, rpb, 0, 0, w.feats_out,
+                                      w.status, ctx->num_sms, st));
+  }
   // rows read over the link, for the counters (read after the hyperbatch is done)
   CK(ctx, cudaMemcpyAsync(ctx->h_rm + 1, ctx->d_host_rows, sizeof(int64_t),
                           cudaMemcpyDeviceToHost, st));

@@ -191,20 +191,22 @@ cudaError_t launch_tile_bitmaps(const int32_t* fb_id, const int32_t* cell_off,
                                 const int32_t* tile_first, int32_t T, int32_t H, uint32_t* bitmap,
                                 uint16_t* wpref, int32_t* dcnt, const int32_t* status,
                                 cudaStream_t st);
-// Copies every distinct requested row (doff = exclusive scan of dcnt, T + 1
-// entries) of a block outside the feature cache [cache_lo, cache_hi) from its
-// block's address to staging, counting them in *host_rows.
+// Copies the distinct requested rows of tiles [t_lo, t_hi) (doff = exclusive
+// scan of dcnt, T + 1 entries) of blocks outside the feature cache
+// [cache_lo, cache_hi) from their block's address to staging, counting them
+// in *host_rows; at most max_blocks CTAs.
 cudaError_t launch_load_distinct_rows(const unsigned long long* addr, int64_t row_bytes,
                                       int64_t rpb, const uint32_t* bitmap, const uint16_t* wpref,
-                                      const int32_t* doff, int32_t T, const int32_t* tile_first,
-                                      void* staging, unsigned long long cache_lo,
-                                      unsigned long long cache_hi, unsigned long long* host_rows,
-                                      const int32_t* status, int num_sms, cudaStream_t st);
-// Gathers every entry of the final bucket from the staging row of its id,
-// or in place from the feature cache when its block's address (addr, one per
-// feature block of rpb rows) lies in [cache_lo, cache_hi).
+                                      const int32_t* doff, int32_t t_lo, int32_t t_hi,
+                                      const int32_t* tile_first, void* staging,
+                                      unsigned long long cache_lo, unsigned long long cache_hi,
+                                      unsigned long long* host_rows, const int32_t* status,
+                                      int max_blocks, int num_sms, cudaStream_t st);
+// Gathers the entries [*lo, *hi) of the final bucket from the staging row of
+// their id, or in place from the feature cache when its block's address (addr,
+// one per feature block of rpb rows) lies in [cache_lo, cache_hi).
 cudaError_t launch_gather_staged_rows(const void* staging, int64_t row_bytes, const int32_t* fb_id,
-                                      const int32_t* fb_pos, const int32_t* total,
+                                      const int32_t* fb_pos, const int32_t* lo, const int32_t* hi,
                                       const int32_t* tile_first, const int32_t* chunk_tile,
                                       int32_t T, const uint32_t* bitmap, const uint16_t* wpref,
                                       const int32_t* doff, const unsigned long long* addr,
