@@ -142,6 +142,9 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (ctx->own_indices) cudaFree(ctx->indices);
   if (ctx->own_features) cudaFree(ctx->features);
   if (ctx->done) cudaEventDestroy(ctx->done);
+  if (ctx->aux_fork) cudaEventDestroy(ctx->aux_fork);
+  if (ctx->aux_join) cudaEventDestroy(ctx->aux_join);
+  if (ctx->aux) cudaStreamDestroy(ctx->aux);
   for (int i = 0; i < kStreamSlots; ++i) {
     if (ctx->slot_copied[i]) cudaEventDestroy(ctx->slot_copied[i]);
     if (ctx->slot_free[i]) cudaEventDestroy(ctx->slot_free[i]);
@@ -380,8 +383,12 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   if (rc == AGNES_OK && d->topology_on_host && d->num_edges > 0 &&
       d->topology_io == AGNES_TOPOLOGY_IO_ROWS && d->graph_buffer_bytes > 0)
     rc = setup_topology_cache(ctx, d, st);
-  if (rc == AGNES_OK && cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess) {
-    set_err(ctx, "cudaEventCreate failed");
+  if (rc == AGNES_OK && (cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess ||
+                         cudaEventCreateWithFlags(&ctx->aux_fork, cudaEventDisableTiming) != cudaSuccess ||
+                         cudaEventCreateWithFlags(&ctx->aux_join, cudaEventDisableTiming) != cudaSuccess ||
+                         cudaStreamCreateWithFlags(&ctx->aux, cudaStreamNonBlocking) != cudaSuccess)) {
+    cudaGetLastError();
+    set_err(ctx, "creating events or the side stream failed");
     rc = AGNES_ECUDA;
   }
   if (rc != AGNES_OK) {

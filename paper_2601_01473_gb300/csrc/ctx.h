@@ -136,6 +136,10 @@ struct agnes_ctx {
   cudaEvent_t ev[agnes::kEventRing][agnes::kMaxPhases + 1] = {{nullptr}};
   bool ev_created = false;
   uint64_t ws_gen = 0;  // bumped whenever the workspace is reallocated
+  // side stream of a hyperbatch: each hop's col fix-up runs on it (forked
+  // after the new-id scan, joined before the next hop's sampling)
+  cudaStream_t aux = nullptr;
+  cudaEvent_t aux_fork = nullptr, aux_join = nullptr;
 
   // The resident path's launch sequence, captured once per hyperbatch shape
   // and replayed as one CUDA graph launch (agnes_set_launch_mode).

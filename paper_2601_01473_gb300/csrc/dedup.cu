@@ -558,6 +558,16 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   // frontier) the distinct sampled ids, numbered by their own column scan
   e = col_scan(d.newcnt, d.newbase, a.T, a.H, d.nsz_prev, d.srcsz, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
+  // final col of new nodes: needs only newbase from here on, so it may run
+  // beside the rest of the hop
+  cudaStream_t fix_st = st;
+  if (d.side) {
+    if ((e = cudaEventRecord(d.fork, st)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(d.side, d.fork, 0)) != cudaSuccess) return e;
+    fix_st = d.side;
+  }
+  dedup_fix_col_kernel<<<egrid, kThreads, 0, fix_st>>>(d.col, d.ecnt, a.ecap, d.scell, d.newbase,
+                                                       d.nsz_prev, a.status);
   if (d.frontier_sampled)
     e = col_scan(d.nfcnt, d.noutbase, a.T, a.H, nullptr, d.nsz_next, d.scan_scratch, a.status,
                  st);
@@ -567,8 +577,6 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   e = seg_scan<int32_t, int32_t>(d.nfcnt, 0, d.nfcell_off, 0, nullptr, ncells, 1, ncells, true,
                                  nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
-  dedup_fix_col_kernel<<<egrid, kThreads, 0, st>>>(d.col, d.ecnt, a.ecap, d.scell, d.newbase,
-                                                   d.nsz_prev, a.status);
   CompactArgs k;
   k.ncells = ncells;
   k.H = a.H;

@@ -157,6 +157,11 @@ struct DedupBufs {
   const int32_t* tile_adj_block;
   uint8_t* adj_flags;       // per topology block: touched at this hop
   int64_t* scan_scratch;
+  // If side is set, the col fix-up (which needs only newbase, col and scell)
+  // runs on it, forked from st through the event fork; the caller joins side
+  // back before anything rewrites scell, newbase or the hop's col.
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork = nullptr;
 };
 
 cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cudaStream_t st);

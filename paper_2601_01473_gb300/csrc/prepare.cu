@@ -253,6 +253,11 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
                                          cap[h], true, ecnt, w.scan_scratch, w.status, st)));
     mark();
     CK(ctx, cudaMemsetAsync(w.scnt, 0, sizeof(int32_t) * cells, st));
+    // the previous hop's col fix-up still reads scell and newbase
+    if (h > 0) {
+      CK(ctx, cudaEventRecord(ctx->aux_join, ctx->aux));
+      CK(ctx, cudaStreamWaitEvent(st, ctx->aux_join, 0));
+    }
     if (ctx->topo.on) {
       rc = fill_streamed(ctx, a, cur, h, st);
       if (rc != AGNES_OK) return rc;
@@ -307,12 +312,21 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.tile_adj_block = ctx->bt.tile_adj_block;
     d.adj_flags = w.adj_flags + (int64_t)h * ctx->bt.n_blocks;
     d.scan_scratch = w.scan_scratch;
+    d.side = ctx->aux;
+    d.fork = ctx->aux_fork;
     CK(ctx, launch_dedup(a, d, nsm, st));
     cur = 1 - cur;
   }
-  // feature blocks touched by the hyperbatch (stats; also the streaming list)
+  // blocks touched by the hyperbatch (the statistics), on the side stream
+  // beside the gather: feature blocks from the final bucket, topology blocks
+  // from the flags the dedup of each hop set
+  CK(ctx, cudaEventRecord(ctx->aux_fork, st));
+  CK(ctx, cudaStreamWaitEvent(ctx->aux, ctx->aux_fork, 0));
   CK(ctx, launch_mark_count(w.fcell_off[cur], T, H, ctx->bt.tile_feat_block, w.feat_flags,
-                            ctx->bt.n_feat_blocks, w.stats + K, w.status, st));
+                            ctx->bt.n_feat_blocks, w.stats + K, w.status, ctx->aux));
+  for (int h = 0; h < K; ++h)
+    CK(ctx, launch_mark_count(nullptr, T, H, nullptr, w.adj_flags + (int64_t)h * ctx->bt.n_blocks,
+                              ctx->bt.n_blocks, w.stats + h, w.status, ctx->aux));
   mark();
   if (ctx->features_on_host) {
     rc = gather_streamed(ctx, cur, st);
@@ -322,9 +336,10 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
                           w.fcell_off[cur] + cells, w.feats_out, w.status, nsm, st));
   }
   mark();
-  for (int h = 0; h < K; ++h)
-    CK(ctx, launch_mark_count(nullptr, T, H, nullptr, w.adj_flags + (int64_t)h * ctx->bt.n_blocks,
-                              ctx->bt.n_blocks, w.stats + h, w.status, st));
+  // the last hop's col fix-up and the statistics ran beside the compaction
+  // and the gather
+  CK(ctx, cudaEventRecord(ctx->aux_join, ctx->aux));
+  CK(ctx, cudaStreamWaitEvent(st, ctx->aux_join, 0));
   const Back b = back_of(w);
   CK(ctx, cudaMemcpyAsync(b.status, w.status, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(b.nsz, w.nsz, sizeof(int32_t) * (K + 1) * H, cudaMemcpyDeviceToHost, st));
@@ -350,7 +365,9 @@ static bool stream_capturing(cudaStream_t st) {
   return cs != cudaStreamCaptureStatusNone;
 }
 
-// Turns every kernel-to-kernel edge of the captured sequence into a
+// Turns every kernel-to-kernel link of the captured chain (an edge whose
+// source has no other successor and whose destination no other predecessor;
+// fork and join edges of the side stream stay as they are) into a
 // programmatic one from the programmatic port: the kernels trigger nothing
 // early, so the next kernel is launched as soon as every block of its
 // predecessor has exited, and its blocks wait at their first statement
@@ -368,7 +385,24 @@ static cudaError_t make_programmatic(cudaGraph_t graph, int64_t* converted) {
   std::vector<cudaGraphEdgeData> data(n);
   e = cudaGraphGetEdges(graph, from.data(), to.data(), data.data(), &n);
   if (e != cudaSuccess) return e;
+  std::vector<std::pair<cudaGraphNode_t, int>> outs, ins;  // edge counts per node
+  auto bump = [](std::vector<std::pair<cudaGraphNode_t, int>>& v, cudaGraphNode_t nd) {
+    for (auto& p : v)
+      if (p.first == nd) return ++p.second;
+    v.emplace_back(nd, 1);
+    return 1;
+  };
+  auto count = [](const std::vector<std::pair<cudaGraphNode_t, int>>& v, cudaGraphNode_t nd) {
+    for (const auto& p : v)
+      if (p.first == nd) return p.second;
+    return 0;
+  };
   for (size_t i = 0; i < n; ++i) {
+    bump(outs, from[i]);
+    bump(ins, to[i]);
+  }
+  for (size_t i = 0; i < n; ++i) {
+    if (count(outs, from[i]) != 1 || count(ins, to[i]) != 1) continue;
     cudaGraphNodeType tf, tt;
     if ((e = cudaGraphNodeGetType(from[i], &tf)) != cudaSuccess) return e;
     if ((e = cudaGraphNodeGetType(to[i], &tt)) != cudaSuccess) return e;
