@@ -144,6 +144,7 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   if (ctx->done) cudaEventDestroy(ctx->done);
   if (ctx->aux_fork) cudaEventDestroy(ctx->aux_fork);
   if (ctx->aux_join) cudaEventDestroy(ctx->aux_join);
+  if (ctx->aux_ready) cudaEventDestroy(ctx->aux_ready);
   if (ctx->aux) cudaStreamDestroy(ctx->aux);
   for (int i = 0; i < kStreamSlots; ++i) {
     if (ctx->slot_copied[i]) cudaEventDestroy(ctx->slot_copied[i]);
@@ -386,6 +387,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
   if (rc == AGNES_OK && (cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming) != cudaSuccess ||
                          cudaEventCreateWithFlags(&ctx->aux_fork, cudaEventDisableTiming) != cudaSuccess ||
                          cudaEventCreateWithFlags(&ctx->aux_join, cudaEventDisableTiming) != cudaSuccess ||
+                         cudaEventCreateWithFlags(&ctx->aux_ready, cudaEventDisableTiming) != cudaSuccess ||
                          cudaStreamCreateWithFlags(&ctx->aux, cudaStreamNonBlocking) != cudaSuccess)) {
     cudaGetLastError();
     set_err(ctx, "creating events or the side stream failed");

@@ -68,6 +68,7 @@ struct Workspace {
   uint8_t* feat_flags = nullptr;
   int64_t* stats = nullptr;  // K+1
   int64_t* scan_scratch = nullptr;
+  int64_t* side_scratch = nullptr;  // scans on the side stream
   int32_t* status = nullptr;
   unsigned long long* distinct = nullptr;
   uint64_t* key = nullptr;  // sampling key {seed, first minibatch id}
@@ -139,7 +140,7 @@ struct agnes_ctx {
   // side stream of a hyperbatch: each hop's col fix-up runs on it (forked
   // after the new-id scan, joined before the next hop's sampling)
   cudaStream_t aux = nullptr;
-  cudaEvent_t aux_fork = nullptr, aux_join = nullptr;
+  cudaEvent_t aux_fork = nullptr, aux_join = nullptr, aux_ready = nullptr;
 
   // The resident path's launch sequence, captured once per hyperbatch shape
   // and replayed as one CUDA graph launch (agnes_set_launch_mode).

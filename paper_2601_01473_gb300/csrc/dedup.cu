@@ -555,28 +555,37 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   // per-minibatch offsets of the new ids: scan down the tiles of the
   // tile-major [T x H] count matrix; totals give the next frontier sizes
   // |src_h| = |dst_h| + new ids; the next frontier is src_h, or (sampled
-  // frontier) the distinct sampled ids, numbered by their own column scan
-  e = col_scan(d.newcnt, d.newbase, a.T, a.H, d.nsz_prev, d.srcsz, d.scan_scratch, a.status, st);
-  if (e != cudaSuccess) return e;
-  // final col of new nodes: needs only newbase from here on, so it may run
-  // beside the rest of the hop
-  cudaStream_t fix_st = st;
+  // frontier) the distinct sampled ids, numbered by their own column scan.
+  // With a side stream, the new-id scan and the col fix-up (which needs only
+  // its result) run there, beside the scans of the next-frontier counts; the
+  // side stream has its own scan scratch, and the compaction waits for the
+  // new-id offsets.
+  cudaStream_t nst = st;
+  int64_t* nscratch = d.scan_scratch;
   if (d.side) {
     if ((e = cudaEventRecord(d.fork, st)) != cudaSuccess) return e;
     if ((e = cudaStreamWaitEvent(d.side, d.fork, 0)) != cudaSuccess) return e;
-    fix_st = d.side;
+    nst = d.side;
+    nscratch = d.side_scratch;
   }
-  dedup_fix_col_kernel<<<egrid, kThreads, 0, fix_st>>>(d.col, d.ecnt, a.ecap, d.scell, d.newbase,
-                                                       d.nsz_prev, a.status);
-  if (d.frontier_sampled)
+  e = col_scan(d.newcnt, d.newbase, a.T, a.H, d.nsz_prev, d.srcsz, nscratch, a.status, nst);
+  if (e != cudaSuccess) return e;
+  if (d.side && (e = cudaEventRecord(d.ready, d.side)) != cudaSuccess) return e;
+  dedup_fix_col_kernel<<<egrid, kThreads, 0, nst>>>(d.col, d.ecnt, a.ecap, d.scell, d.newbase,
+                                                    d.nsz_prev, a.status);
+  if (d.frontier_sampled) {
     e = col_scan(d.nfcnt, d.noutbase, a.T, a.H, nullptr, d.nsz_next, d.scan_scratch, a.status,
                  st);
-  else
-    e = cudaMemcpyAsync(d.nsz_next, d.srcsz, sizeof(int32_t) * a.H, cudaMemcpyDeviceToDevice, st);
-  if (e != cudaSuccess) return e;
+    if (e != cudaSuccess) return e;
+  }
   e = seg_scan<int32_t, int32_t>(d.nfcnt, 0, d.nfcell_off, 0, nullptr, ncells, 1, ncells, true,
                                  nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
+  if (d.side && (e = cudaStreamWaitEvent(st, d.ready, 0)) != cudaSuccess) return e;
+  if (!d.frontier_sampled) {
+    e = cudaMemcpyAsync(d.nsz_next, d.srcsz, sizeof(int32_t) * a.H, cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return e;
+  }
   CompactArgs k;
   k.ncells = ncells;
   k.H = a.H;

@@ -157,11 +157,14 @@ struct DedupBufs {
   const int32_t* tile_adj_block;
   uint8_t* adj_flags;       // per topology block: touched at this hop
   int64_t* scan_scratch;
-  // If side is set, the col fix-up (which needs only newbase, col and scell)
-  // runs on it, forked from st through the event fork; the caller joins side
-  // back before anything rewrites scell, newbase or the hop's col.
+  // If side is set, the new-id scan (into newbase, with side_scratch) and the
+  // col fix-up (which needs only newbase, col and scell) run on it, forked
+  // from st through the event fork; st waits for the scan through the event
+  // ready, and the caller joins side back before anything rewrites scell,
+  // newbase or the hop's col.
   cudaStream_t side = nullptr;
-  cudaEvent_t fork = nullptr;
+  cudaEvent_t fork = nullptr, ready = nullptr;
+  int64_t* side_scratch = nullptr;  // col_scan_scratch_elems(T, H) int64
 };
 
 cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cudaStream_t st);

@@ -67,6 +67,7 @@ void free_workspace(Workspace* w) {
   cudaFree(w->feat_flags);
   cudaFree(w->stats);
   cudaFree(w->scan_scratch);
+  cudaFree(w->side_scratch);
   cudaFree(w->status);
   cudaFree(w->distinct);
   cudaFree(w->key);
@@ -164,6 +165,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.feat_flags, nfb);
   WA(w.stats, K + 1);
   WA(w.scan_scratch, scratch);
+  WA(w.side_scratch, s4);
   WA(w.status, 1);
   WA(w.distinct, 1);
   WA(w.key, 2);
@@ -178,6 +180,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
     return AGNES_ENOMEM;
   }
   if (cudaMemset(w.scan_scratch, 0, sizeof(int64_t) * scratch) != cudaSuccess ||
+      cudaMemset(w.side_scratch, 0, sizeof(int64_t) * s4) != cudaSuccess ||
       cudaMemset(w.fcnt, 0, sizeof(int32_t) * cells) != cudaSuccess ||
       cudaMemset(w.scnt, 0, sizeof(int32_t) * cells) != cudaSuccess) {
     free_workspace(&w);
@@ -314,6 +317,8 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.scan_scratch = w.scan_scratch;
     d.side = ctx->aux;
     d.fork = ctx->aux_fork;
+    d.ready = ctx->aux_ready;
+    d.side_scratch = w.side_scratch;
     CK(ctx, launch_dedup(a, d, nsm, st));
     cur = 1 - cur;
   }
