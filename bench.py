@@ -266,6 +266,9 @@ def main():
                     help="time the GraphSAGE-mean consumer layer on a prepared hyperbatch")
     ap.add_argument("--sage-d-out", type=int, default=128)
     ap.add_argument("--sage-out", default="f32", choices=["f32", "f16"])
+    ap.add_argument("--frontier", default="src", choices=["src", "sampled"],
+                    help="next-hop frontier: src_h (default) or Algorithm 1's literal N_out "
+                         "(the path byte model then counts dst_{h+1} as src_h)")
     ap.add_argument("--launch-mode", default="graph_pdl", choices=["direct", "graph", "graph_pdl"],
                     help="resident path: direct launches, one CUDA graph per hyperbatch shape, "
                          "or the graph with programmatic kernel edges")
@@ -332,6 +335,7 @@ def main():
               feature_cache_threshold=args.feature_cache_threshold,
               feature_io=args.feature_io if args.stream else "blocks")
     g.set_launch_mode(args.launch_mode)
+    g.set_frontier(args.frontier)
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
@@ -484,7 +488,7 @@ def main():
                                  "adj_blocks": info["adj_blocks"], "tiles": info["tiles"],
                                  "feat_blocks": info["feat_blocks"]},
                        "H": w.H, "B": w.B, "fanouts": fan, "parallelism": f"replicas{world}",
-                       "launch_mode": args.launch_mode,
+                       "launch_mode": args.launch_mode, "frontier": args.frontier,
                        "l2": "inputs larger than L2 (graph ~%.0f GB vs 129 MB L2), no flush"
                              % ((offsets.numel() * offsets.element_size()
                                  + indices.numel() * 4

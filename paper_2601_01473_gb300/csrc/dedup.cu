@@ -586,6 +586,12 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
     e = cudaMemcpyAsync(d.nsz_next, d.srcsz, sizeof(int32_t) * a.H, cudaMemcpyDeviceToDevice, st);
     if (e != cudaSuccess) return e;
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dedup_compact(const HopArgs& a, const DedupBufs& d, int num_sms,
+                                 cudaStream_t st) {
+  const int64_t ncells = (int64_t)a.T * a.H;
   CompactArgs k;
   k.ncells = ncells;
   k.H = a.H;

@@ -167,7 +167,13 @@ struct DedupBufs {
   int64_t* side_scratch = nullptr;  // col_scan_scratch_elems(T, H) int64
 };
 
+// One hop's dedup up to the next-frontier offsets (nfcell_off, nsz_next) and
+// the new-id offsets (newbase): scatter, cells, big cells, scans, col fix-up.
 cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cudaStream_t st);
+// Then the compaction: the next frontier bucket (nfb_id / nfb_pos) and the
+// new nodes' ids in the node lists.
+cudaError_t launch_dedup_compact(const HopArgs& a, const DedupBufs& d, int num_sms,
+                                 cudaStream_t st);
 
 // ---- gather.cu -------------------------------------------------------------
 cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,

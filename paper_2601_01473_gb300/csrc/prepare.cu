@@ -320,18 +320,22 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.ready = ctx->aux_ready;
     d.side_scratch = w.side_scratch;
     CK(ctx, launch_dedup(a, d, nsm, st));
+    if (h + 1 == K) {
+      // blocks touched by the hyperbatch (the statistics), on the side stream
+      // beside the last compaction: feature blocks from the final bucket's
+      // offsets, topology blocks from the flags the dedup of each hop set
+      CK(ctx, cudaEventRecord(ctx->aux_fork, st));
+      CK(ctx, cudaStreamWaitEvent(ctx->aux, ctx->aux_fork, 0));
+      CK(ctx, launch_mark_count(w.fcell_off[1 - cur], T, H, ctx->bt.tile_feat_block, w.feat_flags,
+                                ctx->bt.n_feat_blocks, w.stats + K, w.status, ctx->aux));
+      for (int hh = 0; hh < K; ++hh)
+        CK(ctx, launch_mark_count(nullptr, T, H, nullptr,
+                                  w.adj_flags + (int64_t)hh * ctx->bt.n_blocks, ctx->bt.n_blocks,
+                                  w.stats + hh, w.status, ctx->aux));
+    }
+    CK(ctx, launch_dedup_compact(a, d, nsm, st));
     cur = 1 - cur;
   }
-  // blocks touched by the hyperbatch (the statistics), on the side stream
-  // beside the gather: feature blocks from the final bucket, topology blocks
-  // from the flags the dedup of each hop set
-  CK(ctx, cudaEventRecord(ctx->aux_fork, st));
-  CK(ctx, cudaStreamWaitEvent(ctx->aux, ctx->aux_fork, 0));
-  CK(ctx, launch_mark_count(w.fcell_off[cur], T, H, ctx->bt.tile_feat_block, w.feat_flags,
-                            ctx->bt.n_feat_blocks, w.stats + K, w.status, ctx->aux));
-  for (int h = 0; h < K; ++h)
-    CK(ctx, launch_mark_count(nullptr, T, H, nullptr, w.adj_flags + (int64_t)h * ctx->bt.n_blocks,
-                              ctx->bt.n_blocks, w.stats + h, w.status, ctx->aux));
   mark();
   if (ctx->features_on_host) {
     rc = gather_streamed(ctx, cur, st);
@@ -341,8 +345,7 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
                           w.fcell_off[cur] + cells, w.feats_out, w.status, nsm, st));
   }
   mark();
-  // the last hop's col fix-up and the statistics ran beside the compaction
-  // and the gather
+  // the last hop's col fix-up and the statistics ran beside its compaction
   CK(ctx, cudaEventRecord(ctx->aux_join, ctx->aux));
   CK(ctx, cudaStreamWaitEvent(st, ctx->aux_join, 0));
   const Back b = back_of(w);
