@@ -336,15 +336,22 @@ agnes_status agnes_get_graph_info(agnes_ctx* ctx, agnes_graph_info* out);
 agnes_status agnes_copy_adj_blocks(agnes_ctx* ctx, int32_t* start_node, int32_t* start_block,
                                    int64_t cap);
 
-/* Optional per-phase timing of later prepares with CUDA events on the
- * caller's stream (off by default; the events of the last 64 prepares are
- * kept).  agnes_phase_times writes up to n milliseconds of the prepare
- * issued `ago` calls before the latest one (0 = the latest, < 64), in
- * order: [0] bucketing of the targets, then per hop h (3 each): [1+3h]
- * count+scan, [2+3h] sampling, [3+3h] dedup+relabel, then [1+3K] gather;
- * *n_out receives the count (0 if that prepare was not profiled).  Waits
- * for the latest prepare like fetch.  Errors: EINVAL (ago out of range). */
-agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable);
+/* Optional timing of later prepares with CUDA events on the caller's stream
+ * (off by default; the events of the last 64 prepares are kept).
+ * AGNES_PROFILE_PHASES: agnes_phase_times writes, in order, [0] bucketing of
+ *   the targets, then per hop h (3 each): [1+3h] count+scan, [2+3h]
+ *   sampling, [3+3h] dedup+relabel, then [1+3K] gather.
+ * AGNES_PROFILE_GATHER: only [0] the gather.  Each event splits the launch
+ *   sequence at that point (it is a dependency of what follows), so fewer
+ *   events cost less: two instead of 3K + 3.
+ * agnes_phase_times writes up to n milliseconds of the prepare issued `ago`
+ * calls before the latest one (0 = the latest, < 64); *n_out receives the
+ * count (0 if that prepare was not profiled).  Waits for the latest prepare
+ * like fetch.  Errors: EINVAL (mode unknown, ago out of range). */
+#define AGNES_PROFILE_OFF 0
+#define AGNES_PROFILE_PHASES 1
+#define AGNES_PROFILE_GATHER 2
+agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t mode);
 agnes_status agnes_phase_times(agnes_ctx* ctx, int32_t ago, float* ms, int32_t n,
                                int32_t* n_out);
 

@@ -432,8 +432,18 @@ class Graph:
         _check(lib().agnes_copy_adj_blocks(self._ctx, sn.data_ptr(), sb.data_ptr(), n), self._ctx)
         return sn[:n], sb[:n]
 
-    def set_profiling(self, enable: bool):
-        _check(lib().agnes_set_profiling(self._ctx, int(enable)), self._ctx)
+    def set_profiling(self, mode):
+        """CUDA-event timing of later prepares: True or "phases" (every phase),
+        "gather" (the gather only, two events), False or "off"."""
+        if mode is True or mode == "phases":
+            m = 1
+        elif mode == "gather":
+            m = 2
+        elif mode is False or mode == "off":
+            m = 0
+        else:
+            raise ValueError("profiling mode must be True/'phases', 'gather' or False/'off'")
+        _check(lib().agnes_set_profiling(self._ctx, m), self._ctx)
 
     def phase_times(self, ago: int = 0) -> list:
         """Per-phase milliseconds of the prepare issued ``ago`` calls before

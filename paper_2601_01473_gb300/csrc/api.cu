@@ -567,9 +567,13 @@ agnes_status agnes_copy_adj_blocks(agnes_ctx* ctx, int32_t* start_node, int32_t*
   return AGNES_OK;
 }
 
-agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t enable) {
+agnes_status agnes_set_profiling(agnes_ctx* ctx, int32_t mode) {
   if (!ctx) return AGNES_EINVAL;
-  ctx->profiling = enable != 0;
+  if (mode != AGNES_PROFILE_OFF && mode != AGNES_PROFILE_PHASES && mode != AGNES_PROFILE_GATHER) {
+    set_err(ctx, "profiling mode must be AGNES_PROFILE_OFF, _PHASES or _GATHER");
+    return AGNES_EINVAL;
+  }
+  ctx->profiling = mode;
   return AGNES_OK;
 }
 

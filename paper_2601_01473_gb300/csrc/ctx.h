@@ -131,7 +131,7 @@ struct agnes_ctx {
   int cur = 0;  // which frontier buffer holds the final bucket
   cudaEvent_t done = nullptr;
 
-  bool profiling = false;
+  int32_t profiling = AGNES_PROFILE_OFF;
   int64_t n_prepared = 0;                  // prepares issued so far
   int n_phases[agnes::kEventRing] = {0};          // per ring slot; 0 = not profiled
   cudaEvent_t ev[agnes::kEventRing][agnes::kMaxPhases + 1] = {{nullptr}};
@@ -151,7 +151,7 @@ struct agnes_ctx {
     cudaGraphExec_t exec = nullptr;
     // what the capture depends on
     int32_t H = 0, B = 0, K = 0, fan[AGNES_MAX_HOPS] = {0}, frontier_mode = 0, built_mode = 0;
-    bool profiling = false;
+    int32_t profiling = AGNES_PROFILE_OFF;
     uint64_t ws_gen = 0;
     // phase-event nodes, re-pointed at each launch's ring slot
     cudaGraphNode_t phase_node[agnes::kMaxPhases + 1] = {nullptr};

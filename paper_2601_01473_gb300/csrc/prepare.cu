@@ -215,8 +215,11 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
   const int64_t cells = (int64_t)T * H;
   const int nsm = ctx->num_sms;
   int ph = 0;
-  auto mark = [&]() {
-    if (ctx->profiling) cudaEventRecordWithFlags(ctx->ev[ring][ph++], st, mark_flags);
+  // a phase boundary; with AGNES_PROFILE_GATHER only the gather's two count
+  auto mark = [&](bool gather_edge = false) {
+    if (ctx->profiling == AGNES_PROFILE_PHASES ||
+        (ctx->profiling == AGNES_PROFILE_GATHER && gather_edge))
+      cudaEventRecordWithFlags(ctx->ev[ring][ph++], st, mark_flags);
   };
 
   mark();
@@ -336,7 +339,7 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     CK(ctx, launch_dedup_compact(a, d, nsm, st));
     cur = 1 - cur;
   }
-  mark();
+  mark(true);
   if (ctx->features_on_host) {
     rc = gather_streamed(ctx, cur, st);
     if (rc != AGNES_OK) return rc;
@@ -344,7 +347,7 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     CK(ctx, launch_gather(ctx->features, ctx->row_bytes, w.fb_id[cur], w.fb_pos[cur],
                           w.fcell_off[cur] + cells, w.feats_out, w.status, nsm, st));
   }
-  mark();
+  mark(true);
   // the last hop's col fix-up and the statistics ran beside its compaction
   CK(ctx, cudaEventRecord(ctx->aux_join, ctx->aux));
   CK(ctx, cudaStreamWaitEvent(st, ctx->aux_join, 0));

@@ -69,7 +69,8 @@ def test_graph_replays_match_the_oracle_and_direct_launches(cuda_device):
            (3, [5, 5], 7, 0, "src", False),         # new shape: capture
            (6, [6, 4, 3], 9, 12, "sampled", False),  # new shape and frontier: capture
            (6, [6, 4, 3], 9, 18, "src", True),      # frontier and profiling: capture
-           (6, [6, 4, 3], 3, 24, "src", True)]      # replay, phase events re-pointed
+           (6, [6, 4, 3], 3, 24, "src", True),      # replay, phase events re-pointed
+           (6, [6, 4, 3], 4, 30, "src", "gather")]  # gather events only: capture
     for step, (H, fan, seed, gid, frontier, prof) in enumerate(seq):
         targets = synth.hyperbatch_targets(pool, H, 150, 3, step)
         for g in ctxs:
@@ -83,10 +84,11 @@ def test_graph_replays_match_the_oracle_and_direct_launches(cuda_device):
         if prof:
             for g in ctxs:
                 t = g.phase_times(0)
-                assert len(t) == 2 + 3 * len(fan) and all(x >= 0 for x in t)
+                n = 1 if prof == "gather" else 2 + 3 * len(fan)
+                assert len(t) == n and all(x >= 0 for x in t)
     for g in ctxs[:2]:
         c = g.counters()
-        assert c["graph_captures"] == 4 and c["graph_launches"] == len(seq)
+        assert c["graph_captures"] == 5 and c["graph_launches"] == len(seq)
     assert pdl.counters()["graph_programmatic_edges"] > 20
     assert graphed.counters()["graph_programmatic_edges"] == 0
     d = direct.counters()
