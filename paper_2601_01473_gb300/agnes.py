@@ -220,7 +220,7 @@ class HyperbatchView:
     buffer ([H, capacity, ...]) plus host size tables; ``view(j)`` slices
     minibatch j out of them."""
 
-    def __init__(self, v: _HyperbatchView, device):
+    def __init__(self, v: _HyperbatchView, device, tensors=None):
         K, H = v.K, v.H
         self.K, self.H = K, H
         import numpy as np
@@ -231,12 +231,25 @@ class HyperbatchView:
         ss = np.ctypeslib.as_array(ctypes.cast(v.src_size, ctypes.POINTER(ctypes.c_int32)),
                                    shape=(K * H,)).reshape(K, H).copy()
         self.node_size, self.edges, self.src_size = sz, ed, ss
-        self.indptr = [_wrap(v.indptr[h], (H, v.indptr_stride[h]), torch.int64, device)
-                       for h in range(K)]
-        self.col = [_wrap(v.col[h], (H, v.col_stride[h]), torch.int32, device) for h in range(K)]
-        self.nodes = _wrap(v.nodes, (H, v.nodes_stride), torch.int32, device)
-        self.feats = _wrap(v.feats, (H, v.feats_stride_rows, v.feat_dim),
-                           _TORCH_OF[v.feat_dtype], device)
+        if tensors is None:  # wrappers of the ctx's output buffers
+            tensors = ([_wrap(v.indptr[h], (H, v.indptr_stride[h]), torch.int64, device)
+                        for h in range(K)],
+                       [_wrap(v.col[h], (H, v.col_stride[h]), torch.int32, device)
+                        for h in range(K)],
+                       _wrap(v.nodes, (H, v.nodes_stride), torch.int32, device),
+                       _wrap(v.feats, (H, v.feats_stride_rows, v.feat_dim),
+                             _TORCH_OF[v.feat_dtype], device))
+        self.indptr, self.col, self.nodes, self.feats = tensors
+        self._tensors = tensors
+
+    @staticmethod
+    def _key(v: _HyperbatchView):
+        """What the buffer wrappers depend on: addresses, strides, shapes."""
+        K = v.K
+        return (K, v.H, v.nodes, v.nodes_stride, v.feats, v.feats_stride_rows, v.feat_dim,
+                v.feat_dtype, tuple(v.indptr[h] for h in range(K)),
+                tuple(v.indptr_stride[h] for h in range(K)), tuple(v.col[h] for h in range(K)),
+                tuple(v.col_stride[h] for h in range(K)))
 
     def view(self, j: int) -> "MinibatchView":
         hops = []
@@ -346,10 +359,16 @@ class Graph:
         return MinibatchView(hops, nodes, feats)
 
     def fetch_all(self) -> HyperbatchView:
-        """All minibatches of the last hyperbatch (one wait, one size read-back)."""
+        """All minibatches of the last hyperbatch (one wait, one size read-back).
+        The output buffers' tensor wrappers are reused while the ctx's
+        workspace stays where it is (same hyperbatch shape)."""
         v = _HyperbatchView()
         _check(lib().agnes_fetch_hyperbatch(self._ctx, ctypes.byref(v)), self._ctx)
-        return HyperbatchView(v, self.device)
+        key = HyperbatchView._key(v)
+        cached = getattr(self, "_hv_cache", None)
+        hv = HyperbatchView(v, self.device, cached[1] if cached and cached[0] == key else None)
+        self._hv_cache = (key, hv._tensors)
+        return hv
 
     def set_frontier(self, mode: str) -> None:
         """"src" (dst_{h+1} = src_h, the default) or "sampled" (dst_{h+1} =
