@@ -505,7 +505,7 @@ def main():
                        "gen_seconds": round(gen_s, 1)},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "host_link": host_link,
             "topology_streaming": topo,
-            # counted for the HBM-resident path (the ncu launch list has 59 per hyperbatch
+            # counted for the HBM-resident path (the ncu launch list has 61 per hyperbatch
             # at K = 3); the host-resident modes add per-batch loads and gathers
             "gpu_launches": kernel_launches_per_step(K) * args.steps
             if not (args.stream or args.stream_topology) else None,
