@@ -71,8 +71,10 @@ def test_fullsize_parity(cuda_device, name, sample):
 def test_config5_variants_parity(cuda_device):
     """Config 5 at full size: rmat100m's graph as a sweep point (256 KB blocks,
     H = 16), with its features in pinned host memory (row I/O through a 4 GB
-    feature cache, then block I/O), and with its neighbour lists read in place
-    from pinned host memory.  Sampled minibatches bit-exact against the oracle."""
+    feature cache, block I/O, row I/O pipelined over tile ranges), and with
+    its neighbour lists read in place from pinned host memory (without and
+    with a 1 GB topology cache).  Sampled minibatches bit-exact against the
+    oracle."""
     w = WORKLOADS["rmat100m"]
     offsets, indices, features = build_graph(w, cuda_device)
     pool = target_pool(w, cuda_device)
@@ -90,8 +92,13 @@ def test_config5_variants_parity(cuda_device):
                            feature_cache_bytes=4 << 30),
         "blocks": dict(offsets=offsets, indices=indices, features=host_feats,
                        features_on_host=True),
+        "rows": dict(offsets=offsets, indices=indices, features=host_feats,
+                     features_on_host=True, feature_io="rows"),
         "topology rows": dict(offsets=offsets, indices=host_ind, features=features,
                               topology_on_host=True, topology_io="rows"),
+        "topology rows+cache": dict(offsets=offsets, indices=host_ind, features=features,
+                                    topology_on_host=True, topology_io="rows",
+                                    graph_buffer_bytes=1 << 30),
     }
     for name, kw in variants.items():
         g = Graph(adj_block_bytes=ws.adj_block_bytes, feat_block_bytes=ws.feat_block_bytes, **kw)
@@ -102,6 +109,8 @@ def test_config5_variants_parity(cuda_device):
                          _bytes(g.fetch(j).feats)) for j in sample}
         if name == "rows+cache":
             assert g.counters()["fcache_hit_blocks"] > 0
+        if name == "topology rows+cache":
+            assert g.counters()["topo_cached_requests"] > 0
         g.close()
     og = oracle.Graph(offsets.cpu().numpy(), host_ind.numpy(), host_feats.numpy())
     t = targets.cpu().numpy()
