@@ -208,12 +208,16 @@ agnes_status agnes_set_frontier_mode(agnes_ctx* ctx, int32_t mode);
  *   caller's stream for every later hyperbatch of that shape; the targets
  *   copy and the sampling key {seed, first_minibatch_id} are written to
  *   device memory ahead of it.
- * AGNES_LAUNCH_GRAPH_PDL (default): as AGNES_LAUNCH_GRAPH, with each
- *   kernel-to-kernel edge of the graph made programmatic (programmatic
- *   dependent launch: a kernel is launched once every block of the previous
- *   one has exited, and first waits for its writes to become visible), so
- *   each launch overlaps the previous kernel's completion.
- * Results are identical in every mode.  A caller stream that is itself being
+ * AGNES_LAUNCH_GRAPH_PDL (default): as AGNES_LAUNCH_GRAPH, with each link of
+ *   the graph's kernel chain (one predecessor, one successor) made
+ *   programmatic (programmatic dependent launch: a kernel is launched once
+ *   every block of the previous one has exited, and first waits for its
+ *   writes to become visible), so each launch overlaps the previous kernel's
+ *   completion.
+ * In every mode, work off the critical chain (each hop's new-id scan and col
+ * fix-up, the touched-block statistics) runs on a side stream the ctx owns,
+ * forked from and joined back into the caller's stream within the call's
+ * work.  Results are identical in every mode.  A caller stream that is itself being
  * captured, and the host-resident modes (whose calls read sizes back
  * mid-sequence), always take the direct path.  Errors: EINVAL. */
 #define AGNES_LAUNCH_DIRECT 0
