@@ -10,7 +10,6 @@
 
 using namespace agnes;
 
-// Graph buffer, tables and copy stream for topology in pinned host memory.
 // Host copies of the block tables the topology modes plan with: the edge
 // range of every physical block and the blocks of every block run.
 static agnes_status topology_host_tables(agnes_ctx* ctx, const agnes_graph_desc* d,
@@ -74,6 +73,8 @@ agnes_status setup_topology_cache(agnes_ctx* ctx, const agnes_graph_desc* d,
   return AGNES_OK;
 }
 
+// Graph buffer, tables and copy stream for topology in pinned host memory
+// with block I/O.
 agnes_status setup_topology(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStream_t st) {
   agnes_ctx::Topo& tp = ctx->topo;
   const int64_t nb = ctx->bt.n_blocks, ns = ctx->bt.n_starts;
@@ -138,10 +139,11 @@ static void lru_touch(agnes_ctx::Topo& tp, int32_t i) {
 }
 
 // Sampling with the topology in pinned host memory.  The block runs the
-// frontier touches are read back; runs are taken in ascending order into
-// waves that fit the graph buffer: each needed block is either resident
-// (a hit: pinned and moved to the recent end of the LRU list) or copied into
-// the least recently used unpinned slot on the side stream.  The slot table
+// frontier touches are read back; runs are taken in order (ascending and
+// descending in turn, hop by hop) into waves that fit the graph buffer: each
+// needed block is either resident (a hit: pinned and moved to the recent end
+// of the LRU list) or copied into the least recently used unpinned slot on
+// the topology's copy stream.  The slot table
 // is uploaded, the wave's cells are sampled, and the wave's blocks unpin when
 // the next wave starts (its copies wait for this wave's sampling to finish).
 agnes_status fill_streamed(agnes_ctx* ctx, const HopArgs& a, int cur, int h,
