@@ -137,8 +137,11 @@ struct agnes_ctx {
   cudaEvent_t ev[agnes::kEventRing][agnes::kMaxPhases + 1] = {{nullptr}};
   bool ev_created = false;
   uint64_t ws_gen = 0;  // bumped whenever the workspace is reallocated
-  // side stream of a hyperbatch: each hop's col fix-up runs on it (forked
-  // after the new-id scan, joined before the next hop's sampling)
+  // side stream of a hyperbatch: each hop's new-id scan and col fix-up run on
+  // it (forked after the cells are resolved; the compaction waits for the
+  // scan through aux_ready; joined before the next hop's sampling), and the
+  // touched-block statistics (forked before the last compaction, joined
+  // before the size read-back)
   cudaStream_t aux = nullptr;
   cudaEvent_t aux_fork = nullptr, aux_join = nullptr, aux_ready = nullptr;
 

@@ -83,7 +83,7 @@ static int64_t feat_block_bytes_of(const agnes_ctx* ctx, int32_t b) {
 // host link standing in for the SSD).  A touched block that is cached and
 // resident is read in place; one admitted to the cache but not yet loaded is
 // loaded into its cache slot; any other is loaded into the ring of HBM
-// staging slots.  Batch by batch, a loader kernel on the side stream reads
+// staging slots.  Batch by batch, a loader kernel on the copy stream reads
 // the batch's blocks over the host link; the batch's gather waits for it and
 // the next load into a slot waits for the gather that last read it.
 static agnes_status gather_blocks_io(agnes_ctx* ctx, int cur, int32_t n, int64_t* bytes_out,
