@@ -36,7 +36,9 @@
  * enqueued on the caller's CUDA stream (NULL = the legacy default stream);
  * calls on one ctx must not overlap.  Pointers are host or device memory as
  * stated per argument; the library detects which with
- * cudaPointerGetAttributes where both are allowed.
+ * cudaPointerGetAttributes where both are allowed.  A call that works on the
+ * GPU makes the ctx's device current for its duration and restores the
+ * calling thread's current device before it returns.
  */
 #ifndef AGNES_H
 #define AGNES_H
@@ -409,12 +411,13 @@ agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const void* x, i
  *  fanout  1 <= fanout <= AGNES_MAX_FANOUT.
  * Its scratch (64 KiB: per-chunk partial sums and an error word) is a
  * static device array that every GPU loading the library holds until the
- * process exits; nothing is allocated per call.  The first call on a device
- * looks up that array's device address, so make that first call before any
- * stream capture.  All calls on a device share the array: calls that overlap
- * on the GPU race and must be serialised by the caller.  The call enqueues its
- * work on cuda_stream and then waits for it (to report node ids outside
- * [0, N) as EINVAL).  Errors: EINVAL, ERANGE, ECUDA. */
+ * process exits; nothing is allocated per call.  Each call looks up that
+ * array's device address on the ctx's device (a host-side query).  All calls
+ * on a device share the array: calls that overlap on the GPU race and must be
+ * serialised by the caller.  The call enqueues its work on cuda_stream and
+ * then synchronises that stream (to report node ids outside [0, N) as
+ * EINVAL), so it must not be made while cuda_stream is being captured into a
+ * CUDA graph.  Errors: EINVAL, ERANGE, ECUDA. */
 #define AGNES_NOALLOC_MAX_NODES (1LL << 24)
 agnes_status agnes_hop_indptr_noalloc(agnes_ctx* ctx, const int32_t* nodes, int64_t n,
                                       int32_t fanout, int64_t* indptr, void* cuda_stream);

@@ -17,9 +17,11 @@
  *     src_h = dst_h ++ new_h; col[e] = index of the e-th neighbour in src_h
  *     dst_{h+1} = src_h
  *   feats = features[src_K]  (Gather)
- * The readings taken where the paper is silent (without-replacement
- * sampling, dst kept as a prefix of src, ascending order of new nodes, the
- * Philox key layout, the block packing rule) are listed in the design doc.
+ * Where the paper is silent this file takes these readings: sampling is
+ * without replacement over adjacency positions, dst is kept as a prefix of
+ * src, new nodes are in ascending id order, Philox is keyed as stated above,
+ * and blocks are packed greedily in id order.  Each is a choice the paper
+ * leaves open, not a result it fixes.
  */
 #include "agnes_oracle.h"
 

@@ -83,7 +83,7 @@ static agnes_status wait_prepared(agnes_ctx* ctx) {
     return AGNES_ESTATE;
   }
   if (!ctx->synced) {
-    cudaSetDevice(ctx->device);
+    DeviceGuard dg(ctx->device);
     cudaError_t e = cudaEventSynchronize(ctx->done);
     if (e != cudaSuccess) {
       set_err(ctx, "waiting for the hyperbatch failed: %s", cudaGetErrorString(e));
@@ -132,7 +132,7 @@ const char* agnes_last_error(agnes_ctx* ctx) { return ctx ? ctx->err : g_err; }
 
 agnes_status agnes_free(agnes_ctx* ctx) {
   if (!ctx) return AGNES_OK;
-  cudaSetDevice(ctx->device);
+  DeviceGuard dg(ctx->device);
   cudaDeviceSynchronize();
   drop_launch_graph(&ctx->lg);
   if (ctx->lg.cap) cudaStreamDestroy(ctx->lg.cap);
@@ -290,8 +290,8 @@ agnes_status agnes_load_graph(const agnes_graph_desc* d, int device, void* cuda_
                      "feature cache needs features_on_host");
     return AGNES_EINVAL;
   }
-  if (cudaSetDevice(device) != cudaSuccess) {
-    cudaGetLastError();
+  DeviceGuard dg(device);
+  if (!dg.ok()) {
     set_err(nullptr, "invalid device %d", device);
     return AGNES_EINVAL;
   }
@@ -512,7 +512,7 @@ agnes_status agnes_hyperbatch_counters(agnes_ctx* ctx, agnes_counters* out) {
     }
   for (int j = 0; j < w.H; ++j) out->rows += b.nsz[(size_t)w.K * w.H + j];
   out->row_bytes = ctx->row_bytes;
-  cudaSetDevice(ctx->device);
+  DeviceGuard dg(ctx->device);
   unsigned long long distinct = 0;
   CK(ctx, cudaMemset(w.distinct, 0, sizeof(unsigned long long)));
   CK(ctx, launch_distinct_rows(w.fb_id[ctx->cur], w.fcell_off[ctx->cur], ctx->bt.tile_first,
@@ -560,7 +560,7 @@ agnes_status agnes_copy_adj_blocks(agnes_ctx* ctx, int32_t* start_node, int32_t*
     return AGNES_EINVAL;
   }
   const int64_t n = cap < ctx->bt.n_starts ? cap : ctx->bt.n_starts;
-  cudaSetDevice(ctx->device);
+  DeviceGuard dg(ctx->device);
   CK(ctx, cudaMemcpy(start_node, ctx->bt.start_node, sizeof(int32_t) * n, cudaMemcpyDeviceToHost));
   CK(ctx, cudaMemcpy(start_block, ctx->bt.start_block, sizeof(int32_t) * n,
                      cudaMemcpyDeviceToHost));

@@ -274,6 +274,33 @@ cudaError_t launch_distinct_rows(const int32_t* fb_id, const int32_t* cell_off,
                                  const int32_t* tile_first, int32_t T, int32_t H,
                                  unsigned long long* count, cudaStream_t st);
 
+// Makes `device` current for the lifetime of the guard and then restores the
+// device that was current when it was made, so that an entry point never
+// leaves the calling thread on another GPU.
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int device) {
+    if (cudaGetDevice(&prev_) != cudaSuccess) {
+      cudaGetLastError();
+      prev_ = -1;
+    }
+    ok_ = prev_ == device || cudaSetDevice(device) == cudaSuccess;
+    if (!ok_) cudaGetLastError();
+    switched_ = ok_ && prev_ >= 0 && prev_ != device;
+  }
+  ~DeviceGuard() {
+    if (switched_) cudaSetDevice(prev_);
+  }
+  DeviceGuard(const DeviceGuard&) = delete;
+  DeviceGuard& operator=(const DeviceGuard&) = delete;
+  bool ok() const { return ok_; }
+
+ private:
+  int prev_ = -1;
+  bool ok_ = false;
+  bool switched_ = false;
+};
+
 // ---- api.cu: read-only view of a loaded graph for other translation units --
 struct GraphView {
   int device;

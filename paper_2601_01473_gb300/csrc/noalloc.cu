@@ -7,14 +7,12 @@
 // segmented scan), kept separate so that path stays as it is.
 //
 // Scratch: the per-chunk partial sums and an error word live in g_scratch.
-// Host code may not use the name g_scratch as a device address: the first
-// call on each device looks the array's address up with
-// cudaGetSymbolAddress (with that device current) and every launch gets that
-// pointer.  Every call on a device shares the array, so calls that overlap on
-// the GPU race; the error word is cleared at the start of each call and the
-// partial sums are fully rewritten by each call.
-#include <mutex>
-
+// Host code may not use the name g_scratch as a device address: every call
+// looks the array's address up with cudaGetSymbolAddress (with the ctx's
+// device current) and every launch gets that pointer.  Every call on a device
+// shares the array, so calls that overlap on the GPU race; the error word is
+// cleared at the start of each call and the partial sums are fully rewritten
+// by each call.
 #include "../../include/agnes.h"
 #include "common.cuh"
 #include "internal.h"
@@ -121,22 +119,15 @@ na_down_kernel(const OffT* __restrict__ off, int64_t N, const int32_t* __restric
   }
 }
 
-constexpr int kNaMaxDevices = 64;
-std::mutex g_na_mu;
-int64_t* g_na_ptr[kNaMaxDevices] = {nullptr};
-
-// Device address of g_scratch on `device` (which must be current), looked up
-// once per device.
-cudaError_t na_scratch(int device, int64_t** out) {
-  if (device < 0 || device >= kNaMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_na_mu);
-  if (!g_na_ptr[device]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
-    if (e != cudaSuccess) return e;
-    g_na_ptr[device] = (int64_t*)p;
-  }
-  *out = g_na_ptr[device];
+// Device address of g_scratch on the current device.  Looked up on every
+// call (a host-side query, no device work), so that no address outlives the
+// context it was taken in: after a cudaDeviceReset the next call gets the
+// array of the new context.
+cudaError_t na_scratch(int64_t** out) {
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
+  if (e != cudaSuccess) return e;
+  *out = (int64_t*)p;
   return cudaSuccess;
 }
 
@@ -173,8 +164,8 @@ extern "C" agnes_status agnes_hop_indptr_noalloc(agnes_ctx* ctx, const int32_t* 
   }
   GraphView g;
   ctx_graph_view(ctx, &g);
-  if (cudaSetDevice(g.device) != cudaSuccess) {
-    cudaGetLastError();
+  DeviceGuard dg(g.device);
+  if (!dg.ok()) {
     ctx_set_error(ctx, "cudaSetDevice(%d) failed", g.device);
     return AGNES_ECUDA;
   }
@@ -183,7 +174,7 @@ extern "C" agnes_status agnes_hop_indptr_noalloc(agnes_ctx* ctx, const int32_t* 
     return AGNES_EINVAL;
   }
   int64_t* scratch = nullptr;
-  cudaError_t e = na_scratch(g.device, &scratch);
+  cudaError_t e = na_scratch(&scratch);
   if (e != cudaSuccess) {
     ctx_set_error(ctx, "cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
     return AGNES_ECUDA;

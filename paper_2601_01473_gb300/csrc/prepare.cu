@@ -552,9 +552,9 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     set_err(ctx, "H x node capacity (%lld) exceeds 2^31", (long long)(H * cap[K]));
     return AGNES_ERANGE;
   }
-  if (cudaSetDevice(ctx->device) != cudaSuccess) {
-    cudaGetLastError();
-    set_err(ctx, "cudaSetDevice failed");
+  DeviceGuard dg(ctx->device);
+  if (!dg.ok()) {
+    set_err(ctx, "cudaSetDevice(%d) failed", ctx->device);
     return AGNES_ECUDA;
   }
   agnes_status rc = ensure_workspace(ctx, H, B, fanouts, K, cap);

@@ -507,6 +507,13 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
     ctx_set_error(ctx, "ctx, x, w and out must be non-NULL");
     return AGNES_EINVAL;
   }
+  GraphView g;
+  ctx_graph_view(ctx, &g);
+  DeviceGuard dg(g.device);
+  if (!dg.ok()) {
+    ctx_set_error(ctx, "cudaSetDevice(%d) failed", g.device);
+    return AGNES_ECUDA;
+  }
   agnes_hyperbatch_view v;
   agnes_status rc = agnes_fetch_hyperbatch(ctx, &v);
   if (rc != AGNES_OK) return rc;
@@ -573,8 +580,6 @@ extern "C" agnes_status agnes_sage_mean_layer(agnes_ctx* ctx, int32_t hop, const
     ctx_set_error(ctx, "x, w, bias and out must be device memory");
     return AGNES_EINVAL;
   }
-  GraphView g;
-  ctx_graph_view(ctx, &g);
   cudaStream_t st = (cudaStream_t)cuda_stream;
   // device scratch: error word and tables, then (256-byte aligned) the A tiles
   const size_t a_off = (16 + tab_bytes + 255) & ~(size_t)255;

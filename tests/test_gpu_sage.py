@@ -30,7 +30,8 @@ def _weights(d_in, d_out, seed, device):
 
 
 def _check_layer(allv, hop, x, w, b, out, x_f16, out_f16):
-    """Every dst row of every minibatch within 2x the oracle's bound."""
+    """Every dst row of every minibatch within the oracle's derived bound;
+    returns the largest err / bound over all of them."""
     wn = w.float().cpu().numpy().astype(np.float64)
     bn = b.cpu().numpy().astype(np.float64) if b is not None else None
     xs = x.float().cpu().numpy()
@@ -46,7 +47,7 @@ def _check_layer(allv, hop, x, w, b, out, x_f16, out_f16):
         ref, a, m = sage_mean(indptr, col, xs[j, :ns].astype(np.float64), wn, bn, nd)
         bound = error_bound(a, m, wn, bn, ref, x_exact_f16=x_f16, out_f16=out_f16)
         err = np.abs(outs[j, :nd].astype(np.float64) - ref)
-        assert np.all(err <= 2 * bound + 1e-30), (
+        assert np.all(err <= bound), (
             f"minibatch {j}: max err {err.max()} at {np.unravel_index(err.argmax(), err.shape)}")
         if nd:
             worst = max(worst, float((err / (bound + 1e-30)).max()))
@@ -69,14 +70,16 @@ def test_sage_layer_matches_oracle(cuda_device, dim, dtype, d_out, out_dtype):
     w, b = _weights(dim, d_out, 1, cuda_device)
     out = g.sage_mean_layer(K - 1, allv.feats, w, b, out_dtype=out_dtype)
     torch.cuda.synchronize()
-    _check_layer(allv, K - 1, allv.feats, w, b, out, dtype == torch.float16,
-                 out_dtype == torch.float16)
+    worst = _check_layer(allv, K - 1, allv.feats, w, b, out, dtype == torch.float16,
+                         out_dtype == torch.float16)
     # the next layer consumes the first one's output (rows = src_{K-2})
     w2, b2 = _weights(d_out, 64, 2, cuda_device)
     x2 = out.contiguous()
     out2 = g.sage_mean_layer(K - 2, x2, w2, None, out_dtype=torch.float32)
     torch.cuda.synchronize()
-    _check_layer(allv, K - 2, x2, w2, None, out2, out_dtype == torch.float16, False)
+    worst = max(worst, _check_layer(allv, K - 2, x2, w2, None, out2,
+                                    out_dtype == torch.float16, False))
+    print(f"sage layer worst err/bound: {worst:.3g}")
     g.close()
 
 

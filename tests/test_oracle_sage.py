@@ -98,3 +98,67 @@ def test_error_bound_covers_fp16_rounding_of_the_inputs():
     approx = np.maximum(pre, 0).astype(np.float64)
     bound = error_bound(a, m, w, b, out, x_exact_f16=True, out_f16=False)
     assert np.all(np.abs(approx - out) <= bound)
+
+
+def _trunc_f32(v):
+    """Rounds float64 values to float32 toward zero."""
+    r = v.astype(np.float32)
+    over = np.abs(r.astype(np.float64)) > np.abs(v)
+    r[over] = np.nextafter(r[over], np.float32(0))
+    return r
+
+
+def test_error_bound_covers_truncating_accumulation_subnormals_and_f16_output():
+    """A simulated kernel at the bound's worst assumptions: the mean summed in
+    fp32, inputs rounded to fp16 (some aggregates cancel to fp16 subnormals),
+    every product added into an fp32 accumulator that truncates, the bias
+    added in fp32, the result rounded to fp16; fp32 features, so the self half
+    is rounded too."""
+    rng = np.random.default_rng(6)
+    n_src, n_dst, d = 120, 60, 24
+    indptr, col, x = _random_block(rng, n_src, n_dst, 6, d)
+    # the first 20 dst rows take a pair of nearly opposite neighbours, so
+    # their means cancel to about 1e-6 (fp16 subnormals)
+    x[1::2] = -x[0::2] + rng.standard_normal((n_src // 2, d)) * 1e-6
+    deg = np.diff(indptr)
+    deg[:20] = 2
+    rest = col[indptr[20]:]
+    indptr = np.concatenate([[0], np.cumsum(deg)])
+    col = np.concatenate([np.stack([np.arange(20) * 2, np.arange(20) * 2 + 1], 1).ravel(),
+                          rest])
+    w = rng.standard_normal((16, 2 * d)).astype(np.float16).astype(np.float64)
+    b = rng.standard_normal(16).astype(np.float32).astype(np.float64)
+    out, a, m = sage_mean(indptr, col, x, w, b, n_dst)
+    x32 = x.astype(np.float32)
+    agg32 = np.zeros((n_dst, d), np.float32)
+    for i in range(n_dst):
+        s, e = indptr[i], indptr[i + 1]
+        if e > s:
+            acc = np.zeros(d, np.float32)
+            for u in col[s:e]:
+                acc = (acc + x32[u]).astype(np.float32)
+            agg32[i] = (acc / np.float32(e - s)).astype(np.float32)
+    a16 = np.concatenate([x32[:n_dst], agg32], axis=1).astype(np.float16).astype(np.float64)
+    assert np.any((a16 != 0) & (np.abs(a16) < 2.0 ** -14))  # subnormals occur
+    acc = np.zeros((n_dst, 16), np.float32)
+    for k in range(2 * d):
+        acc = _trunc_f32(acc.astype(np.float64) + np.outer(a16[:, k], w[:, k]))
+    pre = (acc + b.astype(np.float32)).astype(np.float32)
+    approx = np.maximum(pre, 0).astype(np.float16).astype(np.float64)
+    bound = error_bound(a, m, w, b, out, x_exact_f16=False, out_f16=True)
+    assert np.all(np.abs(approx - out) <= bound)
+
+
+def test_error_bound_rejects_a_kernel_that_rounds_its_inputs_to_bf16():
+    """The bound is tight enough to catch a real precision loss: inputs
+    rounded to bf16 (8 significant bits) instead of fp16 break it."""
+    rng = np.random.default_rng(7)
+    indptr, col, x = _random_block(rng, 200, 100, 10, 16)
+    x = x.astype(np.float16).astype(np.float64)
+    w = rng.standard_normal((8, 32)).astype(np.float16).astype(np.float64)
+    out, a, m = sage_mean(indptr, col, x, w, None, 100)
+    bits = a.astype(np.float32).view(np.uint32)
+    a_bf16 = ((bits + 0x7FFF + ((bits >> 16) & 1)) & 0xFFFF0000).view(np.float32)
+    approx = np.maximum(a_bf16.astype(np.float64) @ w.T, 0)
+    bound = error_bound(a, m, w, None, out, x_exact_f16=True, out_f16=False)
+    assert np.any(np.abs(approx - out) > bound)

@@ -63,3 +63,27 @@ def test_noalloc_rejects_oversized_and_bad_input(cuda_device):
     deg = (off[1:11] - off[:10]).clamp(max=3).to(torch.int64)
     assert torch.equal(out.cpu(), torch.cat([torch.zeros(1, dtype=torch.int64), deg.cumsum(0)]))
     g.close()
+
+
+@pytest.mark.parametrize("n", [600_000, 1 << 24])
+def test_noalloc_carries_partials_across_chunk_groups(cuda_device, n):
+    """Node lists longer than one 256-chunk group of the partial-sum scan
+    (524,288 nodes), up to the stated maximum of 2^24 nodes, against a torch
+    prefix sum of min(deg, fanout); ids repeat, which the call allows."""
+    N = 50000
+    off, ind = synth.rmat_csr(N, 12, 0.57, 0.19, 0.19, seed=46, offsets_dtype=torch.int64)
+    feats = synth.normal_features(N, 8, torch.float32, 47)
+    g = Graph(off.to(cuda_device), ind.to(cuda_device), feats.to(cuda_device),
+              adj_block_bytes=16384, feat_block_bytes=16384)
+    gen = torch.Generator().manual_seed(n)
+    nodes = torch.randint(0, N, (n,), generator=gen, dtype=torch.int32)
+    deg = (off[1:] - off[:-1]).to(torch.int64)
+    for fanout in (5, 1000):  # two calls in a row on the shared scratch
+        out = torch.full((n + 1,), -3, dtype=torch.int64, device=cuda_device)
+        assert _noalloc(g, nodes.to(cuda_device), fanout, out) == 0, \
+            agnes.lib().agnes_last_error(g._ctx)
+        torch.cuda.synchronize()
+        ref = torch.cat([torch.zeros(1, dtype=torch.int64),
+                         deg[nodes.long()].clamp(max=fanout).cumsum(0)])
+        assert torch.equal(out.cpu(), ref)
+    g.close()
