@@ -59,6 +59,11 @@ struct Workspace {
   int2* sb = nullptr;
   int2* tmp = nullptr;
   int32_t* big_list = nullptr;
+  int32_t* q_cells = nullptr;  // default frontier's dedup queue (internal.h, DedupBufs)
+  int32_t* q_cnt = nullptr;
+  int32_t* q_off = nullptr;
+  int32_t* q_dense = nullptr;
+  int32_t q_warps_cap = 0;
   int32_t* big_n = nullptr;
   int32_t* tmp_id = nullptr;
   int32_t* tmp_pos = nullptr;

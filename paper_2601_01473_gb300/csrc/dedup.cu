@@ -11,7 +11,10 @@
 // with ranks local to the cell, each sampled edge's col and the cell of the
 // next hop's frontier bucket (D | new in ascending id); after the scans, a
 // fix-up pass and a compaction pass turn the local ranks into final indices.
-// The bucket is carried from hop to hop and never rebuilt.
+// The bucket is carried from hop to hop and never rebuilt.  This file holds
+// the scatter, the scans, the fix-up and the compaction, and the cell kernels
+// of the sampled frontier; the default frontier's cells are resolved in
+// dedup_cells.cu.
 #include "common.cuh"
 #include "internal.h"
 
@@ -524,8 +527,6 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   if (e != cudaSuccess) return e;
   dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, d.scell, d.srank,
                                                    d.soff, d.sb, a.status);
-  e = cudaMemsetAsync(d.big_n, 0, sizeof(int32_t), st);
-  if (e != cudaSuccess) return e;
 
   CellArgs c;
   c.tm = tm;
@@ -548,10 +549,16 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   c.big_n = d.big_n;
   c.sampled = d.frontier_sampled;
   c.status = a.status;
-  dedup_cells_kernel<<<resident_grid((const void*)dedup_cells_kernel, kCellThreads, num_sms),
-                       kCellThreads, 0, st>>>(c);
-  dedup_big_kernel<<<resident_grid((const void*)dedup_big_kernel, kThreads, num_sms), kThreads, 0,
-                     st>>>(c);
+  if (d.frontier_sampled) {
+    if ((e = cudaMemsetAsync(d.big_n, 0, sizeof(int32_t), st)) != cudaSuccess) return e;
+    dedup_cells_kernel<<<resident_grid((const void*)dedup_cells_kernel, kCellThreads, num_sms),
+                         kCellThreads, 0, st>>>(c);
+    dedup_big_kernel<<<resident_grid((const void*)dedup_big_kernel, kThreads, num_sms), kThreads,
+                       0, st>>>(c);
+  } else {
+    e = launch_dedup_cells(a, d, num_sms, st);  // dedup_cells.cu
+    if (e != cudaSuccess) return e;
+  }
   // per-minibatch offsets of the new ids: scan down the tiles of the
   // tile-major [T x H] count matrix; totals give the next frontier sizes
   // |src_h| = |dst_h| + new ids; the next frontier is src_h, or (sampled

@@ -126,6 +126,10 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
 // on bitmaps, one warp each; the rest entry-parallel.  The big-cell list
 // therefore holds at most (entries) / (kDedupSmallMax + 1) cells.
 constexpr int kDedupSmallMax = 32;
+// With the default frontier, cells of at most this many entries are resolved
+// by one thread each; larger cells with samples are queued (q_dense), so the
+// queue holds at most (entries) / (kDedupLaneMax + 1) cells.
+constexpr int kDedupLaneMax = 8;
 
 struct DedupBufs {
   const int32_t* nbr;       // H x ecap sampled ids
@@ -138,6 +142,15 @@ struct DedupBufs {
   int2* tmp;                // per cell: next-frontier entries with local ranks
   int32_t* big_list;        // cells with more than kDedupSmallMax entries
   int32_t* big_n;           // their count
+  // default frontier: the queue of cells with samples and more than
+  // kDedupLaneMax entries: per warp of the lane kernel a run in q_cells (T*H),
+  // their counts and offsets (q_warps_cap, q_warps_cap + 1), and the queue in
+  // cell order (q_dense)
+  int32_t* q_cells;
+  int32_t* q_cnt;
+  int32_t* q_off;
+  int32_t* q_dense;
+  int32_t q_warps_cap;
   const int32_t* fb_id;     // current frontier bucket
   const int32_t* fb_pos;
   const int32_t* fcell_off;
@@ -174,6 +187,14 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
 // new nodes' ids in the node lists.
 cudaError_t launch_dedup_compact(const HopArgs& a, const DedupBufs& d, int num_sms,
                                  cudaStream_t st);
+
+// ---- dedup_cells.cu --------------------------------------------------------
+// The default frontier's resolution of one hop's cells (launch_dedup calls
+// it in place of the sampled frontier's cell kernels): newcnt, nfcnt, col
+// with local new-id ranks, the next frontier cells in tmp, the touched-block
+// flags; it builds and uses the queue in q_cells / q_cnt / q_off / q_dense.
+cudaError_t launch_dedup_cells(const HopArgs& a, const DedupBufs& d, int num_sms,
+                               cudaStream_t st);
 
 // ---- gather.cu -------------------------------------------------------------
 cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,

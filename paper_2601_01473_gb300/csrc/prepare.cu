@@ -58,6 +58,10 @@ void free_workspace(Workspace* w) {
   cudaFree(w->sb);
   cudaFree(w->tmp);
   cudaFree(w->big_list);
+  cudaFree(w->q_cells);
+  cudaFree(w->q_cnt);
+  cudaFree(w->q_off);
+  cudaFree(w->q_dense);
   cudaFree(w->big_n);
   cudaFree(w->tmp_id);
   cudaFree(w->tmp_pos);
@@ -153,6 +157,11 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.tmp, rows + edges);
   WA(w.big_list, (rows + edges) / (kDedupSmallMax + 1) + 1);
   WA(w.big_n, 1);
+  w.q_warps_cap = ctx->num_sms * 64;  // warps resident at most (64 per SM)
+  WA(w.q_cells, cells);
+  WA(w.q_cnt, w.q_warps_cap);
+  WA(w.q_off, w.q_warps_cap + 1);
+  WA(w.q_dense, (rows + edges) / (kDedupLaneMax + 1) + 1);
   WA(w.tmp_id, (int64_t)H * B);
   WA(w.tmp_pos, (int64_t)H * B);
   WA(w.cnt, (int64_t)H * w.cap_prev_max);
@@ -298,6 +307,12 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.sb = w.sb;
     d.tmp = w.tmp;
     d.big_list = w.big_list;
+    d.q_cells = w.q_cells;
+    d.q_cnt = w.q_cnt;
+    d.q_off = w.q_off;
+    d.q_dense = w.q_dense;
+    d.q_warps_cap = w.q_warps_cap;
+
     d.big_n = w.big_n;
     d.fb_id = w.fb_id[cur];
     d.fb_pos = w.fb_pos[cur];
