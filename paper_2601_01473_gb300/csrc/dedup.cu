@@ -24,6 +24,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+constexpr int kIlp = 4;  // independent elements per thread in the streaming passes
 
 // Places every sampled edge of minibatch j at soff[cell] + rank (cell and
 // rank were recorded while sampling), building the sampled bucket.
@@ -427,10 +428,21 @@ dedup_fix_col_kernel(int32_t* __restrict__ col, const int32_t* __restrict__ ecnt
   const int64_t E = ecnt[j];
   const int64_t o = (int64_t)j * ecap;
   const int32_t base = nsz_prev[j];
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < E;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const int32_t v = col[o + e];
-    if (v < 0) col[o + e] = base + newbase[scell[o + e]] + (-1 - v);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e0 < E;
+       e0 += kIlp * stride) {  // kIlp edges per thread: their base loads in flight together
+    int32_t v[kIlp], cell[kIlp], nb[kIlp];
+#pragma unroll
+    for (int k = 0; k < kIlp; ++k) {
+      const int64_t e = e0 + k * stride;
+      v[k] = e < E ? col[o + e] : 0;
+      cell[k] = e < E ? scell[o + e] : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < kIlp; ++k) nb[k] = v[k] < 0 ? newbase[cell[k]] : 0;
+#pragma unroll
+    for (int k = 0; k < kIlp; ++k)
+      if (v[k] < 0) col[o + e0 + k * stride] = base + nb[k] + (-1 - v[k]);
   }
 }
 

@@ -243,7 +243,7 @@ struct TileScratch {
   int32_t* pN;  // new ids below word w
 };
 
-__global__ void __launch_bounds__(kThreads) dedup_tile_kernel(CellsArgs a, int32_t nw) {
+__global__ void __launch_bounds__(kThreads, 8) dedup_tile_kernel(CellsArgs a, int32_t nw) {
   grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ __align__(16) uint32_t D_s[kWarps][kTileWords];
