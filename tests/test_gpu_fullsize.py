@@ -1,8 +1,8 @@
 """Full-size parity: each workload at its full size, in the launch
 configuration bench.py times (one hyperbatch of H minibatches through the C
-ABI), checked against the oracle on the host: sampled minibatches bit-exact
-(subgraphs, node lists, gathered feature bytes) and the blocks-touched
-statistics over the whole hyperbatch."""
+ABI), checked against the oracle run over the whole hyperbatch on the host:
+every minibatch bit-exact (subgraphs, node lists, gathered feature bytes) and
+the blocks-touched statistics of the hyperbatch."""
 import os
 
 import numpy as np
@@ -21,13 +21,45 @@ def _bytes(t):
     return t.view(torch.uint8).numpy().reshape(-1)
 
 
+def _check_hyperbatch(g, og, targets, fanouts, seed, gid0, adj_bb, feat_bb, features, byte_sample):
+    """Every minibatch of g's last hyperbatch against the oracle run over the
+    whole hyperbatch on the host cores: subgraph sizes, indptr, col and node
+    lists element by element, the blocks-touched statistics exactly.  Feature
+    rows: every minibatch's gathered bytes equal the feature rows of the
+    oracle's node list (indexed on the device), and the minibatches of
+    byte_sample are also compared with the oracle's own gather."""
+    t = np.ascontiguousarray(targets.cpu().numpy())
+    ref, ref_stats = oracle.hyperbatch(og, t, fanouts, seed, gid0, False, adj_bb, feat_bb,
+                                       threads=os.cpu_count() or 1)
+    assert g.stats() == ref_stats
+    hv = g.fetch_all()
+    K = len(fanouts)
+    word = {2: torch.int16, 4: torch.int32}[features.element_size()]
+    feats_words = features.view(word)
+    for j in range(t.shape[0]):
+        r = ref[j]
+        n = int(hv.node_size[K, j])
+        nodes = hv.nodes[j, :n].cpu().numpy()
+        assert np.array_equal(nodes, r["nodes"]), f"nodes of minibatch {j}"
+        for h in range(K):
+            nd, ns, ne = int(hv.node_size[h, j]), int(hv.src_size[h, j]), int(hv.edges[h, j])
+            rh = r["hops"][h]
+            assert (nd, ns, ne) == (rh["num_dst"], rh["num_src"], rh["num_edges"]), (h, j)
+            assert np.array_equal(hv.indptr[h][j, :nd + 1].cpu().numpy(), rh["indptr"]), (h, j)
+            assert np.array_equal(hv.col[h][j, :ne].cpu().numpy(), rh["col"]), (h, j)
+        want = feats_words.index_select(0, torch.from_numpy(r["nodes"]).to(features.device).long())
+        assert torch.equal(hv.feats[j, :n].view(word), want), f"feats of minibatch {j}"
+    for j in byte_sample:
+        r = oracle.sample_minibatch(og, t[j], fanouts, seed, gid0 + j)
+        n = int(hv.node_size[K, j])
+        assert np.array_equal(_bytes(hv.feats[j, :n]), r["feats"].view(np.uint8).reshape(-1)), j
+
+
 @pytest.mark.timeout(900)
-@pytest.mark.parametrize("name,sample", [
-    ("rmat10m", (0, 31, 63)),
-    ("rmat100m", (0, 77, 127)),
-    ("rmat65m_skew", (0, 40, 63)),
-])
-def test_fullsize_parity(cuda_device, name, sample):
+@pytest.mark.parametrize("name", ["rmat10m", "rmat100m", "rmat65m_skew"])
+def test_fullsize_parity(cuda_device, name):
+    """Configs 2-4 at full size, in bench.py's launch configuration: every
+    minibatch of one hyperbatch."""
     w = WORKLOADS[name]
     offsets, indices, features = build_graph(w, cuda_device)
     targets = targets_for_step(w, target_pool(w, cuda_device), 0)
@@ -37,34 +69,35 @@ def test_fullsize_parity(cuda_device, name, sample):
     if name == "rmat65m_skew":
         assert max_deg > 1_000_000
     torch.cuda.empty_cache()
+    og = oracle.Graph(offsets.cpu().numpy(), indices.cpu().numpy(), features.cpu().numpy())
     g = Graph(offsets, indices, features, w.adj_block_bytes, w.feat_block_bytes)
     gid0 = 1000
     g.prepare(targets, list(w.fanouts), w.seed, gid0)
-    got_stats = g.stats()
-    views = {j: g.fetch(j) for j in sample}
-    got = {j: (v.nodes.cpu().numpy(), [(h.num_dst, h.num_src, h.num_edges, h.indptr.cpu().numpy(),
-                                        h.col.cpu().numpy()) for h in v.hops], _bytes(v.feats))
-           for j, v in views.items()}
-    del views
-    og = oracle.Graph(offsets.cpu().numpy(), indices.cpu().numpy(), features.cpu().numpy())
+    _check_hyperbatch(g, og, targets, list(w.fanouts), w.seed, gid0, w.adj_block_bytes,
+                      w.feat_block_bytes, features, (0, w.H - 1))
     g.close()
-    del offsets, indices, features
+
+
+@pytest.mark.timeout(1200)
+@pytest.mark.parametrize("H,block", [(256, 4 << 20), (1, 256 << 10), (64, 512 << 10)])
+def test_config5_extremes_parity(cuda_device, H, block):
+    """Config 5's sweep at its extremes on rmat100m's graph: the largest
+    hyperbatch with the largest blocks (the largest workspace, H x capK of
+    about 277M output rows), one minibatch per hyperbatch with the smallest
+    blocks, and a middle point; every minibatch checked."""
+    w = WORKLOADS["rmat100m"]
+    offsets, indices, features = build_graph(w, cuda_device)
+    ws = w.with_(H=H, adj_block_bytes=block, feat_block_bytes=block)
+    targets = targets_for_step(ws, target_pool(w, cuda_device), 7)
     torch.cuda.empty_cache()
-    t = targets.cpu().numpy()
-    for j in sample:
-        r = oracle.sample_minibatch(og, t[j], list(w.fanouts), w.seed, gid0 + j)
-        nodes, hops, feats = got[j]
-        assert np.array_equal(nodes, r["nodes"]), f"nodes of minibatch {j}"
-        for h, (nd, ns, ne, ip, col) in enumerate(hops):
-            rh = r["hops"][h]
-            assert (nd, ns, ne) == (rh["num_dst"], rh["num_src"], rh["num_edges"])
-            assert np.array_equal(ip, rh["indptr"]), f"indptr hop {h} mb {j}"
-            assert np.array_equal(col, rh["col"]), f"col hop {h} mb {j}"
-        assert np.array_equal(feats, r["feats"].view(np.uint8).reshape(-1)), f"feats mb {j}"
-    _, ref_stats = oracle.hyperbatch(og, t, list(w.fanouts), w.seed, gid0, False,
-                                     w.adj_block_bytes, w.feat_block_bytes,
-                                     threads=os.cpu_count() or 1)
-    assert got_stats == ref_stats
+    og = oracle.Graph(offsets.cpu().numpy(), indices.cpu().numpy(), features.cpu().numpy())
+    g = Graph(offsets, indices, features, block, block)
+    gid0 = 77_000
+    for step in range(2):  # a second hyperbatch replays the captured launch sequence
+        g.prepare(targets, list(w.fanouts), w.seed, gid0)
+    _check_hyperbatch(g, og, targets, list(w.fanouts), w.seed, gid0, block, block, features,
+                      (0, H - 1) if H > 1 else (0,))
+    g.close()
 
 
 @pytest.mark.timeout(1200)
