@@ -50,7 +50,7 @@ extern "C" {
 #endif
 
 #define AGNES_MAX_HOPS 8
-#define AGNES_MAX_FANOUT 1024
+#define AGNES_MAX_FANOUT 65536
 
 typedef enum {
   AGNES_OK = 0,
@@ -169,6 +169,9 @@ agnes_status agnes_load_graph(const agnes_graph_desc* desc, int device, void* cu
  *            inside the call (pinned memory makes that copy asynchronous).
  *  fanouts   K host int32 values, fanouts[0] for the targets' hop;
  *            1 <= fanouts[h] <= AGNES_MAX_FANOUT, 1 <= K <= AGNES_MAX_HOPS.
+ *            A hop with a fanout above 1024 also uses ctx-owned device
+ *            memory for the sampler's per-warp sets of chosen positions
+ *            (at most 1 GiB, allocated with the workspace).
  *  seed, first_minibatch_id  key the random draws (see above).
  * Stream-ordered: returns once the work is enqueued, after the ctx's previous
  * prepare (on whatever stream) and before anything later on cuda_stream.

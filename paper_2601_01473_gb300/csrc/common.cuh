@@ -14,7 +14,7 @@ namespace agnes {
 constexpr int kTileShift = 12;
 constexpr int kTileSpan = 1 << kTileShift;
 constexpr int kTileWords = kTileSpan / 32;
-constexpr int kMaxFanout = 1024;  // largest fanout accepted by the API
+constexpr int kWideMax = 1024;  // fanouts the warp sampler handles with its choices in shared memory
 
 // Bits of the device status word.
 enum : int32_t {

@@ -59,6 +59,8 @@ struct Workspace {
   int2* sb = nullptr;
   int2* tmp = nullptr;
   int32_t* big_list = nullptr;
+  int32_t* hset = nullptr;     // fanouts above kWideMax: the sampler's per-warp hash sets
+  int64_t hset_elems = 0;
   int32_t* q_cells = nullptr;  // default frontier's dedup queue (internal.h, DedupBufs)
   int32_t* q_cnt = nullptr;
   int32_t* q_off = nullptr;

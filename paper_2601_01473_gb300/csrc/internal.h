@@ -82,7 +82,17 @@ struct HopArgs {
   int32_t hop;       // 1-based
   const uint64_t* key;  // device: {seed, first minibatch id} (launch_set_key)
   int32_t* status;
+  // fanouts above kWideMax: per-warp hash sets of chosen positions, 2^hset_log2
+  // int32 entries each, for the hset_grid CTAs of the sampler
+  int32_t* hset = nullptr;
+  int32_t hset_log2 = 0;
+  int32_t hset_grid = 0;
 };
+
+// The hash sets the sampler needs for a fanout k > kWideMax: 2^log2 >= 2k
+// entries per warp and the CTAs of its grid (capped so the tables stay within
+// 1 GiB); returns the int32 entries to allocate (0 when k <= kWideMax).
+int64_t huge_fanout_tables(int32_t k, int num_sms, int32_t* log2, int32_t* grid);
 
 // Writes the sampling key {seed, first minibatch id} to device memory ahead
 // of a hyperbatch (one 1-thread kernel: the arguments travel with the launch).

@@ -59,6 +59,7 @@ void free_workspace(Workspace* w) {
   cudaFree(w->tmp);
   cudaFree(w->big_list);
   cudaFree(w->q_cells);
+  cudaFree(w->hset);
   cudaFree(w->q_cnt);
   cudaFree(w->q_off);
   cudaFree(w->q_dense);
@@ -162,6 +163,13 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.q_cnt, w.q_warps_cap);
   WA(w.q_off, w.q_warps_cap + 1);
   WA(w.q_dense, (rows + edges) / (kDedupLaneMax + 1) + 1);
+  w.hset_elems = 0;
+  for (int h = 0; h < K; ++h) {
+    int32_t l2 = 0, g = 0;
+    const int64_t e = huge_fanout_tables(fan[h], ctx->num_sms, &l2, &g);
+    if (e > w.hset_elems) w.hset_elems = e;
+  }
+  if (w.hset_elems > 0) WA(w.hset, w.hset_elems);
   WA(w.tmp_id, (int64_t)H * B);
   WA(w.tmp_pos, (int64_t)H * B);
   WA(w.cnt, (int64_t)H * w.cap_prev_max);
@@ -261,6 +269,8 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     a.hop = h + 1;
     a.key = w.key;
     a.status = w.status;
+    a.hset = w.hset;
+    huge_fanout_tables(fanouts[h], nsm, &a.hset_log2, &a.hset_grid);
     int32_t* nsz_prev = w.nsz + (int64_t)h * H;
     int32_t* ecnt = w.ecnt + (int64_t)h * H;
     CK(ctx, launch_sample_count(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.cnt, nsm, st));

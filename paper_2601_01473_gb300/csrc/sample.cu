@@ -14,6 +14,9 @@
 // Philox4x32-10 draws keyed on (seed; v, hop, slot, g).  A group of G >= k
 // lanes handles one frontier node: lane s draws slot s's candidate in
 // parallel and the k-step collision resolution runs over in-group shuffles.
+// Above 32 a warp takes 32 slots at a time, checking each candidate against
+// the earlier chunks' choices (in shared memory up to kWideMax, in a hash set
+// in global memory beyond).
 #include "common.cuh"
 #include "internal.h"
 
@@ -212,6 +215,8 @@ struct FillArgs {
   int32_t k, hop;
   const uint64_t* key;  // device: {seed, first minibatch id}
   int32_t* status;
+  int32_t* hset;      // fanouts above kWideMax: per-warp hash sets of chosen positions
+  int32_t hset_log2;  // each of 2^hset_log2 entries
 };
 
 // The sampling key, read from device memory once per thread, so that one
@@ -340,7 +345,7 @@ __global__ void __launch_bounds__(kThreads)
 sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
   grid_dep_wait();
   if (failed(a.status)) return;
-  __shared__ int32_t chosen_s[kWarps][kMaxFanout];
+  __shared__ int32_t chosen_s[kWarps][kWideMax];
   const int warp = threadIdx.x >> 5, lane = lane_id();
   int32_t* chosen = chosen_s[warp];
   const Key key = load_key(a.key);
@@ -385,7 +390,112 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
   }
 }
 
+// ---- fanouts above kWideMax -----------------------------------------------------
+//
+// One warp per frontier node, slots drawn 32 at a time as in the wide sampler;
+// the positions chosen by earlier chunks live in the warp's own open-addressing
+// hash set in global memory (2^hset_log2 >= 2k entries, so it is at most half
+// full and every probe sequence ends at an empty entry within the table),
+// cleared for each node.  Lookups bypass L1 (__ldcg): the set's entries are
+// written by the warp's atomics at L2.
+constexpr int32_t kHsetEmpty = -1;
+
+__device__ __forceinline__ uint32_t hset_slot(int32_t key, uint32_t mask) {
+  return ((uint32_t)key * 0x9E3779B1u) & mask;  // Fibonacci hashing, low bits
+}
+
+__device__ __forceinline__ bool hset_contains(const int32_t* T, uint32_t mask, int32_t key) {
+  uint32_t h = hset_slot(key, mask);
+  for (uint32_t probe = 0; probe <= mask; ++probe) {
+    const int32_t v = __ldcg(T + h);
+    if (v == key) return true;
+    if (v == kHsetEmpty) return false;
+    h = (h + 1u) & mask;
+  }
+  return false;
+}
+
+// Inserts key (distinct from the keys other lanes insert at the same time).
+__device__ __forceinline__ void hset_insert(int32_t* T, uint32_t mask, int32_t key) {
+  uint32_t h = hset_slot(key, mask);
+  for (uint32_t probe = 0; probe <= mask; ++probe) {
+    const int32_t old = atomicCAS(T + h, kHsetEmpty, key);
+    if (old == kHsetEmpty || old == key) return;
+    h = (h + 1u) & mask;
+  }
+}
+
+template <typename OffT, int kSrc>
+__global__ void __launch_bounds__(kThreads)
+sample_fill_huge_kernel(FillArgs a, const OffT* __restrict__ off) {
+  grid_dep_wait();
+  if (failed(a.status)) return;
+  const int lane = lane_id();
+  const Key key = load_key(a.key);
+  const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
+  const uint32_t capk32 = (uint32_t)a.capK;
+  const int64_t gw = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const uint32_t mask = (1u << a.hset_log2) - 1u;
+  int32_t* T = a.hset + (gw << a.hset_log2);
+  for (int64_t i = E0 + gw; i < E1; i += nwarps) {
+    const int32_t v = a.fb_id[i];
+    const uint32_t g = (uint32_t)a.fb_pos[i];
+    const uint32_t j = g / capk32;
+    const uint32_t pos = g - j * capk32;
+    const int64_t base = (int64_t)__ldg(off + v);
+    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
+    const int64_t ebase = a.indptr[j * (a.cap_prev + 1) + pos];
+    if (d <= a.k) {
+      for (int64_t q0 = 0; q0 < d; q0 += 32) {
+        const int64_t q = q0 + lane;
+        const bool has = q < d;
+        emit_edges(a, has, has ? edge_at<kSrc>(a, v, base, d, q) : 0, j, ebase + q);
+      }
+      continue;
+    }
+    for (uint32_t w = (uint32_t)lane; w <= (mask >> 2); w += 32)
+      reinterpret_cast<int4*>(T)[w] = make_int4(kHsetEmpty, kHsetEmpty, kHsetEmpty, kHsetEmpty);
+    __syncwarp();
+    for (int c0 = 0; c0 < a.k; c0 += 32) {
+      const int s = c0 + lane;
+      const bool valid = s < a.k;
+      const int64_t J = d - a.k + s;
+      const int64_t t = valid ? draw(a, key, v, s, key.gid0 + j, J) : -1;
+      bool collided = valid && hset_contains(T, mask, (int32_t)t);
+      const int m = min(32, a.k - c0);
+      for (int q = 0; q < m; ++q) {
+        const int64_t mine = collided ? J : t;
+        const int64_t cq = __shfl_sync(0xffffffffu, mine, q);
+        if (lane > q && t == cq) collided = true;
+      }
+      const int64_t c = collided ? J : t;
+      if (valid) hset_insert(T, mask, (int32_t)c);
+      emit_edges(a, valid, valid ? edge_at<kSrc>(a, v, base, d, c) : 0, j, ebase + s);
+      __syncwarp();  // the chunk's inserts are seen by the next chunk's lookups
+    }
+    __syncwarp();  // every lookup of this node is done before the next clear
+  }
+}
+
 }  // namespace
+
+int64_t huge_fanout_tables(int32_t k, int num_sms, int32_t* log2, int32_t* grid) {
+  *log2 = 0;
+  *grid = 0;
+  if (k <= kWideMax) return 0;
+  int32_t l = 2;
+  while ((1 << l) < 2 * k) ++l;
+  int g = resident_grid((const void*)sample_fill_huge_kernel<int64_t, kEdgesInPlace>, kThreads,
+                        num_sms);
+  const int64_t budget_entries = (int64_t)1 << 28;  // 1 GiB of tables at most
+  const int64_t max_warps = budget_entries >> l;
+  if ((int64_t)g * kWarps > max_warps) g = (int)(max_warps / kWarps);
+  if (g < 1) g = 1;
+  *log2 = l;
+  *grid = g;
+  return ((int64_t)g * kWarps) << l;
+}
 
 cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32_t B, int32_t N,
                                   const int32_t* tile_first, const int32_t* chunk_tile, int32_t T,
@@ -438,8 +548,8 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
 }
 
 template <typename OffT, int kSrc>
-static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int num_sms,
-                              cudaStream_t st) {
+static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int huge_grid,
+                              int num_sms, cudaStream_t st) {
 #define AGNES_FILL(KERNEL)                                                                   \
   KERNEL<<<resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st>>>(f, off)
   if (k <= 4)
@@ -450,8 +560,10 @@ static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int num
     AGNES_FILL((sample_fill_kernel<OffT, 16, kSrc>));
   else if (k <= 32)
     AGNES_FILL((sample_fill_kernel<OffT, 32, kSrc>));
-  else
+  else if (k <= kWideMax)
     AGNES_FILL((sample_fill_wide_kernel<OffT, kSrc>));
+  else
+    sample_fill_huge_kernel<OffT, kSrc><<<huge_grid, kThreads, 0, st>>>(f, off);
 #undef AGNES_FILL
 }
 
@@ -487,17 +599,20 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.hop = a.hop;
   f.key = a.key;
   f.status = a.status;
+  f.hset = a.hset;
+  f.hset_log2 = a.hset_log2;
+  if (a.k > kWideMax && (a.hset == nullptr || a.hset_grid < 1)) return cudaErrorInvalidValue;
   const int src = r.gbuf == nullptr ? kEdgesInPlace : r.in_place_fallback ? kEdgesCached
                                                                             : kEdgesBuffer;
 #define AGNES_FILL_SRC(OFF)                                                                  \
   do {                                                                                      \
     const OFF* off = (const OFF*)a.offsets;                                                 \
     if (src == kEdgesInPlace)                                                               \
-      launch_fill_typed<OFF, kEdgesInPlace>(f, off, a.k, num_sms, st);                      \
+      launch_fill_typed<OFF, kEdgesInPlace>(f, off, a.k, a.hset_grid, num_sms, st);                      \
     else if (src == kEdgesBuffer)                                                           \
-      launch_fill_typed<OFF, kEdgesBuffer>(f, off, a.k, num_sms, st);                       \
+      launch_fill_typed<OFF, kEdgesBuffer>(f, off, a.k, a.hset_grid, num_sms, st);                       \
     else                                                                                    \
-      launch_fill_typed<OFF, kEdgesCached>(f, off, a.k, num_sms, st);                       \
+      launch_fill_typed<OFF, kEdgesCached>(f, off, a.k, a.hset_grid, num_sms, st);                       \
   } while (0)
   if (a.offsets_bits == 32)
     AGNES_FILL_SRC(int32_t);

@@ -108,6 +108,53 @@ def test_parity_extreme_fanouts_and_hops(cuda_device, fanouts, H, B):
     g.close()
 
 
+def _hub_graph(N: int, hub_degrees, seed: int):
+    """A sparse RMAT graph plus hub nodes with the given numbers of distinct
+    random neighbours (as CSR)."""
+    off, ind = synth.rmat_csr(N, 6, 0.57, 0.19, 0.19, seed)
+    deg = (off[1:] - off[:-1]).long()
+    src = torch.repeat_interleave(torch.arange(N, dtype=torch.int64), deg)
+    keys = [src * N + ind.long()]
+    hubs = []
+    for i, d in enumerate(hub_degrees):
+        h = int(synth.permutation(N, seed + 1)[i])
+        nbrs = synth.permutation(N, seed + 10 + i)[:d + 1].long()
+        nbrs = nbrs[nbrs != h][:d]
+        keys.append(h * N + nbrs)
+        hubs.append(h)
+    keys = torch.unique(torch.cat(keys))
+    off, ind = synth.csr_from_keys(keys, N)
+    return off, ind, hubs
+
+
+@pytest.mark.parametrize("fanouts,H,B", [
+    ((4096, 6), 3, 12),   # four chunks of 1024 past the shared-memory sampler, then a small hop
+    ((65536,), 2, 4),     # the largest fanout
+])
+def test_parity_fanouts_past_shared_memory(cuda_device, fanouts, H, B):
+    """Fanouts above 1024 up to the 2^16 maximum, where each warp keeps the
+    positions Floyd's algorithm has chosen in a hash set in global memory, on
+    a graph whose hubs have more than 2^17 neighbours; every minibatch holds
+    two hubs and is bit-exact against the oracle."""
+    N = 300_000
+    off, ind, hubs = _hub_graph(N, [140_000, 180_000, 220_000, 260_000], 21)
+    deg = off[1:] - off[:-1]
+    assert all(int(deg[h]) > 1 << 17 for h in hubs)
+    feats = synth.normal_features(N, 8, torch.float32, 22)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    targets = synth.hyperbatch_targets(torch.arange(N, dtype=torch.int32), H, B, 23, 0)
+    for j in range(H):  # two hubs per minibatch, targets kept distinct
+        row = [t for t in targets[j].tolist() if t not in hubs][:B - 2]
+        targets[j] = torch.tensor([hubs[(2 * j) % 4], hubs[(2 * j + 1) % 4]] + row,
+                                  dtype=torch.int32)
+    g = load(off, ind, feats, 1 << 20, 1 << 16)
+    g.prepare(targets.to(cuda_device), list(fanouts), 5, 31)
+    compare(g, og, targets.numpy(), list(fanouts), 5, 31, 1 << 20, 1 << 16)
+    g.prepare(targets.to(cuda_device), list(fanouts), 6, 31)  # the sets are cleared per node
+    compare(g, og, targets.numpy(), list(fanouts), 6, 31, 1 << 20, 1 << 16, check_stats=False)
+    g.close()
+
+
 @pytest.mark.parametrize("bits,dtype,fanouts", [
     (32, torch.float32, (10, 5)),
     (64, torch.float16, (15, 10, 5)),
@@ -227,7 +274,7 @@ def test_invalid_targets_are_reported_and_ctx_stays_usable(cuda_device):
     with pytest.raises(AgnesError):
         g.prepare(torch.tensor([[1]], dtype=torch.int32, device=cuda_device), [0], 1, 0)
     with pytest.raises(AgnesError):
-        g.prepare(torch.tensor([[1]], dtype=torch.int32, device=cuda_device), [2000], 1, 0)
+        g.prepare(torch.tensor([[1]], dtype=torch.int32, device=cuda_device), [65537], 1, 0)
     og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
     ok = np.array([[1, 2, 3, 4]], np.int32)
     g.prepare(torch.tensor(ok).to(cuda_device), [3, 2], 1, 0)
