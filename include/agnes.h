@@ -195,7 +195,11 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
  *   node reached so far, so the layer of eq. (1) over each hop has an input
  *   row for each of its src nodes from the layer below.
  * AGNES_FRONTIER_SAMPLED: dst_{h+1} = N_out, the distinct ids sampled at hop
- *   h in ascending order (Algorithm 1 read literally: N_in <- N_out).
+ *   h in ascending order (Algorithm 1's frontier update N_in <- N_out read
+ *   literally).  Only the frontier update is literal: the output is still
+ *   the per-hop blocks and the rows of the last hop's src list (below), not
+ *   Algorithm 1's N_s, the union of every hop's N_out, which would drop the
+ *   rows the lower hops' blocks index.
  * In both, hop h's block has src_h = dst_h ++ new_h (new_h = the sampled ids
  * not in dst_h, ascending) and col indexes src_h; the gathered rows are
  * src_{K-1}.  Errors: EINVAL. */
