@@ -290,6 +290,8 @@ def main():
     ap.add_argument("--launch-mode", default="graph_pdl", choices=["direct", "graph", "graph_pdl"],
                     help="resident path: direct launches, one CUDA graph per hyperbatch shape, "
                          "or the graph with programmatic kernel edges")
+    ap.add_argument("--pipeline-depth", type=int, default=2, choices=[1, 2],
+                    help="hyperbatches in flight inside the library (resident graph only)")
     ap.add_argument("--feature-io", default="blocks", choices=["blocks", "rows"],
                     help="with --stream: load whole feature blocks, or read requested rows in place")
     args = ap.parse_args()
@@ -356,6 +358,8 @@ def main():
               feature_io=args.feature_io if args.stream else "blocks")
     g.set_launch_mode(args.launch_mode)
     g.set_frontier(args.frontier)
+    depth = args.pipeline_depth if not (args.stream or args.stream_topology) else 1
+    g.set_pipeline_depth(depth)
     info = g.info()
     fan = list(w.fanouts)
     K = len(fan)
@@ -383,6 +387,7 @@ def main():
         ev0.record(stream)
         for s in range(args.warmup, n_steps):
             g.prepare(step_targets[s], fan, w.seed, gid(s), stream)
+        g.wait(stream)  # the hyperbatches still in flight on the library's streams
         ev1.record(stream)
         torch.cuda.synchronize()
     if pg:
@@ -420,6 +425,11 @@ def main():
         t0 = time.perf_counter()
         for s in range(args.warmup, n_steps):
             g.prepare(host_targets[s], fan, w.seed, gid(s), stream)
+            if depth == 1:
+                g.fetch_all()
+            elif s > args.warmup:  # the previous hyperbatch, while this one runs
+                g.fetch_previous()
+        if depth == 2:
             g.fetch_all()
         torch.cuda.synchronize()
         e2e_s = time.perf_counter() - t0
@@ -519,6 +529,7 @@ def main():
                                  "feat_blocks": info["feat_blocks"]},
                        "H": w.H, "B": w.B, "fanouts": fan, "parallelism": f"replicas{world}",
                        "launch_mode": args.launch_mode, "frontier": args.frontier,
+                       "pipeline_depth": depth,
                        "l2": "inputs larger than L2 (graph ~%.0f GB vs 129 MB L2), no flush"
                              % ((offsets.numel() * offsets.element_size()
                                  + indices.numel() * 4

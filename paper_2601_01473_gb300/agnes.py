@@ -137,6 +137,9 @@ SIGNATURES = {
     "agnes_hop_indptr_noalloc": ([_P, _P, ctypes.c_int64, ctypes.c_int32, _P, _P], ctypes.c_int),
     "agnes_set_frontier_mode": ([_P, ctypes.c_int32], ctypes.c_int),
     "agnes_set_launch_mode": ([_P, ctypes.c_int32], ctypes.c_int),
+    "agnes_set_pipeline_depth": ([_P, ctypes.c_int32], ctypes.c_int),
+    "agnes_wait_hyperbatches": ([_P, _P], ctypes.c_int),
+    "agnes_fetch_previous_hyperbatch": ([_P, _P], ctypes.c_int),
     "agnes_sage_mean_layer": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int64,
                                ctypes.c_int64, _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
                                ctypes.c_int64, _P], ctypes.c_int),
@@ -386,6 +389,23 @@ class Graph:
         if mode not in LAUNCH:
             raise ValueError(f"launch mode must be one of {sorted(LAUNCH)}")
         _check(lib().agnes_set_launch_mode(self._ctx, LAUNCH[mode]), self._ctx)
+
+    def fetch_previous(self) -> HyperbatchView:
+        """At pipeline depth 2: the hyperbatch prepared before the last one
+        (agnes_fetch_previous_hyperbatch)."""
+        v = _HyperbatchView()
+        _check(lib().agnes_fetch_previous_hyperbatch(self._ctx, ctypes.byref(v)), self._ctx)
+        return HyperbatchView(v, self.device)
+
+    def set_pipeline_depth(self, depth: int) -> None:
+        """Hyperbatches in flight (agnes_set_pipeline_depth): 1, or 2 to let
+        consecutive prepares overlap on the ctx's two internal streams."""
+        _check(lib().agnes_set_pipeline_depth(self._ctx, int(depth)), self._ctx)
+
+    def wait(self, stream=None) -> None:
+        """Orders ``stream`` (default: the current stream) after every
+        hyperbatch still in flight (agnes_wait_hyperbatches)."""
+        _check(lib().agnes_wait_hyperbatches(self._ctx, _stream_handle(stream)), self._ctx)
 
     def sage_mean_layer(self, hop: int, x: torch.Tensor, w: torch.Tensor, bias=None,
                         out_dtype: torch.dtype = torch.float32, stream=None) -> torch.Tensor:

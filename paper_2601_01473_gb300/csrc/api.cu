@@ -137,6 +137,9 @@ agnes_status agnes_free(agnes_ctx* ctx) {
   drop_launch_graph(&ctx->lg);
   if (ctx->lg.cap) cudaStreamDestroy(ctx->lg.cap);
   free_workspace(&ctx->ws);
+  free_spare_state(ctx);
+  if (ctx->pipe_st) cudaStreamDestroy(ctx->pipe_st);
+  if (ctx->pipe_in) cudaEventDestroy(ctx->pipe_in);
   free_block_tables(&ctx->bt);
   if (ctx->own_offsets) cudaFree(ctx->offsets);
   if (ctx->own_indices) cudaFree(ctx->indices);
@@ -449,6 +452,54 @@ agnes_status agnes_set_launch_mode(agnes_ctx* ctx, int32_t mode) {
     return AGNES_EINVAL;
   }
   ctx->lg.mode = mode;
+  ctx->spare.lg.mode = mode;
+  return AGNES_OK;
+}
+
+agnes_status agnes_set_pipeline_depth(agnes_ctx* ctx, int32_t depth) {
+  if (!ctx) return AGNES_EINVAL;
+  if (depth != 1 && depth != 2) {
+    set_err(ctx, "pipeline depth must be 1 or 2");
+    return AGNES_EINVAL;
+  }
+  if (depth == 2 && (ctx->features_on_host || ctx->topo.on)) {
+    set_err(ctx, "a pipeline depth of 2 needs the graph resident in device memory");
+    return AGNES_EINVAL;
+  }
+  if (depth == ctx->pipe_depth) return AGNES_OK;
+  DeviceGuard dg(ctx->device);
+  CK(ctx, cudaDeviceSynchronize());
+  if (depth == 2) {
+    const agnes_status rc = make_spare_state(ctx);
+    if (rc != AGNES_OK) return rc;
+  } else {
+    free_spare_state(ctx);
+  }
+  ctx->pipe_depth = depth;
+  return AGNES_OK;
+}
+
+agnes_status agnes_fetch_previous_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  if (ctx->pipe_depth != 2 || !ctx->spare.prepared) {
+    set_err(ctx, "no earlier hyperbatch in flight (needs a pipeline depth of 2 and two prepares)");
+    return AGNES_ESTATE;
+  }
+  swap_hyperbatch_state(ctx);
+  const agnes_status rc = agnes_fetch_hyperbatch(ctx, out);
+  swap_hyperbatch_state(ctx);
+  return rc;
+}
+
+agnes_status agnes_wait_hyperbatches(agnes_ctx* ctx, void* cuda_stream) {
+  if (!ctx) return AGNES_EINVAL;
+  DeviceGuard dg(ctx->device);
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  if (ctx->done) CK(ctx, cudaStreamWaitEvent(st, ctx->done, 0));
+  if (ctx->pipe_depth == 2 && ctx->spare.done) CK(ctx, cudaStreamWaitEvent(st, ctx->spare.done, 0));
   return AGNES_OK;
 }
 

@@ -169,6 +169,27 @@ struct agnes_ctx {
     int64_t captures = 0, launches = 0, programmatic_edges = 0;
   } lg;
 
+  // Hyperbatches in flight (agnes_set_pipeline_depth): with a depth of 2 the
+  // ctx keeps a second set of the per-hyperbatch state -- workspace, launch
+  // graph, completion and side-stream events, side stream, its own internal
+  // stream and the fetch state -- and swaps it with the active set at every
+  // prepare, so consecutive hyperbatches use alternate sets and run on
+  // alternate internal streams, overlapping.  The active set (the fields
+  // above and pipe_st) always belongs to the last prepare.
+  int32_t pipe_depth = 1;
+  cudaStream_t pipe_st = nullptr;  // the active set's internal stream (depth 2)
+  cudaEvent_t pipe_in = nullptr;   // orders an internal stream after the caller's
+  struct Spare {
+    agnes::Workspace ws;
+    LaunchGraph lg;
+    uint64_t ws_gen = 0;
+    cudaEvent_t done = nullptr, aux_fork = nullptr, aux_join = nullptr, aux_ready = nullptr;
+    cudaStream_t aux = nullptr;
+    cudaStream_t pipe_st = nullptr;
+    int cur = 0;
+    bool prepared = false, synced = false;
+  } spare;
+
   // streaming of host-resident features (features_on_host)
   cudaStream_t copy_stream = nullptr;
   char* slots = nullptr;
@@ -271,6 +292,11 @@ struct agnes_ctx {
 // prepare.cu
 void free_workspace(agnes::Workspace* w);
 void drop_launch_graph(agnes_ctx::LaunchGraph* g);
+// Swaps the active per-hyperbatch state with the spare one (pipeline depth 2).
+void swap_hyperbatch_state(agnes_ctx* ctx);
+// Creates the spare set's events and streams (once); frees the spare set.
+agnes_status make_spare_state(agnes_ctx* ctx);
+void free_spare_state(agnes_ctx* ctx);
 
 // host_features.cu
 agnes_status setup_streaming(agnes_ctx* ctx, const agnes_graph_desc* d, cudaStream_t st);

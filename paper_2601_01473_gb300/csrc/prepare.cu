@@ -14,6 +14,7 @@
 // and replayed as one CUDA graph launch.
 #include <string.h>
 
+#include <utility>
 #include <vector>
 
 #include "ctx.h"
@@ -206,6 +207,60 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   }
   w.valid = true;
   return AGNES_OK;
+}
+
+void swap_hyperbatch_state(agnes_ctx* ctx) {
+  agnes_ctx::Spare& o = ctx->spare;
+  std::swap(ctx->ws, o.ws);
+  std::swap(ctx->lg, o.lg);
+  std::swap(ctx->ws_gen, o.ws_gen);
+  std::swap(ctx->done, o.done);
+  std::swap(ctx->aux_fork, o.aux_fork);
+  std::swap(ctx->aux_join, o.aux_join);
+  std::swap(ctx->aux_ready, o.aux_ready);
+  std::swap(ctx->aux, o.aux);
+  std::swap(ctx->pipe_st, o.pipe_st);
+  std::swap(ctx->cur, o.cur);
+  std::swap(ctx->prepared, o.prepared);
+  std::swap(ctx->synced, o.synced);
+}
+
+agnes_status make_spare_state(agnes_ctx* ctx) {
+  agnes_ctx::Spare& o = ctx->spare;
+  if (o.done) return AGNES_OK;
+  const unsigned f = cudaEventDisableTiming;
+  if (cudaEventCreateWithFlags(&o.done, f) != cudaSuccess ||
+      cudaEventCreateWithFlags(&o.aux_fork, f) != cudaSuccess ||
+      cudaEventCreateWithFlags(&o.aux_join, f) != cudaSuccess ||
+      cudaEventCreateWithFlags(&o.aux_ready, f) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&o.aux, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&o.pipe_st, cudaStreamNonBlocking) != cudaSuccess ||
+      (!ctx->pipe_st && cudaStreamCreateWithFlags(&ctx->pipe_st, cudaStreamNonBlocking) !=
+                            cudaSuccess) ||
+      (!ctx->pipe_in && cudaEventCreateWithFlags(&ctx->pipe_in, f) != cudaSuccess)) {
+    cudaGetLastError();
+    set_err(ctx, "creating the second hyperbatch's events or streams failed");
+    return AGNES_ECUDA;
+  }
+  o.lg.mode = ctx->lg.mode;
+  return AGNES_OK;
+}
+
+void free_spare_state(agnes_ctx* ctx) {
+  agnes_ctx::Spare& o = ctx->spare;
+  drop_launch_graph(&o.lg);
+  if (o.lg.cap) cudaStreamDestroy(o.lg.cap);
+  o.lg.cap = nullptr;
+  free_workspace(&o.ws);
+  if (o.done) cudaEventDestroy(o.done);
+  if (o.aux_fork) cudaEventDestroy(o.aux_fork);
+  if (o.aux_join) cudaEventDestroy(o.aux_join);
+  if (o.aux_ready) cudaEventDestroy(o.aux_ready);
+  if (o.aux) cudaStreamDestroy(o.aux);
+  if (o.pipe_st) cudaStreamDestroy(o.pipe_st);
+  const int32_t mode = o.lg.mode;
+  o = agnes_ctx::Spare();
+  o.lg.mode = mode;
 }
 
 void drop_launch_graph(agnes_ctx::LaunchGraph* g) {
@@ -582,10 +637,22 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     set_err(ctx, "cudaSetDevice(%d) failed", ctx->device);
     return AGNES_ECUDA;
   }
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const bool capturing = stream_capturing(st);
+  const bool resident = !ctx->features_on_host && !ctx->topo.on;
+  const bool pipelined = ctx->pipe_depth == 2 && resident && !capturing;
+  if (pipelined) {
+    // the other set of per-hyperbatch state: its internal stream starts once
+    // the caller's stream reaches this call, and is already ordered after the
+    // set's previous hyperbatch
+    swap_hyperbatch_state(ctx);
+    CK(ctx, cudaEventRecord(ctx->pipe_in, st));
+    CK(ctx, cudaStreamWaitEvent(ctx->pipe_st, ctx->pipe_in, 0));
+    st = ctx->pipe_st;
+  }
   agnes_status rc = ensure_workspace(ctx, H, B, fanouts, K, cap);
   if (rc != AGNES_OK) return rc;
   Workspace& w = ctx->ws;
-  cudaStream_t st = (cudaStream_t)cuda_stream;
   ctx->prepared = false;
   ctx->synced = false;
   if (ctx->profiling && !ctx->ev_created) {
@@ -595,9 +662,8 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   }
   const int ring = (int)(ctx->n_prepared % kEventRing);
   ctx->n_phases[ring] = 0;
-  // a prepare on another stream than the last one still runs after it: both
-  // use the ctx's buffers (a caller's own capture orders its replays itself)
-  const bool capturing = stream_capturing(st);
+  // a prepare on another stream than the last one on these buffers still runs
+  // after it (a caller's own capture orders its replays itself)
   if (ctx->n_prepared > 0 && !capturing) CK(ctx, cudaStreamWaitEvent(st, ctx->done, 0));
   if (!capturing) {
     rc = update_topology_cache(ctx, st);
@@ -607,7 +673,6 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
                             sizeof(int32_t) * B, H, cudaMemcpyDefault, st));
   CK(ctx, launch_set_key(w.key, seed, first_minibatch_id, st));
   int n_marks = 0;
-  const bool resident = !ctx->features_on_host && !ctx->topo.on;
   if (resident && ctx->lg.mode != AGNES_LAUNCH_DIRECT && !capturing)
     rc = launch_graphed(ctx, fanouts, K, cap, ring, st, &n_marks);
   else

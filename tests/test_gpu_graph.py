@@ -138,3 +138,57 @@ def test_prepares_on_two_streams_run_in_call_order(cuda_device):
         g.prepare(t2, fan, 5, 5, s2)  # waits for the prepare on s1
     compare(g, og, t2.cpu().numpy(), fan, 5, 5, ADJ, FEAT)
     g.close()
+
+
+def test_pipeline_depth_two_matches_oracle_and_overlaps_safely(cuda_device):
+    """Two hyperbatches in flight (agnes_set_pipeline_depth 2): a sequence of
+    prepares on one caller stream, each checked against the oracle through
+    fetch, the hyperbatch before the last through agnes_fetch_previous_hyperbatch
+    while the last is in flight, a device-side consumer ordered with
+    agnes_wait_hyperbatches, and a return to depth 1."""
+    off, ind, feats = make(30000, 12, seed=51, dim=32)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    g = load(off, ind, feats, ADJ, FEAT)
+    g.set_pipeline_depth(2)
+    pool = torch.arange(30000, dtype=torch.int32)
+    fan = [6, 4, 3]
+    tgts = [synth.hyperbatch_targets(pool, 6, 200, 53, s) for s in range(5)]
+    st = torch.cuda.Stream(cuda_device)
+    with torch.cuda.stream(st):
+        dev = [t.to(cuda_device, non_blocking=True) for t in tgts]
+    for s in range(5):
+        g.prepare(dev[s], fan, 7, 100 * s, st)
+        if s >= 1:  # the previous hyperbatch, while this one may still run
+            prev = g.fetch_previous()
+            r = oracle.sample_minibatch(og, tgts[s - 1][2].numpy(), fan, 7, 100 * (s - 1) + 2)
+            n = int(prev.node_size[3, 2])
+            assert np.array_equal(prev.nodes[2, :n].cpu().numpy(), r["nodes"])
+        compare(g, og, tgts[s].numpy(), fan, 7, 100 * s, ADJ, FEAT)
+    # a device consumer on the caller's stream, ordered by the wait call
+    g.prepare(dev[0], fan, 9, 0, st)
+    g.prepare(dev[1], fan, 9, 600, st)
+    g.wait(st)
+    with torch.cuda.stream(st):
+        v = g.fetch_all()
+        copy = v.nodes.clone()
+    st.synchronize()
+    assert torch.equal(copy, v.nodes)
+    compare(g, og, tgts[1].numpy(), fan, 9, 600, ADJ, FEAT)
+    g.set_pipeline_depth(1)
+    g.prepare(dev[2], fan, 9, 900, st)
+    compare(g, og, tgts[2].numpy(), fan, 9, 900, ADJ, FEAT)
+    g.close()
+
+
+def test_pipeline_depth_two_needs_a_resident_graph(cuda_device):
+    off, ind, feats = make(3000, 6, seed=52)
+    dev = torch.device("cuda:0")
+    from paper_2601_01473_gb300 import AgnesError, Graph
+    g = Graph(off.to(dev), ind.to(dev), feats.pin_memory(), adj_block_bytes=4096,
+              feat_block_bytes=4096, features_on_host=True)
+    with pytest.raises(AgnesError) as e:
+        g.set_pipeline_depth(2)
+    assert e.value.status == 1
+    with pytest.raises(AgnesError):
+        g.set_pipeline_depth(3)
+    g.close()
