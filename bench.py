@@ -127,14 +127,14 @@ class ClockSampler:
 
 
 def kernel_launches_per_step(K: int) -> int:
-    """Kernels libagnes launches per hyperbatch with the graph in HBM (61 at
+    """Kernels libagnes launches per hyperbatch with the graph in HBM (67 at
     K = 3): the sampling-key write and the dst-size fill 2; target bucketing 5
-    (count, 2-kernel scan, scatter, sort); per hop 16
-    (count, 2-kernel scan, fill, 2-kernel scan, scatter, cells, big cells,
-    3-kernel column scan, 2-kernel scan, col fix-up, compaction); after the
-    last hop 3 (feature-block marks, their count, gather) and K counts of
-    touched topology blocks."""
-    return 2 + 5 + 16 * K + 3 + K
+    (count, 2-kernel scan, scatter, sort); per hop 18 (count, 2-kernel scan,
+    fill, 2-kernel scan, scatter, the cells' lane kernel, queue offsets, queue
+    copy, tile kernel, 3-kernel column scan, 2-kernel scan, col fix-up,
+    compaction); after the last hop 3 (feature-block marks, their count,
+    gather) and K counts of touched topology blocks."""
+    return 2 + 5 + 18 * K + 3 + K
 
 
 def algorithmic_bytes(c: dict, off_bytes: int) -> dict:
@@ -410,6 +410,8 @@ def main():
     algo = [algorithmic_bytes(c, off_bytes) for c in counters]
     gather_bytes = statistics.mean(a["gather"] for a in algo)
     total_bytes = statistics.mean(a["total"] for a in algo)
+    iso = [p[-1] for p in phases if p]
+    iso_ms = statistics.mean(iso) if iso else None
     stats = g.stats()
 
     # end to end through the C ABI: host (pinned) targets in, views out
@@ -450,6 +452,11 @@ def main():
                 "traffic": gather_traffic_from_profile(w.name),
                 "algorithmic_bytes_per_launch": gather_bytes,
                 "avg_launch_ms": g_ms,
+                # the gather alone: the untimed re-run fetches each hyperbatch's
+                # counters before the next prepare, so nothing overlaps it there
+                "isolated_launch_ms": iso_ms,
+                "isolated_achieved": gather_bytes / (iso_ms / 1e3) / 1e9 if iso_ms else None,
+                "isolated_frac": gather_bytes / (iso_ms / 1e3) / 1e9 / peak if iso_ms else None,
                 "path_algorithmic_bytes_per_step": total_bytes,
                 "path_GBps": total_bytes / (elapsed_ms / args.steps / 1e3) / 1e9}
     # the whole sample+gather path (every kernel of the step) against the same
@@ -539,7 +546,7 @@ def main():
                        "gen_seconds": round(gen_s, 1)},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "host_link": host_link,
             "topology_streaming": topo,
-            # counted for the HBM-resident path (the ncu launch list has 61 per hyperbatch
+            # counted for the HBM-resident path (the ncu launch list has 67 per hyperbatch
             # at K = 3); the host-resident modes add per-batch loads and gathers
             "gpu_launches": kernel_launches_per_step(K) * args.steps
             if not (args.stream or args.stream_topology) else None,

@@ -156,7 +156,7 @@ __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, co
 // takes a contiguous range of batches and appends its queued cells (with
 // samples and more than kLaneMax entries) in order at the start of its own
 // range of q_cells (q_cnt[warp] of them).
-__global__ void __launch_bounds__(kThreads) dedup_lane_kernel(CellsArgs a) {
+__global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
   grid_dep_wait();
   if (failed(a.status)) return;
   const int lane = lane_id();
