@@ -576,6 +576,7 @@ def run_sweep(args, w):
     fan = list(w.fanouts)
     for bb in [int(x) for x in args.sweep_blocks.split(",")]:
         g = Graph(offsets, indices, features, bb, bb, device=0, stream=stream)
+        g.set_pipeline_depth(args.pipeline_depth)
         info = g.info()
         for H in [int(x) for x in args.sweep_H.split(",")]:
             wh = w.with_(H=H, adj_block_bytes=bb, feat_block_bytes=bb)
@@ -588,6 +589,7 @@ def run_sweep(args, w):
             e0.record(stream)
             for s in range(args.warmup, args.warmup + args.steps):
                 g.prepare(steps[s], fan, w.seed, s * H, stream)
+            g.wait(stream)
             e1.record(stream)
             torch.cuda.synchronize()
             ms = e0.elapsed_time(e1) / args.steps
