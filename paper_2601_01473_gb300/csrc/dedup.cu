@@ -27,12 +27,13 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kIlp = 4;  // independent elements per thread in the streaming passes
 
 // Places every sampled edge of minibatch j at soff[cell] + rank (cell and
-// rank were recorded while sampling), building the sampled bucket.
+// rank were recorded while sampling), building the sampled bucket: (id, edge
+// index) pairs, or packed 4-byte entries edge index << 12 | tile-local id.
 __global__ void __launch_bounds__(kThreads)
 dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict__ ecnt,
                      int64_t ecap, const int32_t* __restrict__ scell,
                      const int32_t* __restrict__ srank, const int32_t* __restrict__ soff,
-                     int2* __restrict__ sb, const int32_t* status) {
+                     int2* __restrict__ sb, bool packed, const int32_t* status) {
   grid_dep_wait();
   if (failed(status)) return;
   const int32_t j = blockIdx.y;
@@ -41,7 +42,10 @@ dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict_
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < E;
        e += (int64_t)gridDim.x * blockDim.x) {
     const int32_t slot = soff[scell[o + e]] + srank[o + e];
-    sb[slot] = make_int2(nbr[o + e], (int32_t)e);
+    if (packed)  // nbr holds the tile-local id (< 2^12), e < 2^20
+      reinterpret_cast<uint32_t*>(sb)[slot] = ((uint32_t)e << 12) | (uint32_t)nbr[o + e];
+    else
+      sb[slot] = make_int2(nbr[o + e], (int32_t)e);
   }
 }
 
@@ -538,7 +542,7 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
                                              true, nullptr, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
   dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, d.scell, d.srank,
-                                                   d.soff, d.sb, a.status);
+                                                   d.soff, d.sb, a.sb_packed, a.status);
 
   CellArgs c;
   c.tm = tm;

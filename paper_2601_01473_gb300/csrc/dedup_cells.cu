@@ -49,7 +49,8 @@ struct CellsArgs {
   const int32_t* fb_id;  // frontier bucket: ids ascending inside a cell
   const int32_t* fb_pos;
   const int32_t* fcell_off;
-  const int2* sb;  // sampled bucket: (id, edge index in the minibatch)
+  const int2* sb;  // sampled bucket: (id, edge index in the minibatch), or packed 4-byte
+                   // entries edge index << 12 | tile-local id (the kernels' kPacked)
   const int32_t* soff;
   const int32_t* tile_adj_block;
   uint8_t* adj_flags;
@@ -79,6 +80,19 @@ __device__ __forceinline__ CellFacts cell_facts(const CellsArgs& a, int64_t cell
   return c;
 }
 
+// Sampled entry i of the bucket as (tile-local id, edge index); base is the
+// tile's first id.
+template <bool kPacked>
+__device__ __forceinline__ int2 sampled_entry(const CellsArgs& a, int32_t i, int32_t base) {
+  if constexpr (kPacked) {
+    const uint32_t v = reinterpret_cast<const uint32_t*>(a.sb)[i];
+    return make_int2((int32_t)(v & 0xfffu), (int32_t)(v >> 12));
+  } else {
+    const int2 e = a.sb[i];
+    return make_int2(e.x - base, e.y);
+  }
+}
+
 // ---- cells of at most kLaneMax entries: a thread each ---------------------------
 
 template <int I, int J>
@@ -103,6 +117,7 @@ __device__ __forceinline__ void sort8(int32_t (&k)[kLaneMax], int32_t (&p)[kLane
 }
 
 // Resolves one cell with samples and at most kLaneMax entries in one thread.
+template <bool kPacked>
 __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, const CellFacts& c) {
   const int32_t n = c.fn + c.sn;
   const int32_t tb = __ldg(a.tile_first + c.t);
@@ -115,8 +130,8 @@ __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, co
       key[q] = (a.fb_id[c.fo + q] - tb) << 1;
       pay[q] = a.fb_pos[c.fo + q];
     } else if (q < n) {
-      const int2 e = a.sb[c.so + (q - c.fn)];
-      key[q] = ((e.x - tb) << 1) | 1;
+      const int2 e = sampled_entry<kPacked>(a, c.so + (q - c.fn), tb);
+      key[q] = (e.x << 1) | 1;
       pay[q] = e.y;
     }
   }
@@ -156,6 +171,7 @@ __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, co
 // takes a contiguous range of batches and appends its queued cells (with
 // samples and more than kLaneMax entries) in order at the start of its own
 // range of q_cells (q_cnt[warp] of them).
+template <bool kPacked>
 __global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
   grid_dep_wait();
   if (failed(a.status)) return;
@@ -180,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
     if ((qm >> lane) & 1u)
       a.q_cells[(b_lo << 5) + queued + __popc(qm & ((1u << lane) - 1u))] = (int32_t)cell;
     queued += __popc(qm);
-    if (has && c.sn > 0 && n <= kLaneMax) thread_cell(a, cell, c);
+    if (has && c.sn > 0 && n <= kLaneMax) thread_cell<kPacked>(a, cell, c);
   }
   if (lane == 0) a.q_cnt[gw] = queued;
 }
@@ -243,6 +259,7 @@ struct TileScratch {
   int32_t* pN;  // new ids below word w
 };
 
+template <bool kPacked>
 __global__ void __launch_bounds__(kThreads, 8) dedup_tile_kernel(CellsArgs a, int32_t nw) {
   grid_dep_wait();
   if (failed(a.status)) return;
@@ -278,7 +295,7 @@ __global__ void __launch_bounds__(kThreads, 8) dedup_tile_kernel(CellsArgs a, in
       int32_t v[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k)
-        v[k] = i0 + 32 * k < c.sn ? a.sb[c.so + i0 + 32 * k].x - base : -1;
+        v[k] = i0 + 32 * k < c.sn ? sampled_entry<kPacked>(a, c.so + i0 + 32 * k, base).x : -1;
 #pragma unroll
       for (int k = 0; k < 4; ++k)
         if (v[k] >= 0) atomicOr(t.S + (v[k] >> 5), 1u << (v[k] & 31));
@@ -317,8 +334,8 @@ __global__ void __launch_bounds__(kThreads, 8) dedup_tile_kernel(CellsArgs a, in
     }
     int32_t* col = a.col + (int64_t)c.j * a.ecap;
     for (int32_t i = lane; i < c.sn; i += 32) {
-      const int2 e = a.sb[c.so + i];
-      const int32_t v = e.x - base;
+      const int2 e = sampled_entry<kPacked>(a, c.so + i, base);
+      const int32_t v = e.x;
       const int32_t w = v >> 5;
       const uint32_t bit = 1u << (v & 31), below = bit - 1u;
       const uint32_t dw = t.D[w];
@@ -362,21 +379,28 @@ CellsArgs cells_args(const HopArgs& h, const DedupBufs& d) {
   return a;
 }
 
+template <bool kPacked>
+cudaError_t launch_cells(const CellsArgs& a, int32_t q_warps_cap, int num_sms, cudaStream_t st) {
+  const int grid = resident_grid((const void*)dedup_lane_kernel<kPacked>, kThreads, num_sms);
+  const int nw = grid * kWarps;
+  if (nw > q_warps_cap) return cudaErrorInvalidValue;
+  dedup_lane_kernel<kPacked><<<grid, kThreads, 0, st>>>(a);
+  queue_offsets_kernel<<<1, 1024, 0, st>>>(a.q_cnt, nw, a.q_off, a.status);
+  queue_compact_kernel<<<resident_grid((const void*)queue_compact_kernel, kThreads, num_sms),
+                         kThreads, 0, st>>>(a, nw);
+  dedup_tile_kernel<kPacked><<<resident_grid((const void*)dedup_tile_kernel<kPacked>, kThreads,
+                                             num_sms),
+                               kThreads, 0, st>>>(a, nw);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_dedup_cells(const HopArgs& h, const DedupBufs& d, int num_sms,
                                cudaStream_t st) {
   const CellsArgs a = cells_args(h, d);
-  const int grid = resident_grid((const void*)dedup_lane_kernel, kThreads, num_sms);
-  const int nw = grid * kWarps;
-  if (nw > d.q_warps_cap) return cudaErrorInvalidValue;
-  dedup_lane_kernel<<<grid, kThreads, 0, st>>>(a);
-  queue_offsets_kernel<<<1, 1024, 0, st>>>(a.q_cnt, nw, a.q_off, a.status);
-  queue_compact_kernel<<<resident_grid((const void*)queue_compact_kernel, kThreads, num_sms),
-                         kThreads, 0, st>>>(a, nw);
-  dedup_tile_kernel<<<resident_grid((const void*)dedup_tile_kernel, kThreads, num_sms), kThreads,
-                      0, st>>>(a, nw);
-  return cudaGetLastError();
+  return h.sb_packed ? launch_cells<true>(a, d.q_warps_cap, num_sms, st)
+                     : launch_cells<false>(a, d.q_warps_cap, num_sms, st);
 }
 
 }  // namespace agnes

@@ -87,7 +87,13 @@ struct HopArgs {
   int32_t* hset = nullptr;
   int32_t hset_log2 = 0;
   int32_t hset_grid = 0;
+  // the sampled bucket holds 4-byte entries (edge index << 12 | tile-local
+  // id): the default frontier with ecap <= kPackedEdgeMax; the sampler then
+  // records tile-local ids
+  bool sb_packed = false;
 };
+
+constexpr int64_t kPackedEdgeMax = (int64_t)1 << 20;
 
 // The hash sets the sampler needs for a fanout k > kWideMax: 2^log2 >= 2k
 // entries per warp and the CTAs of its grid (capped so the tables stay within

@@ -326,6 +326,8 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     a.status = w.status;
     a.hset = w.hset;
     huge_fanout_tables(fanouts[h], nsm, &a.hset_log2, &a.hset_grid);
+    const bool frontier_sampled = ctx->frontier_mode == AGNES_FRONTIER_SAMPLED && h + 1 < K;
+    a.sb_packed = !frontier_sampled && a.ecap <= kPackedEdgeMax;
     int32_t* nsz_prev = w.nsz + (int64_t)h * H;
     int32_t* ecnt = w.ecnt + (int64_t)h * H;
     CK(ctx, launch_sample_count(a, w.fb_id[cur], w.fb_pos[cur], w.fcell_off[cur], w.cnt, nsm, st));
@@ -392,7 +394,7 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.nsz_next = w.nsz + (int64_t)(h + 1) * H;
     d.srcsz = w.srcsz + (int64_t)h * H;
     d.noutbase = w.noutbase;
-    d.frontier_sampled = ctx->frontier_mode == AGNES_FRONTIER_SAMPLED && h + 1 < K;
+    d.frontier_sampled = frontier_sampled;
     d.nodes = w.nodes;
     d.col = w.col[h];
     d.tile_adj_block = ctx->bt.tile_adj_block;

@@ -215,6 +215,7 @@ struct FillArgs {
   int32_t k, hop;
   const uint64_t* key;  // device: {seed, first minibatch id}
   int32_t* status;
+  bool packed;        // record tile-local ids (the dedup's sampled bucket is packed)
   int32_t* hset;      // fanouts above kWideMax: per-warp hash sets of chosen positions
   int32_t hset_log2;  // each of 2^hset_log2 entries
 };
@@ -273,12 +274,17 @@ __device__ __forceinline__ int64_t draw(const FillArgs& a, const Key& key, int32
 __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t u, uint32_t j,
                                            int64_t eidx) {
   int64_t cell = 0;
-  if (has) cell = (int64_t)tile_of(a.tm, u) * a.H + j;
+  int32_t val = u;  // the id, or with a packed sampled bucket its tile-local id
+  if (has) {
+    const int32_t t = tile_of(a.tm, u);
+    cell = (int64_t)t * a.H + j;
+    if (a.packed) val = u - __ldg(a.tm.tile_first + t);
+  }
   const unsigned m = __ballot_sync(0xffffffffu, has);
   if (has) {
     const int32_t rank = warp_agg_add(a.scnt, cell, m);
     const int64_t at = (int64_t)j * a.ecap + eidx;
-    a.nbr[at] = u;
+    a.nbr[at] = val;
     a.scell[at] = (int32_t)cell;
     a.srank[at] = rank;
   }
@@ -601,6 +607,7 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.status = a.status;
   f.hset = a.hset;
   f.hset_log2 = a.hset_log2;
+  f.packed = a.sb_packed;
   if (a.k > kWideMax && (a.hset == nullptr || a.hset_grid < 1)) return cudaErrorInvalidValue;
   const int src = r.gbuf == nullptr ? kEdgesInPlace : r.in_place_fallback ? kEdgesCached
                                                                             : kEdgesBuffer;
