@@ -70,6 +70,7 @@ struct Workspace {
   int32_t* tmp_id = nullptr;
   int32_t* tmp_pos = nullptr;
   int32_t* cnt = nullptr;
+  int64_t* fbd = nullptr;  // 2 per frontier entry: (first edge, degree)
   void* feats_out = nullptr;
   uint8_t* adj_flags = nullptr;
   uint8_t* feat_flags = nullptr;

@@ -91,6 +91,9 @@ struct HopArgs {
   // id): the default frontier with ecap <= kPackedEdgeMax; the sampler then
   // records tile-local ids
   bool sb_packed = false;
+  // per frontier entry (bucket order): its node's first edge and degree, two
+  // int64 each, written by the count kernel and read by the fill
+  int64_t* fbd = nullptr;
 };
 
 constexpr int64_t kPackedEdgeMax = (int64_t)1 << 20;

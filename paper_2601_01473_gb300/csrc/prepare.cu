@@ -68,6 +68,7 @@ void free_workspace(Workspace* w) {
   cudaFree(w->tmp_id);
   cudaFree(w->tmp_pos);
   cudaFree(w->cnt);
+  cudaFree(w->fbd);
   cudaFree(w->feats_out);
   cudaFree(w->adj_flags);
   cudaFree(w->feat_flags);
@@ -174,6 +175,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.tmp_id, (int64_t)H * B);
   WA(w.tmp_pos, (int64_t)H * B);
   WA(w.cnt, (int64_t)H * w.cap_prev_max);
+  WA(w.fbd, 2 * (int64_t)H * w.cap_prev_max);
   {
     uint8_t* f = nullptr;
     WA(f, rows * ctx->row_bytes);
@@ -325,6 +327,7 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     a.key = w.key;
     a.status = w.status;
     a.hset = w.hset;
+    a.fbd = w.fbd;
     huge_fanout_tables(fanouts[h], nsm, &a.hset_log2, &a.hset_grid);
     const bool frontier_sampled = ctx->frontier_mode == AGNES_FRONTIER_SAMPLED && h + 1 < K;
     a.sb_packed = !frontier_sampled && a.ecap <= kPackedEdgeMax;

@@ -169,12 +169,16 @@ targets_sort_kernel(const int32_t* __restrict__ fcell_off, int64_t ncells, int32
 
 // ---- sampling --------------------------------------------------------------------
 
+// Per frontier entry i (bucket order): the node's count of sampled edges
+// min(deg, k) at its minibatch position (for the edge offsets' scan), and
+// (first edge, degree) in fbd[i] for the fill, which then reads them
+// coalesced instead of the offsets at random.
 template <typename OffT>
 __global__ void __launch_bounds__(kThreads)
 sample_count_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict__ fb_pos,
                     const int32_t* total_ptr, const OffT* __restrict__ off, int64_t capK,
                     int64_t cap_prev, int32_t k, int32_t* __restrict__ cnt,
-                    const int32_t* status) {
+                    longlong2* __restrict__ fbd, const int32_t* status) {
   grid_dep_wait();
   if (failed(status)) return;
   const int64_t total = *total_ptr;
@@ -185,8 +189,10 @@ sample_count_kernel(const int32_t* __restrict__ fb_id, const int32_t* __restrict
     const uint32_t g = (uint32_t)fb_pos[i];
     const uint32_t j = g / capk32;
     const uint32_t pos = g - j * capk32;
-    const int64_t d = (int64_t)__ldg(off + v + 1) - (int64_t)__ldg(off + v);
+    const int64_t base = (int64_t)__ldg(off + v);
+    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
     cnt[j * cap_prev + pos] = (int32_t)(d < k ? d : k);
+    fbd[i] = make_longlong2(base, d);
   }
 }
 
@@ -208,6 +214,7 @@ struct FillArgs {
   int32_t* srank;  // per edge: its rank within the cell
   const int32_t* fb_id;
   const int32_t* fb_pos;
+  const longlong2* fbd;  // per frontier entry: (first edge, degree) of its node
   const int64_t* indptr;
   const int32_t* indices;
   int32_t* nbr;
@@ -290,53 +297,54 @@ __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t 
   }
 }
 
-// G lanes per frontier node, k <= G.
-template <typename OffT, int G, int kSrc>
-__global__ void __launch_bounds__(kThreads)
-sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
+// k <= 32: k lanes per frontier node (lane s draws slot s), 32 / k nodes per
+// warp round; the lanes past them (32 mod k) idle.
+template <int kSrc>
+__global__ void __launch_bounds__(kThreads, 8) sample_fill_kernel(FillArgs a) {
   grid_dep_wait();
   if (failed(a.status)) return;
   const Key key = load_key(a.key);
   const int64_t E0 = a.fcell_off[a.cell_lo], E1 = a.fcell_off[a.cell_hi];
-  constexpr int kGroups = 32 / G;
+  const int k = a.k;
+  const int groups = 32 / k;
   const int lane = lane_id();
-  const int sub = lane / G, s = lane % G;
-  const unsigned gmask = G == 32 ? 0xffffffffu : (((1u << G) - 1u) << (sub * G));
+  const int sub = lane / k, s = lane - sub * k;
+  const int g0 = sub * k;  // the group's first lane
+  const bool member = sub < groups;
+  const unsigned gmask = k == 32 ? 0xffffffffu : (((1u << k) - 1u) << g0);
   const uint32_t capk32 = (uint32_t)a.capK;
   const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t e0 = E0 + warp0 * kGroups; e0 < E1; e0 += nwarps * kGroups) {
+  for (int64_t e0 = E0 + warp0 * groups; e0 < E1; e0 += nwarps * groups) {
     const int64_t i = e0 + sub;
     bool has = false;
     int32_t u = 0;
     uint32_t j = 0;
     int64_t eidx = 0;
-    if (i < E1) {  // whole group takes the same branches
+    if (member && i < E1) {  // whole group takes the same branches
       const int32_t v = a.fb_id[i];
       const uint32_t g = (uint32_t)a.fb_pos[i];
+      const longlong2 bd = a.fbd[i];
+      const int64_t base = bd.x, d = bd.y;
       j = g / capk32;
       const uint32_t pos = g - j * capk32;
-      const int64_t base = (int64_t)__ldg(off + v);
-      const int64_t d = (int64_t)__ldg(off + v + 1) - base;
       eidx = a.indptr[j * (a.cap_prev + 1) + pos] + s;
-      if (d <= a.k) {
+      if (d <= k) {
         if (s < d) {
           u = edge_at<kSrc>(a, v, base, d, s);
           has = true;
         }
       } else {
-        const int64_t J = d - a.k + s;
-        const int64_t t = s < a.k ? draw(a, key, v, s, key.gid0 + j, J) : -1;
+        const int64_t J = d - k + s;
+        const int64_t t = draw(a, key, v, s, key.gid0 + j, J);
         bool collided = false;
-        for (int q = 0; q < a.k; ++q) {
+        for (int q = 0; q < k; ++q) {
           const int64_t mine = collided ? J : t;
-          const int64_t cq = __shfl_sync(gmask, mine, q, G);
+          const int64_t cq = __shfl_sync(gmask, mine, g0 + q);
           if (s > q && t == cq) collided = true;
         }
-        if (s < a.k) {
-          u = edge_at<kSrc>(a, v, base, d, collided ? J : t);
-          has = true;
-        }
+        u = edge_at<kSrc>(a, v, base, d, collided ? J : t);
+        has = true;
       }
     }
     emit_edges(a, has, u, j, eidx);
@@ -346,9 +354,8 @@ sample_fill_kernel(FillArgs a, const OffT* __restrict__ off) {
 // One warp per frontier node for fanouts above 32: slots are drawn 32 at a
 // time; each candidate is checked against the choices of earlier chunks (kept
 // in shared memory) and then resolved within its chunk by shuffles.
-template <typename OffT, int kSrc>
-__global__ void __launch_bounds__(kThreads)
-sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
+template <int kSrc>
+__global__ void __launch_bounds__(kThreads) sample_fill_wide_kernel(FillArgs a) {
   grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ int32_t chosen_s[kWarps][kWideMax];
@@ -364,8 +371,8 @@ sample_fill_wide_kernel(FillArgs a, const OffT* __restrict__ off) {
     const uint32_t g = (uint32_t)a.fb_pos[i];
     const uint32_t j = g / capk32;
     const uint32_t pos = g - j * capk32;
-    const int64_t base = (int64_t)__ldg(off + v);
-    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
+    const longlong2 bd = a.fbd[i];
+    const int64_t base = bd.x, d = bd.y;
     const int64_t ebase = a.indptr[j * (a.cap_prev + 1) + pos];
     if (d <= a.k) {
       for (int64_t q0 = 0; q0 < d; q0 += 32) {
@@ -431,9 +438,8 @@ __device__ __forceinline__ void hset_insert(int32_t* T, uint32_t mask, int32_t k
   }
 }
 
-template <typename OffT, int kSrc>
-__global__ void __launch_bounds__(kThreads)
-sample_fill_huge_kernel(FillArgs a, const OffT* __restrict__ off) {
+template <int kSrc>
+__global__ void __launch_bounds__(kThreads) sample_fill_huge_kernel(FillArgs a) {
   grid_dep_wait();
   if (failed(a.status)) return;
   const int lane = lane_id();
@@ -449,8 +455,8 @@ sample_fill_huge_kernel(FillArgs a, const OffT* __restrict__ off) {
     const uint32_t g = (uint32_t)a.fb_pos[i];
     const uint32_t j = g / capk32;
     const uint32_t pos = g - j * capk32;
-    const int64_t base = (int64_t)__ldg(off + v);
-    const int64_t d = (int64_t)__ldg(off + v + 1) - base;
+    const longlong2 bd = a.fbd[i];
+    const int64_t base = bd.x, d = bd.y;
     const int64_t ebase = a.indptr[j * (a.cap_prev + 1) + pos];
     if (d <= a.k) {
       for (int64_t q0 = 0; q0 < d; q0 += 32) {
@@ -492,8 +498,7 @@ int64_t huge_fanout_tables(int32_t k, int num_sms, int32_t* log2, int32_t* grid)
   if (k <= kWideMax) return 0;
   int32_t l = 2;
   while ((1 << l) < 2 * k) ++l;
-  int g = resident_grid((const void*)sample_fill_huge_kernel<int64_t, kEdgesInPlace>, kThreads,
-                        num_sms);
+  int g = resident_grid((const void*)sample_fill_huge_kernel<kEdgesInPlace>, kThreads, num_sms);
   const int64_t budget_entries = (int64_t)1 << 28;  // 1 GiB of tables at most
   const int64_t max_warps = budget_entries >> l;
   if ((int64_t)g * kWarps > max_warps) g = (int)(max_warps / kWarps);
@@ -544,33 +549,30 @@ cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const in
     sample_count_kernel<int32_t><<<resident_grid((const void*)sample_count_kernel<int32_t>,
                                                  kThreads, num_sms),
                                    kThreads, 0, st>>>(
-        fb_id, fb_pos, total, (const int32_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt, a.status);
+        fb_id, fb_pos, total, (const int32_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt,
+        reinterpret_cast<longlong2*>(a.fbd), a.status);
   else
     sample_count_kernel<int64_t><<<resident_grid((const void*)sample_count_kernel<int64_t>,
                                                  kThreads, num_sms),
                                    kThreads, 0, st>>>(
-        fb_id, fb_pos, total, (const int64_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt, a.status);
+        fb_id, fb_pos, total, (const int64_t*)a.offsets, a.capK, a.cap_prev, a.k, cnt,
+        reinterpret_cast<longlong2*>(a.fbd), a.status);
   return cudaGetLastError();
 }
 
-template <typename OffT, int kSrc>
-static void launch_fill_typed(const FillArgs& f, const OffT* off, int k, int huge_grid,
-                              int num_sms, cudaStream_t st) {
-#define AGNES_FILL(KERNEL)                                                                   \
-  KERNEL<<<resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st>>>(f, off)
-  if (k <= 4)
-    AGNES_FILL((sample_fill_kernel<OffT, 4, kSrc>));
-  else if (k <= 8)
-    AGNES_FILL((sample_fill_kernel<OffT, 8, kSrc>));
-  else if (k <= 16)
-    AGNES_FILL((sample_fill_kernel<OffT, 16, kSrc>));
-  else if (k <= 32)
-    AGNES_FILL((sample_fill_kernel<OffT, 32, kSrc>));
+template <int kSrc>
+static void launch_fill_typed(const FillArgs& f, int k, int huge_grid, int num_sms,
+                              cudaStream_t st) {
+  if (k <= 32)
+    sample_fill_kernel<kSrc><<<resident_grid((const void*)sample_fill_kernel<kSrc>, kThreads,
+                                             num_sms),
+                               kThreads, 0, st>>>(f);
   else if (k <= kWideMax)
-    AGNES_FILL((sample_fill_wide_kernel<OffT, kSrc>));
+    sample_fill_wide_kernel<kSrc><<<resident_grid((const void*)sample_fill_wide_kernel<kSrc>,
+                                                  kThreads, num_sms),
+                                    kThreads, 0, st>>>(f);
   else
-    sample_fill_huge_kernel<OffT, kSrc><<<huge_grid, kThreads, 0, st>>>(f, off);
-#undef AGNES_FILL
+    sample_fill_huge_kernel<kSrc><<<huge_grid, kThreads, 0, st>>>(f);
 }
 
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
@@ -595,6 +597,7 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   f.srank = srank;
   f.fb_id = fb_id;
   f.fb_pos = fb_pos;
+  f.fbd = reinterpret_cast<const longlong2*>(a.fbd);
   f.indptr = indptr;
   f.indices = a.indices;
   f.nbr = nbr;
@@ -611,21 +614,12 @@ cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int
   if (a.k > kWideMax && (a.hset == nullptr || a.hset_grid < 1)) return cudaErrorInvalidValue;
   const int src = r.gbuf == nullptr ? kEdgesInPlace : r.in_place_fallback ? kEdgesCached
                                                                             : kEdgesBuffer;
-#define AGNES_FILL_SRC(OFF)                                                                  \
-  do {                                                                                      \
-    const OFF* off = (const OFF*)a.offsets;                                                 \
-    if (src == kEdgesInPlace)                                                               \
-      launch_fill_typed<OFF, kEdgesInPlace>(f, off, a.k, a.hset_grid, num_sms, st);                      \
-    else if (src == kEdgesBuffer)                                                           \
-      launch_fill_typed<OFF, kEdgesBuffer>(f, off, a.k, a.hset_grid, num_sms, st);                       \
-    else                                                                                    \
-      launch_fill_typed<OFF, kEdgesCached>(f, off, a.k, a.hset_grid, num_sms, st);                       \
-  } while (0)
-  if (a.offsets_bits == 32)
-    AGNES_FILL_SRC(int32_t);
+  if (src == kEdgesInPlace)
+    launch_fill_typed<kEdgesInPlace>(f, a.k, a.hset_grid, num_sms, st);
+  else if (src == kEdgesBuffer)
+    launch_fill_typed<kEdgesBuffer>(f, a.k, a.hset_grid, num_sms, st);
   else
-    AGNES_FILL_SRC(int64_t);
-#undef AGNES_FILL_SRC
+    launch_fill_typed<kEdgesCached>(f, a.k, a.hset_grid, num_sms, st);
   return cudaGetLastError();
 }
 
