@@ -276,29 +276,34 @@ __device__ __forceinline__ int64_t draw(const FillArgs& a, const Key& key, int32
 }
 
 // Records sampled edge e = (j, eidx) with neighbour u: its id, its
-// (tile, minibatch) cell and its rank within the cell (warp-aggregated
-// atomic), so the bucketing scatter after the scan needs no atomics.
+// (tile, minibatch) cell and its rank within the cell (one atomic per distinct
+// cell of the warp), so the bucketing scatter after the scan needs no atomics.
+// Called by all 32 lanes; lanes without an edge pass has = false.  Cell
+// indices fit 31 bits (T * H < 2^31).
 __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t u, uint32_t j,
                                            int64_t eidx) {
-  int64_t cell = 0;
-  int32_t val = u;  // the id, or with a packed sampled bucket its tile-local id
+  const int32_t t = tile_of(a.tm, has ? u : 0);
+  const uint32_t cell = (uint32_t)t * (uint32_t)a.H + j;
+  // the id, or with a packed sampled bucket its tile-local id
+  const int32_t val = a.packed ? u - __ldg(a.tm.tile_first + t) : u;
+  const unsigned peers = __match_any_sync(0xffffffffu, has ? cell : 0xffffffffu);
+  const int lane = lane_id();
+  const int leader = __ffs(peers) - 1;
+  int32_t old = 0;
+  if (has && lane == leader) old = atomicAdd(a.scnt + cell, __popc(peers));
+  old = __shfl_sync(0xffffffffu, old, leader);
   if (has) {
-    const int32_t t = tile_of(a.tm, u);
-    cell = (int64_t)t * a.H + j;
-    if (a.packed) val = u - __ldg(a.tm.tile_first + t);
-  }
-  const unsigned m = __ballot_sync(0xffffffffu, has);
-  if (has) {
-    const int32_t rank = warp_agg_add(a.scnt, cell, m);
     const int64_t at = (int64_t)j * a.ecap + eidx;
     a.nbr[at] = val;
     a.scell[at] = (int32_t)cell;
-    a.srank[at] = rank;
+    a.srank[at] = old + __popc(peers & ((1u << lane) - 1u));
   }
 }
 
 // k <= 32: k lanes per frontier node (lane s draws slot s), 32 / k nodes per
-// warp round; the lanes past them (32 mod k) idle.
+// warp round; the lanes past them (32 mod k) idle.  The round runs without
+// divergent branches: every lane draws (a node of degree <= k takes its
+// first d edges instead) and the collision shuffles span the whole warp.
 template <int kSrc>
 __global__ void __launch_bounds__(kThreads, 8) sample_fill_kernel(FillArgs a) {
   grid_dep_wait();
@@ -309,44 +314,48 @@ __global__ void __launch_bounds__(kThreads, 8) sample_fill_kernel(FillArgs a) {
   const int groups = 32 / k;
   const int lane = lane_id();
   const int sub = lane / k, s = lane - sub * k;
-  const int g0 = sub * k;  // the group's first lane
+  const int g0 = sub * k;  // the group's first lane (>= 32 - k for idle lanes)
   const bool member = sub < groups;
-  const unsigned gmask = k == 32 ? 0xffffffffu : (((1u << k) - 1u) << g0);
   const uint32_t capk32 = (uint32_t)a.capK;
   const int64_t warp0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t e0 = E0 + warp0 * groups; e0 < E1; e0 += nwarps * groups) {
     const int64_t i = e0 + sub;
-    bool has = false;
-    int32_t u = 0;
-    uint32_t j = 0;
-    int64_t eidx = 0;
-    if (member && i < E1) {  // whole group takes the same branches
-      const int32_t v = a.fb_id[i];
-      const uint32_t g = (uint32_t)a.fb_pos[i];
-      const longlong2 bd = a.fbd[i];
-      const int64_t base = bd.x, d = bd.y;
-      j = g / capk32;
-      const uint32_t pos = g - j * capk32;
-      eidx = a.indptr[j * (a.cap_prev + 1) + pos] + s;
-      if (d <= k) {
-        if (s < d) {
-          u = edge_at<kSrc>(a, v, base, d, s);
-          has = true;
-        }
-      } else {
-        const int64_t J = d - k + s;
-        const int64_t t = draw(a, key, v, s, key.gid0 + j, J);
-        bool collided = false;
-        for (int q = 0; q < k; ++q) {
-          const int64_t mine = collided ? J : t;
-          const int64_t cq = __shfl_sync(gmask, mine, g0 + q);
-          if (s > q && t == cq) collided = true;
-        }
-        u = edge_at<kSrc>(a, v, base, d, collided ? J : t);
-        has = true;
+    const bool live = member && i < E1;
+    int32_t v = 0;
+    uint32_t g = 0;
+    longlong2 bd = make_longlong2(0, 0);
+    if (live) {
+      v = a.fb_id[i];
+      g = (uint32_t)a.fb_pos[i];
+      bd = a.fbd[i];
+    }
+    const int64_t base = bd.x, d = bd.y;
+    const uint32_t j = g / capk32;
+    const uint32_t pos = g - j * capk32;
+    int64_t eidx = s;
+    if (live) eidx += a.indptr[j * (a.cap_prev + 1) + pos];
+    // Floyd's algorithm: slot s draws t in [0, J], J = d - k + s, and takes J
+    // when an earlier slot of the node holds t
+    const int64_t J = d - k + s;
+    const int64_t t = draw(a, key, v, s, key.gid0 + j, J);
+    bool collided = false;
+    if (__any_sync(0xffffffffu, d > (int64_t)0xffffffffu)) {  // positions past 32 bits
+      for (int q = 0; q < k; ++q) {
+        const int64_t cq = __shfl_sync(0xffffffffu, collided ? J : t, g0 + q);
+        if (s > q && t == cq) collided = true;
+      }
+    } else {
+      const uint32_t t32 = (uint32_t)t, J32 = (uint32_t)J;
+      for (int q = 0; q < k; ++q) {
+        const uint32_t cq = __shfl_sync(0xffffffffu, collided ? J32 : t32, g0 + q);
+        if (s > q && t32 == cq) collided = true;
       }
     }
+    const bool small = d <= k;
+    const bool has = live && (!small || s < d);
+    int32_t u = 0;
+    if (has) u = edge_at<kSrc>(a, v, base, d, small ? (int64_t)s : collided ? J : t);
     emit_edges(a, has, u, j, eidx);
   }
 }
