@@ -183,7 +183,7 @@ agnes_status agnes_load_graph(const agnes_graph_desc* desc, int device, void* cu
  * targets (range, distinctness) run on the device and are reported by the
  * next agnes_fetch_minibatch / agnes_hyperbatch_stats call as EINVAL.
  * Errors here: EINVAL (bad scalar args), ERANGE (H * capacity >= 2^31 output
- * rows), ENOMEM, ECUDA. */
+ * rows, or H * the graph's tiles >= 2^31 bucket cells), ENOMEM, ECUDA. */
 agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, int32_t H,
                                       int32_t B, const int32_t* fanouts, int32_t K,
                                       uint64_t seed, uint64_t first_minibatch_id,

@@ -86,7 +86,7 @@ __device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell*
   c->fn = a.fcell_off[cell + 1] - c->fo;
   c->so = a.soff[cell];
   c->sn = a.soff[cell + 1] - c->so;
-  c->t = (int32_t)(cell / a.H);
+  c->t = (int32_t)((uint32_t)cell / (uint32_t)a.H);  // cells < 2^31
   c->j = (int32_t)(cell - (int64_t)c->t * a.H);
   return true;
 }
@@ -490,7 +490,7 @@ __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs
       const int32_t fo = a.fcell_off[cell];
       const int32_t so = a.soff[cell];
       const int32_t sn = a.soff[cell + 1] - so;
-      const int32_t j = (int32_t)(cell % a.H);
+      const int32_t j = (int32_t)((uint32_t)cell % (uint32_t)a.H);
       s_nfo[tid] = a.nfcell_off[cell];
       s_src[tid] = sn == 0 && !a.sampled ? fo : ~(fo + so);
       s_row[tid] = (int32_t)((int64_t)j * a.capK +

@@ -69,15 +69,22 @@ struct CellFacts {
   int32_t fo, fn, so, sn, t, j;
 };
 
-__device__ __forceinline__ CellFacts cell_facts(const CellsArgs& a, int64_t cell) {
+// Cell (t, j) = t * H + j.
+__device__ __forceinline__ CellFacts cell_facts(const CellsArgs& a, int64_t cell, int32_t t,
+                                                int32_t j) {
   CellFacts c;
   c.fo = a.fcell_off[cell];
   c.fn = a.fcell_off[cell + 1] - c.fo;
   c.so = a.soff[cell];
   c.sn = a.soff[cell + 1] - c.so;
-  c.t = (int32_t)(cell / a.H);
-  c.j = (int32_t)(cell - (int64_t)c.t * a.H);
+  c.t = t;
+  c.j = j;
   return c;
+}
+
+__device__ __forceinline__ CellFacts cell_facts(const CellsArgs& a, int64_t cell) {
+  const int32_t t = (int32_t)((uint32_t)cell / (uint32_t)a.H);  // cells < 2^31
+  return cell_facts(a, cell, t, (int32_t)cell - t * a.H);
 }
 
 // Sampled entry i of the bucket as (tile-local id, edge index); base is the
@@ -181,11 +188,15 @@ __global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
   const int64_t nw = (int64_t)gridDim.x * kWarps;
   const int64_t b_lo = gw * nbatch / nw, b_hi = (gw + 1) * nbatch / nw;
   int32_t queued = 0;
+  // the lane's cell (t, j), advanced by 32 cells per batch
+  int32_t t = (int32_t)((uint32_t)((b_lo << 5) + lane) / (uint32_t)a.H);  // cells < 2^31
+  int32_t j = (int32_t)((b_lo << 5) + lane) - t * a.H;
   for (int64_t b = b_lo; b < b_hi; ++b) {
     const int64_t cell = (b << 5) + lane;
     const bool has = cell < a.ncells;
     CellFacts c{0, 0, 0, 0, 0, 0};
-    if (has) c = cell_facts(a, cell);
+    if (has) c = cell_facts(a, cell, t, j);
+    for (j += 32; j >= a.H; j -= a.H) ++t;
     const int32_t n = c.fn + c.sn;
     if (has && c.fn > 0) a.adj_flags[a.tile_adj_block[c.t]] = 1;
     if (has && c.sn == 0) {  // nothing sampled: the compaction copies the frontier cell

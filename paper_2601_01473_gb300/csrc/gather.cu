@@ -124,7 +124,7 @@ __global__ void mark_kernel(const int32_t* __restrict__ cell_off, int32_t T, int
   const int64_t ncells = (int64_t)T * H;
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < ncells;
        c += (int64_t)gridDim.x * blockDim.x)
-    if (cell_off[c + 1] > cell_off[c]) flags[map[c / H]] = 1;
+    if (cell_off[c + 1] > cell_off[c]) flags[map[(uint32_t)c / (uint32_t)H]] = 1;
 }
 
 // Requests per feature block: counts[tile_feat_block[t]] += entries of tile t.

@@ -637,6 +637,10 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
     set_err(ctx, "H x node capacity (%lld) exceeds 2^31", (long long)(H * cap[K]));
     return AGNES_ERANGE;
   }
+  if ((int64_t)H * ctx->bt.T >= lim) {  // cell indices are 31-bit in the kernels
+    set_err(ctx, "H x tiles (%lld) exceeds 2^31", (long long)(H * ctx->bt.T));
+    return AGNES_ERANGE;
+  }
   DeviceGuard dg(ctx->device);
   if (!dg.ok()) {
     set_err(ctx, "cudaSetDevice(%d) failed", ctx->device);
