@@ -444,7 +444,7 @@ def main():
     peak, peak_kind = measured_peak()
     g_ms = statistics.mean(gather_ms) if gather_ms else None
     achieved = gather_bytes / (g_ms / 1e3) / 1e9 if g_ms else None
-    roofline = {"bound": "hbm", "kernel": "gather_vec_kernel<16,4>",
+    roofline = {"bound": "hbm", "kernel": "gather_vec_kernel<16,8>",
                 "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak if achieved else None,
                 "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"

@@ -17,6 +17,12 @@ namespace agnes {
 namespace {
 
 constexpr int kThreads = 256;
+// CTAs per SM of the gather (0: as many as fit) and rows in flight per lane.
+// A few CTAs with several rows each keep HBM busy and leave the rest of each
+// SM to the kernels of the next hyperbatch, which run beside the gather when
+// two hyperbatches are in flight.
+constexpr int kGatherCtasPerSm = 3;
+constexpr int kU = 8;
 
 // LPR lanes per row, row = LPR 16-byte vectors, U rows in flight per lane.
 template <int LPR, int U>
@@ -86,6 +92,11 @@ gather_bytes_kernel(const uint8_t* __restrict__ feats, int64_t row_bytes,
   }
 }
 
+int gather_grid(const void* kernel, int num_sms) {
+  const int g = resident_grid(kernel, kThreads, num_sms);
+  return kGatherCtasPerSm > 0 && g > kGatherCtasPerSm * num_sms ? kGatherCtasPerSm * num_sms : g;
+}
+
 }  // namespace
 
 cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* fb_id,
@@ -97,16 +108,16 @@ cudaError_t launch_gather(const void* feats, int64_t row_bytes, const int32_t* f
     const int64_t vecs = row_bytes / 16;
     const uint4* f = (const uint4*)feats;
     uint4* o = (uint4*)out;
-#define AGNES_GRID(KERNEL) resident_grid((const void*)KERNEL, kThreads, num_sms), kThreads, 0, st
+#define AGNES_GRID(KERNEL) gather_grid((const void*)KERNEL, num_sms), kThreads, 0, st
     if (vecs == 8)
-      gather_vec_kernel<8, 4><<<AGNES_GRID((gather_vec_kernel<8, 4>))>>>(f, fb_id, fb_pos, total, o,
-                                                                         status);
+      gather_vec_kernel<8, kU><<<AGNES_GRID((gather_vec_kernel<8, kU>))>>>(f, fb_id, fb_pos, total,
+                                                                           o, status);
     else if (vecs == 16)
-      gather_vec_kernel<16, 4><<<AGNES_GRID((gather_vec_kernel<16, 4>))>>>(f, fb_id, fb_pos, total,
-                                                                           o, status);
+      gather_vec_kernel<16, kU><<<AGNES_GRID((gather_vec_kernel<16, kU>))>>>(f, fb_id, fb_pos,
+                                                                             total, o, status);
     else if (vecs == 32)
-      gather_vec_kernel<32, 4><<<AGNES_GRID((gather_vec_kernel<32, 4>))>>>(f, fb_id, fb_pos, total,
-                                                                           o, status);
+      gather_vec_kernel<32, kU><<<AGNES_GRID((gather_vec_kernel<32, kU>))>>>(f, fb_id, fb_pos,
+                                                                             total, o, status);
     else
       gather_rows_kernel<<<AGNES_GRID(gather_rows_kernel)>>>(f, vecs, fb_id, fb_pos, total, o,
                                                              status);
