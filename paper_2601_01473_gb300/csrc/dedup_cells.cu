@@ -259,108 +259,164 @@ __global__ void __launch_bounds__(kThreads) queue_compact_kernel(CellsArgs a, in
 
 // ---- queued cells: a warp each, on bitmaps over the tile --------------------------
 
-// A warp's shared-memory scratch: kTileWords (128) words each, lane l owning
-// words 4l .. 4l+3, which it reads and writes as one 16-byte vector
-// (conflict-free).
-struct TileScratch {
-  uint32_t* D;  // frontier ids
-  uint32_t* S;  // sampled ids, then N = S & ~D, the new ids
-  uint32_t* C;  // new ids already entered in the next frontier cell
-  int32_t* pD;  // frontier ids below word w
-  int32_t* pN;  // new ids below word w
+// Marks entries 0 .. n-1 of a cell in a bitmap: put(get(i)) per entry, the
+// lanes taking entries lane, lane + 32, ...; past 64 entries four loads per
+// lane are issued before their marks.
+template <typename Get, typename Put>
+__device__ __forceinline__ void mark_entries(int32_t n, int lane, Get get, Put put) {
+  if (n <= 64) {
+    for (int32_t i = lane; i < n; i += 32) put(get(i));
+    return;
+  }
+  for (int32_t i0 = lane; i0 < n; i0 += 128) {
+    int32_t v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = i0 + 32 * k < n ? get(i0 + 32 * k) : -1;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v[k] >= 0) put(v[k]);
+  }
+}
+
+// A warp's shared-memory scratch, lane l owning words 4l .. 4l+3 of each
+// bitmap over the tile (kTileWords = 128 words), read and written as one
+// 16-byte vector (conflict-free):
+//   D[w]   frontier ids of word w;
+//   N[w]   sampled ids, then the new ids S & ~D once both are marked;
+//   P[w]   frontier ids below word w << 16 | new ids below word w (each at
+//          most 4096, so the two halves add without carries);
+//   C[w]   new ids already entered in the next frontier cell.
+struct TileResolver {
+  const uint32_t* D;
+  const uint32_t* N;
+  const uint32_t* P;
+  uint32_t* C;
+  int2* tmp;            // the cell's next-frontier entries
+  int32_t* col;         // the minibatch's col
+  const int32_t* fpos;  // the cell's frontier rows
+  int32_t base, jrow;
+
+  // Frontier entry i (sorted: i frontier ids lie below it) with tile-local id
+  // v keeps its row; below it in the next cell also lie the new ids below v.
+  __device__ __forceinline__ void frontier(int32_t i, int32_t v, int32_t row) const {
+    const int32_t w = v >> 5;
+    const uint32_t below = (1u << (v & 31)) - 1u;
+    tmp[i + (int32_t)(P[w] & 0xffffu) + __popc(N[w] & below)] = make_int2(base + v, row);
+  }
+
+  // Sampled entry (tile-local id, edge index): col is its frontier twin's
+  // row in dst, or -(1 + r) for the r-th new id of the cell, whose first
+  // entry enters the next frontier cell.
+  __device__ __forceinline__ void sampled(int2 e) const {
+    const int32_t v = e.x;
+    const int32_t w = v >> 5;
+    const uint32_t bit = 1u << (v & 31), below = bit - 1u;
+    const uint32_t dw = D[w];
+    const uint32_t pw = P[w];
+    const int32_t rd = (int32_t)(pw >> 16) + __popc(dw & below);  // frontier ids below
+    if (dw & bit) {
+      col[e.y] = fpos[rd] - jrow;
+    } else {
+      const int32_t rn = (int32_t)(pw & 0xffffu) + __popc(N[w] & below);  // new ids below
+      col[e.y] = -1 - rn;
+      if ((atomicOr(C + w, bit) & bit) == 0u) tmp[rd + rn] = make_int2(base + v, -1 - rn);
+    }
+  }
 };
 
+// One warp per queued cell.  A cell of at most 32 frontier and 64 sampled
+// entries (most queued cells) is read once into registers, with all its loads
+// in flight together, and resolved from there; larger cells are walked twice
+// (mark, resolve).  Each warp loads the next queued cell's offsets while it
+// resolves the current one.
 template <bool kPacked>
-__global__ void __launch_bounds__(kThreads, 8) dedup_tile_kernel(CellsArgs a, int32_t nw) {
+__global__ void __launch_bounds__(kThreads, 5) dedup_tile_kernel(CellsArgs a, int32_t nw) {
   grid_dep_wait();
   if (failed(a.status)) return;
   __shared__ __align__(16) uint32_t D_s[kWarps][kTileWords];
-  __shared__ __align__(16) uint32_t S_s[kWarps][kTileWords];
+  __shared__ __align__(16) uint32_t N_s[kWarps][kTileWords];
+  __shared__ __align__(16) uint32_t P_s[kWarps][kTileWords];
   __shared__ __align__(16) uint32_t C_s[kWarps][kTileWords];
-  __shared__ __align__(16) int32_t pD_s[kWarps][kTileWords];
-  __shared__ __align__(16) int32_t pN_s[kWarps][kTileWords];
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  const TileScratch t{D_s[warp], S_s[warp], C_s[warp], pD_s[warp], pN_s[warp]};
+  uint32_t* D = D_s[warp];
+  uint32_t* N = N_s[warp];
+  uint32_t* P = P_s[warp];
+  uint32_t* C = C_s[warp];
   const int32_t total = a.q_off[nw];
-  const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-  for (int64_t q = blockIdx.x * (int64_t)kWarps + warp; q < total; q += nwarps) {
-    const int64_t cell = a.q_dense[q];
-    const CellFacts c = cell_facts(a, cell);
+  const int32_t nwarps = (int32_t)gridDim.x * kWarps;
+  int32_t q = (int32_t)blockIdx.x * kWarps + warp;
+  int32_t cell = q < total ? a.q_dense[q] : 0;
+  CellFacts c = cell_facts(a, cell);
+  for (; q < total; q += nwarps) {
+    const int32_t next = q + nwarps < total ? a.q_dense[q + nwarps] : cell;
+    const CellFacts cn = cell_facts(a, next);
     const int32_t base = __ldg(a.tile_first + c.t);
+    const int32_t* fid = a.fb_id + c.fo;
+    const int32_t* fpos = a.fb_pos + c.fo;
+    const bool small = c.fn <= 32 && c.sn <= 64;  // warp-uniform
+    int32_t fv = -1, fr = 0;
+    int2 s0 = make_int2(-1, 0), s1 = make_int2(-1, 0);
+    if (small) {
+      if (lane < c.fn) {
+        fv = fid[lane] - base;
+        fr = fpos[lane];
+      }
+      if (lane < c.sn) s0 = sampled_entry<kPacked>(a, c.so + lane, base);
+      if (lane + 32 < c.sn) s1 = sampled_entry<kPacked>(a, c.so + lane + 32, base);
+    }
     // mark D and S
     const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-    reinterpret_cast<uint4*>(t.D)[lane] = z;
-    reinterpret_cast<uint4*>(t.S)[lane] = z;
-    reinterpret_cast<uint4*>(t.C)[lane] = z;
+    reinterpret_cast<uint4*>(D)[lane] = z;
+    reinterpret_cast<uint4*>(N)[lane] = z;
+    reinterpret_cast<uint4*>(C)[lane] = z;
     __syncwarp();
-    for (int32_t i0 = lane; i0 < c.fn; i0 += 128) {  // four entries in flight per lane
-      int32_t v[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        v[k] = i0 + 32 * k < c.fn ? a.fb_id[c.fo + i0 + 32 * k] - base : -1;
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        if (v[k] >= 0) atomicOr(t.D + (v[k] >> 5), 1u << (v[k] & 31));
-    }
-    for (int32_t i0 = lane; i0 < c.sn; i0 += 128) {
-      int32_t v[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        v[k] = i0 + 32 * k < c.sn ? sampled_entry<kPacked>(a, c.so + i0 + 32 * k, base).x : -1;
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        if (v[k] >= 0) atomicOr(t.S + (v[k] >> 5), 1u << (v[k] & 31));
+    if (small) {
+      if (fv >= 0) atomicOr(D + (fv >> 5), 1u << (fv & 31));
+      if (s0.x >= 0) atomicOr(N + (s0.x >> 5), 1u << (s0.x & 31));
+      if (s1.x >= 0) atomicOr(N + (s1.x >> 5), 1u << (s1.x & 31));
+    } else {
+      mark_entries(
+          c.fn, lane, [&](int32_t i) { return fid[i] - base; },
+          [&](int32_t v) { atomicOr(D + (v >> 5), 1u << (v & 31)); });
+      mark_entries(
+          c.sn, lane, [&](int32_t i) { return sampled_entry<kPacked>(a, c.so + i, base).x; },
+          [&](int32_t v) { atomicOr(N + (v >> 5), 1u << (v & 31)); });
     }
     __syncwarp();
-    // N = S & ~D and the per-word prefix counts of D and N
-    const uint4 d = reinterpret_cast<const uint4*>(t.D)[lane];
-    const uint4 sv = reinterpret_cast<const uint4*>(t.S)[lane];
-    const uint4 nv = make_uint4(sv.x & ~d.x, sv.y & ~d.y, sv.z & ~d.z, sv.w & ~d.w);
-    const int32_t cd0 = __popc(d.x), cd1 = __popc(d.y), cd2 = __popc(d.z), cd3 = __popc(d.w);
-    const int32_t cn0 = __popc(nv.x), cn1 = __popc(nv.y), cn2 = __popc(nv.z), cn3 = __popc(nv.w);
-    const int32_t lane_d = cd0 + cd1 + cd2 + cd3, lane_n = cn0 + cn1 + cn2 + cn3;
-    const int32_t ed = warp_incl_scan(lane_d) - lane_d;
-    const int32_t en_incl = warp_incl_scan(lane_n);
-    const int32_t en = en_incl - lane_n;
-    reinterpret_cast<int4*>(t.pD)[lane] =
-        make_int4(ed, ed + cd0, ed + cd0 + cd1, ed + cd0 + cd1 + cd2);
-    reinterpret_cast<int4*>(t.pN)[lane] =
-        make_int4(en, en + cn0, en + cn0 + cn1, en + cn0 + cn1 + cn2);
-    reinterpret_cast<uint4*>(t.S)[lane] = nv;
+    // N = S & ~D and the per-word prefix counts, both halves in one scan
+    const uint4 d = reinterpret_cast<const uint4*>(D)[lane];
+    uint4 nv = reinterpret_cast<const uint4*>(N)[lane];
+    nv.x &= ~d.x;
+    nv.y &= ~d.y;
+    nv.z &= ~d.z;
+    nv.w &= ~d.w;
+    const uint32_t k0 = ((uint32_t)__popc(d.x) << 16) | (uint32_t)__popc(nv.x);
+    const uint32_t k1 = ((uint32_t)__popc(d.y) << 16) | (uint32_t)__popc(nv.y);
+    const uint32_t k2 = ((uint32_t)__popc(d.z) << 16) | (uint32_t)__popc(nv.z);
+    const uint32_t k3 = ((uint32_t)__popc(d.w) << 16) | (uint32_t)__popc(nv.w);
+    const uint32_t mine = k0 + k1 + k2 + k3;
+    const uint32_t incl = warp_incl_scan(mine);
+    const uint32_t ex = incl - mine;
+    reinterpret_cast<uint4*>(P)[lane] = make_uint4(ex, ex + k0, ex + k0 + k1, ex + k0 + k1 + k2);
+    reinterpret_cast<uint4*>(N)[lane] = nv;
     if (lane == 31) {
-      a.newcnt[cell] = en_incl;
-      a.nfcnt[cell] = c.fn + en_incl;
+      a.newcnt[cell] = (int32_t)(incl & 0xffffu);
+      a.nfcnt[cell] = c.fn + (int32_t)(incl & 0xffffu);
     }
     __syncwarp();
-    const uint32_t* N = t.S;
-    const int64_t jrow = (int64_t)c.j * a.capK;
-    int2* tmp = a.tmp + c.fo + c.so;
-    // frontier entries (sorted: entry i has i frontier ids below it) keep
-    // their rows; below them in the next cell also lie the new ids below
-    for (int32_t i = lane; i < c.fn; i += 32) {
-      const int32_t v = a.fb_id[c.fo + i] - base;
-      const int32_t w = v >> 5;
-      const uint32_t below = (1u << (v & 31)) - 1u;
-      tmp[i + t.pN[w] + __popc(N[w] & below)] = make_int2(base + v, a.fb_pos[c.fo + i]);
-    }
-    int32_t* col = a.col + (int64_t)c.j * a.ecap;
-    for (int32_t i = lane; i < c.sn; i += 32) {
-      const int2 e = sampled_entry<kPacked>(a, c.so + i, base);
-      const int32_t v = e.x;
-      const int32_t w = v >> 5;
-      const uint32_t bit = 1u << (v & 31), below = bit - 1u;
-      const uint32_t dw = t.D[w];
-      const int32_t rd = t.pD[w] + __popc(dw & below);  // frontier ids below
-      if (dw & bit) {
-        col[e.y] = (int32_t)(a.fb_pos[c.fo + rd] - jrow);
-      } else {
-        const int32_t rn = t.pN[w] + __popc(N[w] & below);  // new ids below
-        col[e.y] = -1 - rn;
-        if ((atomicOr(t.C + w, bit) & bit) == 0u)  // the id's first entry enters the cell
-          tmp[rd + rn] = make_int2(base + v, -1 - rn);
-      }
+    const TileResolver r{D, N, P, C, a.tmp + c.fo + c.so, a.col + (int64_t)c.j * a.ecap, fpos,
+                         base, (int32_t)((int64_t)c.j * a.capK)};
+    if (small) {
+      if (fv >= 0) r.frontier(lane, fv, fr);
+      if (s0.x >= 0) r.sampled(s0);
+      if (s1.x >= 0) r.sampled(s1);
+    } else {
+      for (int32_t i = lane; i < c.fn; i += 32) r.frontier(i, fid[i] - base, fpos[i]);
+      for (int32_t i = lane; i < c.sn; i += 32) r.sampled(sampled_entry<kPacked>(a, c.so + i, base));
     }
     __syncwarp();  // the scratch is rewritten by the next cell
+    cell = next;
+    c = cn;
   }
 }
 
