@@ -59,7 +59,7 @@ typedef enum {
   AGNES_ENOMEM = 3,   /* device or pinned host allocation failed */
   AGNES_ECUDA = 4,    /* a CUDA runtime call failed */
   AGNES_ESTATE = 5,   /* call out of order (e.g. fetch before prepare) */
-  AGNES_ETIMEOUT = 6, /* a bounded host-side wait ran out */
+  AGNES_ETIMEOUT = 6, /* a bounded wait ran out (on the host, or between CTAs of a kernel) */
   AGNES_EKERNEL = 7   /* a kernel reported an internal inconsistency */
 } agnes_status;
 

@@ -102,6 +102,10 @@ static agnes_status wait_prepared(agnes_ctx* ctx) {
       set_err(ctx, "a target id is repeated within a minibatch");
       return AGNES_EINVAL;
     }
+    if (s & kErrWaitTimeout) {
+      set_err(ctx, "a bounded wait between CTAs ran out (device status word 0x%x)", s);
+      return AGNES_ETIMEOUT;
+    }
     set_err(ctx, "device status word 0x%x", s);
     return AGNES_EKERNEL;
   }

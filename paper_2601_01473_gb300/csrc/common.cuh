@@ -21,6 +21,7 @@ enum : int32_t {
   kErrTargetRange = 1,  // a target id outside [0, N)
   kErrTargetDup = 2,    // a target repeated within a minibatch
   kErrInternal = 4,     // a capacity or consistency check failed
+  kErrWaitTimeout = 8,  // a bounded wait on another CTA's progress ran out
 };
 
 struct TileMap {

@@ -65,12 +65,15 @@ struct Workspace {
   int32_t* q_cnt = nullptr;
   int32_t* q_off = nullptr;
   int32_t* q_dense = nullptr;
-  int32_t q_warps_cap = 0;
+  int32_t* q_next = nullptr;
+  int32_t q_chunks_cap = 0;
   int32_t* big_n = nullptr;
   int32_t* tmp_id = nullptr;
   int32_t* tmp_pos = nullptr;
   int32_t* cnt = nullptr;
   int64_t* fbd = nullptr;  // 2 per frontier entry: (first edge, degree)
+  uint64_t* flat_scratch = nullptr;  // single-pass scans of the cell counts (zero between scans)
+  int64_t flat_elems = 0;
   void* feats_out = nullptr;
   uint8_t* adj_flags = nullptr;
   uint8_t* feat_flags = nullptr;

@@ -538,8 +538,7 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
   int gx = (num_sms * 8 + a.H - 1) / a.H;
   if (gx < 1) gx = 1;
   const dim3 egrid(gx, a.H);
-  cudaError_t e = seg_scan<int32_t, int32_t>(d.scnt, 0, d.soff, 0, nullptr, ncells, 1, ncells,
-                                             true, nullptr, d.scan_scratch, a.status, st);
+  cudaError_t e = cells_scan(d.scnt, d.soff, ncells, d.flat_scratch, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
   dedup_scatter_kernel<<<egrid, kThreads, 0, st>>>(d.nbr, d.ecnt, a.ecap, d.scell, d.srank,
                                                    d.soff, d.sb, a.sb_packed, a.status);
@@ -601,8 +600,7 @@ cudaError_t launch_dedup(const HopArgs& a, const DedupBufs& d, int num_sms, cuda
                  st);
     if (e != cudaSuccess) return e;
   }
-  e = seg_scan<int32_t, int32_t>(d.nfcnt, 0, d.nfcell_off, 0, nullptr, ncells, 1, ncells, true,
-                                 nullptr, d.scan_scratch, a.status, st);
+  e = cells_scan(d.nfcnt, d.nfcell_off, ncells, d.flat_scratch, d.scan_scratch, a.status, st);
   if (e != cudaSuccess) return e;
   if (d.side && (e = cudaStreamWaitEvent(st, d.ready, 0)) != cudaSuccess) return e;
   if (!d.frontier_sampled) {

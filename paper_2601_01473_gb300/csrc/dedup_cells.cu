@@ -58,10 +58,11 @@ struct CellsArgs {
   int32_t* nfcnt;
   int2* tmp;     // per cell at fcell_off + soff: next-frontier entries, local ranks
   int32_t* col;  // H x ecap
-  int32_t* q_cells;  // per warp of the lane kernel: its queued cells, at its range's start
-  int32_t* q_cnt;    // per warp: how many
-  int32_t* q_off;    // exclusive scan of q_cnt (nw + 1)
+  int32_t* q_cells;  // per chunk of kChunkCells cells: its queued cells, at the chunk's start
+  int32_t* q_cnt;    // per chunk: how many
+  int32_t* q_off;    // exclusive scan of q_cnt (nchunks + 1)
   int32_t* q_dense;  // the queue, in cell order
+  int32_t* q_next;   // the lane kernel's next chunk (zero between launches)
   const int32_t* status;
 };
 
@@ -174,19 +175,18 @@ __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, co
   a.nfcnt[cell] = c.fn + cnt_new;
 }
 
-// Walks every cell, a warp over 32 consecutive cells at a time; each warp
-// takes a contiguous range of batches and appends its queued cells (with
-// samples and more than kLaneMax entries) in order at the start of its own
-// range of q_cells (q_cnt[warp] of them).
+// Walks every cell, a warp over 32 consecutive cells at a time.  Warps take
+// chunks of kChunkCells cells from a counter (cells differ widely in cost, so
+// fixed ranges would leave warps idle); each appends its queued cells (with
+// samples and more than kLaneMax entries) in order at the start of the
+// chunk's range of q_cells (q_cnt[chunk] of them).
+constexpr int kChunkCells = kDedupChunkCells;
+constexpr int kChunkBatches = kChunkCells / 32;
+
+// Batches [b_lo, b_hi) of one chunk.
 template <bool kPacked>
-__global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
-  grid_dep_wait();
-  if (failed(a.status)) return;
-  const int lane = lane_id();
-  const int64_t nbatch = (a.ncells + 31) >> 5;
-  const int64_t gw = blockIdx.x * (int64_t)kWarps + (threadIdx.x >> 5);
-  const int64_t nw = (int64_t)gridDim.x * kWarps;
-  const int64_t b_lo = gw * nbatch / nw, b_hi = (gw + 1) * nbatch / nw;
+__device__ __forceinline__ void lane_chunk(const CellsArgs& a, int lane, int64_t b_lo,
+                                           int64_t b_hi, int32_t chunk) {
   int32_t queued = 0;
   // the lane's cell (t, j), advanced by 32 cells per batch
   int32_t t = (int32_t)((uint32_t)((b_lo << 5) + lane) / (uint32_t)a.H);  // cells < 2^31
@@ -209,25 +209,47 @@ __global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
     queued += __popc(qm);
     if (has && c.sn > 0 && n <= kLaneMax) thread_cell<kPacked>(a, cell, c);
   }
-  if (lane == 0) a.q_cnt[gw] = queued;
+  if (lane == 0) a.q_cnt[chunk] = queued;
 }
 
-// The queue in cell order: q_off = the exclusive scan of the warps' counts
-// (one CTA) ...
+template <bool kPacked>
+__global__ void __launch_bounds__(kThreads, 6) dedup_lane_kernel(CellsArgs a) {
+  grid_dep_wait();
+  if (failed(a.status)) return;
+  const int lane = lane_id();
+  const int64_t nbatch = (a.ncells + 31) >> 5;
+  const int32_t nchunks = (int32_t)((a.ncells + kChunkCells - 1) / kChunkCells);
+  for (;;) {
+    int32_t chunk = 0;
+    if (lane == 0) chunk = atomicAdd(a.q_next, 1);
+    chunk = __shfl_sync(kFull, chunk, 0);
+    if (chunk >= nchunks) break;
+    lane_chunk<kPacked>(a, lane, (int64_t)chunk * kChunkBatches,
+                        min((int64_t)(chunk + 1) * kChunkBatches, nbatch), chunk);
+  }
+}
+
+// The queue in cell order: q_off = the exclusive scan of the chunks' counts
+// (one CTA, four counts per thread and round; it also rewinds the lane
+// kernel's chunk counter) ...
 __global__ void __launch_bounds__(1024) queue_offsets_kernel(const int32_t* q_cnt, int32_t nw,
-                                                             int32_t* q_off,
+                                                             int32_t* q_off, int32_t* q_next,
                                                              const int32_t* status) {
   grid_dep_wait();
+  if (threadIdx.x == 0) *q_next = 0;
   if (failed(status)) return;
   __shared__ int32_t wsum[32];
   __shared__ int32_t carry;
   if (threadIdx.x == 0) carry = 0;
   __syncthreads();
   const int lane = lane_id(), w = threadIdx.x >> 5;
-  for (int32_t base = 0; base < nw; base += 1024) {
-    const int32_t i = base + threadIdx.x;
-    const int32_t v = i < nw ? q_cnt[i] : 0;
-    const int32_t incl = warp_incl_scan(v);
+  for (int32_t base = 0; base < nw; base += 4096) {
+    const int32_t i = base + 4 * (int32_t)threadIdx.x;
+    int32_t v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = i + k < nw ? q_cnt[i + k] : 0;
+    const int32_t mine = v[0] + v[1] + v[2] + v[3];
+    const int32_t incl = warp_incl_scan(mine);
     if (lane == 31) wsum[w] = incl;
     __syncthreads();
     if (w == 0) {
@@ -235,23 +257,27 @@ __global__ void __launch_bounds__(1024) queue_offsets_kernel(const int32_t* q_cn
       wsum[lane] = warp_incl_scan(t) - t;
     }
     __syncthreads();
-    if (i < nw) q_off[i] = carry + wsum[w] + incl - v;
+    int32_t run = carry + wsum[w] + incl - mine;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (i + k < nw) q_off[i + k] = run;
+      run += v[k];
+    }
     __syncthreads();
-    if (threadIdx.x == 1023) carry += wsum[31] + incl;
+    if (threadIdx.x == 1023) carry = run;
     __syncthreads();
   }
   if (threadIdx.x == 0) q_off[nw] = carry;
 }
 
-// ... then each warp's run copied to q_dense[q_off[warp] ...).
+// ... then each chunk's run copied to q_dense[q_off[chunk] ...).
 __global__ void __launch_bounds__(kThreads) queue_compact_kernel(CellsArgs a, int32_t nw) {
   grid_dep_wait();
   if (failed(a.status)) return;
   const int lane = lane_id();
-  const int64_t nbatch = (a.ncells + 31) >> 5;
   const int64_t nwarps = (int64_t)gridDim.x * kWarps;
   for (int64_t r = blockIdx.x * (int64_t)kWarps + (threadIdx.x >> 5); r < nw; r += nwarps) {
-    const int64_t src = (r * nbatch / nw) << 5;
+    const int64_t src = r * kChunkCells;
     const int32_t dst = a.q_off[r], cnt = a.q_off[r + 1] - dst;
     for (int32_t i = lane; i < cnt; i += 32) a.q_dense[dst + i] = a.q_cells[src + i];
   }
@@ -442,22 +468,23 @@ CellsArgs cells_args(const HopArgs& h, const DedupBufs& d) {
   a.q_cnt = d.q_cnt;
   a.q_off = d.q_off;
   a.q_dense = d.q_dense;
+  a.q_next = d.q_next;
   a.status = h.status;
   return a;
 }
 
 template <bool kPacked>
-cudaError_t launch_cells(const CellsArgs& a, int32_t q_warps_cap, int num_sms, cudaStream_t st) {
+cudaError_t launch_cells(const CellsArgs& a, int32_t q_chunks_cap, int num_sms, cudaStream_t st) {
   const int grid = resident_grid((const void*)dedup_lane_kernel<kPacked>, kThreads, num_sms);
-  const int nw = grid * kWarps;
-  if (nw > q_warps_cap) return cudaErrorInvalidValue;
+  const int64_t nw = (a.ncells + kChunkCells - 1) / kChunkCells;  // chunks
+  if (nw > q_chunks_cap) return cudaErrorInvalidValue;
   dedup_lane_kernel<kPacked><<<grid, kThreads, 0, st>>>(a);
-  queue_offsets_kernel<<<1, 1024, 0, st>>>(a.q_cnt, nw, a.q_off, a.status);
+  queue_offsets_kernel<<<1, 1024, 0, st>>>(a.q_cnt, (int32_t)nw, a.q_off, a.q_next, a.status);
   queue_compact_kernel<<<resident_grid((const void*)queue_compact_kernel, kThreads, num_sms),
-                         kThreads, 0, st>>>(a, nw);
+                         kThreads, 0, st>>>(a, (int32_t)nw);
   dedup_tile_kernel<kPacked><<<resident_grid((const void*)dedup_tile_kernel<kPacked>, kThreads,
                                              num_sms),
-                               kThreads, 0, st>>>(a, nw);
+                               kThreads, 0, st>>>(a, (int32_t)nw);
   return cudaGetLastError();
 }
 
@@ -466,8 +493,8 @@ cudaError_t launch_cells(const CellsArgs& a, int32_t q_warps_cap, int num_sms, c
 cudaError_t launch_dedup_cells(const HopArgs& h, const DedupBufs& d, int num_sms,
                                cudaStream_t st) {
   const CellsArgs a = cells_args(h, d);
-  return h.sb_packed ? launch_cells<true>(a, d.q_warps_cap, num_sms, st)
-                     : launch_cells<false>(a, d.q_warps_cap, num_sms, st);
+  return h.sb_packed ? launch_cells<true>(a, d.q_chunks_cap, num_sms, st)
+                     : launch_cells<false>(a, d.q_chunks_cap, num_sms, st);
 }
 
 }  // namespace agnes

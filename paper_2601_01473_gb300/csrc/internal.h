@@ -27,6 +27,28 @@ cudaError_t seg_scan(const InT* in, int64_t in_stride, OutT* out, int64_t out_st
                      bool write_end, int32_t* seg_total, int64_t* scratch,
                      const int32_t* status, cudaStream_t st);
 
+// Single-pass exclusive scan of n int32 values (decoupled look-back): out[i]
+// = sum of in[i'] for i' < i; with write_end out[n] = the total; total_out
+// (if non-null) gets it too.  in and out 16-byte aligned
+// (flat_scan_supported).  scratch needs flat_scan_scratch_elems(n) uint64s,
+// zero before first use (the scan leaves it zero again).  Scans sharing a
+// scratch must be ordered on one stream.
+int64_t flat_scan_scratch_elems(int64_t max_n);
+bool flat_scan_supported(const int32_t* in, const int32_t* out);
+cudaError_t flat_scan(const int32_t* in, int32_t* out, int64_t n, bool write_end,
+                      int32_t* total_out, uint64_t* scratch, int32_t* status, cudaStream_t st);
+
+// Exclusive scan of n int32 cell counts into out (n + 1 entries, the total
+// last): single pass where flat_scratch is given and the arrays allow it,
+// else the three-phase seg_scan with scan_scratch.
+inline cudaError_t cells_scan(const int32_t* in, int32_t* out, int64_t n, uint64_t* flat_scratch,
+                              int64_t* scan_scratch, int32_t* status, cudaStream_t st) {
+  if (flat_scratch && flat_scan_supported(in, out))
+    return flat_scan(in, out, n, true, nullptr, flat_scratch, status, st);
+  return seg_scan<int32_t, int32_t>(in, 0, out, 0, nullptr, n, 1, n, true, nullptr, scan_scratch,
+                                    status, st);
+}
+
 // Exclusive scan down each column of a row-major [rows x cols] matrix:
 // out[r*cols + c] = sum of in[r'*cols + c] over r' < r (coalesced along
 // rows).  total_out[c] (if non-null) = column total + add_in[c] (add_in may be
@@ -111,8 +133,8 @@ cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32
                                   const int32_t* tile_first, const int32_t* chunk_tile, int32_t T,
                                   int32_t* fcnt, int32_t* fcell_off, int32_t* tmp_id,
                                   int32_t* tmp_pos, int32_t* fb_id, int32_t* fb_pos,
-                                  int64_t* scan_scratch, int32_t* status, int num_sms,
-                                  cudaStream_t st);
+                                  int64_t* scan_scratch, uint64_t* flat_scratch, int32_t* status,
+                                  int num_sms, cudaStream_t st);
 
 cudaError_t launch_sample_count(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
                                 const int32_t* fcell_off, int32_t* cnt, int num_sms,
@@ -149,6 +171,8 @@ constexpr int kDedupSmallMax = 32;
 // by one thread each; larger cells with samples are queued (q_dense), so the
 // queue holds at most (entries) / (kDedupLaneMax + 1) cells.
 constexpr int kDedupLaneMax = 8;
+// The lane kernel's unit of dynamically scheduled work: 256 consecutive cells.
+constexpr int kDedupChunkCells = 256;
 
 struct DedupBufs {
   const int32_t* nbr;       // H x ecap sampled ids
@@ -162,14 +186,16 @@ struct DedupBufs {
   int32_t* big_list;        // cells with more than kDedupSmallMax entries
   int32_t* big_n;           // their count
   // default frontier: the queue of cells with samples and more than
-  // kDedupLaneMax entries: per warp of the lane kernel a run in q_cells (T*H),
-  // their counts and offsets (q_warps_cap, q_warps_cap + 1), and the queue in
-  // cell order (q_dense)
+  // kDedupLaneMax entries: per chunk of kDedupChunkCells cells a run in
+  // q_cells (T*H), the runs' counts and offsets (q_chunks_cap,
+  // q_chunks_cap + 1), the queue in cell order (q_dense), and the lane
+  // kernel's chunk counter (q_next, zero between launches)
   int32_t* q_cells;
   int32_t* q_cnt;
   int32_t* q_off;
   int32_t* q_dense;
-  int32_t q_warps_cap;
+  int32_t* q_next;
+  int32_t q_chunks_cap;
   const int32_t* fb_id;     // current frontier bucket
   const int32_t* fb_pos;
   const int32_t* fcell_off;
@@ -189,6 +215,7 @@ struct DedupBufs {
   const int32_t* tile_adj_block;
   uint8_t* adj_flags;       // per topology block: touched at this hop
   int64_t* scan_scratch;
+  uint64_t* flat_scratch = nullptr;  // flat_scan_scratch_elems(T*H), or null
   // If side is set, the new-id scan (into newbase, with side_scratch) and the
   // col fix-up (which needs only newbase, col and scell) run on it, forked
   // from st through the event fork; st waits for the scan through the event

@@ -63,12 +63,14 @@ void free_workspace(Workspace* w) {
   cudaFree(w->hset);
   cudaFree(w->q_cnt);
   cudaFree(w->q_off);
+  cudaFree(w->q_next);
   cudaFree(w->q_dense);
   cudaFree(w->big_n);
   cudaFree(w->tmp_id);
   cudaFree(w->tmp_pos);
   cudaFree(w->cnt);
   cudaFree(w->fbd);
+  cudaFree(w->flat_scratch);
   cudaFree(w->feats_out);
   cudaFree(w->adj_flags);
   cudaFree(w->feat_flags);
@@ -160,10 +162,11 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.tmp, rows + edges);
   WA(w.big_list, (rows + edges) / (kDedupSmallMax + 1) + 1);
   WA(w.big_n, 1);
-  w.q_warps_cap = ctx->num_sms * 64;  // warps resident at most (64 per SM)
+  w.q_chunks_cap = (int32_t)((cells + kDedupChunkCells - 1) / kDedupChunkCells);
   WA(w.q_cells, cells);
-  WA(w.q_cnt, w.q_warps_cap);
-  WA(w.q_off, w.q_warps_cap + 1);
+  WA(w.q_cnt, w.q_chunks_cap);
+  WA(w.q_off, w.q_chunks_cap + 1);
+  WA(w.q_next, 1);
   WA(w.q_dense, (rows + edges) / (kDedupLaneMax + 1) + 1);
   w.hset_elems = 0;
   for (int h = 0; h < K; ++h) {
@@ -176,6 +179,8 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   WA(w.tmp_pos, (int64_t)H * B);
   WA(w.cnt, (int64_t)H * w.cap_prev_max);
   WA(w.fbd, 2 * (int64_t)H * w.cap_prev_max);
+  w.flat_elems = flat_scan_scratch_elems(cells);
+  WA(w.flat_scratch, w.flat_elems);
   {
     uint8_t* f = nullptr;
     WA(f, rows * ctx->row_bytes);
@@ -202,7 +207,9 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   if (cudaMemset(w.scan_scratch, 0, sizeof(int64_t) * scratch) != cudaSuccess ||
       cudaMemset(w.side_scratch, 0, sizeof(int64_t) * s4) != cudaSuccess ||
       cudaMemset(w.fcnt, 0, sizeof(int32_t) * cells) != cudaSuccess ||
-      cudaMemset(w.scnt, 0, sizeof(int32_t) * cells) != cudaSuccess) {
+      cudaMemset(w.scnt, 0, sizeof(int32_t) * cells) != cudaSuccess ||
+      cudaMemset(w.q_next, 0, sizeof(int32_t)) != cudaSuccess ||
+      cudaMemset(w.flat_scratch, 0, sizeof(uint64_t) * w.flat_elems) != cudaSuccess) {
     free_workspace(&w);
     set_err(ctx, "cudaMemset failed");
     return AGNES_ECUDA;
@@ -306,7 +313,8 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
   CK(ctx, cudaGetLastError());
   CK(ctx, launch_bucket_targets(w.nodes, w.capK, H, B, (int32_t)ctx->N, ctx->bt.tile_first,
                                 ctx->bt.chunk_tile, T, w.fcnt, w.fcell_off[0], w.tmp_id, w.tmp_pos,
-                                w.fb_id[0], w.fb_pos[0], w.scan_scratch, w.status, nsm, st));
+                                w.fb_id[0], w.fb_pos[0], w.scan_scratch, w.flat_scratch, w.status,
+                                nsm, st));
   int cur = 0;
   for (int h = 0; h < K; ++h) {
     mark();
@@ -381,7 +389,8 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.q_cnt = w.q_cnt;
     d.q_off = w.q_off;
     d.q_dense = w.q_dense;
-    d.q_warps_cap = w.q_warps_cap;
+    d.q_next = w.q_next;
+    d.q_chunks_cap = w.q_chunks_cap;
 
     d.big_n = w.big_n;
     d.fb_id = w.fb_id[cur];
@@ -403,6 +412,7 @@ static agnes_status enqueue_hyperbatch(agnes_ctx* ctx, const int32_t* fanouts, i
     d.tile_adj_block = ctx->bt.tile_adj_block;
     d.adj_flags = w.adj_flags + (int64_t)h * ctx->bt.n_blocks;
     d.scan_scratch = w.scan_scratch;
+    d.flat_scratch = w.flat_scratch;
     d.side = ctx->aux;
     d.fork = ctx->aux_fork;
     d.ready = ctx->aux_ready;

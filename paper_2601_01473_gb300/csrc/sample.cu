@@ -521,14 +521,13 @@ cudaError_t launch_bucket_targets(int32_t* nodes, int64_t capK, int32_t H, int32
                                   const int32_t* tile_first, const int32_t* chunk_tile, int32_t T,
                                   int32_t* fcnt, int32_t* fcell_off, int32_t* tmp_id,
                                   int32_t* tmp_pos, int32_t* fb_id, int32_t* fb_pos,
-                                  int64_t* scan_scratch, int32_t* status, int num_sms,
-                                  cudaStream_t st) {
+                                  int64_t* scan_scratch, uint64_t* flat_scratch, int32_t* status,
+                                  int num_sms, cudaStream_t st) {
   const TileMap tm{tile_first, chunk_tile, T};
   const int64_t ncells = (int64_t)T * H;
   const int grid = resident_grid((const void*)targets_count_kernel, kThreads, num_sms);
   targets_count_kernel<<<grid, kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, status);
-  cudaError_t e = seg_scan<int32_t, int32_t>(fcnt, 0, fcell_off, 0, nullptr, ncells, 1, ncells,
-                                             true, nullptr, scan_scratch, status, st);
+  cudaError_t e = cells_scan(fcnt, fcell_off, ncells, flat_scratch, scan_scratch, status, st);
   if (e != cudaSuccess) return e;
   targets_scatter_kernel<<<resident_grid((const void*)targets_scatter_kernel, kThreads, num_sms),
                            kThreads, 0, st>>>(nodes, capK, H, B, N, tm, fcnt, fcell_off,

@@ -247,6 +247,146 @@ col_down_kernel(const int32_t* __restrict__ in, int32_t* __restrict__ out, int64
   }
 }
 
+// ---- single-pass flat scan (decoupled look-back) ----------------------------------
+//
+// Merrill & Garland's single-pass prefix scan (2016): every CTA takes the next
+// tile of kFlatTile elements from a counter, publishes its tile's sum, and
+// derives its exclusive prefix by walking back over its predecessors' flags
+// until it meets an inclusive prefix; it then publishes that as well.  CTAs
+// take tiles in the order they start, so a CTA waits only on tiles of CTAs
+// that are already running; each wait is still bounded (kFlatSpinLimit
+// polls), after which the CTA records kErrWaitTimeout and carries on.
+//
+// Scratch (uint64, zero between scans): [0] tile counter, [1] finished
+// CTAs, [2 + t] flag of tile t = state << 62 | value, state 1 = the tile's
+// sum, 2 = the inclusive prefix through the tile.  The last CTA to finish
+// clears the flags and the counters.
+constexpr int kFlatItems = 16;  // consecutive elements per thread (four 16-byte vectors)
+constexpr int64_t kFlatTile = (int64_t)kThreads * kFlatItems;
+constexpr unsigned long long kFlagAgg = 1ull << 62;
+constexpr unsigned long long kFlagInc = 2ull << 62;
+constexpr unsigned long long kFlagVal = (1ull << 62) - 1;
+constexpr int kFlatSpinLimit = 1 << 20;
+
+__device__ __forceinline__ unsigned long long flag_load(const unsigned long long* p) {
+  return *(const volatile unsigned long long*)p;
+}
+
+__global__ void __launch_bounds__(kThreads)
+flat_scan_kernel(const int32_t* __restrict__ in, int32_t* __restrict__ out, int64_t n,
+                 bool write_end, int32_t* total_out, unsigned long long* scratch,
+                 int32_t* status) {
+  grid_dep_wait();
+  // no early return on a failed status: every CTA takes its tile and counts
+  // itself finished, so the scratch is left zero for the next scan
+  __shared__ int64_t s_tile, s_excl;
+  __shared__ int64_t warp_tot[kThreads / 32];
+  __shared__ bool s_last;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t ntiles = (int64_t)gridDim.x;
+  unsigned long long* flags = scratch + 2;
+  if (tid == 0) {
+    const int64_t t = (int64_t)atomicAdd(scratch, 1ull);
+    if (t == ntiles - 1) scratch[0] = 0;  // every CTA has taken its tile
+    s_tile = t;
+  }
+  __syncthreads();
+  const int64_t tile = s_tile;
+  // the thread's 16 consecutive elements
+  const int64_t i0 = tile * kFlatTile + (int64_t)tid * kFlatItems;
+  int32_t v[kFlatItems];
+  if (i0 + kFlatItems <= n) {
+    const int4* p = reinterpret_cast<const int4*>(in + i0);
+#pragma unroll
+    for (int q = 0; q < kFlatItems / 4; ++q) {
+      const int4 x = p[q];
+      v[4 * q] = x.x;
+      v[4 * q + 1] = x.y;
+      v[4 * q + 2] = x.z;
+      v[4 * q + 3] = x.w;
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < kFlatItems; ++k) v[k] = i0 + k < n ? in[i0 + k] : 0;
+  }
+  int64_t mine = 0;
+#pragma unroll
+  for (int k = 0; k < kFlatItems; ++k) mine += v[k];
+  // block scan of the threads' sums
+  const int64_t incl = warp_incl_scan(mine);
+  if (lane == 31) warp_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const int64_t w = lane < kThreads / 32 ? warp_tot[lane] : 0;
+    const int64_t wi = warp_incl_scan(w);
+    if (lane < kThreads / 32) warp_tot[lane] = wi - w;
+    const int64_t agg = __shfl_sync(0xffffffffu, wi, kThreads / 32 - 1);
+    // publish, look back, publish the inclusive prefix
+    int64_t excl = 0;
+    if (tile == 0) {
+      if (lane == 0) atomicExch(flags, kFlagInc | (unsigned long long)agg);
+    } else {
+      if (lane == 0) atomicExch(flags + tile, kFlagAgg | (unsigned long long)agg);
+      for (int64_t j = tile - 1;; j -= 32) {
+        const int64_t idx = j - lane;  // lane 0 the nearest predecessor
+        unsigned long long f = kFlagInc;  // before tile 0: an inclusive prefix of 0
+        if (idx >= 0) {
+          f = flag_load(flags + idx);
+          for (int spin = 0; (f >> 62) == 0; ++spin) {
+            if (spin == kFlatSpinLimit) {
+              atomicOr(status, kErrWaitTimeout);
+              f = kFlagInc;
+              break;
+            }
+            __nanosleep(64);
+            f = flag_load(flags + idx);
+          }
+        }
+        const unsigned inc = __ballot_sync(0xffffffffu, (f >> 62) == 2);
+        const int stop = inc ? __ffs(inc) - 1 : 31;  // lanes 0 .. stop contribute
+        excl += warp_sum(lane <= stop ? (int64_t)(f & kFlagVal) : (int64_t)0);
+        if (inc) break;
+      }
+      if (lane == 0) atomicExch(flags + tile, kFlagInc | (unsigned long long)(excl + agg));
+    }
+    if (lane == 0) {
+      s_excl = excl;
+      if (tile == ntiles - 1) {
+        if (write_end) out[n] = (int32_t)(excl + agg);
+        if (total_out) *total_out = (int32_t)(excl + agg);
+      }
+    }
+  }
+  __syncthreads();
+  int64_t run = s_excl + warp_tot[warp] + incl - mine;
+  int32_t o[kFlatItems];
+#pragma unroll
+  for (int k = 0; k < kFlatItems; ++k) {
+    o[k] = (int32_t)run;
+    run += v[k];
+  }
+  if (i0 + kFlatItems <= n) {
+    int4* p = reinterpret_cast<int4*>(out + i0);
+#pragma unroll
+    for (int q = 0; q < kFlatItems / 4; ++q)
+      p[q] = make_int4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+  } else {
+#pragma unroll
+    for (int k = 0; k < kFlatItems; ++k)
+      if (i0 + k < n) out[i0 + k] = o[k];
+  }
+  // the last CTA to finish (all look-backs done) clears the scratch
+  if (tid == 0) {
+    __threadfence();
+    s_last = atomicAdd(scratch + 1, 1ull) == (unsigned long long)(ntiles - 1);
+  }
+  __syncthreads();
+  if (s_last) {
+    for (int64_t t = tid; t < ntiles; t += kThreads) flags[t] = 0;
+    if (tid == 0) scratch[1] = 0;
+  }
+}
+
 }  // namespace
 
 int64_t col_scan_scratch_elems(int64_t rows, int32_t cols) {
@@ -292,6 +432,24 @@ int64_t scan_scratch_elems(int64_t nseg, int64_t max_len) {
   int64_t chunks = (max_len + kChunk - 1) / kChunk;
   if (chunks < 1) chunks = 1;
   return kTicketElems + nseg * chunks;
+}
+
+int64_t flat_scan_scratch_elems(int64_t max_n) {
+  return 2 + (max_n + kFlatTile - 1) / kFlatTile + 1;
+}
+
+bool flat_scan_supported(const int32_t* in, const int32_t* out) {
+  return (uintptr_t)in % 16 == 0 && (uintptr_t)out % 16 == 0;
+}
+
+cudaError_t flat_scan(const int32_t* in, int32_t* out, int64_t n, bool write_end,
+                      int32_t* total_out, uint64_t* scratch, int32_t* status, cudaStream_t st) {
+  if (!flat_scan_supported(in, out)) return cudaErrorInvalidValue;
+  const int64_t ntiles = n > 0 ? (n + kFlatTile - 1) / kFlatTile : 1;
+  if (ntiles > 0x7fffffff) return cudaErrorInvalidValue;
+  flat_scan_kernel<<<(unsigned)ntiles, kThreads, 0, st>>>(
+      in, out, n, write_end, total_out, reinterpret_cast<unsigned long long*>(scratch), status);
+  return cudaGetLastError();
 }
 
 template <typename InT, typename OutT>
