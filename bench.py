@@ -127,14 +127,14 @@ class ClockSampler:
 
 
 def kernel_launches_per_step(K: int) -> int:
-    """Kernels libagnes launches per hyperbatch with the graph in HBM (67 at
-    K = 3): the sampling-key write and the dst-size fill 2; target bucketing 5
-    (count, 2-kernel scan, scatter, sort); per hop 18 (count, 2-kernel scan,
-    fill, 2-kernel scan, scatter, the cells' lane kernel, queue offsets, queue
-    copy, tile kernel, 3-kernel column scan, 2-kernel scan, col fix-up,
-    compaction); after the last hop 3 (feature-block marks, their count,
-    gather) and K counts of touched topology blocks."""
-    return 2 + 5 + 18 * K + 3 + K
+    """Kernels libagnes launches per hyperbatch with the graph in HBM (60 at
+    K = 3): the sampling-key write and the dst-size fill 2; target bucketing 4
+    (count, single-pass scan, scatter, sort); per hop 16 (count, 2-kernel
+    segmented scan, fill, single-pass scan, scatter, the cells' lane kernel,
+    queue offsets, queue copy, tile kernel, 3-kernel column scan, single-pass
+    scan, col fix-up, compaction); after the last hop 3 (feature-block marks,
+    their count, gather) and K counts of touched topology blocks."""
+    return 2 + 4 + 16 * K + 3 + K
 
 
 def algorithmic_bytes(c: dict, off_bytes: int) -> dict:

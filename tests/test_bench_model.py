@@ -24,10 +24,10 @@ def test_algorithmic_bytes_by_hand():
 
 
 def test_launch_count_per_step():
-    # key + size fill, 5 for the targets, 18 per hop, mark + count + gather, one count per hop;
-    # 67 at K = 3 is the count of the ncu launch list of one rmat100m hyperbatch
-    assert bench.kernel_launches_per_step(3) == 67
-    assert bench.kernel_launches_per_step(1) == 2 + 5 + 18 + 3 + 1
+    # key + size fill, 4 for the targets, 16 per hop, mark + count + gather, one count per hop;
+    # 60 at K = 3 is the count of the ncu launch list of one rmat100m hyperbatch
+    assert bench.kernel_launches_per_step(3) == 60
+    assert bench.kernel_launches_per_step(1) == 2 + 4 + 16 + 3 + 1
 
 
 def test_profiled_traffic_only_for_its_workload_and_source():
