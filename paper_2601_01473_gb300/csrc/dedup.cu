@@ -499,32 +499,51 @@ __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs
     if (tid == 0) s_nfo[last - c0] = a.nfcell_off[last];
     __syncthreads();
     const int32_t k0 = s_nfo[0], k1 = s_nfo[last - c0];
-    for (int32_t k = k0 + tid; k < k1; k += kCellThreads) {
-      int32_t lo = 0, hi = (int32_t)(last - c0);  // last cell with nfo <= k
-      while (hi - lo > 1) {
-        const int32_t mid = (lo + hi) >> 1;
-        if (s_nfo[mid] <= k) lo = mid; else hi = mid;
-      }
-      const int32_t r = k - s_nfo[lo];
-      const int32_t src = s_src[lo];
-      int32_t id, pos;
-      if (src >= 0) {
-        id = a.fb_id[src + r];
-        pos = a.fb_pos[src + r];
-      } else {
-        const int2 e = a.tmp[~src + r];
-        id = e.x;
-        pos = e.y;
-        if (a.sampled) {
-          pos = s_row[lo] + r;
-          a.nodes[pos] = id;
-        } else if (pos < 0) {
-          pos = s_row[lo] + (-1 - pos);
-          a.nodes[pos] = id;
+    // two entries per thread and round: both loads in flight before the stores
+    for (int32_t kb = k0 + tid; kb < k1; kb += 2 * kCellThreads) {
+      int32_t cl[2], r[2], id[2], pos[2];
+      bool in[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int32_t k = kb + u * kCellThreads;
+        in[u] = k < k1;
+        int32_t lo = 0, hi = (int32_t)(last - c0);  // last cell with nfo <= k
+        while (hi - lo > 1) {
+          const int32_t mid = (lo + hi) >> 1;
+          if (s_nfo[mid] <= k) lo = mid; else hi = mid;
+        }
+        cl[u] = lo;
+        r[u] = k - s_nfo[lo];
+        id[u] = 0;
+        pos[u] = 0;
+        if (in[u]) {
+          const int32_t src = s_src[lo];
+          if (src >= 0) {
+            id[u] = a.fb_id[src + r[u]];
+            pos[u] = a.fb_pos[src + r[u]];
+          } else {
+            const int2 e = a.tmp[~src + r[u]];
+            id[u] = e.x;
+            pos[u] = e.y;
+          }
         }
       }
-      a.nfb_id[k] = id;
-      a.nfb_pos[k] = pos;
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        if (!in[u]) continue;
+        const int32_t k = kb + u * kCellThreads;
+        if (s_src[cl[u]] < 0) {
+          if (a.sampled) {
+            pos[u] = s_row[cl[u]] + r[u];
+            a.nodes[pos[u]] = id[u];
+          } else if (pos[u] < 0) {
+            pos[u] = s_row[cl[u]] + (-1 - pos[u]);
+            a.nodes[pos[u]] = id[u];
+          }
+        }
+        a.nfb_id[k] = id[u];
+        a.nfb_pos[k] = pos[u];
+      }
     }
     __syncthreads();
   }
