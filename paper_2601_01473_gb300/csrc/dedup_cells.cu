@@ -103,8 +103,8 @@ __device__ __forceinline__ int2 sampled_entry(const CellsArgs& a, int32_t i, int
 
 // ---- cells of at most kLaneMax entries: a thread each ---------------------------
 
-template <int I, int J>
-__device__ __forceinline__ void cmp_swap(int32_t (&k)[kLaneMax], int32_t (&p)[kLaneMax]) {
+template <int I, int J, int W>
+__device__ __forceinline__ void cmp_swap(int32_t (&k)[W], int32_t (&p)[W]) {
   const bool sw = k[I] > k[J];
   const int32_t ki = k[I], pi = p[I];
   k[I] = sw ? k[J] : ki;
@@ -113,9 +113,16 @@ __device__ __forceinline__ void cmp_swap(int32_t (&k)[kLaneMax], int32_t (&p)[kL
   p[J] = sw ? pi : p[J];
 }
 
+// Sorts 4 (key, payload) pairs by key in registers: 5 comparators.
+__device__ __forceinline__ void sort_net(int32_t (&k)[4], int32_t (&p)[4]) {
+  cmp_swap<0, 1>(k, p); cmp_swap<2, 3>(k, p);
+  cmp_swap<0, 2>(k, p); cmp_swap<1, 3>(k, p);
+  cmp_swap<1, 2>(k, p);
+}
+
 // Sorts 8 (key, payload) pairs by key in registers: a 19-comparator network
 // in six layers.
-__device__ __forceinline__ void sort8(int32_t (&k)[kLaneMax], int32_t (&p)[kLaneMax]) {
+__device__ __forceinline__ void sort_net(int32_t (&k)[8], int32_t (&p)[8]) {
   cmp_swap<0, 2>(k, p); cmp_swap<1, 3>(k, p); cmp_swap<4, 6>(k, p); cmp_swap<5, 7>(k, p);
   cmp_swap<0, 4>(k, p); cmp_swap<1, 5>(k, p); cmp_swap<2, 6>(k, p); cmp_swap<3, 7>(k, p);
   cmp_swap<0, 1>(k, p); cmp_swap<2, 3>(k, p); cmp_swap<4, 5>(k, p); cmp_swap<6, 7>(k, p);
@@ -124,14 +131,15 @@ __device__ __forceinline__ void sort8(int32_t (&k)[kLaneMax], int32_t (&p)[kLane
   cmp_swap<1, 2>(k, p); cmp_swap<3, 4>(k, p); cmp_swap<5, 6>(k, p);
 }
 
-// Resolves one cell with samples and at most kLaneMax entries in one thread.
-template <bool kPacked>
+// Resolves one cell with samples and at most W (4 or 8, kLaneMax at most)
+// entries in one thread.
+template <bool kPacked, int W>
 __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, const CellFacts& c) {
   const int32_t n = c.fn + c.sn;
   const int32_t tb = __ldg(a.tile_first + c.t);
-  int32_t key[kLaneMax], pay[kLaneMax];
+  int32_t key[W], pay[W];
 #pragma unroll
-  for (int q = 0; q < kLaneMax; ++q) {
+  for (int q = 0; q < W; ++q) {
     key[q] = kNoKey;
     pay[q] = 0;
     if (q < c.fn) {
@@ -143,7 +151,7 @@ __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, co
       pay[q] = e.y;
     }
   }
-  sort8(key, pay);
+  sort_net(key, pay);
   // sweep: the first entry of each id is its frontier twin (sorted first) or,
   // without one, the new id's first occurrence
   const int64_t jrow = (int64_t)c.j * a.capK;
@@ -151,7 +159,7 @@ __device__ __forceinline__ void thread_cell(const CellsArgs& a, int64_t cell, co
   int2* tmp = a.tmp + c.fo + c.so;
   int32_t prev = -1, cnt_new = 0, cnt_keep = 0, cur = 0;  // cur: col of the current id
 #pragma unroll
-  for (int q = 0; q < kLaneMax; ++q) {
+  for (int q = 0; q < W; ++q) {
     if (key[q] != kNoKey) {
       const int32_t lu = key[q] >> 1;
       const bool sampled = key[q] & 1;
@@ -207,7 +215,13 @@ __device__ __forceinline__ void lane_chunk(const CellsArgs& a, int lane, int64_t
     if ((qm >> lane) & 1u)
       a.q_cells[(b_lo << 5) + queued + __popc(qm & ((1u << lane) - 1u))] = (int32_t)cell;
     queued += __popc(qm);
-    if (has && c.sn > 0 && n <= kLaneMax) thread_cell<kPacked>(a, cell, c);
+    // the warp takes the 4-entry network unless one of its cells needs 8
+    const bool mine = has && c.sn > 0 && n <= kLaneMax;
+    if (__any_sync(kFull, mine && n > 4)) {
+      if (mine) thread_cell<kPacked, 8>(a, cell, c);
+    } else if (mine) {
+      thread_cell<kPacked, 4>(a, cell, c);
+    }
   }
   if (lane == 0) a.q_cnt[chunk] = queued;
 }
