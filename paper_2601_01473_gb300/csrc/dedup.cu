@@ -41,11 +41,13 @@ dedup_scatter_kernel(const int32_t* __restrict__ nbr, const int32_t* __restrict_
   const int64_t o = (int64_t)j * ecap;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < E;
        e += (int64_t)gridDim.x * blockDim.x) {
-    const int32_t slot = soff[scell[o + e]] + srank[o + e];
-    if (packed)  // nbr holds the tile-local id (< 2^12), e < 2^20
-      reinterpret_cast<uint32_t*>(sb)[slot] = ((uint32_t)e << 12) | (uint32_t)nbr[o + e];
-    else
-      sb[slot] = make_int2(nbr[o + e], (int32_t)e);
+    if (packed) {  // nbr holds rank << 12 | tile-local id; e < 2^20
+      const uint32_t v = (uint32_t)nbr[o + e];
+      reinterpret_cast<uint32_t*>(sb)[soff[scell[o + e]] + (v >> 12)] =
+          ((uint32_t)e << 12) | (v & 0xfffu);
+    } else {
+      sb[soff[scell[o + e]] + srank[o + e]] = make_int2(nbr[o + e], (int32_t)e);
+    }
   }
 }
 

@@ -156,7 +156,9 @@ struct FillRange {
 
 // Samples the frontier entries of cells [r.cell_lo, r.cell_hi) and records,
 // per sampled edge, its neighbour id (nbr), its (tile, minibatch) cell (scell)
-// and its rank within that cell (srank), counting the cells in scnt.
+// and its rank within that cell (srank), counting the cells in scnt.  With
+// HopArgs::sb_packed, nbr holds rank << 12 | tile-local id and srank is not
+// written.
 cudaError_t launch_sample_fill(const HopArgs& a, const int32_t* fb_id, const int32_t* fb_pos,
                                const int32_t* fcell_off, const int64_t* indptr, int32_t* nbr,
                                int32_t* scnt, int32_t* scell, int32_t* srank,
@@ -175,10 +177,10 @@ constexpr int kDedupLaneMax = 8;
 constexpr int kDedupChunkCells = 256;
 
 struct DedupBufs {
-  const int32_t* nbr;       // H x ecap sampled ids
+  const int32_t* nbr;       // H x ecap sampled ids (packed: rank << 12 | tile-local id)
   const int32_t* ecnt;      // H edge counts
   const int32_t* scell;     // H x ecap: cell of each sampled id
-  const int32_t* srank;     // H x ecap: its rank within the cell
+  const int32_t* srank;     // H x ecap: its rank within the cell (not packed)
   const int32_t* scnt;      // T*H per-cell counts of sampled ids
   int32_t* soff;            // T*H+1
   int2* sb;                 // bucketed (sampled id, edge index in the minibatch)

@@ -222,7 +222,8 @@ struct FillArgs {
   int32_t k, hop;
   const uint64_t* key;  // device: {seed, first minibatch id}
   int32_t* status;
-  bool packed;        // record tile-local ids (the dedup's sampled bucket is packed)
+  bool packed;        // record rank << 12 | tile-local id in nbr, no srank (the dedup's
+                      // sampled bucket is packed)
   int32_t* hset;      // fanouts above kWideMax: per-warp hash sets of chosen positions
   int32_t hset_log2;  // each of 2^hset_log2 entries
 };
@@ -294,9 +295,14 @@ __device__ __forceinline__ void emit_edges(const FillArgs& a, bool has, int32_t 
   old = __shfl_sync(0xffffffffu, old, leader);
   if (has) {
     const int64_t at = (int64_t)j * a.ecap + eidx;
-    a.nbr[at] = val;
+    const int32_t rank = old + __popc(peers & ((1u << lane) - 1u));
     a.scell[at] = (int32_t)cell;
-    a.srank[at] = old + __popc(peers & ((1u << lane) - 1u));
+    if (a.packed) {  // rank < ecap <= 2^20 beside the 12-bit tile-local id
+      a.nbr[at] = (rank << 12) | val;
+    } else {
+      a.nbr[at] = val;
+      a.srank[at] = rank;
+    }
   }
 }
 
