@@ -108,6 +108,7 @@ __device__ __forceinline__ bool load_cell(const CellArgs& a, int64_t cell, Cell*
 //            among the cell's new ids is lessN.
 // Cells with more than 32 entries go to the big-cell list.
 constexpr int kCellThreads = 128;  // threads per CTA of the cells kernel
+constexpr int kCompactIlp = 2;     // bucket entries per thread and round of the compaction (4 and 8 measured slower)
 constexpr int kGroupCells = kCellThreads;
 constexpr int kSlotCap = 1024;
 constexpr int kSmallMax = kDedupSmallMax;
@@ -501,12 +502,12 @@ __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs
     if (tid == 0) s_nfo[last - c0] = a.nfcell_off[last];
     __syncthreads();
     const int32_t k0 = s_nfo[0], k1 = s_nfo[last - c0];
-    // two entries per thread and round: both loads in flight before the stores
-    for (int32_t kb = k0 + tid; kb < k1; kb += 2 * kCellThreads) {
-      int32_t cl[2], r[2], id[2], pos[2];
-      bool in[2];
+    // kCompactIlp entries per thread and round: their loads in flight before the stores
+    for (int32_t kb = k0 + tid; kb < k1; kb += kCompactIlp * kCellThreads) {
+      int32_t cl[kCompactIlp], r[kCompactIlp], id[kCompactIlp], pos[kCompactIlp];
+      bool in[kCompactIlp];
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
+      for (int u = 0; u < kCompactIlp; ++u) {
         const int32_t k = kb + u * kCellThreads;
         in[u] = k < k1;
         int32_t lo = 0, hi = (int32_t)(last - c0);  // last cell with nfo <= k
@@ -531,7 +532,7 @@ __global__ void __launch_bounds__(kCellThreads) dedup_compact_kernel(CompactArgs
         }
       }
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
+      for (int u = 0; u < kCompactIlp; ++u) {
         if (!in[u]) continue;
         const int32_t k = kb + u * kCellThreads;
         if (s_src[cl[u]] < 0) {
