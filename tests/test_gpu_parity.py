@@ -176,6 +176,24 @@ def test_parity_small_rmat(cuda_device, bits, dtype, fanouts):
     g.close()
 
 
+@pytest.mark.parametrize("frontier", ["src", "sampled"])
+def test_parity_edge_capacity_past_packed_bucket(cuda_device, frontier):
+    """Hop 2's edge capacity per minibatch (41,984 frontier slots x 30) passes
+    2^20, so that hop keeps the sampled bucket as (id, edge index) pairs and
+    the sampler's separate rank array; hop 1 packs its entries into 4 bytes.
+    Both layouts in one hyperbatch, every minibatch against the oracle."""
+    n, B, fanouts = 60000, 1024, [40, 30]
+    assert min(n, B * (1 + fanouts[0])) * fanouts[1] > 1 << 20 > B * fanouts[0]
+    off, ind, feats = make(n, 12, seed=77, bits=64, dtype=torch.float16)
+    og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
+    targets = synth.hyperbatch_targets(torch.arange(n, dtype=torch.int32), 2, B, 12, 64)
+    g = load(off, ind, feats, 8192, 4096)
+    g.set_frontier(frontier)
+    g.prepare(targets.to(cuda_device), fanouts, 0x5EED, 40)
+    compare(g, og, targets.numpy(), fanouts, 0x5EED, 40, 8192, 4096, frontier=frontier)
+    g.close()
+
+
 def test_block_table_matches_oracle(cuda_device):
     for bits, bb in ((32, 64), (64, 256), (64, 4096), (32, 65536)):
         off, ind, feats = make(20000, 20, a=0.6, b=0.2, c=0.15, seed=bb, bits=bits)
