@@ -290,7 +290,7 @@ def main():
     ap.add_argument("--launch-mode", default="graph_pdl", choices=["direct", "graph", "graph_pdl"],
                     help="resident path: direct launches, one CUDA graph per hyperbatch shape, "
                          "or the graph with programmatic kernel edges")
-    ap.add_argument("--pipeline-depth", type=int, default=2, choices=[1, 2],
+    ap.add_argument("--pipeline-depth", type=int, default=3, choices=[1, 2, 3, 4],
                     help="hyperbatches in flight inside the library (resident graph only)")
     ap.add_argument("--feature-io", default="blocks", choices=["blocks", "rows"],
                     help="with --stream: load whole feature blocks, or read requested rows in place")
@@ -429,10 +429,10 @@ def main():
             g.prepare(host_targets[s], fan, w.seed, gid(s), stream)
             if depth == 1:
                 g.fetch_all()
-            elif s > args.warmup:  # the previous hyperbatch, while this one runs
-                g.fetch_previous()
-        if depth == 2:
-            g.fetch_all()
+            elif s - args.warmup >= depth - 1:  # the oldest one held, while the later ones run
+                g.fetch_earlier(depth - 1)
+        for ago in range(min(depth, args.steps) - 2, -1, -1):  # the ones still unread
+            g.fetch_earlier(ago)
         torch.cuda.synchronize()
         e2e_s = time.perf_counter() - t0
         e2e_s = reduce_max(e2e_s, pg, dev)
@@ -576,7 +576,8 @@ def run_sweep(args, w):
     fan = list(w.fanouts)
     for bb in [int(x) for x in args.sweep_blocks.split(",")]:
         g = Graph(offsets, indices, features, bb, bb, device=0, stream=stream)
-        g.set_pipeline_depth(args.pipeline_depth)
+        # at most two in flight here: H = 256 needs twice config 3's workspace per set
+        g.set_pipeline_depth(min(args.pipeline_depth, 2))
         info = g.info()
         for H in [int(x) for x in args.sweep_H.split(",")]:
             wh = w.with_(H=H, adj_block_bytes=bb, feat_block_bytes=bb)

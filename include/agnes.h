@@ -50,6 +50,7 @@ extern "C" {
 #endif
 
 #define AGNES_MAX_HOPS 8
+#define AGNES_MAX_PIPELINE_DEPTH 4 /* hyperbatches in flight (agnes_set_pipeline_depth) */
 #define AGNES_MAX_FANOUT 65536
 
 typedef enum {
@@ -295,33 +296,45 @@ typedef struct {
 agnes_status agnes_fetch_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out);
 
 /* Hyperbatches in flight.  depth 1 (the default): each prepare is ordered on
- * the caller's stream as described at agnes_prepare_hyperbatch.  depth 2:
- * the ctx keeps a second workspace (as much device memory again) and a
- * second set of internal streams, and consecutive prepares use the two sets
- * in turn, each on its own internal stream that starts when the caller's
- * stream reaches the call; the caller's stream is not made to wait for the
- * hyperbatch, so one hyperbatch's sampling and dedup overlap the previous
- * one's gather (Sec. 3.4 (4): one stage's latency hidden behind another's
- * transfers).  Then: fetch, stats and counters wait for and describe the last
- * prepared hyperbatch (host side, as before); a stream that consumes the
- * views on the device must first be ordered with
- * agnes_wait_hyperbatches; views stay valid until the second prepare after
- * the one they come from.  depth 2 needs the graph resident in device memory
- * (no features_on_host, no topology_on_host); a prepare issued while the
- * caller's stream is being captured runs as at depth 1.  The call waits for
- * the device.  Errors: EINVAL, ECUDA. */
+ * the caller's stream as described at agnes_prepare_hyperbatch.  depth d in
+ * 2 .. AGNES_MAX_PIPELINE_DEPTH: the ctx keeps d workspaces (d times the
+ * device memory of one) and d sets of internal streams, and consecutive
+ * prepares use the sets in turn, each on its own internal stream that starts
+ * when the caller's stream reaches the call and once the set's previous
+ * hyperbatch (d prepares earlier) is done; the caller's stream is not made to
+ * wait for the hyperbatch, so consecutive hyperbatches overlap (Sec. 3.4 (4):
+ * one stage's latency hidden behind another's work).  Then: fetch, stats and
+ * counters wait for and describe the last prepared hyperbatch (host side, as
+ * before); a stream that consumes the views on the device must first be
+ * ordered with agnes_wait_hyperbatches; views stay valid until the d-th
+ * prepare after the one they come from.  depth > 1 needs the graph resident
+ * in device memory (no features_on_host, no topology_on_host); a prepare
+ * issued while the caller's stream is being captured runs as at depth 1.
+ * The call waits for the device; changing the depth releases the spare sets,
+ * so only the last hyperbatch's views survive it.  Errors: EINVAL, ECUDA. */
 agnes_status agnes_set_pipeline_depth(agnes_ctx* ctx, int32_t depth);
 
-/* At depth 2: the views of the hyperbatch prepared before the last one
+/* At depth > 1: the views of the hyperbatch prepared before the last one
  * (waiting for it like agnes_fetch_hyperbatch), so a caller can take one
  * hyperbatch's results while the next is being prepared.  They stay valid
- * until the next prepare.  Errors: EINVAL, ESTATE (depth 1, or fewer than
- * two prepares), ECUDA, and what agnes_fetch_hyperbatch reports. */
+ * until the (depth - 1)-th prepare after this call.  Errors: EINVAL, ESTATE
+ * (depth 1, or fewer than two prepares), ECUDA, and what
+ * agnes_fetch_hyperbatch reports. */
 agnes_status agnes_fetch_previous_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_view* out);
 
+/* At depth d: the views of the hyperbatch prepared `ago` prepares before the
+ * last one, 0 <= ago < d (0: as agnes_fetch_hyperbatch; 1: as
+ * agnes_fetch_previous_hyperbatch), waiting for it, so a caller can take the
+ * oldest hyperbatch still held while the later ones run.  They stay valid
+ * until the (d - ago)-th prepare after this call.  Errors: EINVAL (ago out
+ * of range), ESTATE (fewer than ago + 1 prepares at this depth), ECUDA, and
+ * what agnes_fetch_hyperbatch reports. */
+agnes_status agnes_fetch_earlier_hyperbatch(agnes_ctx* ctx, int32_t ago,
+                                            agnes_hyperbatch_view* out);
+
 /* Makes cuda_stream wait (on the device) for every hyperbatch prepared and
- * still in flight on the ctx: at depth 2 the two last prepares, at depth 1
- * the last one.  Errors: EINVAL, ECUDA. */
+ * still in flight on the ctx: the last depth prepares.  Errors: EINVAL,
+ * ECUDA. */
 agnes_status agnes_wait_hyperbatches(agnes_ctx* ctx, void* cuda_stream);
 
 /* Blocks touched by the last hyperbatch (the block-wise I/Os of Sec. 3.3 and

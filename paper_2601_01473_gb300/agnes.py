@@ -140,6 +140,7 @@ SIGNATURES = {
     "agnes_set_pipeline_depth": ([_P, ctypes.c_int32], ctypes.c_int),
     "agnes_wait_hyperbatches": ([_P, _P], ctypes.c_int),
     "agnes_fetch_previous_hyperbatch": ([_P, _P], ctypes.c_int),
+    "agnes_fetch_earlier_hyperbatch": ([_P, ctypes.c_int32, _P], ctypes.c_int),
     "agnes_sage_mean_layer": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int64,
                                ctypes.c_int64, _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
                                ctypes.c_int64, _P], ctypes.c_int),
@@ -391,15 +392,24 @@ class Graph:
         _check(lib().agnes_set_launch_mode(self._ctx, LAUNCH[mode]), self._ctx)
 
     def fetch_previous(self) -> HyperbatchView:
-        """At pipeline depth 2: the hyperbatch prepared before the last one
+        """At pipeline depth > 1: the hyperbatch prepared before the last one
         (agnes_fetch_previous_hyperbatch)."""
         v = _HyperbatchView()
         _check(lib().agnes_fetch_previous_hyperbatch(self._ctx, ctypes.byref(v)), self._ctx)
         return HyperbatchView(v, self.device)
 
+    def fetch_earlier(self, ago: int) -> HyperbatchView:
+        """At pipeline depth d: the hyperbatch prepared ``ago`` prepares
+        before the last one, 0 <= ago < d (agnes_fetch_earlier_hyperbatch)."""
+        v = _HyperbatchView()
+        _check(lib().agnes_fetch_earlier_hyperbatch(self._ctx, int(ago), ctypes.byref(v)),
+               self._ctx)
+        return HyperbatchView(v, self.device)
+
     def set_pipeline_depth(self, depth: int) -> None:
-        """Hyperbatches in flight (agnes_set_pipeline_depth): 1, or 2 to let
-        consecutive prepares overlap on the ctx's two internal streams."""
+        """Hyperbatches in flight (agnes_set_pipeline_depth): 1, or up to
+        AGNES_MAX_PIPELINE_DEPTH (4) to let consecutive prepares overlap on
+        the ctx's internal streams, one workspace each."""
         _check(lib().agnes_set_pipeline_depth(self._ctx, int(depth)), self._ctx)
 
     def wait(self, stream=None) -> None:

@@ -456,28 +456,28 @@ agnes_status agnes_set_launch_mode(agnes_ctx* ctx, int32_t mode) {
     return AGNES_EINVAL;
   }
   ctx->lg.mode = mode;
-  ctx->spare.lg.mode = mode;
+  for (agnes_ctx::Spare& o : ctx->spares) o.lg.mode = mode;
   return AGNES_OK;
 }
 
 agnes_status agnes_set_pipeline_depth(agnes_ctx* ctx, int32_t depth) {
   if (!ctx) return AGNES_EINVAL;
-  if (depth != 1 && depth != 2) {
-    set_err(ctx, "pipeline depth must be 1 or 2");
+  if (depth < 1 || depth > AGNES_MAX_PIPELINE_DEPTH) {
+    set_err(ctx, "pipeline depth must be 1 .. %d", AGNES_MAX_PIPELINE_DEPTH);
     return AGNES_EINVAL;
   }
-  if (depth == 2 && (ctx->features_on_host || ctx->topo.on)) {
-    set_err(ctx, "a pipeline depth of 2 needs the graph resident in device memory");
+  if (depth > 1 && (ctx->features_on_host || ctx->topo.on)) {
+    set_err(ctx, "a pipeline depth above 1 needs the graph resident in device memory");
     return AGNES_EINVAL;
   }
   if (depth == ctx->pipe_depth) return AGNES_OK;
   DeviceGuard dg(ctx->device);
   CK(ctx, cudaDeviceSynchronize());
-  if (depth == 2) {
-    const agnes_status rc = make_spare_state(ctx);
+  // the spare sets restart empty (the active set keeps the last hyperbatch)
+  free_spare_state(ctx);
+  if (depth > 1) {
+    const agnes_status rc = make_spare_state(ctx, depth);
     if (rc != AGNES_OK) return rc;
-  } else {
-    free_spare_state(ctx);
   }
   ctx->pipe_depth = depth;
   return AGNES_OK;
@@ -488,13 +488,37 @@ agnes_status agnes_fetch_previous_hyperbatch(agnes_ctx* ctx, agnes_hyperbatch_vi
     set_err(ctx, "ctx and out must be non-NULL");
     return AGNES_EINVAL;
   }
-  if (ctx->pipe_depth != 2 || !ctx->spare.prepared) {
-    set_err(ctx, "no earlier hyperbatch in flight (needs a pipeline depth of 2 and two prepares)");
+  if (ctx->pipe_depth < 2 || !ctx->spares[ctx->pipe_depth - 2].prepared) {
+    set_err(ctx, "no earlier hyperbatch in flight (needs a pipeline depth above 1 and two prepares)");
     return AGNES_ESTATE;
   }
-  swap_hyperbatch_state(ctx);
+  agnes_ctx::Spare& prev = ctx->spares[ctx->pipe_depth - 2];
+  swap_hyperbatch_state(ctx, prev);
   const agnes_status rc = agnes_fetch_hyperbatch(ctx, out);
-  swap_hyperbatch_state(ctx);
+  swap_hyperbatch_state(ctx, prev);
+  return rc;
+}
+
+agnes_status agnes_fetch_earlier_hyperbatch(agnes_ctx* ctx, int32_t ago,
+                                            agnes_hyperbatch_view* out) {
+  if (!ctx || !out) {
+    set_err(ctx, "ctx and out must be non-NULL");
+    return AGNES_EINVAL;
+  }
+  if (ago < 0 || ago >= ctx->pipe_depth) {
+    set_err(ctx, "ago = %d outside [0, %d) (the pipeline depth)", ago, ctx->pipe_depth);
+    return AGNES_EINVAL;
+  }
+  if (ago == 0) return agnes_fetch_hyperbatch(ctx, out);
+  // spares[d - 2] holds the previous hyperbatch, spares[0] the oldest
+  agnes_ctx::Spare& o = ctx->spares[ctx->pipe_depth - 1 - ago];
+  if (!o.prepared) {
+    set_err(ctx, "no hyperbatch %d prepares before the last one", ago);
+    return AGNES_ESTATE;
+  }
+  swap_hyperbatch_state(ctx, o);
+  const agnes_status rc = agnes_fetch_hyperbatch(ctx, out);
+  swap_hyperbatch_state(ctx, o);
   return rc;
 }
 
@@ -503,7 +527,8 @@ agnes_status agnes_wait_hyperbatches(agnes_ctx* ctx, void* cuda_stream) {
   DeviceGuard dg(ctx->device);
   cudaStream_t st = (cudaStream_t)cuda_stream;
   if (ctx->done) CK(ctx, cudaStreamWaitEvent(st, ctx->done, 0));
-  if (ctx->pipe_depth == 2 && ctx->spare.done) CK(ctx, cudaStreamWaitEvent(st, ctx->spare.done, 0));
+  for (int i = 0; i + 1 < ctx->pipe_depth; ++i)
+    if (ctx->spares[i].done) CK(ctx, cudaStreamWaitEvent(st, ctx->spares[i].done, 0));
   return AGNES_OK;
 }
 

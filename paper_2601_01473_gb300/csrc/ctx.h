@@ -173,15 +173,17 @@ struct agnes_ctx {
     int64_t captures = 0, launches = 0, programmatic_edges = 0;
   } lg;
 
-  // Hyperbatches in flight (agnes_set_pipeline_depth): with a depth of 2 the
-  // ctx keeps a second set of the per-hyperbatch state -- workspace, launch
-  // graph, completion and side-stream events, side stream, its own internal
-  // stream and the fetch state -- and swaps it with the active set at every
-  // prepare, so consecutive hyperbatches use alternate sets and run on
-  // alternate internal streams, overlapping.  The active set (the fields
-  // above and pipe_st) always belongs to the last prepare.
+  // Hyperbatches in flight (agnes_set_pipeline_depth): with a depth of d > 1
+  // the ctx keeps d - 1 more sets of the per-hyperbatch state -- workspace,
+  // launch graph, completion and side-stream events, side stream, its own
+  // internal stream and the fetch state -- and rotates them with the active
+  // set at every prepare, so consecutive hyperbatches use the sets in turn
+  // and run on their internal streams, overlapping.  The active set (the
+  // fields above and pipe_st) always belongs to the last prepare; spares[0]
+  // to the oldest hyperbatch still held, spares[d - 2] to the one before the
+  // last.
   int32_t pipe_depth = 1;
-  cudaStream_t pipe_st = nullptr;  // the active set's internal stream (depth 2)
+  cudaStream_t pipe_st = nullptr;  // the active set's internal stream (depth > 1)
   cudaEvent_t pipe_in = nullptr;   // orders an internal stream after the caller's
   struct Spare {
     agnes::Workspace ws;
@@ -192,7 +194,7 @@ struct agnes_ctx {
     cudaStream_t pipe_st = nullptr;
     int cur = 0;
     bool prepared = false, synced = false;
-  } spare;
+  } spares[AGNES_MAX_PIPELINE_DEPTH - 1];
 
   // streaming of host-resident features (features_on_host)
   cudaStream_t copy_stream = nullptr;
@@ -296,10 +298,14 @@ struct agnes_ctx {
 // prepare.cu
 void free_workspace(agnes::Workspace* w);
 void drop_launch_graph(agnes_ctx::LaunchGraph* g);
-// Swaps the active per-hyperbatch state with the spare one (pipeline depth 2).
-void swap_hyperbatch_state(agnes_ctx* ctx);
-// Creates the spare set's events and streams (once); frees the spare set.
-agnes_status make_spare_state(agnes_ctx* ctx);
+// Swaps the active per-hyperbatch state with spare set o.
+void swap_hyperbatch_state(agnes_ctx* ctx, agnes_ctx::Spare& o);
+// Before a prepare at depth d > 1: the oldest set (spares[0]) becomes the
+// active one and the active one the newest spare (spares[d - 2]).
+void rotate_hyperbatch_state(agnes_ctx* ctx);
+// Creates the events and streams of spares[0 .. depth - 2] (once); frees
+// every spare set.
+agnes_status make_spare_state(agnes_ctx* ctx, int32_t depth);
 void free_spare_state(agnes_ctx* ctx);
 
 // host_features.cu

@@ -218,8 +218,7 @@ static agnes_status ensure_workspace(agnes_ctx* ctx, int32_t H, int32_t B, const
   return AGNES_OK;
 }
 
-void swap_hyperbatch_state(agnes_ctx* ctx) {
-  agnes_ctx::Spare& o = ctx->spare;
+void swap_hyperbatch_state(agnes_ctx* ctx, agnes_ctx::Spare& o) {
   std::swap(ctx->ws, o.ws);
   std::swap(ctx->lg, o.lg);
   std::swap(ctx->ws_gen, o.ws_gen);
@@ -234,8 +233,12 @@ void swap_hyperbatch_state(agnes_ctx* ctx) {
   std::swap(ctx->synced, o.synced);
 }
 
-agnes_status make_spare_state(agnes_ctx* ctx) {
-  agnes_ctx::Spare& o = ctx->spare;
+void rotate_hyperbatch_state(agnes_ctx* ctx) {
+  swap_hyperbatch_state(ctx, ctx->spares[0]);
+  for (int i = 0; i + 2 < ctx->pipe_depth; ++i) std::swap(ctx->spares[i], ctx->spares[i + 1]);
+}
+
+static agnes_status make_one_spare(agnes_ctx* ctx, agnes_ctx::Spare& o) {
   if (o.done) return AGNES_OK;
   const unsigned f = cudaEventDisableTiming;
   if (cudaEventCreateWithFlags(&o.done, f) != cudaSuccess ||
@@ -243,33 +246,47 @@ agnes_status make_spare_state(agnes_ctx* ctx) {
       cudaEventCreateWithFlags(&o.aux_join, f) != cudaSuccess ||
       cudaEventCreateWithFlags(&o.aux_ready, f) != cudaSuccess ||
       cudaStreamCreateWithFlags(&o.aux, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&o.pipe_st, cudaStreamNonBlocking) != cudaSuccess ||
-      (!ctx->pipe_st && cudaStreamCreateWithFlags(&ctx->pipe_st, cudaStreamNonBlocking) !=
-                            cudaSuccess) ||
-      (!ctx->pipe_in && cudaEventCreateWithFlags(&ctx->pipe_in, f) != cudaSuccess)) {
+      cudaStreamCreateWithFlags(&o.pipe_st, cudaStreamNonBlocking) != cudaSuccess) {
     cudaGetLastError();
-    set_err(ctx, "creating the second hyperbatch's events or streams failed");
+    set_err(ctx, "creating a further hyperbatch's events or streams failed");
     return AGNES_ECUDA;
   }
   o.lg.mode = ctx->lg.mode;
   return AGNES_OK;
 }
 
+agnes_status make_spare_state(agnes_ctx* ctx, int32_t depth) {
+  for (int i = 0; i + 1 < depth; ++i) {
+    const agnes_status rc = make_one_spare(ctx, ctx->spares[i]);
+    if (rc != AGNES_OK) return rc;
+  }
+  const unsigned f = cudaEventDisableTiming;
+  if ((!ctx->pipe_st && cudaStreamCreateWithFlags(&ctx->pipe_st, cudaStreamNonBlocking) !=
+                            cudaSuccess) ||
+      (!ctx->pipe_in && cudaEventCreateWithFlags(&ctx->pipe_in, f) != cudaSuccess)) {
+    cudaGetLastError();
+    set_err(ctx, "creating the pipeline's stream or event failed");
+    return AGNES_ECUDA;
+  }
+  return AGNES_OK;
+}
+
 void free_spare_state(agnes_ctx* ctx) {
-  agnes_ctx::Spare& o = ctx->spare;
-  drop_launch_graph(&o.lg);
-  if (o.lg.cap) cudaStreamDestroy(o.lg.cap);
-  o.lg.cap = nullptr;
-  free_workspace(&o.ws);
-  if (o.done) cudaEventDestroy(o.done);
-  if (o.aux_fork) cudaEventDestroy(o.aux_fork);
-  if (o.aux_join) cudaEventDestroy(o.aux_join);
-  if (o.aux_ready) cudaEventDestroy(o.aux_ready);
-  if (o.aux) cudaStreamDestroy(o.aux);
-  if (o.pipe_st) cudaStreamDestroy(o.pipe_st);
-  const int32_t mode = o.lg.mode;
-  o = agnes_ctx::Spare();
-  o.lg.mode = mode;
+  for (agnes_ctx::Spare& o : ctx->spares) {
+    drop_launch_graph(&o.lg);
+    if (o.lg.cap) cudaStreamDestroy(o.lg.cap);
+    o.lg.cap = nullptr;
+    free_workspace(&o.ws);
+    if (o.done) cudaEventDestroy(o.done);
+    if (o.aux_fork) cudaEventDestroy(o.aux_fork);
+    if (o.aux_join) cudaEventDestroy(o.aux_join);
+    if (o.aux_ready) cudaEventDestroy(o.aux_ready);
+    if (o.aux) cudaStreamDestroy(o.aux);
+    if (o.pipe_st) cudaStreamDestroy(o.pipe_st);
+    const int32_t mode = o.lg.mode;
+    o = agnes_ctx::Spare();
+    o.lg.mode = mode;
+  }
 }
 
 void drop_launch_graph(agnes_ctx::LaunchGraph* g) {
@@ -659,12 +676,12 @@ agnes_status agnes_prepare_hyperbatch(agnes_ctx* ctx, const int32_t* targets, in
   cudaStream_t st = (cudaStream_t)cuda_stream;
   const bool capturing = stream_capturing(st);
   const bool resident = !ctx->features_on_host && !ctx->topo.on;
-  const bool pipelined = ctx->pipe_depth == 2 && resident && !capturing;
+  const bool pipelined = ctx->pipe_depth > 1 && resident && !capturing;
   if (pipelined) {
-    // the other set of per-hyperbatch state: its internal stream starts once
-    // the caller's stream reaches this call, and is already ordered after the
-    // set's previous hyperbatch
-    swap_hyperbatch_state(ctx);
+    // the least recently used set of per-hyperbatch state: its internal
+    // stream starts once the caller's stream reaches this call, and is
+    // already ordered after the set's previous hyperbatch
+    rotate_hyperbatch_state(ctx);
     CK(ctx, cudaEventRecord(ctx->pipe_in, st));
     CK(ctx, cudaStreamWaitEvent(ctx->pipe_st, ctx->pipe_in, 0));
     st = ctx->pipe_st;

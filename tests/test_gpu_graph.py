@@ -140,16 +140,19 @@ def test_prepares_on_two_streams_run_in_call_order(cuda_device):
     g.close()
 
 
-def test_pipeline_depth_two_matches_oracle_and_overlaps_safely(cuda_device):
-    """Two hyperbatches in flight (agnes_set_pipeline_depth 2): a sequence of
-    prepares on one caller stream, each checked against the oracle through
-    fetch, the hyperbatch before the last through agnes_fetch_previous_hyperbatch
-    while the last is in flight, a device-side consumer ordered with
+@pytest.mark.parametrize("depth", [2, 3, 4])
+def test_pipeline_depth_matches_oracle_and_overlaps_safely(cuda_device, depth):
+    """Several hyperbatches in flight (agnes_set_pipeline_depth 2 .. 4): a
+    sequence of prepares on one caller stream (more than the sets, so every
+    set is reused), each checked against the oracle through fetch, the
+    hyperbatch before the last through agnes_fetch_previous_hyperbatch while
+    the last is in flight, a device-side consumer ordered with
     agnes_wait_hyperbatches, and a return to depth 1."""
+    from paper_2601_01473_gb300 import AgnesError
     off, ind, feats = make(30000, 12, seed=51, dim=32)
     og = oracle.Graph(off.numpy(), ind.numpy(), feats.numpy())
     g = load(off, ind, feats, ADJ, FEAT)
-    g.set_pipeline_depth(2)
+    g.set_pipeline_depth(depth)
     pool = torch.arange(30000, dtype=torch.int32)
     fan = [6, 4, 3]
     tgts = [synth.hyperbatch_targets(pool, 6, 200, 53, s) for s in range(5)]
@@ -163,7 +166,15 @@ def test_pipeline_depth_two_matches_oracle_and_overlaps_safely(cuda_device):
             r = oracle.sample_minibatch(og, tgts[s - 1][2].numpy(), fan, 7, 100 * (s - 1) + 2)
             n = int(prev.node_size[3, 2])
             assert np.array_equal(prev.nodes[2, :n].cpu().numpy(), r["nodes"])
+        if s >= depth - 1:  # the oldest one still held
+            old = g.fetch_earlier(depth - 1)
+            a = s - (depth - 1)
+            r = oracle.sample_minibatch(og, tgts[a][4].numpy(), fan, 7, 100 * a + 4)
+            n = int(old.node_size[3, 4])
+            assert np.array_equal(old.nodes[4, :n].cpu().numpy(), r["nodes"])
         compare(g, og, tgts[s].numpy(), fan, 7, 100 * s, ADJ, FEAT)
+    with pytest.raises(AgnesError):
+        g.fetch_earlier(depth)
     # a device consumer on the caller's stream, ordered by the wait call
     g.prepare(dev[0], fan, 9, 0, st)
     g.prepare(dev[1], fan, 9, 600, st)
@@ -192,3 +203,10 @@ def test_pipeline_depth_two_needs_a_resident_graph(cuda_device):
     with pytest.raises(AgnesError):
         g.set_pipeline_depth(3)
     g.close()
+    r = load(off, ind, feats, 4096, 4096)
+    for bad in (0, 5):  # 1 .. AGNES_MAX_PIPELINE_DEPTH
+        with pytest.raises(AgnesError) as e:
+            r.set_pipeline_depth(bad)
+        assert e.value.status == 1
+    r.set_pipeline_depth(4)
+    r.close()
