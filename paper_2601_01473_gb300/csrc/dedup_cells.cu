@@ -14,17 +14,20 @@
 // Work layout.  Cells are small on average, but the entries concentrate in
 // the larger cells of the tiles that hold the graph's hubs (at rmat100m's hop
 // 3, cells of more than 32 entries hold over half of them), so:
-//   - a lane kernel walks all cells, a warp over 32 consecutive cells at a
-//     time; a cell of at most 8 entries is resolved by its own thread: its
-//     entries become keys (tile-local id << 1 | sampled) in registers,
-//     carried with their rows or edge indices through a 19-comparator sorting
-//     network, and swept once -- equal ids are adjacent with the frontier
-//     entry first, so the first entry of each id is its frontier twin or the
-//     new id's first occurrence;
-//   - larger cells with samples are queued in cell order (each warp appends
-//     its cells in order into its own range; a scan and a copy concatenate
+//   - a lane kernel walks all cells in chunks of 256 taken from a counter, a
+//     warp over 32 consecutive cells at a time; a cell of at most 8 entries
+//     is resolved by its own thread: its entries become keys (tile-local id
+//     << 1 | sampled) in registers, carried with their rows or edge indices
+//     through a 5- or 19-comparator sorting network, and swept once -- equal
+//     ids are adjacent with the frontier entry first, so the first entry of
+//     each id is its frontier twin or the new id's first occurrence;
+//   - larger cells with samples are queued in cell order (each chunk's cells
+//     in order at the start of its own range; a scan and a copy concatenate
 //     the ranges) and resolved one warp per cell on bitmaps over the tile,
 //     where every rank is a popcount over per-word prefix counts.
+// The sampled bucket is either (id, edge index) pairs or, when the hop's
+// edge indices fit 20 bits, packed words edge index << 12 | tile-local id
+// (the kernels' kPacked).
 #include "common.cuh"
 #include "internal.h"
 

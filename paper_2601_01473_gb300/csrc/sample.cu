@@ -11,12 +11,14 @@
 // Sampling (Sec. 3.1, Algorithm 1's Sample): up to k neighbours per frontier
 // node, uniformly without replacement; all of them in CSR order when
 // deg <= k, else Floyd's algorithm (Bentley & Floyd, CACM 1987) with
-// Philox4x32-10 draws keyed on (seed; v, hop, slot, g).  A group of G >= k
-// lanes handles one frontier node: lane s draws slot s's candidate in
-// parallel and the k-step collision resolution runs over in-group shuffles.
-// Above 32 a warp takes 32 slots at a time, checking each candidate against
-// the earlier chunks' choices (in shared memory up to kWideMax, in a hash set
-// in global memory beyond).
+// Philox4x32-10 draws keyed on (seed; v, hop, slot, g).  For k <= 32 a group
+// of k lanes handles one frontier node (32 / k nodes per warp round): lane s
+// draws slot s's candidate in parallel and the k-step collision resolution
+// runs over warp shuffles.  Above 32 a warp takes 32 slots at a time,
+// checking each candidate against the earlier chunks' choices (in shared
+// memory up to kWideMax, in a hash set in global memory beyond).  The count
+// kernel's (first edge, degree) per frontier entry lets the fill read them
+// coalesced.
 #include "common.cuh"
 #include "internal.h"
 
