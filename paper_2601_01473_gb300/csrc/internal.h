@@ -111,7 +111,7 @@ struct HopArgs {
   int32_t hset_grid = 0;
   // the sampled bucket holds 4-byte entries (edge index << 12 | tile-local
   // id): the default frontier with ecap <= kPackedEdgeMax; the sampler then
-  // records tile-local ids
+  // records rank << 12 | tile-local id per edge (no rank array)
   bool sb_packed = false;
   // per frontier entry (bucket order): its node's first edge and degree, two
   // int64 each, written by the count kernel and read by the fill
@@ -183,7 +183,8 @@ struct DedupBufs {
   const int32_t* srank;     // H x ecap: its rank within the cell (not packed)
   const int32_t* scnt;      // T*H per-cell counts of sampled ids
   int32_t* soff;            // T*H+1
-  int2* sb;                 // bucketed (sampled id, edge index in the minibatch)
+  int2* sb;                 // bucketed (sampled id, edge index in the minibatch), or packed
+                            // 4-byte entries edge index << 12 | tile-local id (sb_packed)
   int2* tmp;                // per cell: next-frontier entries with local ranks
   int32_t* big_list;        // cells with more than kDedupSmallMax entries
   int32_t* big_n;           // their count
